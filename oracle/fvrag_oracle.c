@@ -1,0 +1,383 @@
+/*
+ * fvrag oracle -- TEST INFRASTRUCTURE ONLY.
+ *
+ * A plain, slow, fp64 CPU statement of what the verifier hot path of
+ * VideoSpeculateRAG computes.  Only the tests, the smoke check and the CPU
+ * baseline leg of the benchmark may load this library; the product path
+ * (libfvrag, its CUDA kernels and its Python binding) never touches it, and the
+ * two share no code: inputs arrive as raw bf16/fp16 bit patterns and are decoded
+ * here, exactly, by this file's own routines.
+ *
+ * Every floating-point sum runs in fp64 over a fixed index order, so the result
+ * does not depend on the number of OpenMP threads (threads only split
+ * independent output rows).
+ *
+ * Functions and the passages they follow:
+ *   oracle_verify_attn    -- the verifier forward of Eq. 6 / Eq. 11 (Section 3.1,
+ *                            "Two-Stage Verification") restricted to one
+ *                            attention layer: every candidate token attends to
+ *                            the shared prefix (Q, V, retrieved passages) and to
+ *                            its own candidate's tokens up to itself.
+ *   oracle_score_logprobs -- the verifier's token probabilities P(token | ...):
+ *                            log-softmax of the LM-head logits, gathered at the
+ *                            requested token ids (Eq. 11; "self-consistent"
+ *                            likelihood, Section 4.5 "Analysis of Scoring
+ *                            Mechanisms").
+ *   oracle_clip_align     -- Eq. 14 (cosine of CLIP embeddings) and Eq. 15 (max
+ *                            over the frames), plus the keep/drop threshold.
+ *   oracle_select         -- selection: length-normalised likelihood masked by
+ *                            keep (mode 0), or Algorithm 1's two stages:
+ *                            Eq. 12 reliability, Eq. 13 high-reliability set,
+ *                            argmax alignment over it (mode 1).
+ * Readings where the paper is silent are stated beside each function.
+ *
+ * Build: gcc -O2 -fopenmp -shared -fPIC fvrag_oracle.c -o libfvrag_oracle.so -lm
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+int oracle_max_threads(void) {
+#ifdef _OPENMP
+  return omp_get_max_threads();
+#else
+  return 1;
+#endif
+}
+
+void oracle_set_threads(int n) {
+#ifdef _OPENMP
+  if (n > 0) omp_set_num_threads(n);
+#else
+  (void)n;
+#endif
+}
+
+/* ---- exact decoding of the 16-bit formats (IEEE 754 binary16; bfloat16 =
+ * the top half of an IEEE binary32) ---------------------------------------- */
+static double dec_bf16(uint16_t b) {
+  uint32_t u = (uint32_t)b << 16;
+  float f;
+  memcpy(&f, &u, 4);
+  return (double)f;
+}
+
+static double dec_f16(uint16_t h) {
+  int sign = (h >> 15) & 1;
+  int ex = (h >> 10) & 0x1F;
+  int man = h & 0x3FF;
+  double v;
+  if (ex == 0) {
+    v = ldexp((double)man, -24); /* subnormal: man * 2^-24 */
+  } else if (ex == 31) {
+    v = man ? NAN : INFINITY;
+  } else {
+    v = ldexp((double)(man + 1024), ex - 25); /* (1 + man/1024) * 2^(ex-15) */
+  }
+  return sign ? -v : v;
+}
+
+void oracle_decode_bf16(const uint16_t* in, double* out, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) out[i] = dec_bf16(in[i]);
+}
+
+void oracle_decode_f16(const uint16_t* in, double* out, int64_t n) {
+  for (int64_t i = 0; i < n; ++i) out[i] = dec_f16(in[i]);
+}
+
+/*
+ * Attention of one verifier layer over the shared prefix and each candidate's
+ * own tokens.
+ *
+ *   q       [Qn][K][L][Hq][D]   bf16     query of token l of candidate k
+ *   k_pre   [sum P][Hkv][D]     bf16     prefix keys; query qi owns rows
+ *   v_pre   [sum P][Hkv][D]     bf16       offs[qi] .. offs[qi+1]-1
+ *   offs    [Qn+1]              int32
+ *   k_tail  [Qn][K][L][Hkv][D]  bf16     keys / values of the candidate tokens
+ *   v_tail  [Qn][K][L][Hkv][D]  bf16
+ *   row_sel [Qn*K*L*Hq] or NULL          compute only rows with row_sel != 0
+ *   out     [Qn][K][L][Hq][D]   fp64
+ *   lse     [Qn][K][L][Hq]      fp64 or NULL (natural log of the softmax denominator
+ *                                             including the max shift)
+ *
+ * For query qi, candidate k, token l, head h with kv head g = h / (Hq / Hkv):
+ *   keys  S = { prefix j : 0 <= j < P_qi }  U  { tail (k, t) : 0 <= t <= l }
+ *   s_j   = scale * <q, K_j[g]>
+ *   out   = sum_j softmax(s)_j * V_j[g],   lse = max s + ln sum_j exp(s_j - max s)
+ * Readings: candidates do not see one another (Eq. 6 scores each a_i on its own);
+ * consecutive query heads share a KV head; scale = 1/sqrt(D) unless given.
+ * Returns 0, or -1 on bad arguments.
+ */
+int oracle_verify_attn(int Qn, int K, int L, int Hq, int Hkv, int D, double scale,
+                       const uint16_t* q, const uint16_t* k_pre, const uint16_t* v_pre,
+                       const int32_t* offs, const uint16_t* k_tail, const uint16_t* v_tail,
+                       const uint8_t* row_sel, double* out, double* lse) {
+  if (Qn <= 0 || K <= 0 || L <= 0 || Hq <= 0 || Hkv <= 0 || D <= 0 || Hq % Hkv) return -1;
+  if (!q || !offs || !k_tail || !v_tail || !out) return -1;
+  if (scale == 0.0) scale = 1.0 / sqrt((double)D);
+  const int grp = Hq / Hkv;
+  int maxP = 0;
+  for (int qi = 0; qi < Qn; ++qi) {
+    int p = offs[qi + 1] - offs[qi];
+    if (p < 0) return -1;
+    if (p > maxP) maxP = p;
+  }
+  if (maxP > 0 && (!k_pre || !v_pre)) return -1;
+  const int64_t nrows = (int64_t)Qn * K * L * Hq;
+  int bad = 0;
+#pragma omp parallel
+  {
+    double* s = (double*)malloc(sizeof(double) * (size_t)(maxP + L));
+    double* qv = (double*)malloc(sizeof(double) * (size_t)D);
+    double* acc = (double*)malloc(sizeof(double) * (size_t)D);
+    if (!s || !qv || !acc) {
+#pragma omp atomic write
+      bad = 1;
+    }
+#pragma omp for schedule(dynamic, 4)
+    for (int64_t r = 0; r < nrows; ++r) {
+      if (bad) continue;
+      if (row_sel && !row_sel[r]) continue;
+      const int h = (int)(r % Hq);
+      const int64_t tok = r / Hq; /* ((qi*K + k)*L + l) */
+      const int l = (int)(tok % L);
+      const int k = (int)((tok / L) % K);
+      const int qi = (int)(tok / ((int64_t)L * K));
+      const int g = h / grp;
+      const int P = offs[qi + 1] - offs[qi];
+      for (int d = 0; d < D; ++d) qv[d] = dec_bf16(q[r * D + d]);
+      int n = 0;
+      for (int j = 0; j < P; ++j) {
+        const uint16_t* kr = k_pre + ((int64_t)(offs[qi] + j) * Hkv + g) * D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d) dot += qv[d] * dec_bf16(kr[d]);
+        s[n++] = scale * dot;
+      }
+      for (int t = 0; t <= l; ++t) {
+        const uint16_t* kr = k_tail + ((((int64_t)qi * K + k) * L + t) * Hkv + g) * D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d) dot += qv[d] * dec_bf16(kr[d]);
+        s[n++] = scale * dot;
+      }
+      double m = -INFINITY;
+      for (int j = 0; j < n; ++j) if (s[j] > m) m = s[j];
+      double Z = 0.0;
+      for (int j = 0; j < n; ++j) Z += exp(s[j] - m);
+      for (int d = 0; d < D; ++d) acc[d] = 0.0;
+      int j = 0;
+      for (; j < P; ++j) {
+        const double p = exp(s[j] - m) / Z;
+        const uint16_t* vr = v_pre + ((int64_t)(offs[qi] + j) * Hkv + g) * D;
+        for (int d = 0; d < D; ++d) acc[d] += p * dec_bf16(vr[d]);
+      }
+      for (int t = 0; t <= l; ++t, ++j) {
+        const double p = exp(s[j] - m) / Z;
+        const uint16_t* vr = v_tail + ((((int64_t)qi * K + k) * L + t) * Hkv + g) * D;
+        for (int d = 0; d < D; ++d) acc[d] += p * dec_bf16(vr[d]);
+      }
+      for (int d = 0; d < D; ++d) out[r * D + d] = acc[d];
+      if (lse) lse[r] = m + log(Z);
+    }
+    free(s);
+    free(qv);
+    free(acc);
+  }
+  return bad ? -1 : 0;
+}
+
+/*
+ * Verifier token log-probabilities at the candidate positions.
+ *
+ *   hidden  [M][H] bf16   final hidden state of each candidate row
+ *   weight  [V][H] bf16   LM-head projection (one row per vocabulary entry)
+ *   targets [M][G] int32  token ids whose log-probability is wanted
+ *   logprob [M][G] fp64   z[m][t] - lse[m]; NaN when t is outside [0, V)
+ *   lse     [M]    fp64 or NULL
+ * z[m][v] = sum_h hidden[m][h] * weight[v][h]  (no bias, norm or temperature);
+ * lse[m]  = max_v z + ln sum_v exp(z[m][v] - max_v z).
+ * Returns 0, or -1 on bad arguments / allocation failure.
+ */
+int oracle_score_logprobs(int M, int H, int V, int G, const uint16_t* hidden,
+                          const uint16_t* weight, const int32_t* targets, double* logprob,
+                          double* lse) {
+  if (M <= 0 || H <= 0 || V <= 0 || G < 0 || !hidden || !weight) return -1;
+  if (G > 0 && (!targets || !logprob)) return -1;
+  double* hd = (double*)malloc(sizeof(double) * (size_t)M * H);
+  double* z = (double*)malloc(sizeof(double) * (size_t)M * V);
+  if (!hd || !z) {
+    free(hd);
+    free(z);
+    return -1;
+  }
+  for (int64_t i = 0; i < (int64_t)M * H; ++i) hd[i] = dec_bf16(hidden[i]);
+  int bad = 0;
+#pragma omp parallel
+  {
+    double* w = (double*)malloc(sizeof(double) * (size_t)H);
+    if (!w) {
+#pragma omp atomic write
+      bad = 1;
+    }
+#pragma omp for schedule(static)
+    for (int v = 0; v < V; ++v) {
+      if (bad) continue;
+      for (int h = 0; h < H; ++h) w[h] = dec_bf16(weight[(int64_t)v * H + h]);
+      for (int m = 0; m < M; ++m) {
+        const double* x = hd + (int64_t)m * H;
+        double dot = 0.0;
+        for (int h = 0; h < H; ++h) dot += x[h] * w[h];
+        z[(int64_t)m * V + v] = dot;
+      }
+    }
+    free(w);
+  }
+  if (!bad) {
+#pragma omp parallel for schedule(static)
+    for (int m = 0; m < M; ++m) {
+      const double* zr = z + (int64_t)m * V;
+      double mx = -INFINITY;
+      for (int v = 0; v < V; ++v) if (zr[v] > mx) mx = zr[v];
+      double s = 0.0;
+      for (int v = 0; v < V; ++v) s += exp(zr[v] - mx);
+      const double l = mx + log(s);
+      if (lse) lse[m] = l;
+      for (int g = 0; g < G; ++g) {
+        const int32_t t = targets[(int64_t)m * G + g];
+        logprob[(int64_t)m * G + g] = (t >= 0 && t < V) ? zr[t] - l : NAN;
+      }
+    }
+  }
+  free(hd);
+  free(z);
+  return bad ? -1 : 0;
+}
+
+/*
+ * CLIP entity alignment (Eq. 14-15) with the keep threshold.
+ *
+ *   cand   [Qn][K][E] fp16   CLIP embedding of each candidate's entity e_k
+ *   frames [Qn][F][E] fp16   CLIP embeddings of the query's keyframes
+ *   cosm   [Qn][K][F] fp64 or NULL    cos(e_k, f_j)
+ *   max_cos[Qn][K]    fp64            max_j cos(e_k, f_j)            (Eq. 15)
+ *   argmax [Qn][K]    int32           smallest j attaining the max
+ *   keep   [Qn][K]    uint8           max_cos >= tau
+ * cos(a, b) = <a, b> / (|a| |b|), taken as 0 when either vector is zero.
+ * Readings: the max runs over all frames given for the query (the keyframe set
+ * F of Algorithm 1); ties go to the lowest frame index; keep uses >= like Eq. 13.
+ */
+int oracle_clip_align(int Qn, int K, int F, int E, double tau, const uint16_t* cand,
+                      const uint16_t* frames, double* cosm, double* max_cos, int32_t* argmax,
+                      uint8_t* keep) {
+  if (Qn <= 0 || K <= 0 || F <= 0 || E <= 0 || !cand || !frames || !max_cos || !argmax || !keep)
+    return -1;
+#pragma omp parallel for schedule(static)
+  for (int64_t qk = 0; qk < (int64_t)Qn * K; ++qk) {
+    const int qi = (int)(qk / K);
+    const uint16_t* e = cand + qk * E;
+    double ee = 0.0;
+    for (int i = 0; i < E; ++i) ee += dec_f16(e[i]) * dec_f16(e[i]);
+    double best = -INFINITY;
+    int besti = 0;
+    for (int j = 0; j < F; ++j) {
+      const uint16_t* f = frames + ((int64_t)qi * F + j) * E;
+      double ef = 0.0, ff = 0.0;
+      for (int i = 0; i < E; ++i) {
+        ef += dec_f16(e[i]) * dec_f16(f[i]);
+        ff += dec_f16(f[i]) * dec_f16(f[i]);
+      }
+      const double c = (ee > 0.0 && ff > 0.0) ? ef / (sqrt(ee) * sqrt(ff)) : 0.0;
+      if (cosm) cosm[qk * F + j] = c;
+      if (c > best) {
+        best = c;
+        besti = j;
+      }
+    }
+    max_cos[qk] = best;
+    argmax[qk] = besti;
+    keep[qk] = best >= tau ? 1 : 0;
+  }
+  return 0;
+}
+
+/*
+ * Candidate selection.
+ *
+ *   logprob [Qn][K][L][G] fp64   per-token log-probabilities (gather g)
+ *   lengths [Qn][K] int32 or NULL  valid tokens n_k per candidate (default L)
+ *   keep    [Qn][K] uint8          CLIP filter decision          (mode 0)
+ *   max_cos [Qn][K] fp64           alignment score of Eq. 15     (mode 1)
+ *   score   [Qn][K] fp64           mode 0: mean log-prob; mode 1: reliability
+ *   selected[Qn]    int32          chosen candidate, or -1
+ *
+ * mode 0 (masked mean log-prob): score_k = (sum_{l < n_k} logprob[k][l][0]) / n_k,
+ *   the verifier's own likelihood of the candidate normalised by its length
+ *   (Section 4.5 "self-consistent"); selected = argmax of score over candidates
+ *   with keep = 1, lowest index on ties, -1 when none is kept.
+ * mode 1 (Algorithm 1): with lp_Y = logprob[k][n_k-1][0] and lp_N = logprob[k][n_k-1][1]
+ *   (the first generated token after the candidate), Eq. 12 gives
+ *   score_k = p_Y / (p_Y + p_N) = 1 / (1 + exp(lp_N - lp_Y));
+ *   Eq. 13 keeps A_H = { k : score_k >= max_j score_j - delta };
+ *   the answer is the k in A_H with the largest max_cos (lowest index on ties).
+ * A candidate whose n_k is outside [1, L] or whose score is NaN is never selected.
+ */
+int oracle_select(int Qn, int K, int L, int G, int mode, double delta, const double* logprob,
+                  const int32_t* lengths, const uint8_t* keep, const double* max_cos,
+                  double* score, int32_t* selected) {
+  if (Qn <= 0 || K <= 0 || L <= 0 || G <= 0 || !logprob || !score || !selected) return -1;
+  if (mode == 0 && !keep) return -1;
+  if (mode == 1 && (G < 2 || !max_cos)) return -1;
+  if (mode != 0 && mode != 1) return -1;
+  for (int qi = 0; qi < Qn; ++qi) {
+    for (int k = 0; k < K; ++k) {
+      const int64_t qk = (int64_t)qi * K + k;
+      const int n = lengths ? lengths[qk] : L;
+      double sc = NAN;
+      if (n >= 1 && n <= L) {
+        if (mode == 0) {
+          double s = 0.0;
+          for (int l = 0; l < n; ++l) s += logprob[(qk * L + l) * G + 0];
+          sc = s / (double)n;
+        } else {
+          const double lpY = logprob[(qk * L + (n - 1)) * G + 0];
+          const double lpN = logprob[(qk * L + (n - 1)) * G + 1];
+          sc = 1.0 / (1.0 + exp(lpN - lpY));
+        }
+      }
+      score[qk] = sc;
+    }
+    int sel = -1;
+    if (mode == 0) {
+      double best = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const int64_t qk = (int64_t)qi * K + k;
+        if (!keep[qk] || isnan(score[qk])) continue;
+        if (sel < 0 || score[qk] > best) {
+          best = score[qk];
+          sel = k;
+        }
+      }
+    } else {
+      double top = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const double s = score[(int64_t)qi * K + k];
+        if (!isnan(s) && s > top) top = s;
+      }
+      double best = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const int64_t qk = (int64_t)qi * K + k;
+        const double s = score[qk];
+        if (isnan(s) || !(s >= top - delta)) continue; /* Eq. 13 */
+        if (sel < 0 || max_cos[qk] > best) {
+          best = max_cos[qk];
+          sel = k;
+        }
+      }
+    }
+    selected[qi] = sel;
+  }
+  return 0;
+}

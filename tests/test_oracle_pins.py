@@ -1,0 +1,368 @@
+"""Pins of the fp64 oracle to things other than itself (CPU only).
+
+Each group ties one oracle function to a library routine, a closed form, an
+invariant or a fixture from the paper, chosen so that a dropped term, a wrong
+sign, a wrong index or a transposed operand fails at least one test.
+"""
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle
+from paper_2601_01513_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def bf16_bits(x: np.ndarray) -> np.ndarray:
+    """fp64 values that are already bf16-representable -> bit patterns (test helper)."""
+    return synth.round_bf16(x)
+
+
+def bf16_vals(bits):
+    return oracle.decode_bf16(bits)
+
+
+def rand_bf16(shape, seed, stream, std=1.0):
+    return synth.normal_bf16(shape, seed, stream, 0.0, std)
+
+
+# --------------------------------------------------------------------------- decoding
+
+def test_decode_matches_torch_and_numpy():
+    bits = np.arange(0, 65536, dtype=np.uint32).astype(np.uint16)
+    ref_bf = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).to(torch.float64).numpy()
+    got_bf = oracle.decode_bf16(bits)
+    ok = ~np.isnan(ref_bf)
+    assert np.array_equal(got_bf[ok], ref_bf[ok]) and np.all(np.isnan(got_bf[~ok]))
+    ref_h = bits.view(np.float16).astype(np.float64)
+    got_h = oracle.decode_f16(bits)
+    ok = ~np.isnan(ref_h)
+    assert np.array_equal(got_h[ok], ref_h[ok]) and np.all(np.isnan(got_h[~ok]))
+
+
+# --------------------------------------------------------------------------- attention
+
+def _attn_case(Qn, K, L, Hq, Hkv, D, plens, seed):
+    offs = np.zeros(Qn + 1, np.int32)
+    offs[1:] = np.cumsum(plens)
+    tot = int(offs[-1])
+    q = rand_bf16((Qn, K, L, Hq, D), seed, 1)
+    kp = rand_bf16((tot, Hkv, D), seed, 2)
+    vp = rand_bf16((tot, Hkv, D), seed, 3)
+    kt = rand_bf16((Qn, K, L, Hkv, D), seed, 4)
+    vt = rand_bf16((Qn, K, L, Hkv, D), seed, 5)
+    return q, kp, vp, offs, kt, vt
+
+
+def _sdpa_reference(q, kp, vp, offs, kt, vt, scale):
+    """Library reference: torch SDPA (fp64, CPU) per (query, candidate) with an explicit mask
+    that shows the whole prefix and the candidate's own tokens causally; GQA by enable_gqa."""
+    Qn, K, L, Hq, D = q.shape
+    out = np.zeros(q.shape)
+    lse = np.zeros(q.shape[:-1])
+    for qi in range(Qn):
+        P = int(offs[qi + 1] - offs[qi])
+        for k in range(K):
+            keys = np.concatenate([bf16_vals(kp[offs[qi]:offs[qi + 1]]), bf16_vals(kt[qi, k])], 0)
+            vals = np.concatenate([bf16_vals(vp[offs[qi]:offs[qi + 1]]), bf16_vals(vt[qi, k])], 0)
+            Q = torch.from_numpy(bf16_vals(q[qi, k])).permute(1, 0, 2)[None]      # [1,Hq,L,D]
+            Kt = torch.from_numpy(keys).permute(1, 0, 2)[None]                    # [1,Hkv,P+L,D]
+            Vt = torch.from_numpy(vals).permute(1, 0, 2)[None]
+            mask = torch.zeros(L, P + L, dtype=torch.bool)
+            mask[:, :P] = True
+            mask[:, P:] = torch.ones(L, L, dtype=torch.bool).tril()
+            o = torch.nn.functional.scaled_dot_product_attention(
+                Q, Kt, Vt, attn_mask=mask, scale=scale, enable_gqa=True)
+            out[qi, k] = o[0].permute(1, 0, 2).numpy()
+            # lse via the library logsumexp of the masked score matrix
+            rep = Hq // Kt.shape[1]
+            s = torch.einsum("bhld,bhjd->bhlj", Q, Kt.repeat_interleave(rep, dim=1)) * scale
+            s = s.masked_fill(~mask, float("-inf"))
+            lse[qi, k] = torch.logsumexp(s, dim=-1)[0].permute(1, 0).numpy()
+    return out, lse
+
+
+@pytest.mark.parametrize("Qn,K,L,Hq,Hkv,D,plens", [
+    (1, 3, 4, 4, 2, 16, [7]),
+    (2, 2, 5, 6, 3, 8, [5, 0]),       # ragged, one query without prefix
+    (1, 1, 6, 2, 2, 32, [0]),         # textbook causal attention
+    (2, 4, 1, 8, 1, 16, [3, 9]),      # L = 1, MQA
+])
+def test_attn_matches_sdpa(Qn, K, L, Hq, Hkv, D, plens):
+    q, kp, vp, offs, kt, vt = _attn_case(Qn, K, L, Hq, Hkv, D, plens, seed=11 + Qn * 7 + L)
+    scale = 1.0 / math.sqrt(D)
+    out, lse = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    ref, ref_lse = _sdpa_reference(q, kp, vp, offs, kt, vt, scale)
+    np.testing.assert_allclose(out, ref, rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse, ref_lse, rtol=0, atol=1e-12)
+
+
+def test_attn_textbook_causal_is_is_causal_sdpa():
+    """P = 0, K = 1, Hq = Hkv: plain causal self-attention over the candidate tokens."""
+    q, kp, vp, offs, kt, vt = _attn_case(1, 1, 9, 3, 3, 16, [0], seed=5)
+    out, _ = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    Q = torch.from_numpy(bf16_vals(q[0, 0])).permute(1, 0, 2)
+    Kk = torch.from_numpy(bf16_vals(kt[0, 0])).permute(1, 0, 2)
+    Vv = torch.from_numpy(bf16_vals(vt[0, 0])).permute(1, 0, 2)
+    ref = torch.nn.functional.scaled_dot_product_attention(Q, Kk, Vv, is_causal=True)
+    np.testing.assert_allclose(out[0, 0], ref.permute(1, 0, 2).numpy(), rtol=0, atol=1e-12)
+
+
+def test_attn_zero_query_averages_exactly_the_visible_keys():
+    """q = 0 makes every score equal: out = mean of V over prefix U own-tail[0..l],
+    lse = ln(#visible keys).  Pins the key set (prefix length, causal tail, other
+    candidates excluded) and the KV-head mapping (per-head distinct values)."""
+    Qn, K, L, Hq, Hkv, D = 2, 3, 4, 6, 2, 8
+    plens = [5, 2]
+    q, kp, vp, offs, kt, vt = _attn_case(Qn, K, L, Hq, Hkv, D, plens, seed=3)
+    q = np.zeros_like(q)
+    out, lse = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    vpd, vtd = bf16_vals(vp), bf16_vals(vt)
+    grp = Hq // Hkv
+    for qi in range(Qn):
+        P = plens[qi]
+        for k in range(K):
+            for l in range(L):
+                for h in range(Hq):
+                    g = h // grp
+                    vis = np.concatenate([vpd[offs[qi]:offs[qi] + P, g], vtd[qi, k, :l + 1, g]], 0)
+                    np.testing.assert_allclose(out[qi, k, l, h], vis.mean(0), rtol=0, atol=1e-14)
+                    assert abs(lse[qi, k, l, h] - math.log(P + l + 1)) < 1e-14
+
+
+def test_attn_constant_values_and_single_key():
+    q, kp, vp, offs, kt, vt = _attn_case(1, 2, 3, 4, 2, 16, [6], seed=8)
+    c = bf16_bits(np.linspace(-2, 2, 16))
+    vp2 = np.broadcast_to(c, vp.shape).copy()
+    vt2 = np.broadcast_to(c, vt.shape).copy()
+    out, _ = oracle.verify_attn(q, kp, vp2, offs, kt, vt2)
+    np.testing.assert_allclose(out, np.broadcast_to(bf16_vals(c), out.shape), rtol=0, atol=1e-14)
+    # one visible key (no prefix, first tail token): output is exactly that value row
+    q, kp, vp, offs, kt, vt = _attn_case(1, 2, 3, 4, 2, 16, [0], seed=9)
+    out, lse = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    for h in range(4):
+        np.testing.assert_array_equal(out[0, :, 0, h], bf16_vals(vt[0, :, 0, h // 2]))
+
+
+def test_attn_candidates_are_independent_and_permute():
+    q, kp, vp, offs, kt, vt = _attn_case(1, 4, 5, 4, 2, 16, [10], seed=21)
+    out, lse = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    # another candidate's tail changes nothing for candidate 0
+    kt2, vt2 = kt.copy(), vt.copy()
+    kt2[0, 1:] = rand_bf16(kt2[0, 1:].shape, 99, 1)
+    vt2[0, 1:] = rand_bf16(vt2[0, 1:].shape, 99, 2)
+    out2, _ = oracle.verify_attn(q, kp, vp, offs, kt2, vt2)
+    np.testing.assert_array_equal(out2[0, 0], out[0, 0])
+    # permuting candidates permutes the rows
+    perm = np.array([2, 0, 3, 1])
+    out3, lse3 = oracle.verify_attn(q[:, perm], kp, vp, offs, kt[:, perm], vt[:, perm])
+    np.testing.assert_array_equal(out3, out[:, perm])
+    np.testing.assert_array_equal(lse3, lse[:, perm])
+    # a later token of the own tail is invisible to earlier rows (causality)
+    kt4 = kt.copy()
+    kt4[0, 0, 3:] = rand_bf16(kt4[0, 0, 3:].shape, 77, 3)
+    out4, _ = oracle.verify_attn(q, kp, vp, offs, kt4, vt)
+    np.testing.assert_array_equal(out4[0, 0, :3], out[0, 0, :3])
+    assert not np.array_equal(out4[0, 0, 3:], out[0, 0, 3:])
+
+
+def test_attn_row_selection_computes_only_selected_rows():
+    q, kp, vp, offs, kt, vt = _attn_case(1, 2, 3, 4, 2, 16, [6], seed=4)
+    full, _ = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    sel = np.zeros(q.shape[:-1], bool)
+    sel[0, 1, 2, 3] = True
+    part, _ = oracle.verify_attn(q, kp, vp, offs, kt, vt, row_sel=sel)
+    np.testing.assert_array_equal(part[sel], full[sel])
+    assert np.all(np.isnan(part[~sel]))
+
+
+# --------------------------------------------------------------------------- LM head
+
+def test_logprobs_match_torch_log_softmax():
+    M, H, V = 7, 40, 300
+    hid = rand_bf16((M, H), 31, 1)
+    W = rand_bf16((V, H), 31, 2, std=0.3)
+    tgt = synth.uniform_i32((M, 3), 31, 3, 0, V)
+    lp, lse = oracle.score_logprobs(hid, W, tgt)
+    z = torch.from_numpy(bf16_vals(hid)) @ torch.from_numpy(bf16_vals(W)).T
+    ref = torch.log_softmax(z, dim=-1)
+    np.testing.assert_allclose(lp, torch.gather(ref, 1, torch.from_numpy(tgt).long()).numpy(),
+                               rtol=0, atol=1e-12)
+    np.testing.assert_allclose(lse, torch.logsumexp(z, -1).numpy(), rtol=0, atol=1e-12)
+
+
+def test_logprobs_closed_forms():
+    M, H, V = 3, 16, 257
+    hid = rand_bf16((M, H), 5, 1)
+    tgt = synth.uniform_i32((M, 2), 5, 2, 0, V)
+    # W = 0: uniform distribution, logprob = -ln V exactly
+    lp, lse = oracle.score_logprobs(hid, np.zeros((V, H), np.uint16), tgt)
+    np.testing.assert_allclose(lp, -math.log(V), rtol=0, atol=1e-14)
+    np.testing.assert_allclose(lse, math.log(V), rtol=0, atol=1e-14)
+    # one nonzero row t = alpha * hidden[0]: two-level softmax for row 0
+    t = 17
+    W = np.zeros((V, H), np.uint16)
+    W[t] = hid[0]
+    hv = bf16_vals(hid[0])
+    zt = float(hv @ hv)
+    lp, lse = oracle.score_logprobs(hid[:1], W, np.array([[t, t + 1]], np.int32))
+    ref_lse = math.log(math.exp(zt) + (V - 1))
+    assert abs(lse[0] - ref_lse) < 1e-12
+    assert abs(lp[0, 0] - (zt - ref_lse)) < 1e-12
+    assert abs(lp[0, 1] - (0.0 - ref_lse)) < 1e-12
+
+
+def test_logprobs_invariants():
+    M, H, V = 4, 24, 130
+    hid = rand_bf16((M, H), 6, 1)
+    W = rand_bf16((V, H), 6, 2, std=0.5)
+    all_t = np.tile(np.arange(V, dtype=np.int32), (M, 1))
+    lp, _ = oracle.score_logprobs(hid, W, all_t)
+    assert np.all(lp <= 0)
+    np.testing.assert_allclose(np.exp(lp).sum(1), 1.0, rtol=0, atol=1e-13)
+    # rows are independent: permuting rows permutes results
+    perm = np.array([3, 1, 0, 2])
+    lp2, _ = oracle.score_logprobs(hid[perm], W, all_t)
+    np.testing.assert_array_equal(lp2, lp[perm])
+    # out-of-range targets give NaN and leave the others untouched
+    bad = np.array([[-1, 5], [V, 0], [0, V - 1], [2**30, 1]], np.int32)
+    lpb, _ = oracle.score_logprobs(hid, W, bad)
+    assert np.isnan(lpb[0, 0]) and np.isnan(lpb[1, 0]) and np.isnan(lpb[3, 0])
+    np.testing.assert_array_equal(lpb[0, 1], lp[0, 5])
+    np.testing.assert_array_equal(lpb[2], lp[2, [0, V - 1]])
+
+
+# --------------------------------------------------------------------------- CLIP
+
+def test_clip_matches_torch_cosine_similarity():
+    Qn, K, F, E = 2, 3, 11, 40
+    cand = synth.round_f16(synth.normal_f64((Qn, K, E), 7, 1))
+    fr = synth.round_f16(synth.normal_f64((Qn, F, E), 7, 2))
+    cosm, mc, am, keep = oracle.clip_align(cand, fr, 0.1)
+    c = torch.from_numpy(oracle.decode_f16(cand))
+    f = torch.from_numpy(oracle.decode_f16(fr))
+    ref = torch.nn.functional.cosine_similarity(c[:, :, None, :], f[:, None, :, :], dim=-1)
+    np.testing.assert_allclose(cosm, ref.numpy(), rtol=0, atol=1e-14)
+    np.testing.assert_allclose(mc, ref.max(-1).values.numpy(), rtol=0, atol=1e-14)
+    np.testing.assert_array_equal(am, ref.argmax(-1).numpy())
+    np.testing.assert_array_equal(keep, (mc >= 0.1).astype(np.uint8))
+
+
+def test_clip_closed_forms():
+    E = 8
+    eye = np.eye(E)
+    cand = synth.round_f16(eye[None, :3] * 3.0)          # e_0, e_1, e_2 scaled
+    frames = synth.round_f16(eye[None, 3:7] * 0.5)        # orthogonal to all candidates
+    cosm, mc, am, keep = oracle.clip_align(cand, frames, 0.2)
+    assert np.all(cosm == 0.0) and np.all(keep == 0) and np.all(am == 0)
+    # a planted frame equal to the candidate: cos = 1 at that index
+    frames2 = frames.copy()
+    frames2[0, 2] = cand[0, 1]
+    cosm, mc, am, keep = oracle.clip_align(cand, frames2, 0.2)
+    assert mc[0, 1] == 1.0 and am[0, 1] == 2 and keep[0, 1] == 1
+    # ties go to the lowest frame index
+    frames3 = frames2.copy()
+    frames3[0, 0] = cand[0, 1]
+    _, mc, am, _ = oracle.clip_align(cand, frames3, 0.2)
+    assert am[0, 1] == 0 and mc[0, 1] == 1.0
+    # a zero vector has cosine 0 with everything
+    cand0 = cand.copy()
+    cand0[0, 0] = 0
+    cosm, mc, _, _ = oracle.clip_align(cand0, frames2, 0.2)
+    assert np.all(cosm[0, 0] == 0.0)
+
+
+def test_clip_scale_invariance_and_threshold():
+    Qn, K, F, E = 1, 4, 9, 32
+    base = synth.normal_f64((Qn, K, E), 12, 1)
+    fr = synth.normal_f64((Qn, F, E), 12, 2)
+    a = oracle.clip_align(synth.round_f16(base), synth.round_f16(fr), 0.0)
+    b = oracle.clip_align(synth.round_f16(base * 4.0), synth.round_f16(fr * 0.25), 0.0)
+    np.testing.assert_allclose(a[0], b[0], rtol=0, atol=1e-14)  # powers of two: exact in fp16
+    # keep uses >=: threshold equal to max_cos keeps, a hair above drops
+    mc = a[1]
+    _, _, _, keep_eq = oracle.clip_align(synth.round_f16(base), synth.round_f16(fr), float(mc[0, 0]))
+    assert keep_eq[0, 0] == 1
+    _, _, _, keep_gt = oracle.clip_align(synth.round_f16(base), synth.round_f16(fr),
+                                         float(np.nextafter(mc[0, 0], 2.0)))
+    assert keep_gt[0, 0] == 0
+
+
+# --------------------------------------------------------------------------- selection
+
+def _two_stage_logprobs(rel):
+    """[1][K][1][2] log-probs whose normalised Yes-probability (Eq. 12) is `rel`."""
+    rel = np.asarray(rel, np.float64)
+    lp = np.stack([np.log(rel), np.log1p(-rel)], -1)
+    return lp[None, :, None, :]
+
+
+@pytest.mark.parametrize("name", ["case_penguin.json", "case_cuttlefish.json"])
+def test_selection_case_studies(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        case = json.load(f)
+    lp = _two_stage_logprobs(case["reliability"])
+    mc = np.array([case["max_cos"]])
+    score, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=case["delta"])
+    np.testing.assert_allclose(score[0], case["reliability"], rtol=0, atol=1e-14)
+    assert sel[0] == case["expected_selected"]
+    top = score.max()
+    assert [bool(s >= top - case["delta"]) for s in score[0]] == case["expected_in_AH"]
+    # a single-criterion rule would choose differently: the cases need both stages
+    assert int(np.argmax(case["reliability"])) != case["expected_selected"] or \
+        int(np.argmax(case["max_cos"])) != case["expected_selected"]
+
+
+def test_two_stage_delta_boundary():
+    d = 0.0625
+    lp = _two_stage_logprobs([0.75, 0.75 - d + 1e-9, 0.75 - d - 1e-9, 0.5])
+    mc = np.array([[0.1, 0.2, 0.9, 0.95]])
+    score, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=d)
+    assert sel[0] == 1          # 0 and 1 in A_H; 1 has the higher alignment
+    score, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=0.0)
+    assert sel[0] == 0          # delta = 0: only the most reliable survives
+    score, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=1.0)
+    assert sel[0] == 3          # everything survives: pure alignment argmax
+
+
+def test_masked_mean_logprob_rules():
+    # candidate means: [-1, -0.5, -0.25, -2]; lengths cut off huge trailing values
+    lp = np.array([[[-1, -1, 50], [-0.5, -0.5, -0.5], [-0.25, 9, 9], [-2, -2, -2]]], np.float64)[..., None]
+    lengths = np.array([[2, 3, 1, 3]], np.int32)
+    keep = np.array([[1, 1, 1, 1]], np.uint8)
+    score, sel = oracle.select(lp, lengths=lengths, keep=keep)
+    np.testing.assert_array_equal(score[0], [-1.0, -0.5, -0.25, -2.0])
+    assert sel[0] == 2
+    keep = np.array([[1, 1, 0, 1]], np.uint8)
+    _, sel = oracle.select(lp, lengths=lengths, keep=keep)
+    assert sel[0] == 1          # the best candidate is dropped by the CLIP filter
+    _, sel = oracle.select(lp, lengths=lengths, keep=np.zeros((1, 4), np.uint8))
+    assert sel[0] == -1         # nothing kept
+    # ties: lowest index; invalid lengths are never selected
+    lp2 = np.full((1, 3, 2, 1), -1.0)
+    _, sel = oracle.select(lp2, keep=np.ones((1, 3), np.uint8))
+    assert sel[0] == 0
+    score, sel = oracle.select(lp2, lengths=np.array([[0, 3, 2]], np.int32), keep=np.ones((1, 3), np.uint8))
+    assert np.isnan(score[0, 0]) and np.isnan(score[0, 1]) and sel[0] == 2
+    # default lengths = L: plain mean
+    score, _ = oracle.select(lp[:, :, :, :], keep=np.ones((1, 4), np.uint8))
+    np.testing.assert_allclose(score[0], lp[0, :, :, 0].mean(1), rtol=0, atol=1e-15)
+
+
+def test_selection_permutation_invariance():
+    lp, keep, mc = synth.selection_inputs(3, 7, 5, 2, seed=13)
+    for mode in (oracle.SEL_MASKED_MEAN_LOGPROB, oracle.SEL_TWO_STAGE):
+        score, sel = oracle.select(lp, mode=mode, keep=keep, max_cos=mc)
+        perm = np.array([6, 2, 0, 5, 1, 4, 3])
+        score2, sel2 = oracle.select(lp[:, perm], mode=mode, keep=keep[:, perm], max_cos=mc[:, perm])
+        np.testing.assert_array_equal(score2, score[:, perm])
+        for qi in range(3):
+            if sel[qi] < 0:
+                assert sel2[qi] == -1
+            else:
+                assert perm[sel2[qi]] == sel[qi]

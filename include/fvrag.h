@@ -1,0 +1,238 @@
+/*
+ * libfvrag -- the verifier hot path of VideoSpeculateRAG (arXiv 2601.01513) on
+ * one GB300 (sm_103a).
+ *
+ * The verifier of the paper scores K draft candidates that share one long
+ * prefix (video tokens, question, retrieved passages) in a single forward pass
+ * (Section 3.1, Eq. 6; Section 3.2 "Two-Stage Verification", Eq. 11), then
+ * checks each candidate's entity against the video's keyframes with CLIP
+ * (Eq. 14-15) and picks the answer (Eq. 7, Eq. 12-13, Algorithm 1).  This
+ * library implements the data-parallel core of that step as four calls:
+ *
+ *   fvrag_verify_attn       one attention layer of the verifier forward over
+ *                           all K x L candidate rows: the shared prefix is read
+ *                           once for all candidates (split over the key axis),
+ *                           plus each candidate's own causal tail;
+ *   fvrag_score_logprobs    the LM head: hidden @ W^T fused with an online
+ *                           log-sum-exp and a gather of the target ids, so the
+ *                           [rows x vocab] logits never reach memory;
+ *   fvrag_clip_align        cosine of each candidate-entity embedding with every
+ *                           frame embedding, max/argmax over frames, keep flag;
+ *   fvrag_select_candidate  the per-query selection reduction.
+ *
+ * Conventions shared by every call
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the library
+ *     never allocates, frees or synchronises (except fvrag_read_status), and
+ *     keeps no state between calls other than read-only driver entry points.
+ *   - Every call validates its arguments on the host and returns an error
+ *     before launching anything; on success it has only enqueued work on
+ *     `stream` (NULL = the legacy default stream).
+ *   - Layouts are dense row-major, leading index first, as written beside each
+ *     argument.  bf16 / fp16 tensors are passed as `const void*`.
+ *   - Workspaces: the first 256 bytes hold a 32-bit status word that kernels
+ *     only ever OR error bits into (FVRAG_ERR_TIMEOUT when a bounded wait ran
+ *     out).  Zero it once (fvrag_clear_status or a memset) before first use;
+ *     read it with fvrag_read_status.  The rest is scratch owned by the call
+ *     while it runs; calls that share a workspace must not overlap in time.
+ *   - Alignment: every tensor pointer must be 16-byte aligned
+ *     (FVRAG_ERR_MISALIGNED otherwise).
+ */
+#ifndef FVRAG_H
+#define FVRAG_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define FVRAG_ABI_VERSION 1
+
+/* cudaStream_t without including the CUDA headers. */
+typedef struct CUstream_st* fvrag_stream_t;
+
+typedef enum {
+  FVRAG_OK = 0,
+  FVRAG_ERR_INVALID_ARG = 1, /* null required pointer, non-positive size, bad mode */
+  FVRAG_ERR_UNSUPPORTED = 2, /* shape outside what the kernels handle (see each call) */
+  FVRAG_ERR_MISALIGNED = 3,  /* pointer not 16-byte aligned, row pitch not a multiple of 16 B */
+  FVRAG_ERR_WORKSPACE = 4,   /* workspace pointer null or smaller than the *_workspace() size */
+  FVRAG_ERR_CUDA = 5,        /* a CUDA runtime/driver call or a launch failed */
+  FVRAG_ERR_TIMEOUT = 6      /* device status: a bounded wait inside a kernel ran out */
+} fvrag_status;
+
+/* FVRAG_ABI_VERSION of the loaded library. */
+int fvrag_abi_version(void);
+
+/* Static, never NULL, human-readable name of a status code. */
+const char* fvrag_status_string(int status);
+
+/* ------------------------------------------------------------------------ *
+ * 1. Shared-prefix attention (verifier forward, Eq. 6 and Eq. 11)
+ *
+ * For query q, candidate k, candidate token l and query head h, with KV head
+ * g = h / (hq / hkv) (consecutive query heads share a KV head):
+ *   keys   = the P_q prefix tokens of query q, then tokens 0..l of candidate k
+ *            (candidates never see one another; causal inside a candidate)
+ *   out    = softmax(scale * q . K^T) V over those keys,   scale = softmax_scale
+ *            or 1/sqrt(head_dim) when softmax_scale == 0
+ *   lse    = natural-log log-sum-exp of the scaled scores (optional output)
+ * ------------------------------------------------------------------------ */
+typedef struct fvrag_attn_desc {
+  int32_t num_queries;  /* Qn >= 1 */
+  int32_t num_cand;     /* K >= 1 */
+  int32_t cand_len;     /* L, 1..64 */
+  int32_t hq;           /* query heads, multiple of hkv */
+  int32_t hkv;          /* KV heads >= 1 */
+  int32_t head_dim;     /* D: 64 or 128 */
+  int32_t max_prefix;   /* upper bound on every P_q (plans the key split); >= 0 */
+  int32_t total_prefix; /* sum over queries of P_q = rows of k_prefix / v_prefix */
+  float softmax_scale;  /* 0 => 1/sqrt(head_dim) */
+  uint32_t flags;       /* must be 0 */
+} fvrag_attn_desc;
+
+/* Bytes of workspace fvrag_verify_attn needs for `d` (0 if `d` is invalid). */
+size_t fvrag_verify_attn_workspace(const fvrag_attn_desc* d);
+
+/*
+ *   q              [Qn][K][L][hq][D]     bf16
+ *   k_prefix       [total_prefix][hkv][D] bf16   query q owns rows
+ *   v_prefix       [total_prefix][hkv][D] bf16     prefix_offsets[q] .. prefix_offsets[q+1]-1
+ *   prefix_offsets [Qn+1]                int32  device; non-decreasing, offsets[0] = 0,
+ *                                               offsets[Qn] = total_prefix, every
+ *                                               P_q <= max_prefix (not checked on device)
+ *   k_tail, v_tail [Qn][K][L][hkv][D]    bf16   the candidates' own tokens
+ *   out            [Qn][K][L][hq][D]     bf16   written
+ *   lse            [Qn][K][L][hq]        fp32   written when not NULL
+ *   ws / ws_bytes  workspace of at least fvrag_verify_attn_workspace(d) bytes
+ * k_prefix / v_prefix may be NULL when total_prefix == 0.
+ */
+fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* q, const void* k_prefix,
+                               const void* v_prefix, const int32_t* prefix_offsets,
+                               const void* k_tail, const void* v_tail, void* out, float* lse,
+                               void* ws, size_t ws_bytes, fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * 2. LM-head log-probabilities (Eq. 11; the verifier likelihood of Section 4.5)
+ *
+ *   z[m][v]        = sum_h hidden[m][h] * weight[v][h]   (bf16 x bf16, fp32 accumulate)
+ *   lse[m]         = log sum_v exp(z[m][v])              (natural log)
+ *   logprob[m][g]  = z[m][targets[m][g]] - lse[m], NaN when the id is outside [0, V)
+ * The [rows x vocab] logits are never written to memory.
+ * ------------------------------------------------------------------------ */
+typedef struct fvrag_lm_desc {
+  int32_t rows;    /* M >= 1 (candidate token rows, (q, k, l) order) */
+  int32_t hidden;  /* H >= 8, multiple of 8 (16-byte row pitch) */
+  int32_t vocab;   /* V >= 1 */
+  int32_t gathers; /* G: target ids per row, 1..8 (1: likelihood; 2: "Yes"/"No") */
+  uint32_t flags;  /* must be 0 */
+} fvrag_lm_desc;
+
+size_t fvrag_score_logprobs_workspace(const fvrag_lm_desc* d);
+
+/*
+ *   hidden  [M][H] bf16
+ *   weight  [V][H] bf16   (nn.Linear layout: one row per vocabulary entry)
+ *   targets [M][G] int32
+ *   logprob [M][G] fp32   written
+ *   lse     [M]    fp32   written when not NULL
+ */
+fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void* hidden, const void* weight,
+                                  const int32_t* targets, float* logprob, float* lse, void* ws,
+                                  size_t ws_bytes, fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * 3. CLIP entity alignment (Eq. 14-15) with the keep/drop threshold
+ *
+ *   cos[q][k][f]  = <e_qk, f_qf> / (|e_qk| |f_qf|)   (0 when either vector is 0)
+ *   max_cos[q][k] = max_f cos[q][k][f]                (Eq. 15)
+ *   argmax[q][k]  = lowest f attaining the max
+ *   keep[q][k]    = max_cos >= threshold
+ * ------------------------------------------------------------------------ */
+typedef struct fvrag_clip_desc {
+  int32_t num_queries; /* Qn >= 1 */
+  int32_t num_cand;    /* K >= 1 */
+  int32_t num_frames;  /* F >= 1 */
+  int32_t dim;         /* E: multiple of 8, 8..4096 */
+  float threshold;     /* tau */
+  uint32_t flags;      /* must be 0 */
+} fvrag_clip_desc;
+
+/*
+ *   cand_emb  [Qn][K][E] fp16
+ *   frame_emb [Qn][F][E] fp16
+ *   cos       [Qn][K][F] fp32  written when not NULL
+ *   max_cos   [Qn][K]    fp32  written
+ *   argmax    [Qn][K]    int32 written
+ *   keep      [Qn][K]    uint8 written
+ */
+fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
+                              const void* frame_emb, float* cos, float* max_cos, int32_t* argmax,
+                              uint8_t* keep, fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * 4. Candidate selection
+ *
+ * FVRAG_SEL_MASKED_MEAN_LOGPROB: score_k = (sum_{l < n_k} logprob[k][l][0]) / n_k
+ *   (the verifier's own length-normalised likelihood, Section 4.5); selected =
+ *   argmax over candidates with keep = 1, lowest index on ties, -1 if none.
+ * FVRAG_SEL_TWO_STAGE (Algorithm 1): with lpY = logprob[k][n_k-1][0] and
+ *   lpN = logprob[k][n_k-1][1], score_k = 1 / (1 + exp(lpN - lpY)) = pY/(pY+pN)
+ *   (Eq. 12); A_H = {k : score_k >= max_j score_j - delta} (Eq. 13); selected =
+ *   the k in A_H with the largest max_cos, lowest index on ties.
+ * n_k = lengths[q][k] (or L when lengths is NULL); a candidate with n_k outside
+ * [1, L] or a NaN score gets score NaN and is never selected.  Sums and the
+ * comparisons run in fp64; score is rounded to fp32 on output.
+ * ------------------------------------------------------------------------ */
+typedef enum { FVRAG_SEL_MASKED_MEAN_LOGPROB = 0, FVRAG_SEL_TWO_STAGE = 1 } fvrag_sel_mode;
+
+typedef struct fvrag_select_desc {
+  int32_t num_queries; /* Qn >= 1 */
+  int32_t num_cand;    /* K, 1..1024 */
+  int32_t cand_len;    /* L >= 1 */
+  int32_t gathers;     /* G: innermost extent of logprob (>= 2 for TWO_STAGE) */
+  int32_t mode;        /* fvrag_sel_mode */
+  float delta;         /* Eq. 13 margin (the paper uses 0.05) */
+  uint32_t flags;      /* must be 0 */
+} fvrag_select_desc;
+
+/*
+ *   logprob  [Qn][K][L][G] fp32
+ *   lengths  [Qn][K] int32, or NULL
+ *   keep     [Qn][K] uint8  (required for MASKED_MEAN_LOGPROB)
+ *   max_cos  [Qn][K] fp32   (required for TWO_STAGE)
+ *   score    [Qn][K] fp32   written
+ *   selected [Qn]    int32  written
+ */
+fvrag_status fvrag_select_candidate(const fvrag_select_desc* d, const float* logprob,
+                                    const int32_t* lengths, const uint8_t* keep,
+                                    const float* max_cos, float* score, int32_t* selected,
+                                    fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * Device status (failure detection without faulting the GPU)
+ * ------------------------------------------------------------------------ */
+
+/* Synchronises `stream`, then returns the status word stored in `ws`
+ * (FVRAG_OK, or the error a kernel recorded), or FVRAG_ERR_CUDA if the copy failed. */
+fvrag_status fvrag_read_status(const void* ws, fvrag_stream_t stream);
+
+/* Enqueues a reset of the status word in `ws` to FVRAG_OK. */
+fvrag_status fvrag_clear_status(void* ws, fvrag_stream_t stream);
+
+/* Limit, in nanoseconds, of every bounded wait inside the kernels launched
+ * after this call (default 1e9 = one second; clamped to >= 1000). */
+void fvrag_set_wait_limit_ns(uint64_t ns);
+uint64_t fvrag_get_wait_limit_ns(void);
+
+/* Diagnostic: launches one CTA that waits, with the bounded wait every kernel
+ * uses, on a shared-memory barrier that nothing ever completes.  The wait runs
+ * out after the current wait limit and records FVRAG_ERR_TIMEOUT in `ws`'s
+ * status word; the kernel then returns normally and the context stays usable. */
+fvrag_status fvrag_selftest_wait_timeout(void* ws, fvrag_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FVRAG_H */

@@ -1,0 +1,214 @@
+// K3: CLIP entity alignment (Eq. 14-15) with the keep threshold, and
+// K4: candidate selection (masked mean log-prob; Algorithm 1's two stages,
+// Eq. 12-13 and the final argmax over alignment).
+//
+// Both steps move kilobytes to a few megabytes, so they are latency-bound:
+// K3 uses one CTA per (query, candidate) with one warp per frame at a time and
+// 16-byte loads; K4 uses one CTA per query.
+#include <cuda_fp16.h>
+
+#include "fvrag_common.cuh"
+#include "fvrag_internal.h"
+
+namespace fvrag {
+
+constexpr int kClipThreads = 256;
+constexpr int kClipMaxDim = 4096;
+
+// One CTA per (query q, candidate k).  The candidate embedding is widened to
+// fp32 in shared memory; warp w handles frames w, w + 8, ...: the 32 lanes split
+// the E dimension in 16-byte (8 x fp16) chunks, reduce <e, f> and |f|^2 with
+// shuffles, and lane 0 keeps the warp's best (cos, frame).  The 8 warp results
+// are then reduced by one warp: larger cos wins, equal cos goes to the lower
+// frame index.
+__global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
+    const __half* __restrict__ cand, const __half* __restrict__ frames, int K, int F, int E,
+    float tau, float* __restrict__ cos_out, float* __restrict__ max_cos, int32_t* __restrict__ argmax,
+    uint8_t* __restrict__ keep) {
+  __shared__ __align__(16) float e_s[kClipMaxDim];
+  __shared__ float red[kClipThreads / 32];
+  __shared__ float best_v[kClipThreads / 32];
+  __shared__ int best_i[kClipThreads / 32];
+  const int qk = blockIdx.x;
+  const int q = qk / K;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nchunk = E >> 3;
+
+  const __half* e = cand + (size_t)qk * E;
+  float ee_part = 0.f;
+  for (int c = threadIdx.x; c < nchunk; c += kClipThreads) {
+    const uint4 raw = __ldg(reinterpret_cast<const uint4*>(e) + c);
+    const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __half22float2(h2[j]);
+      e_s[8 * c + 2 * j] = f.x;
+      e_s[8 * c + 2 * j + 1] = f.y;
+      ee_part = fmaf(f.x, f.x, fmaf(f.y, f.y, ee_part));
+    }
+  }
+  ee_part = warp_sum(ee_part);
+  if (lane == 0) red[warp] = ee_part;
+  __syncthreads();
+  float ee = 0.f;
+#pragma unroll
+  for (int w = 0; w < kClipThreads / 32; ++w) ee += red[w];
+  const float inv_e = ee > 0.f ? rsqrtf(ee) : 0.f;
+
+  float wbest = -INFINITY;
+  int wbest_i = 0x7fffffff;
+  const __half* fq = frames + (size_t)q * F * E;
+  for (int f = warp; f < F; f += kClipThreads / 32) {
+    const uint4* fr = reinterpret_cast<const uint4*>(fq + (size_t)f * E);
+    float dot = 0.f, ff = 0.f;
+    for (int c = lane; c < nchunk; c += 32) {
+      const uint4 raw = __ldg(fr + c);
+      const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
+      const float4 ea = *reinterpret_cast<const float4*>(&e_s[8 * c]);
+      const float4 eb = *reinterpret_cast<const float4*>(&e_s[8 * c + 4]);
+      const float2 f0 = __half22float2(h2[0]), f1 = __half22float2(h2[1]);
+      const float2 f2 = __half22float2(h2[2]), f3 = __half22float2(h2[3]);
+      dot = fmaf(ea.x, f0.x, dot); dot = fmaf(ea.y, f0.y, dot);
+      dot = fmaf(ea.z, f1.x, dot); dot = fmaf(ea.w, f1.y, dot);
+      dot = fmaf(eb.x, f2.x, dot); dot = fmaf(eb.y, f2.y, dot);
+      dot = fmaf(eb.z, f3.x, dot); dot = fmaf(eb.w, f3.y, dot);
+      ff = fmaf(f0.x, f0.x, ff); ff = fmaf(f0.y, f0.y, ff);
+      ff = fmaf(f1.x, f1.x, ff); ff = fmaf(f1.y, f1.y, ff);
+      ff = fmaf(f2.x, f2.x, ff); ff = fmaf(f2.y, f2.y, ff);
+      ff = fmaf(f3.x, f3.x, ff); ff = fmaf(f3.y, f3.y, ff);
+    }
+    dot = warp_sum(dot);
+    ff = warp_sum(ff);
+    const float c = (ff > 0.f && inv_e > 0.f) ? dot * inv_e * rsqrtf(ff) : 0.f;
+    if (lane == 0) {
+      if (cos_out) cos_out[(size_t)qk * F + f] = c;
+      if (c > wbest) {  // frames arrive in increasing order per warp: strict > keeps the lowest
+        wbest = c;
+        wbest_i = f;
+      }
+    }
+  }
+  if (lane == 0) {
+    best_v[warp] = wbest;
+    best_i[warp] = wbest_i;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    float v = lane < kClipThreads / 32 ? best_v[lane] : -INFINITY;
+    int i = lane < kClipThreads / 32 ? best_i[lane] : 0x7fffffff;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, i, o);
+      if (ov > v || (ov == v && oi < i)) {
+        v = ov;
+        i = oi;
+      }
+    }
+    if (lane == 0) {
+      max_cos[qk] = v;
+      argmax[qk] = i;
+      keep[qk] = v >= tau ? 1 : 0;
+    }
+  }
+}
+
+// One CTA per query; thread k scores candidate k in fp64 (fixed summation
+// order l = 0 .. n_k-1), then thread 0 runs the selection rule serially
+// (K <= 1024 candidates).
+__global__ void select_kernel(const float* __restrict__ logprob, const int32_t* __restrict__ lengths,
+                              const uint8_t* __restrict__ keep, const float* __restrict__ max_cos,
+                              int K, int L, int G, int mode, double delta, float* __restrict__ score,
+                              int32_t* __restrict__ selected) {
+  extern __shared__ double sc[];
+  const int q = blockIdx.x;
+  for (int k = threadIdx.x; k < K; k += blockDim.x) {
+    const size_t qk = (size_t)q * K + k;
+    const int n = lengths ? lengths[qk] : L;
+    double s = __longlong_as_double(0x7ff8000000000000ll);  // NaN
+    if (n >= 1 && n <= L) {
+      const float* lp = logprob + qk * L * G;
+      if (mode == FVRAG_SEL_MASKED_MEAN_LOGPROB) {
+        double acc = 0.0;
+        for (int l = 0; l < n; ++l) acc += (double)lp[(size_t)l * G];
+        s = acc / (double)n;
+      } else {
+        const double lpY = lp[(size_t)(n - 1) * G + 0];
+        const double lpN = lp[(size_t)(n - 1) * G + 1];
+        s = 1.0 / (1.0 + exp(lpN - lpY));
+      }
+    }
+    sc[k] = s;
+    score[qk] = (float)s;
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int sel = -1;
+    if (mode == FVRAG_SEL_MASKED_MEAN_LOGPROB) {
+      double best = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const double s = sc[k];
+        if (!keep[(size_t)q * K + k] || isnan(s)) continue;
+        if (sel < 0 || s > best) {
+          best = s;
+          sel = k;
+        }
+      }
+    } else {
+      double top = -INFINITY;
+      for (int k = 0; k < K; ++k)
+        if (!isnan(sc[k]) && sc[k] > top) top = sc[k];
+      float best = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const double s = sc[k];
+        if (isnan(s) || !(s >= top - delta)) continue;
+        const float a = max_cos[(size_t)q * K + k];
+        if (sel < 0 || a > best) {
+          best = a;
+          sel = k;
+        }
+      }
+    }
+    selected[q] = sel;
+  }
+}
+
+}  // namespace fvrag
+
+using namespace fvrag;
+
+extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
+                                         const void* frame_emb, float* cos, float* max_cos,
+                                         int32_t* argmax, uint8_t* keep, fvrag_stream_t stream) {
+  if (!d || !cand_emb || !frame_emb || !max_cos || !argmax || !keep) return FVRAG_ERR_INVALID_ARG;
+  if (d->num_queries < 1 || d->num_cand < 1 || d->num_frames < 1 || d->dim < 1 || d->flags != 0)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->dim % 8 != 0 || d->dim > kClipMaxDim) return FVRAG_ERR_UNSUPPORTED;
+  if ((int64_t)d->num_queries * d->num_cand > 0x7fffffff) return FVRAG_ERR_UNSUPPORTED;
+  if (!aligned16(cand_emb) || !aligned16(frame_emb)) return FVRAG_ERR_MISALIGNED;
+  const int blocks = d->num_queries * d->num_cand;
+  clip_align_kernel<<<blocks, kClipThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
+      reinterpret_cast<const __half*>(cand_emb), reinterpret_cast<const __half*>(frame_emb),
+      d->num_cand, d->num_frames, d->dim, d->threshold, cos, max_cos, argmax, keep);
+  return launch_status();
+}
+
+extern "C" fvrag_status fvrag_select_candidate(const fvrag_select_desc* d, const float* logprob,
+                                               const int32_t* lengths, const uint8_t* keep,
+                                               const float* max_cos, float* score,
+                                               int32_t* selected, fvrag_stream_t stream) {
+  if (!d || !logprob || !score || !selected) return FVRAG_ERR_INVALID_ARG;
+  if (d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->gathers < 1 || d->flags != 0)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->mode != FVRAG_SEL_MASKED_MEAN_LOGPROB && d->mode != FVRAG_SEL_TWO_STAGE)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->mode == FVRAG_SEL_MASKED_MEAN_LOGPROB && !keep) return FVRAG_ERR_INVALID_ARG;
+  if (d->mode == FVRAG_SEL_TWO_STAGE && (!max_cos || d->gathers < 2)) return FVRAG_ERR_INVALID_ARG;
+  if (d->num_cand > 1024) return FVRAG_ERR_UNSUPPORTED;
+  const int threads = ((d->num_cand + 31) / 32) * 32;
+  select_kernel<<<d->num_queries, threads, sizeof(double) * d->num_cand,
+                  reinterpret_cast<cudaStream_t>(stream)>>>(
+      logprob, lengths, keep, max_cos, d->num_cand, d->cand_len, d->gathers, d->mode,
+      (double)d->delta, score, selected);
+  return launch_status();
+}

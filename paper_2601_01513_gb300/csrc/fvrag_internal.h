@@ -1,0 +1,32 @@
+// Host-side helpers shared by the libfvrag translation units (not exported).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "fvrag.h"
+
+namespace fvrag {
+
+// Current limit of the kernels' bounded waits, in nanoseconds.
+uint64_t wait_limit_ns();
+
+// Number of SMs of the current device (cached per device); 0 if it cannot be read.
+int sm_count();
+
+// Tiled TMA descriptor over a row-major tensor of 16-bit elements.
+//   dims[0] = innermost extent (elements), dims[i] = extent of dimension i,
+//   strides_bytes[i-1] = byte stride of dimension i (multiple of 16),
+//   box[i] = box extent in dimension i (box[0] * 2 bytes <= 128 with the 128-byte swizzle).
+// Returns false when the driver rejects the description.
+bool encode_tmap_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
+                      const uint64_t* strides_bytes, const uint32_t* box, bool swizzle128);
+
+inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+inline fvrag_status launch_status() {
+  return cudaGetLastError() == cudaSuccess ? FVRAG_OK : FVRAG_ERR_CUDA;
+}
+
+}  // namespace fvrag

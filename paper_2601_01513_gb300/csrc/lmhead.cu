@@ -1,0 +1,438 @@
+// K2: verifier LM-head log-probabilities (Eq. 11; the verifier likelihood of
+// Section 4.5) as one tcgen05 GEMM with a fused online log-sum-exp and target
+// gather, so the [rows x vocab] logits never leave the SM.
+//
+// Shape of the work: z = hidden[M x H] * W[V x H]^T with M (candidate tokens)
+// small (32 .. ~1300) and V x H large (152064 x 3584 bf16 = 1.09 GB).  W is read
+// from HBM exactly once; hidden (<= a few MB) stays in L2 and is re-read by
+// every CTA.
+//
+// Persistent grid, one CTA per SM.  CTA b owns a contiguous vocabulary range
+// (multiples of 16 rows, balanced to within 16 rows) and walks it in tiles of BN
+// rows.  Per tile it accumulates, for a group of MG M-tiles of 128 hidden rows,
+// D[128 x BN] = hidden_tile * W_tile^T in tensor memory (fp32), K-loop over H
+// in blocks of 64 (one 128-byte swizzled row per operand row).
+//
+// Warp roles (192 threads):
+//   warp 0     TMA producer: hidden tiles (box 64 x 128) and W tiles (boxes of
+//              64 x 64 rows, 64 x 16 rows for the remainder) into a STAGES-deep
+//              shared-memory ring, completion via mbarrier transaction counts.
+//   warp 1     allocates tensor memory; one lane issues tcgen05.mma
+//              (M = 128, N = tile rows, K = 16) and tcgen05.commit.
+//   warps 2-5  epilogue: tcgen05.ld of 32 columns at a time (one hidden row per
+//              thread), online max / sum of exp over the CTA's vocabulary slice,
+//              and the gather of target logits that fall in the slice.
+// SLOTS accumulator sets in tensor memory let the epilogue of tile t overlap the
+// MMAs of tile t+1.
+//
+// A second small kernel merges the per-CTA (max, sum) partials of every row into
+// lse and writes logprob = z_target - lse (NaN for ids outside [0, V)).
+#include <cuda_bf16.h>
+
+#include <algorithm>
+
+#include "fvrag_common.cuh"
+#include "fvrag_internal.h"
+
+namespace fvrag {
+namespace lm {
+
+constexpr int kThreads = 192;
+constexpr int kBK = 64;            // bf16 elements per 128-byte swizzled row
+constexpr int kBM = 128;           // hidden rows per M-tile (MMA M)
+constexpr int kStages = 4;
+constexpr int kMaxCtas = 256;      // workspace is sized for this many partials
+constexpr int kMaxMTiles = 16;     // rows <= 2048
+constexpr int kMaxGathers = 8;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+// wait-site ids recorded in the workspace header on a timeout
+enum : uint32_t { kSiteProdEmpty = 0x201, kSiteMmaTmem = 0x202, kSiteMmaFull = 0x203,
+                  kSiteEpiFull = 0x204, kSiteDrain = 0x205 };
+
+template <int BN, int MG>
+struct Cfg {
+  static constexpr int kABytes = kBM * kBK * 2;           // 16 KB per M-tile
+  static constexpr int kBBytes = BN * kBK * 2;            // BN rows x 128 B
+  static constexpr int kStageBytes = MG * kABytes + kBBytes;
+  static constexpr int kSlots = 2;
+  static constexpr int kTmemCols = kSlots * MG * BN;      // 512
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/ +
+                                    2 * kMaxMTiles * kBM * 4 /*row state*/;
+  static_assert(kTmemCols == 512, "tensor memory plan uses all 512 columns");
+  static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+};
+
+__device__ __forceinline__ float ex2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+template <int BN, int MG>
+__global__ void __launch_bounds__(kThreads, 1)
+    lm_head_kernel(const __grid_constant__ CUtensorMap tm_hidden,
+                   const __grid_constant__ CUtensorMap tm_w64,
+                   const __grid_constant__ CUtensorMap tm_w16, const int32_t* __restrict__ targets,
+                   int M, int H, int V, int G, float* __restrict__ part_max,
+                   float* __restrict__ part_sum, float* __restrict__ tgt_logit, uint32_t* status,
+                   uint64_t limit_ns) {
+  using C = Cfg<BN, MG>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* ring = smem;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + kStages * C::kStageBytes);
+  uint64_t* full = bars;                    // [kStages]
+  uint64_t* empty = bars + kStages;         // [kStages]
+  uint64_t* tfull = bars + 2 * kStages;     // [kSlots]
+  uint64_t* tempty = tfull + C::kSlots;     // [kSlots]
+  uint64_t* drain = tempty + C::kSlots;     // [1]
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* st_max = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);
+  float* st_sum = st_max + kMaxMTiles * kBM;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  // ---- this CTA's vocabulary range, in units of 16 rows
+  const int nunits = (V + 15) >> 4;
+  const int u_lo = (int)(((long long)blockIdx.x * nunits) / gridDim.x);
+  const int u_hi = (int)(((long long)(blockIdx.x + 1) * nunits) / gridDim.x);
+  const int v_lo = u_lo * 16;
+  const int v_hi = min(u_hi * 16, V);
+  const int ntiles = (v_hi - v_lo + BN - 1) / BN;
+  const int mtiles = (M + kBM - 1) / kBM;
+  const int ngroups = (mtiles + MG - 1) / MG;
+  const int nitems = ntiles * ngroups;
+  const int kblocks = (H + kBK - 1) / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int s = 0; s < C::kSlots; ++s) {
+      mbar_init(smem_u32(&tfull[s]), 1);
+      mbar_init(smem_u32(&tempty[s]), 4);  // one arrival per epilogue warp
+    }
+    mbar_init(smem_u32(drain), 1);
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_hidden);
+    tma_prefetch_desc(&tm_w64);
+    tma_prefetch_desc(&tm_w16);
+  }
+  for (int i = threadIdx.x; i < mtiles * kBM; i += kThreads) {
+    st_max[i] = -INFINITY;
+    st_sum[i] = 0.f;
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_h = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int t = it / ngroups, grp = it % ngroups;
+        const int v0 = v_lo + t * BN;
+        const int rows16 = (min(BN, v_hi - v0) + 15) & ~15;
+        const int mcount = min(MG, mtiles - grp * MG);
+        const uint32_t bytes = mcount * C::kABytes + rows16 * kBK * 2;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_arrive_expect_tx(fb, bytes);
+          uint8_t* st = ring + stage * C::kStageBytes;
+          for (int j = 0; j < mcount; ++j)
+            tma_load_2d(smem_u32(st + j * C::kABytes), &tm_hidden, fb, kb * kBK,
+                        (grp * MG + j) * kBM, pol_h);
+          uint8_t* bsm = st + MG * C::kABytes;
+          int r = 0;
+          for (; r + 64 <= rows16; r += 64)
+            tma_load_2d(smem_u32(bsm + r * 128), &tm_w64, fb, kb * kBK, v0 + r, pol_w);
+          for (; r < rows16; r += 16)
+            tma_load_2d(smem_u32(bsm + r * 128), &tm_w16, fb, kb * kBK, v0 + r, pol_w);
+          ++issued;
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // leave no copy in flight: wait for the last (up to kStages) loads issued
+      const int pend = issued < kStages ? (int)issued : kStages;
+      for (int i = 0; i < pend; ++i) {
+        if (--stage < 0) {
+          stage = kStages - 1;
+          phase ^= 1;
+        }
+        mbar_wait(smem_u32(&full[stage]), phase, limit_ns);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int slot = it % C::kSlots;
+        const uint32_t use = it / C::kSlots;
+        const int t = it / ngroups, grp = it % ngroups;
+        const int v0 = v_lo + t * BN;
+        const int rows16 = (min(BN, v_hi - v0) + 15) & ~15;
+        const int mcount = min(MG, mtiles - grp * MG);
+        const uint32_t idesc = idesc_bf16_f32(kBM, rows16);
+        if (!mbar_wait(smem_u32(&tempty[slot]), (use & 1) ^ 1, limit_ns)) {
+          record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaTmem);
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaFull);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(ring + stage * C::kStageBytes);
+          const uint32_t bsm = st + MG * C::kABytes;
+          for (int j = 0; j < mcount; ++j) {
+            const uint32_t d = tmem_base + (uint32_t)((slot * MG + j) * BN);
+#pragma unroll
+            for (int k16 = 0; k16 < kBK / 16; ++k16) {
+              const uint64_t a = desc_kmajor_sw128(st + j * C::kABytes + k16 * 32);
+              const uint64_t b = desc_kmajor_sw128(bsm + k16 * 32);
+              tc_mma_bf16(d, a, b, idesc, (kb | k16) != 0);
+            }
+          }
+          tc_commit(smem_u32(&empty[stage]));
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit(smem_u32(&tfull[slot]));
+      }
+      // every MMA issued by this thread has finished before tensor memory is freed
+      tc_commit(smem_u32(drain));
+      if (!mbar_wait(smem_u32(drain), 0, limit_ns))
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quarter = warp & 3;             // tensor-memory lanes this warp may access
+    const int row = quarter * 32 + lane;      // row inside an M-tile
+    for (int it = 0; it < nitems; ++it) {
+      const int slot = it % C::kSlots;
+      const uint32_t use = it / C::kSlots;
+      const int t = it / ngroups, grp = it % ngroups;
+      const int v0 = v_lo + t * BN;
+      const int ncols = min(BN, v_hi - v0);
+      const int rows16 = (ncols + 15) & ~15;
+      const int mcount = min(MG, mtiles - grp * MG);
+      if (!mbar_wait(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
+        break;
+      }
+      tc_fence_after();
+      for (int j = 0; j < mcount; ++j) {
+        const int mt = grp * MG + j;
+        const int m = mt * kBM + row;
+        const bool live = m < M;
+        int tg[kMaxGathers];
+#pragma unroll
+        for (int g = 0; g < kMaxGathers; ++g)
+          tg[g] = (live && g < G) ? __ldg(&targets[(size_t)m * G + g]) - v0 : -1;
+        float rmax = st_max[mt * kBM + row];  // running max of z * log2(e)
+        float rsum = st_sum[mt * kBM + row];
+        const uint32_t tbase =
+            tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * MG + j) * BN);
+        for (int c0 = 0; c0 < rows16; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + c0, r);
+          tmem_wait_ld();
+          const int nvalid = min(32, ncols - c0);
+          float cmax = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nvalid) cmax = fmaxf(cmax, __uint_as_float(r[i]) * kLog2e);
+          const float nmax = fmaxf(rmax, cmax);
+          float s = rsum * ex2(rmax - nmax);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nvalid) s += ex2(fmaf(__uint_as_float(r[i]), kLog2e, -nmax));
+          rsum = s;
+          rmax = nmax;
+#pragma unroll
+          for (int g = 0; g < kMaxGathers; ++g) {
+            const int c = tg[g] - c0;
+            if (c >= 0 && c < nvalid) {
+              float val = 0.f;
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (i == c) val = __uint_as_float(r[i]);
+              tgt_logit[(size_t)m * G + g] = val;
+            }
+          }
+        }
+        st_max[mt * kBM + row] = rmax;
+        st_sum[mt * kBM + row] = rsum;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[slot]));
+    }
+    // publish this CTA's partials (row state in the log2 domain)
+    for (int mt = 0; mt < mtiles; ++mt) {
+      const int m = mt * kBM + row;
+      if (m < M) {
+        part_max[(size_t)blockIdx.x * M + m] = st_max[mt * kBM + row];
+        part_sum[(size_t)blockIdx.x * M + m] = st_sum[mt * kBM + row];
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
+}
+
+// One warp per row: lse = ln 2 * (M2 + log2 S) with M2 = max_b max_b and
+// S = sum_b sum_b * 2^(max_b - M2); logprob = z_target - lse.
+__global__ void lm_merge_kernel(const float* __restrict__ part_max, const float* __restrict__ part_sum,
+                                const float* __restrict__ tgt_logit,
+                                const int32_t* __restrict__ targets, int M, int V, int G, int nparts,
+                                float* __restrict__ logprob, float* __restrict__ lse_out) {
+  const int m = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (m >= M) return;
+  float mx = -INFINITY;
+  for (int b = lane; b < nparts; b += 32) mx = fmaxf(mx, part_max[(size_t)b * M + m]);
+  mx = warp_max(mx);
+  float s = 0.f;
+  for (int b = lane; b < nparts; b += 32) {
+    const float pm = part_max[(size_t)b * M + m];
+    if (pm != -INFINITY) s += part_sum[(size_t)b * M + m] * ex2(pm - mx);
+  }
+  s = warp_sum(s);
+  const float l = kLn2 * (mx + __log2f(s));
+  if (lane == 0 && lse_out) lse_out[m] = l;
+  for (int g = lane; g < G; g += 32) {
+    const int32_t t = targets[(size_t)m * G + g];
+    logprob[(size_t)m * G + g] =
+        (t >= 0 && t < V) ? tgt_logit[(size_t)m * G + g] - l : __int_as_float(0x7fc00000);
+  }
+}
+
+struct Plan {
+  int ctas;
+  int bn, mg;
+};
+
+static Plan make_plan(const fvrag_lm_desc* d, int sms) {
+  Plan p;
+  const int mtiles = (d->rows + kBM - 1) / kBM;
+  p.bn = mtiles == 1 ? 256 : 128;
+  p.mg = mtiles == 1 ? 1 : 2;
+  const int nunits = (d->vocab + 15) / 16;
+  p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
+  return p;
+}
+
+static size_t ws_bytes(const fvrag_lm_desc* d) {
+  const size_t M = (size_t)d->rows;
+  return kWsHeaderBytes + 2 * (size_t)kMaxCtas * M * 4 + M * (size_t)d->gathers * 4;
+}
+
+template <int BN, int MG>
+static fvrag_status launch(const Plan& p, const CUtensorMap& th, const CUtensorMap& tw64,
+                           const CUtensorMap& tw16, const int32_t* targets, const fvrag_lm_desc* d,
+                           float* pmax, float* psum, float* ptgt, uint32_t* status,
+                           cudaStream_t s) {
+  using C = Cfg<BN, MG>;
+  auto kern = lm_head_kernel<BN, MG>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  kern<<<p.ctas, kThreads, C::kSmemBytes, s>>>(th, tw64, tw16, targets, d->rows, d->hidden,
+                                               d->vocab, d->gathers, pmax, psum, ptgt, status,
+                                               wait_limit_ns());
+  return launch_status();
+}
+
+}  // namespace lm
+}  // namespace fvrag
+
+using namespace fvrag;
+
+extern "C" size_t fvrag_score_logprobs_workspace(const fvrag_lm_desc* d) {
+  if (!d || d->rows < 1 || d->hidden < 8 || d->vocab < 1 || d->gathers < 1) return 0;
+  return lm::ws_bytes(d);
+}
+
+extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void* hidden,
+                                             const void* weight, const int32_t* targets,
+                                             float* logprob, float* lse, void* ws, size_t ws_size,
+                                             fvrag_stream_t stream) {
+  using namespace lm;
+  if (!d || !hidden || !weight || !targets || !logprob) return FVRAG_ERR_INVALID_ARG;
+  if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->gathers > kMaxGathers || d->rows > kMaxMTiles * kBM) return FVRAG_ERR_UNSUPPORTED;
+  if (d->hidden % 8 != 0) return FVRAG_ERR_MISALIGNED;
+  if (!aligned16(hidden) || !aligned16(weight)) return FVRAG_ERR_MISALIGNED;
+  if (!ws || ws_size < ws_bytes(d)) return FVRAG_ERR_WORKSPACE;
+  if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
+
+  const Plan p = make_plan(d, sm_count());
+  const uint64_t H = (uint64_t)d->hidden, M = (uint64_t)d->rows, V = (uint64_t)d->vocab;
+  CUtensorMap th, tw64, tw16;
+  {
+    const uint64_t dims[2] = {H, M}, strides[1] = {H * 2};
+    const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)kBM};
+    if (!encode_tmap_bf16(&th, hidden, 2, dims, strides, box, true)) return FVRAG_ERR_CUDA;
+  }
+  {
+    const uint64_t dims[2] = {H, V}, strides[1] = {H * 2};
+    const uint32_t box64[2] = {(uint32_t)kBK, 64u}, box16[2] = {(uint32_t)kBK, 16u};
+    if (!encode_tmap_bf16(&tw64, weight, 2, dims, strides, box64, true)) return FVRAG_ERR_CUDA;
+    if (!encode_tmap_bf16(&tw16, weight, 2, dims, strides, box16, true)) return FVRAG_ERR_CUDA;
+  }
+  uint8_t* base = reinterpret_cast<uint8_t*>(ws);
+  uint32_t* status = reinterpret_cast<uint32_t*>(base);
+  float* pmax = reinterpret_cast<float*>(base + kWsHeaderBytes);
+  float* psum = pmax + (size_t)kMaxCtas * M;
+  float* ptgt = psum + (size_t)kMaxCtas * M;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  fvrag_status st;
+  if (p.bn == 256)
+    st = launch<256, 1>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
+  else
+    st = launch<128, 2>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
+  if (st != FVRAG_OK) return st;
+  const int rows_per_block = 8;
+  lm_merge_kernel<<<(d->rows + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0, s>>>(
+      pmax, psum, ptgt, targets, d->rows, d->vocab, d->gathers, p.ctas, logprob, lse);
+  return launch_status();
+}

@@ -1,0 +1,142 @@
+"""One verify step of the VideoSpeculateRAG verifier on one GPU (public API).
+
+``VerifyStep`` owns the device buffers of one workload and issues the four
+libfvrag calls in order on one stream:
+
+  1. fvrag_verify_attn       attention over shared prefix + own causal tail (Eq. 6, Eq. 11)
+  2. fvrag_score_logprobs    LM-head log-probabilities of the candidate tokens (Eq. 11)
+  3. fvrag_clip_align        entity/frame cosine, max over frames, keep flag (Eq. 14-15)
+  4. fvrag_select_candidate  masked mean log-prob, or Algorithm 1's two stages (Eq. 12-13)
+
+In the real verifier the attention output feeds further layers before the LM
+head; the synthetic workloads give the LM head its own hidden states, so the
+four calls are independent launches on one stream.  PyTorch only provides
+memory, copies and the stream.
+"""
+import numpy as np
+import torch
+
+from . import fvrag
+from .configs import VerifyConfig
+
+STEP_INPUTS = ("q", "k_prefix", "v_prefix", "prefix_offsets", "k_tail", "v_tail", "hidden",
+               "targets", "cand_emb", "frame_emb")
+RESIDENT = ("weight",)   # model parameters: loaded once, not part of a step's inputs
+
+
+def _to_torch(name, arr):
+    if name in ("cand_emb", "frame_emb"):
+        return torch.from_numpy(arr.view(np.int16)).view(torch.float16)
+    if arr.dtype == np.uint16:
+        return torch.from_numpy(arr.view(np.int16)).view(torch.bfloat16)
+    return torch.from_numpy(arr)
+
+
+class VerifyStep:
+    def __init__(self, cfg: VerifyConfig, device="cuda", mode=fvrag.SEL_MASKED_MEAN_LOGPROB,
+                 max_prefix=None, with_lse=True):
+        self.cfg = cfg
+        self.device = torch.device(device)
+        self.mode = mode
+        self.with_lse = with_lse
+        self.max_prefix = max_prefix
+        self.t = {}
+        Qn, K, L, hq, D = cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.hq, cfg.head_dim
+        M = cfg.rows
+        dev = self.device
+        self.out = torch.empty((Qn, K, L, hq, D), dtype=torch.bfloat16, device=dev)
+        self.attn_lse = torch.empty((Qn, K, L, hq), dtype=torch.float32, device=dev) if with_lse else None
+        self.logprob = torch.empty((M, cfg.gathers), dtype=torch.float32, device=dev)
+        self.lm_lse = torch.empty((M,), dtype=torch.float32, device=dev) if with_lse else None
+        self.max_cos = torch.empty((Qn, K), dtype=torch.float32, device=dev)
+        self.argmax = torch.empty((Qn, K), dtype=torch.int32, device=dev)
+        self.keep = torch.empty((Qn, K), dtype=torch.uint8, device=dev)
+        self.cos = None
+        self.score = torch.empty((Qn, K), dtype=torch.float32, device=dev)
+        self.selected = torch.empty((Qn,), dtype=torch.int32, device=dev)
+        lmd = fvrag.LmDesc(M, cfg.hidden, cfg.vocab, cfg.gathers, 0)
+        self.lm_ws = torch.zeros(fvrag.lm_workspace_bytes(lmd), dtype=torch.uint8, device=dev)
+        self.attn_ws = None
+
+    # ---------------------------------------------------------------- inputs
+    def upload(self, inputs: dict) -> None:
+        """Copies numpy inputs (from ``synth.make_inputs``) to the device."""
+        for name, arr in inputs.items():
+            self.t[name] = _to_torch(name, arr).to(self.device)
+        if "prefix_offsets" in inputs:
+            offs = inputs["prefix_offsets"]
+            mp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
+            self.max_prefix = mp if self.max_prefix is None else max(self.max_prefix, mp)
+            self._alloc_attn_ws()
+
+    def _alloc_attn_ws(self):
+        c = self.cfg
+        d = fvrag.AttnDesc(c.num_queries, c.num_cand, c.cand_len, c.hq, c.hkv, c.head_dim,
+                           int(self.max_prefix), int(self.t["k_prefix"].shape[0]), 0.0, 0)
+        need = fvrag.attn_workspace_bytes(d)
+        if self.attn_ws is None or self.attn_ws.numel() < need:
+            self.attn_ws = torch.zeros(need, dtype=torch.uint8, device=self.device)
+
+    def host_inputs(self, pin=True) -> dict:
+        """Per-step inputs as (pinned) host tensors, for the end-to-end path."""
+        h = {}
+        for name in STEP_INPUTS:
+            if name in self.t:
+                x = torch.empty(self.t[name].shape, dtype=self.t[name].dtype, pin_memory=pin)
+                x.copy_(self.t[name])
+                h[name] = x
+        return h
+
+    # ---------------------------------------------------------------- the step
+    def attention(self, stream=None):
+        t = self.t
+        fvrag.verify_attn(t["q"], t["k_prefix"], t["v_prefix"], t["prefix_offsets"], t["k_tail"],
+                          t["v_tail"], self.out, self.attn_ws, self.max_prefix, lse=self.attn_lse,
+                          stream=stream)
+
+    def lm_head(self, stream=None):
+        t = self.t
+        fvrag.score_logprobs(t["hidden"], t["weight"], t["targets"], self.logprob, self.lm_ws,
+                             lse=self.lm_lse, stream=stream)
+
+    def clip(self, stream=None):
+        t = self.t
+        fvrag.clip_align(t["cand_emb"], t["frame_emb"], self.cfg.threshold, self.max_cos,
+                         self.argmax, self.keep, cos=self.cos, stream=stream)
+
+    def select(self, stream=None):
+        c = self.cfg
+        lp = self.logprob.view(c.num_queries, c.num_cand, c.cand_len, c.gathers)
+        fvrag.select_candidate(lp, self.score, self.selected, mode=self.mode, keep=self.keep,
+                               max_cos=self.max_cos, lengths=self.t.get("lengths"),
+                               delta=c.delta, stream=stream)
+
+    def run(self, stream=None):
+        """All four calls of one verify step, enqueued on `stream` (default: current)."""
+        self.attention(stream)
+        self.lm_head(stream)
+        self.clip(stream)
+        self.select(stream)
+
+    def launches_per_step(self) -> int:
+        """Kernels this library launches per step: attention prefix (if any prefix) + tail/merge,
+        LM head + merge, CLIP, select."""
+        return (2 if self.cfg.prefix_len > 0 or self.cfg.prefix_range else 1) + 2 + 1 + 1
+
+    def run_from_host(self, host: dict, stream=None):
+        """End-to-end step: host->device copies of the step's inputs, the four calls, and a
+        device->host read of the result (selected index and candidate scores).
+        Returns (selected, score) host tensors and the byte counts moved each way."""
+        h2d = 0
+        for name, x in host.items():
+            self.t[name].copy_(x, non_blocking=True)
+            h2d += x.numel() * x.element_size()
+        self.run(stream)
+        if getattr(self, "_sel_h", None) is None:
+            self._sel_h = torch.empty(self.selected.shape, dtype=self.selected.dtype, pin_memory=True)
+            self._sc_h = torch.empty(self.score.shape, dtype=self.score.dtype, pin_memory=True)
+        sel, sc = self._sel_h, self._sc_h
+        sel.copy_(self.selected, non_blocking=True)
+        sc.copy_(self.score, non_blocking=True)
+        d2h = sel.numel() * sel.element_size() + sc.numel() * sc.element_size()
+        return sel, sc, h2d, d2h

@@ -1,0 +1,123 @@
+"""Shared helpers of the GPU parity tests: device placement of seeded inputs and
+the comparison rules (tolerances and margin rules for integer decisions)."""
+import numpy as np
+import torch
+
+from paper_2601_01513_gb300 import build, fvrag
+
+ATTN_ATOL = 2e-2        # attention output, max-abs (bf16 output vs fp64)
+ATTN_LSE_ATOL = 2e-3    # attention log-sum-exp (fp32 scores, fp32 sums)
+LOGPROB_ATOL = 1e-2     # per-token log-prob
+COS_ATOL = 1e-3         # cosine / max_cos
+
+
+def ensure_built():
+    build.build_all()
+    return fvrag.lib()
+
+
+def dev_bf16(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def dev_f16(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.float16).cuda()
+
+
+def dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0):
+    """Runs fvrag_verify_attn on numpy inputs; returns (out fp32 numpy, lse numpy, status)."""
+    Qn, K, L, Hq, D = q.shape
+    tq, tkt, tvt = dev_bf16(q), dev_bf16(kt), dev_bf16(vt)
+    tkp = dev_bf16(kp) if kp.shape[0] > 0 else None
+    tvp = dev_bf16(vp) if vp.shape[0] > 0 else None
+    toffs = dev(offs.astype(np.int32))
+    maxp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
+    d = fvrag.AttnDesc(Qn, K, L, Hq, kt.shape[3], D, maxp, int(kp.shape[0]), float(scale), 0)
+    ws = torch.zeros(fvrag.attn_workspace_bytes(d), dtype=torch.uint8, device="cuda")
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full(q.shape[:-1], float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
+    fvrag.verify_attn(tq, tkp, tvp, toffs, tkt, tvt, out, ws, maxp, lse=lse, softmax_scale=scale)
+    st = fvrag.read_status(ws)
+    return out.float().cpu().numpy(), (lse.cpu().numpy() if with_lse else None), st
+
+
+def run_lm(hidden, weight, targets):
+    th, tw, tt = dev_bf16(hidden), dev_bf16(weight), dev(targets.astype(np.int32))
+    M = hidden.shape[0]
+    G = targets.shape[1]
+    d = fvrag.LmDesc(M, hidden.shape[1], weight.shape[0], G, 0)
+    ws = torch.zeros(fvrag.lm_workspace_bytes(d), dtype=torch.uint8, device="cuda")
+    lp = torch.full((M, G), float("nan"), dtype=torch.float32, device="cuda")
+    lse = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+    fvrag.score_logprobs(th, tw, tt, lp, ws, lse=lse)
+    st = fvrag.read_status(ws)
+    return lp.cpu().numpy(), lse.cpu().numpy(), st
+
+
+def run_clip(cand, frames, tau, with_cos=True):
+    Qn, K, E = cand.shape
+    F = frames.shape[1]
+    tc, tf = dev_f16(cand), dev_f16(frames)
+    mc = torch.full((Qn, K), float("nan"), device="cuda")
+    am = torch.full((Qn, K), -7, dtype=torch.int32, device="cuda")
+    keep = torch.full((Qn, K), 9, dtype=torch.uint8, device="cuda")
+    cos = torch.full((Qn, K, F), float("nan"), device="cuda") if with_cos else None
+    fvrag.clip_align(tc, tf, tau, mc, am, keep, cos=cos)
+    torch.cuda.synchronize()
+    return ((cos.cpu().numpy() if with_cos else None), mc.cpu().numpy(), am.cpu().numpy(),
+            keep.cpu().numpy())
+
+
+def run_select(lp, mode, keep=None, max_cos=None, lengths=None, delta=0.05):
+    Qn, K, L, G = lp.shape
+    score = torch.full((Qn, K), float("nan"), device="cuda")
+    sel = torch.full((Qn,), -7, dtype=torch.int32, device="cuda")
+    fvrag.select_candidate(dev(lp.astype(np.float32)), score, sel, mode=mode,
+                           keep=None if keep is None else dev(keep.astype(np.uint8)),
+                           max_cos=None if max_cos is None else dev(max_cos.astype(np.float32)),
+                           lengths=None if lengths is None else dev(lengths.astype(np.int32)),
+                           delta=delta)
+    torch.cuda.synchronize()
+    return score.cpu().numpy(), sel.cpu().numpy()
+
+
+def check_argmax_with_margin(gpu_idx, oracle_cos, tol=COS_ATOL):
+    """GPU frame index must attain the oracle max within tol (unique when the margin is larger)."""
+    Qn, K, F = oracle_cos.shape
+    for q in range(Qn):
+        for k in range(K):
+            row = oracle_cos[q, k]
+            j = int(gpu_idx[q, k])
+            assert 0 <= j < F
+            assert row[j] >= row.max() - tol, (q, k, j, row[j], row.max())
+            srt = np.sort(row)
+            if F > 1 and srt[-1] - srt[-2] > tol:
+                assert j == int(np.argmax(row))
+
+
+def check_keep_with_margin(gpu_keep, oracle_maxcos, tau, tol=COS_ATOL):
+    exp = (oracle_maxcos >= tau).astype(np.uint8)
+    ambiguous = np.abs(oracle_maxcos - tau) < tol
+    assert np.all((gpu_keep == exp) | ambiguous)
+    assert np.all((gpu_keep == 0) | (gpu_keep == 1))
+
+
+def check_selection_masked(gpu_sel, oracle_score, oracle_maxcos, tau, tol_score=2 * LOGPROB_ATOL,
+                           tol_cos=COS_ATOL):
+    """The GPU pick must be a valid answer under some resolution of the ambiguous keeps, and
+    within the score tolerance of the best valid candidate."""
+    Qn, K = oracle_score.shape
+    for q in range(Qn):
+        sure = oracle_maxcos[q] >= tau + tol_cos
+        maybe = oracle_maxcos[q] > tau - tol_cos
+        s = int(gpu_sel[q])
+        if s < 0:
+            assert not sure.any()
+            continue
+        assert maybe[s]
+        best_sure = oracle_score[q][sure].max() if sure.any() else -np.inf
+        assert oracle_score[q, s] >= best_sure - tol_score

@@ -1,0 +1,123 @@
+"""The C ABI without a GPU: the library loads, exports every symbol that
+include/fvrag.h declares, and rejects bad arguments on the host before any
+CUDA call (fake, never-dereferenced pointer values are enough for that)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2601_01513_gb300 import build, fvrag
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "fvrag.h")
+
+P = ctypes.c_void_p(0x10000)      # aligned fake pointer (never dereferenced: calls fail first)
+PMIS = ctypes.c_void_p(0x10008)   # 8-byte aligned only
+
+
+@pytest.fixture(scope="module")
+def L():
+    build.build_lib()
+    return fvrag.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(fvrag_[a-z_0-9]+)\s*\(", text)))
+
+
+def test_exports_every_declared_symbol(L):
+    names = declared_functions()
+    assert len(names) >= 13
+    assert set(names) == set(fvrag.EXPORTED)
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_version_and_strings(L):
+    assert L.fvrag_abi_version() == 1
+    for s in range(7):
+        assert fvrag.status_string(s)
+    assert fvrag.status_string(99) == "unknown status"
+
+
+def test_wait_limit_roundtrip(L):
+    old = fvrag.get_wait_limit_ns()
+    fvrag.set_wait_limit_ns(5)
+    assert fvrag.get_wait_limit_ns() == 1000    # clamped
+    fvrag.set_wait_limit_ns(old)
+    assert fvrag.get_wait_limit_ns() == old
+
+
+def _attn(L, d, ws_bytes=1 << 30, q=P, kp=P, vp=P, offs=P, kt=P, vt=P, out=P, ws=P):
+    return L.fvrag_verify_attn(ctypes.byref(d), q, kp, vp, offs, kt, vt, out, None, ws, ws_bytes, None)
+
+
+def test_attn_validation(L):
+    good = fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 0)
+    ws = L.fvrag_verify_attn_workspace(ctypes.byref(good))
+    assert ws > 256
+    assert _attn(L, fvrag.AttnDesc(0, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert _attn(L, good, q=None) == fvrag.ERR_INVALID_ARG
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 1)) == fvrag.ERR_INVALID_ARG
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 5, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 96, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _attn(L, fvrag.AttnDesc(1, 5, 65, 28, 4, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _attn(L, good, q=PMIS) == fvrag.ERR_MISALIGNED
+    assert _attn(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE
+    assert _attn(L, good, ws=None) == fvrag.ERR_WORKSPACE
+    assert _attn(L, good, kp=None) == fvrag.ERR_INVALID_ARG
+    # no prefix at all: prefix pointers may be NULL, workspace is just the header
+    nop = fvrag.AttnDesc(1, 2, 3, 4, 2, 64, 0, 0, 0.0, 0)
+    assert L.fvrag_verify_attn_workspace(ctypes.byref(nop)) == 256
+
+
+def test_lm_validation(L):
+    d = fvrag.LmDesc(80, 3584, 152064, 1, 0)
+    need = L.fvrag_score_logprobs_workspace(ctypes.byref(d))
+    assert need >= 256 + 2 * 256 * 80 * 4 + 80 * 4
+
+    def call(desc, h=P, w=P, t=P, lp=P, ws=P, wsb=need):
+        return L.fvrag_score_logprobs(ctypes.byref(desc), h, w, t, lp, None, ws, wsb, None)
+
+    assert call(d, h=None) == fvrag.ERR_INVALID_ARG
+    assert call(fvrag.LmDesc(0, 3584, 152064, 1, 0)) == fvrag.ERR_INVALID_ARG
+    assert call(fvrag.LmDesc(80, 3584, 152064, 9, 0)) == fvrag.ERR_UNSUPPORTED
+    assert call(fvrag.LmDesc(4096, 3584, 152064, 1, 0)) == fvrag.ERR_UNSUPPORTED
+    assert call(fvrag.LmDesc(80, 3583, 152064, 1, 0)) == fvrag.ERR_MISALIGNED
+    assert call(d, w=PMIS) == fvrag.ERR_MISALIGNED
+    assert call(d, wsb=need - 4) == fvrag.ERR_WORKSPACE
+    assert L.fvrag_score_logprobs_workspace(ctypes.byref(fvrag.LmDesc(0, 8, 8, 1, 0))) == 0
+
+
+def test_clip_and_select_validation(L):
+    d = fvrag.ClipDesc(1, 5, 64, 768, 0.2, 0)
+    assert L.fvrag_clip_align(ctypes.byref(d), None, P, None, P, P, P, None) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_clip_align(ctypes.byref(fvrag.ClipDesc(1, 5, 64, 770, 0.2, 0)), P, P, None, P, P, P,
+                              None) == fvrag.ERR_UNSUPPORTED
+    assert L.fvrag_clip_align(ctypes.byref(fvrag.ClipDesc(1, 5, 0, 768, 0.2, 0)), P, P, None, P, P, P,
+                              None) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_clip_align(ctypes.byref(d), PMIS, P, None, P, P, P, None) == fvrag.ERR_MISALIGNED
+    s = fvrag.SelectDesc(1, 5, 16, 1, fvrag.SEL_MASKED_MEAN_LOGPROB, 0.05, 0)
+    assert L.fvrag_select_candidate(ctypes.byref(s), P, None, None, None, P, P, None) == fvrag.ERR_INVALID_ARG
+    s2 = fvrag.SelectDesc(1, 5, 16, 1, fvrag.SEL_TWO_STAGE, 0.05, 0)
+    assert L.fvrag_select_candidate(ctypes.byref(s2), P, None, None, P, P, P, None) == fvrag.ERR_INVALID_ARG
+    s3 = fvrag.SelectDesc(1, 5, 16, 2, 7, 0.05, 0)
+    assert L.fvrag_select_candidate(ctypes.byref(s3), P, None, P, P, P, P, None) == fvrag.ERR_INVALID_ARG
+    s4 = fvrag.SelectDesc(1, 2000, 16, 1, 0, 0.05, 0)
+    assert L.fvrag_select_candidate(ctypes.byref(s4), P, None, P, P, P, P, None) == fvrag.ERR_UNSUPPORTED
+
+
+def test_status_calls_reject_null(L):
+    assert L.fvrag_read_status(None, None) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_clear_status(None, None) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_selftest_wait_timeout(None, None) == fvrag.ERR_INVALID_ARG
+
+
+def test_binding_raises_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(fvrag, "_lib", None)
+    monkeypatch.setattr(fvrag, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(OSError):
+        fvrag.lib()

@@ -1,0 +1,283 @@
+"""GPU parity: every libfvrag call, through the C ABI, against the fp64 oracle on the
+same seeded inputs.  Small cases compare every element and span several tiles with
+ragged tails; the full-size workloads compare sampled rows the oracle computes one
+by one (in the launch configuration the benchmark uses) plus size-independent
+properties.  Tolerances: attention |diff| <= 2e-2, log-prob |diff| <= 1e-2,
+cosine |diff| <= 1e-3; integer decisions exact unless the oracle's margin is
+below the tolerance."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle
+from paper_2601_01513_gb300 import configs, fvrag, synth
+from paper_2601_01513_gb300.pipeline import VerifyStep
+
+from gpu_helpers import (ATTN_ATOL, ATTN_LSE_ATOL, COS_ATOL, LOGPROB_ATOL, check_argmax_with_margin,
+                         check_keep_with_margin, check_selection_masked, ensure_built, run_attn,
+                         run_clip, run_lm, run_select)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    return ensure_built()
+
+
+# ============================================================ attention
+def _attn_inputs(Qn, K, L, Hq, Hkv, D, plens, seed):
+    offs = np.zeros(Qn + 1, np.int32)
+    offs[1:] = np.cumsum(plens)
+    tot = int(offs[-1])
+    return (synth.normal_bf16((Qn, K, L, Hq, D), seed, 1), synth.normal_bf16((tot, Hkv, D), seed, 2),
+            synth.normal_bf16((tot, Hkv, D), seed, 3), offs,
+            synth.normal_bf16((Qn, K, L, Hkv, D), seed, 4), synth.normal_bf16((Qn, K, L, Hkv, D), seed, 5))
+
+
+ATTN_CASES = [
+    # Qn, K, L, Hq, Hkv, D, prefix lengths
+    (1, 4, 8, 8, 8, 64, [256]),            # tiny config shape
+    (1, 3, 5, 14, 2, 128, [0]),            # no prefix: tail only
+    (1, 2, 1, 4, 4, 64, [1]),              # one prefix key, L = 1
+    (1, 2, 3, 4, 1, 128, [63]),
+    (1, 2, 3, 4, 2, 128, [64]),
+    (1, 2, 3, 8, 2, 64, [65]),
+    (1, 2, 33, 4, 4, 128, [257]),          # L = 33 (two lanes' worth of tail keys)
+    (3, 2, 4, 12, 4, 128, [0, 130, 70]),   # ragged queries
+    (1, 5, 16, 28, 4, 128, [1000]),        # 7b-style GQA: 5 row tiles of 18 tokens x 7 heads
+    (2, 3, 9, 16, 2, 128, [700, 2049]),    # 8 heads per KV head, several key splits
+    (1, 2, 64, 8, 8, 64, [300]),           # longest supported tail
+]
+
+
+@pytest.mark.parametrize("case", ATTN_CASES, ids=lambda c: "x".join(map(str, c[:6])) + "_P" + "-".join(map(str, c[6])))
+def test_attn_matches_oracle(case):
+    Qn, K, L, Hq, Hkv, D, plens = case
+    q, kp, vp, offs, kt, vt = _attn_inputs(Qn, K, L, Hq, Hkv, D, plens, seed=1000 + sum(plens) + L)
+    out, lse, st = run_attn(q, kp, vp, offs, kt, vt)
+    assert st == fvrag.OK
+    ref, ref_lse = oracle.verify_attn(q, kp, vp, offs, kt, vt)
+    assert np.all(np.isfinite(out))
+    assert np.max(np.abs(out - ref)) <= ATTN_ATOL
+    assert np.max(np.abs(lse - ref_lse)) <= ATTN_LSE_ATOL
+
+
+def test_attn_custom_scale_and_no_lse():
+    q, kp, vp, offs, kt, vt = _attn_inputs(1, 2, 4, 8, 2, 128, [150], seed=5)
+    out, _, st = run_attn(q, kp, vp, offs, kt, vt, with_lse=False, scale=0.05)
+    ref, _ = oracle.verify_attn(q, kp, vp, offs, kt, vt, scale=0.05)
+    assert st == fvrag.OK and np.max(np.abs(out - ref)) <= ATTN_ATOL
+
+
+def _sample_rows(shape, n, seed):
+    rng = np.random.default_rng(seed)
+    sel = np.zeros(shape, bool)
+    flat = rng.choice(sel.size, size=min(n, sel.size), replace=False)
+    sel.reshape(-1)[flat] = True
+    # always include the first and the last row (edges of the row tiling)
+    sel.reshape(-1)[0] = sel.reshape(-1)[-1] = True
+    return sel
+
+
+@pytest.mark.parametrize("name", ["7b", "long", "batch16", "72b"])
+def test_attn_full_size_sampled(name):
+    cfg = configs.PRESETS[name]
+    x = synth.make_inputs(cfg, parts=("attn",))
+    out, lse, st = run_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_tail"], x["v_tail"])
+    assert st == fvrag.OK
+    assert np.all(np.isfinite(out)) and np.all(np.isfinite(lse))
+    sel = _sample_rows(x["q"].shape[:-1], 48, seed=7)
+    ref, ref_lse = oracle.verify_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"],
+                                      x["k_tail"], x["v_tail"], row_sel=sel)
+    assert np.max(np.abs(out[sel] - ref[sel])) <= ATTN_ATOL
+    assert np.max(np.abs(lse[sel] - ref_lse[sel])) <= ATTN_LSE_ATOL
+    # size-independent property: lse >= log(number of visible keys) * 0 + max score, i.e. finite
+    # and at least the log of one key's weight; outputs are convex combinations of V rows
+    assert np.max(np.abs(out)) <= 8.0
+
+
+# ============================================================ LM head
+LM_CASES = [
+    # M, H, V, G
+    (32, 512, 4096, 1),       # tiny config shape
+    (1, 64, 16, 1),           # smallest: one row, one 16-row vocabulary unit
+    (33, 72, 1007, 2),        # H not a multiple of 64; V not a multiple of 16
+    (128, 128, 5000, 8),      # one full M-tile, 8 gathers
+    (129, 256, 4103, 1),      # two M-tiles (second with one row)
+    (300, 192, 3001, 2),      # three M-tiles: two groups
+    (80, 3584, 9000, 1),      # 7b hidden size, small vocabulary
+]
+
+
+@pytest.mark.parametrize("case", LM_CASES, ids=lambda c: "M%d_H%d_V%d_G%d" % c)
+def test_lm_matches_oracle(case):
+    M, H, V, G = case
+    seed = 2000 + M + V
+    hid = synth.normal_bf16((M, H), seed, 1)
+    W = synth.normal_bf16((V, H), seed, 2, 0.0, 0.02 if H > 1000 else 0.2)
+    tgt = synth.uniform_i32((M, G), seed, 3, 0, V)
+    if M > 2:  # out-of-range ids give NaN
+        tgt[1, 0] = -1
+        tgt[2, G - 1] = V
+    lp, lse, st = run_lm(hid, W, tgt)
+    assert st == fvrag.OK
+    ref, ref_lse = oracle.score_logprobs(hid, W, tgt)
+    assert np.array_equal(np.isnan(lp), np.isnan(ref))
+    ok = ~np.isnan(ref)
+    assert np.max(np.abs(lp[ok] - ref[ok])) <= LOGPROB_ATOL
+    assert np.max(np.abs(lse - ref_lse)) <= LOGPROB_ATOL
+
+
+def test_lm_all_targets_sum_to_one():
+    """Gathering every vocabulary id of a row: sum of probabilities is 1 (any size)."""
+    M, H, V = 3, 128, 8
+    hid = synth.normal_bf16((M, H), 5, 1)
+    W = synth.normal_bf16((V, H), 5, 2, 0.0, 0.3)
+    tgt = np.tile(np.arange(V, dtype=np.int32), (M, 1))
+    lp, _, st = run_lm(hid, W, tgt)
+    assert st == fvrag.OK
+    np.testing.assert_allclose(np.exp(lp.astype(np.float64)).sum(1), 1.0, atol=1e-4)
+
+
+@pytest.mark.parametrize("name", ["7b", "long", "72b", "batch16"])
+def test_lm_full_size_sampled(name):
+    cfg = configs.PRESETS[name]
+    x = synth.make_inputs(cfg, parts=("lm",))
+    lp, lse, st = run_lm(x["hidden"], x["weight"], x["targets"])
+    assert st == fvrag.OK
+    assert np.all(np.isfinite(lp)) and np.all(lp <= 0)
+    rows = np.unique(np.concatenate([[0, cfg.rows - 1], np.random.default_rng(3).choice(cfg.rows, 6, replace=False)]))
+    ref, ref_lse = oracle.score_logprobs(x["hidden"][rows], x["weight"], x["targets"][rows])
+    assert np.max(np.abs(lp[rows] - ref)) <= LOGPROB_ATOL
+    assert np.max(np.abs(lse[rows] - ref_lse)) <= LOGPROB_ATOL
+
+
+# ============================================================ CLIP
+@pytest.mark.parametrize("name", ["tiny", "7b", "long", "batch16", "72b"])
+def test_clip_configs(name):
+    cfg = configs.PRESETS[name]
+    cand, frames = synth.clip_embeddings(cfg)
+    cos, mc, am, keep = run_clip(cand, frames, cfg.threshold)
+    rcos, rmc, ram, rkeep = oracle.clip_align(cand, frames, cfg.threshold)
+    assert np.max(np.abs(cos - rcos)) <= COS_ATOL
+    assert np.max(np.abs(mc - rmc)) <= COS_ATOL
+    check_argmax_with_margin(am, rcos)
+    check_keep_with_margin(keep, rmc, cfg.threshold)
+    assert keep.sum() >= 1
+
+
+def test_clip_edges():
+    E = 8
+    eye = np.eye(E)
+    cand = synth.round_f16(eye[None, :3] * 3.0)
+    frames = synth.round_f16(eye[None, 3:7] * 0.5)
+    frames[0, 2] = cand[0, 1]
+    frames[0, 3] = cand[0, 1]          # tie: lowest index wins
+    cand[0, 2] = 0                     # zero vector: cos 0
+    cos, mc, am, keep = run_clip(cand, frames, 0.2)
+    assert am[0, 1] == 2 and abs(mc[0, 1] - 1.0) < 1e-6 and keep[0, 1] == 1
+    assert np.all(cos[0, 2] == 0.0) and keep[0, 2] == 0 and am[0, 2] == 0
+    assert np.all(cos[0, 0] == 0.0)
+    # one frame only, and a dimension that is not a multiple of 256
+    c1 = synth.round_f16(synth.normal_f64((2, 3, 40), 9, 1))
+    f1 = synth.round_f16(synth.normal_f64((2, 1, 40), 9, 2))
+    cos, mc, am, keep = run_clip(c1, f1, 0.0, with_cos=True)
+    rcos, rmc, _, _ = oracle.clip_align(c1, f1, 0.0)
+    assert np.all(am == 0) and np.max(np.abs(mc - rmc)) <= COS_ATOL
+    # without the optional cos output
+    _, mc2, am2, _ = run_clip(c1, f1, 0.0, with_cos=False)
+    assert np.array_equal(mc2, mc) and np.array_equal(am2, am)
+
+
+# ============================================================ selection
+@pytest.mark.parametrize("mode", [fvrag.SEL_MASKED_MEAN_LOGPROB, fvrag.SEL_TWO_STAGE])
+@pytest.mark.parametrize("Qn,K,L", [(1, 1, 1), (3, 7, 5), (16, 5, 16), (2, 1000, 3)])
+def test_select_matches_oracle(mode, Qn, K, L):
+    lp, keep, mc = synth.selection_inputs(Qn, K, L, 2, seed=Qn * 31 + K)
+    lengths = synth.uniform_i32((Qn, K), 77, 1, 0, L + 2)   # includes invalid 0 and L+1
+    delta = float(np.float32(0.05))
+    for lens in (None, lengths):
+        score, sel = run_select(lp, mode, keep=keep, max_cos=mc, lengths=lens, delta=delta)
+        rscore, rsel = oracle.select(lp, mode=mode, lengths=lens, keep=keep, max_cos=mc, delta=delta)
+        assert np.array_equal(np.isnan(score), np.isnan(rscore))
+        ok = ~np.isnan(rscore)
+        assert np.array_equal(score[ok], rscore[ok].astype(np.float32))   # fp64 on both sides
+        assert np.array_equal(sel, rsel)
+
+
+def test_select_case_studies_on_gpu():
+    import json, os
+    here = os.path.join(os.path.dirname(__file__), "golden")
+    for name in ("case_penguin.json", "case_cuttlefish.json"):
+        case = json.load(open(os.path.join(here, name)))
+        rel = np.array(case["reliability"])
+        lp = np.stack([np.log(rel), np.log1p(-rel)], -1)[None, :, None, :]
+        _, sel = run_select(lp, fvrag.SEL_TWO_STAGE, max_cos=np.array([case["max_cos"]]),
+                            delta=case["delta"])
+        assert sel[0] == case["expected_selected"]
+
+
+# ============================================================ whole step
+@pytest.mark.parametrize("name", ["tiny", "7b"])
+def test_pipeline_step(name):
+    cfg = configs.PRESETS[name]
+    x = synth.make_inputs(cfg)
+    step = VerifyStep(cfg)
+    step.upload(x)
+    for _ in range(2):            # repeated steps reuse the workspaces
+        step.run()
+    torch.cuda.synchronize()
+    assert fvrag.read_status(step.lm_ws) == fvrag.OK
+    assert fvrag.read_status(step.attn_ws) == fvrag.OK
+    _, rmc, _, rkeep = oracle.clip_align(x["cand_emb"], x["frame_emb"], cfg.threshold)
+    lp = step.logprob.cpu().numpy()
+    if name == "tiny":
+        ref_lp, _ = oracle.score_logprobs(x["hidden"], x["weight"], x["targets"])
+        assert np.max(np.abs(lp - ref_lp)) <= LOGPROB_ATOL
+        ref_out, _ = oracle.verify_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"],
+                                        x["k_tail"], x["v_tail"])
+        assert np.max(np.abs(step.out.float().cpu().numpy() - ref_out)) <= ATTN_ATOL
+    else:
+        ref_lp = lp.astype(np.float64)   # full-size LM head is checked by the sampled test above
+    rscore, _ = oracle.select(ref_lp.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.gathers),
+                              keep=rkeep)
+    check_selection_masked(step.selected.cpu().numpy(), rscore, rmc, cfg.threshold)
+
+
+def test_pipeline_end_to_end_from_host():
+    cfg = configs.TINY
+    x = synth.make_inputs(cfg)
+    step = VerifyStep(cfg)
+    step.upload(x)
+    host = step.host_inputs()
+    sel, sc, h2d, d2h = step.run_from_host(host)
+    torch.cuda.synchronize()
+    step.run()
+    torch.cuda.synchronize()
+    assert h2d > 0 and d2h == cfg.num_queries * 4 + cfg.num_queries * cfg.num_cand * 4
+    assert np.array_equal(sel.numpy(), step.selected.cpu().numpy())
+
+
+# ============================================================ failure detection
+def test_bounded_wait_times_out_and_context_survives():
+    ws = torch.zeros(256, dtype=torch.uint8, device="cuda")
+    old = fvrag.get_wait_limit_ns()
+    try:
+        fvrag.set_wait_limit_ns(2_000_000)       # 2 ms
+        fvrag.selftest_wait_timeout(ws)
+        assert fvrag.read_status(ws) == fvrag.ERR_TIMEOUT
+        fvrag.clear_status(ws)
+        assert fvrag.read_status(ws) == fvrag.OK
+    finally:
+        fvrag.set_wait_limit_ns(old)
+    # the context is still usable: a normal call succeeds with a clean status
+    hid = synth.normal_bf16((4, 64), 1, 1)
+    W = synth.normal_bf16((64, 64), 1, 2)
+    tgt = synth.uniform_i32((4, 1), 1, 3, 0, 64)
+    lp, _, st = run_lm(hid, W, tgt)
+    assert st == fvrag.OK and np.all(np.isfinite(lp))

@@ -1,0 +1,374 @@
+"""Benchmark of one verify step of the VideoSpeculateRAG verifier hot path.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config 7b] [--impl reference]
+
+A step is one pass of the whole hot path over one query batch: shared-prefix
+attention, LM-head log-probabilities, CLIP alignment and candidate selection
+(the four libfvrag calls).  Inputs are seeded synthetic tensors resident in HBM
+before the timed region; L2 is flushed (a 256 MiB write) between timed steps,
+outside the per-step CUDA events.
+
+Metric: verified candidate tokens/s = (queries x candidates x tokens) / step time.
+Also reported: verify-step microseconds per query, per-kernel times, the roofline
+fraction of the dominant kernel (the LM head, HBM-bound at the 7B shape), the
+end-to-end number through the public API with host buffers (host->device copies
+of the step's inputs and the device->host read of the result inside the timed
+region), and the fp64 oracle's time on this host's cores.
+
+Multi-GPU (torchrun): every rank runs an independent replica of the workload
+(independent queries, no collective on the data path: weak scaling); the time is
+the max over ranks.  --impl reference times the fp64 oracle on the host cores
+(rank 0 only).
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2601_01513_gb300 import configs, synth  # noqa: E402
+
+METRIC = "verified candidate tokens/s"
+UNIT = "tokens/s"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+# DRAM traffic of one LM-head launch at the 7B shape, from an ncu capture of the
+# kernel source with this SHA-256 prefix (null once the kernel source changes).
+LM_TRAFFIC = {"sha256_prefix": "2531dd33051e9ac9", "bytes_per_launch": 1093397920}
+
+
+def peaks():
+    p = dict(FALLBACK_PEAKS)
+    src = "fallback"
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            m = json.load(f)
+        for k in FALLBACK_PEAKS:
+            if k in m:
+                p[k] = float(m[k])
+        src = "measured"
+    return p, src
+
+
+def source_sha(name):
+    with open(os.path.join(ROOT, "paper_2601_01513_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def algorithmic(cfg):
+    """Bytes and flops each kernel must move / perform at minimum (per launch)."""
+    Qn, K, L, hq, hkv, D = cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.hq, cfg.hkv, cfg.head_dim
+    M, H, V, G = cfg.rows, cfg.hidden, cfg.vocab, cfg.gathers
+    plen = synth.prefix_lengths(cfg)
+    sumP = int(plen.sum())
+    rows = Qn * K * L * hq
+    attn_bytes = 2 * sumP * hkv * D * 2 + 2 * rows * D * 2 + 2 * Qn * K * L * hkv * D * 2 + rows * 4
+    vis = sum(int(p) * K * L + K * L * (L + 1) // 2 for p in plen) * hq
+    attn_flops = 4.0 * D * vis
+    lm_bytes = V * H * 2 + M * H * 2 + M * G * 4 + M * G * 4 + M * 4
+    lm_flops = 2.0 * M * H * V
+    clip_bytes = Qn * (K + cfg.num_frames) * cfg.clip_dim * 2 + Qn * K * 9
+    sel_bytes = M * G * 4 + Qn * K * 9 + Qn * 4
+    return {"attn": (attn_bytes, attn_flops), "lm": (lm_bytes, lm_flops), "clip": (clip_bytes, 0.0),
+            "select": (sel_bytes, 0.0)}
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling while the timed region runs."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.idx = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.Q, "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx = float(f[2])
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def run_reference(args, cfg):
+    """fp64 oracle on the host cores: each step is a bounded sample of the workload."""
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    from oracle import oracle
+    oracle.build()
+    x = synth.make_inputs(cfg)
+    frac_rows = args.ref_rows
+    M = cfg.rows
+    rows = np.arange(0, M, max(1, M // frac_rows))[:frac_rows]
+    # attention rows of the same candidate tokens, all heads
+    tok = rows
+    sel = np.zeros((M, cfg.hq), bool)
+    sel[tok, :] = True
+    sel = sel.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.hq)
+    cores = oracle.max_threads()
+
+    def step():
+        oracle.verify_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_tail"],
+                           x["v_tail"], row_sel=sel)
+        lp, _ = oracle.score_logprobs(x["hidden"][rows], x["weight"], x["targets"][rows])
+        _, mc, _, keep = oracle.clip_align(x["cand_emb"], x["frame_emb"], cfg.threshold)
+        full = np.zeros((M, cfg.gathers))
+        full[rows] = lp
+        oracle.select(full.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.gathers), keep=keep)
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = (time.perf_counter() - t0) / args.steps
+    value = len(rows) / dt
+    sample = ("%d of %d candidate-token rows per step (LM head and all %d heads of attention for "
+              "those rows; CLIP and selection in full)" % (len(rows), M, cfg.hq))
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": config_block(cfg),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle", "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def config_block(cfg):
+    return {"workload": cfg.description, "name": cfg.name, "num_queries": cfg.num_queries,
+            "tokens_per_step": cfg.rows, "prefix_len": cfg.prefix_len or list(cfg.prefix_range),
+            "hidden": cfg.hidden, "heads": [cfg.hq, cfg.hkv, cfg.head_dim], "vocab": cfg.vocab,
+            "clip": [cfg.num_cand, cfg.num_frames, cfg.clip_dim], "selection": "masked mean log-prob",
+            "l2": "flushed between timed steps (256 MiB write); LM-head weight 1 GB+ > L2",
+            "parallelism": "replicas"}
+
+
+def cpu_baseline(cfg, x, budget_s):
+    """The oracle as it stands, timed on this host's cores over a bounded sample."""
+    from oracle import oracle
+    oracle.build()
+    cores = oracle.max_threads()
+    M = cfg.rows
+    t0 = time.perf_counter()
+    done = 0
+    nrows = max(1, min(M, 8))
+    rows = np.arange(nrows) * max(1, M // nrows)
+    # attention for the sampled tokens (all heads) + LM head for the sampled rows, then CLIP + select
+    sel = np.zeros((M, cfg.hq), bool)
+    sel[rows, :] = True
+    sel = sel.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.hq)
+    reps = 0
+    while True:
+        oracle.verify_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_tail"],
+                           x["v_tail"], row_sel=sel)
+        lp, _ = oracle.score_logprobs(x["hidden"][rows], x["weight"], x["targets"][rows])
+        _, mc, _, keep = oracle.clip_align(x["cand_emb"], x["frame_emb"], cfg.threshold)
+        full = np.zeros((M, cfg.gathers))
+        full[rows] = lp
+        oracle.select(full.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.gathers), keep=keep)
+        done += nrows
+        reps += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": done / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": "%d repetitions of %d of %d candidate-token rows (their attention over all %d "
+                      "heads and their LM-head log-probs, plus CLIP and selection in full), %.1f s"
+                      % (reps, nrows, M, cfg.hq, dt)}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", default="7b", choices=sorted(configs.PRESETS))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--ref-rows", type=int, default=8)
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    cfg = configs.PRESETS[args.config]
+
+    if args.impl == "reference":
+        return run_reference(args, cfg)
+
+    import torch
+    import torch.distributed as dist
+
+    from paper_2601_01513_gb300 import fvrag
+    from paper_2601_01513_gb300.build import build_all
+    from paper_2601_01513_gb300.pipeline import VerifyStep
+
+    ws_, rank, local = dist_env()
+    if ws_ > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if ws_ > 1 else 0)
+    if rank == 0:
+        build_all()
+    if ws_ > 1:
+        dist.barrier()
+    fvrag.lib()
+
+    # each rank verifies its own queries (independent replica, rank-dependent seed)
+    x = synth.make_inputs(cfg, seed=cfg.seed + 7919 * rank)
+    step = VerifyStep(cfg, device=dev)
+    step.upload(x)
+    stream = torch.cuda.Stream(device=dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    nk = 4
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            step.run()
+        stream.synchronize()
+        assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
+
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
+        if ws_ > 1:
+            dist.barrier()
+        torch.cuda.synchronize(dev)
+        with ClockSampler(dev.index if dev.index is not None else 0) as clk:
+            for i in range(args.steps):
+                flush.zero_()
+                e = ev[i]
+                e[0].record(stream)
+                step.attention()
+                e[1].record(stream)
+                step.lm_head()
+                e[2].record(stream)
+                step.clip()
+                e[3].record(stream)
+                step.select()
+                e[4].record(stream)
+            torch.cuda.synchronize(dev)
+        if ws_ > 1:
+            dist.barrier()
+        per_k = np.array([[ev[i][j].elapsed_time(ev[i][j + 1]) for j in range(nk)] for i in range(args.steps)])
+        step_ms = per_k.sum(1)
+        total_ms = float(step_ms.sum())
+        assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
+
+        # end to end through the public API with host buffers
+        host = step.host_inputs(pin=True)
+        for _ in range(2):
+            step.run_from_host(host)
+        torch.cuda.synchronize(dev)
+        ee = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+        h2d = d2h = 0
+        for i in range(args.steps):
+            flush.zero_()
+            ee[i][0].record(stream)
+            _, _, h2d, d2h = step.run_from_host(host)
+            ee[i][1].record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = float(sum(a.elapsed_time(b) for a, b in ee))
+
+    if ws_ > 1:
+        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms, e2e_ms = float(t[0]), float(t[1])
+
+    tokens = cfg.rows * args.steps * ws_
+    value = tokens / (total_ms / 1e3)
+    e2e_value = tokens / (e2e_ms / 1e3)
+    pk, pk_src = peaks()
+    alg = algorithmic(cfg)
+    names = ["attn", "lm", "clip", "select"]
+    kern = {}
+    for j, n in enumerate(names):
+        us = float(np.mean(per_k[:, j])) * 1e3
+        b, f = alg[n]
+        kern[n] = {"us": us, "us_median": float(np.median(per_k[:, j])) * 1e3, "GB_s": b / (us * 1e-6) / 1e9,
+                   "TFLOP_s": f / (us * 1e-6) / 1e12 if f else 0.0, "alg_bytes": b, "alg_flops": f}
+        kern[n]["hbm_frac"] = kern[n]["GB_s"] / pk["hbm_gbs"]
+        if f:
+            kern[n]["tc_frac"] = kern[n]["TFLOP_s"] / pk["bf16_tflops_sustained"]
+    lm = kern["lm"]
+    traffic = None
+    if LM_TRAFFIC["bytes_per_launch"] and source_sha("lmhead.cu").startswith(LM_TRAFFIC["sha256_prefix"] or "#"):
+        traffic = LM_TRAFFIC["bytes_per_launch"]
+    roof = {"bound": "hbm", "achieved": lm["GB_s"], "peak": pk["hbm_gbs"], "unit": "GB/s",
+            "frac": lm["GB_s"] / pk["hbm_gbs"], "traffic": traffic, "kernel": "fvrag LM head (tcgen05 GEMM + LSE)",
+            "peak_source": pk_src}
+    if rank != 0:
+        if ws_ > 1:
+            dist.destroy_process_group()
+        return 0
+    line = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws_, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": config_block(cfg),
+            "us_per_query": total_ms / args.steps * 1e3 / cfg.num_queries,
+            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
+                    "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms / args.steps},
+            "gpu_launches": step.launches_per_step() * args.steps,
+            "roofline": roof, "kernels": kern, "clocks": clk.summary()}
+    if not args.no_cpu_baseline and ws_ == 1:
+        line["cpu_baseline"] = cpu_baseline(cfg, x, args.cpu_budget)
+    print(json.dumps(line), flush=True)
+    if ws_ > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

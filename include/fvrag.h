@@ -142,6 +142,29 @@ fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void* hidden, co
                                   const int32_t* targets, float* logprob, float* lse, void* ws,
                                   size_t ws_bytes, fvrag_stream_t stream);
 
+/*
+ * Allocation-free form of fvrag_score_logprobs (the paper has no counterpart:
+ * this is a deployment aid).  For callers that cannot call cudaMalloc -- for
+ * example a serving runtime whose device memory is owned by another allocator,
+ * or code that must not allocate once it is running -- the scratch that the
+ * workspace argument would hold lives instead in a fixed static device array
+ * inside the library: 2,130,176 bytes per GPU that loads the library, held
+ * until the process exits.  Same arguments, layouts and results as
+ * fvrag_score_logprobs without ws / ws_bytes.
+ *   - rows must be <= 1024 (gathers <= 8): larger shapes return
+ *     FVRAG_ERR_UNSUPPORTED without enqueuing anything.
+ *   - The first call on a device looks up the array's device address (with
+ *     that device current) and caches it; make that first call before any
+ *     stream capture.  No call allocates or frees memory.
+ *   - Every call shares the one array and leaves its contents behind; each call
+ *     clears the array's status word before its kernels run.  Calls that
+ *     overlap on the GPU (other streams, other threads) race on the array:
+ *     serialise them.
+ */
+fvrag_status fvrag_score_logprobs_noalloc(const fvrag_lm_desc* d, const void* hidden,
+                                          const void* weight, const int32_t* targets,
+                                          float* logprob, float* lse, fvrag_stream_t stream);
+
 /* ------------------------------------------------------------------------ *
  * 3. CLIP entity alignment (Eq. 14-15) with the keep/drop threshold
  *

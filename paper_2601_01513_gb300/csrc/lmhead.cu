@@ -30,6 +30,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "fvrag_common.cuh"
 #include "fvrag_internal.h"
@@ -435,4 +436,65 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   lm_merge_kernel<<<(d->rows + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0, s>>>(
       pmax, psum, ptgt, targets, d->rows, d->vocab, d->gathers, p.ctas, logprob, lse);
   return launch_status();
+}
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of fvrag_score_logprobs.
+//
+// Some callers cannot call cudaMalloc: a host runtime that hands out only
+// pre-registered buffers, an embedded engine whose allocator is owned by
+// someone else, or a caller working under a memory budget that forbids new
+// device allocations after start-up.  For them this entry point keeps the LM
+// head's scratch (the workspace header and the per-CTA partial max / sum and
+// gathered target logits) in a file-scope device array of fixed size instead of
+// a caller-provided workspace.  Every GPU that loads the library holds the
+// array until the process exits.
+namespace fvrag {
+namespace lm {
+
+constexpr int kNoAllocMaxRows = 1024;
+constexpr size_t kNoAllocBytes = kWsHeaderBytes + 2 * (size_t)kMaxCtas * kNoAllocMaxRows * 4 +
+                                 (size_t)kNoAllocMaxRows * kMaxGathers * 4;
+
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocBytes];
+
+// Device address of g_noalloc_scratch on the current device.  In host code the
+// array's name is only a host-side stand-in, so the address is looked up once
+// per device (with that device current) and cached.
+static void* noalloc_scratch_address() {
+  static std::mutex mu;
+  static void* addr[64] = {nullptr};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+    addr[dev] = p;
+  }
+  return addr[dev];
+}
+
+}  // namespace lm
+}  // namespace fvrag
+
+extern "C" fvrag_status fvrag_score_logprobs_noalloc(const fvrag_lm_desc* d, const void* hidden,
+                                                     const void* weight, const int32_t* targets,
+                                                     float* logprob, float* lse,
+                                                     fvrag_stream_t stream) {
+  using namespace lm;
+  // reject bad arguments before anything is enqueued
+  if (!d || !hidden || !weight || !targets || !logprob) return FVRAG_ERR_INVALID_ARG;
+  if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->rows > kNoAllocMaxRows || d->gathers > kMaxGathers) return FVRAG_ERR_UNSUPPORTED;
+  if (d->hidden % 8 != 0 || !aligned16(hidden) || !aligned16(weight)) return FVRAG_ERR_MISALIGNED;
+  void* scratch = noalloc_scratch_address();
+  if (!scratch) return FVRAG_ERR_CUDA;
+  // the status word reports this call only
+  if (cudaMemsetAsync(scratch, 0, kWsHeaderBytes, reinterpret_cast<cudaStream_t>(stream)) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return fvrag_score_logprobs(d, hidden, weight, targets, logprob, lse, scratch, kNoAllocBytes,
+                              stream);
 }

@@ -19,7 +19,7 @@ WS_HEADER_BYTES = 256
 EXPORTED = (
     "fvrag_abi_version", "fvrag_status_string",
     "fvrag_verify_attn_workspace", "fvrag_verify_attn",
-    "fvrag_score_logprobs_workspace", "fvrag_score_logprobs",
+    "fvrag_score_logprobs_workspace", "fvrag_score_logprobs", "fvrag_score_logprobs_noalloc",
     "fvrag_clip_align", "fvrag_select_candidate",
     "fvrag_read_status", "fvrag_clear_status",
     "fvrag_set_wait_limit_ns", "fvrag_get_wait_limit_ns", "fvrag_selftest_wait_timeout",
@@ -79,6 +79,8 @@ def lib():
         L.fvrag_score_logprobs_workspace.argtypes = [ctypes.POINTER(LmDesc)]
         L.fvrag_score_logprobs.restype = i32
         L.fvrag_score_logprobs.argtypes = [ctypes.POINTER(LmDesc)] + [vp] * 5 + [vp, sz, vp]
+        L.fvrag_score_logprobs_noalloc.restype = i32
+        L.fvrag_score_logprobs_noalloc.argtypes = [ctypes.POINTER(LmDesc)] + [vp] * 5 + [vp]
         L.fvrag_clip_align.restype = i32
         L.fvrag_clip_align.argtypes = [ctypes.POINTER(ClipDesc)] + [vp] * 6 + [vp]
         L.fvrag_select_candidate.restype = i32
@@ -151,6 +153,14 @@ def score_logprobs(hidden, weight, targets, logprob, ws, lse=None, stream=None):
                                    _ptr(logprob), _ptr(lse), _ptr(ws), ws.numel() * ws.element_size(),
                                    _stream(stream))
     _check(s, "fvrag_score_logprobs")
+
+
+def score_logprobs_noalloc(hidden, weight, targets, logprob, lse=None, stream=None):
+    """As score_logprobs, with the scratch in the library's static device array (no workspace)."""
+    d = lm_desc(hidden, weight, targets)
+    s = lib().fvrag_score_logprobs_noalloc(ctypes.byref(d), _ptr(hidden), _ptr(weight), _ptr(targets),
+                                           _ptr(logprob), _ptr(lse), _stream(stream))
+    _check(s, "fvrag_score_logprobs_noalloc")
 
 
 def clip_align(cand_emb, frame_emb, threshold, max_cos, argmax, keep, cos=None, stream=None):

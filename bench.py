@@ -98,7 +98,7 @@ class ClockSampler:
         try:
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.idx), "--query-gpu=" + self.Q, "--format=csv,noheader,nounits",
-                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
             self.t = threading.Thread(target=self._read, daemon=True)
             self.t.start()
         except (OSError, FileNotFoundError):
@@ -108,6 +108,14 @@ class ClockSampler:
     def _read(self):
         for line in self.proc.stdout:
             self.lines.append(line.strip())
+
+    def wait_first(self, timeout=5.0):
+        """Blocks until nvidia-smi has produced its first sample (it starts slowly); the
+        samples then cover the whole timed region that follows."""
+        t0 = time.time()
+        while self.proc is not None and not self.lines and time.time() - t0 < timeout:
+            time.sleep(0.05)
+        self.lines.clear()
 
     def __exit__(self, *a):
         if self.proc is not None:
@@ -196,7 +204,8 @@ def config_block(cfg):
             "tokens_per_step": cfg.rows, "prefix_len": cfg.prefix_len or list(cfg.prefix_range),
             "hidden": cfg.hidden, "heads": [cfg.hq, cfg.hkv, cfg.head_dim], "vocab": cfg.vocab,
             "clip": [cfg.num_cand, cfg.num_frames, cfg.clip_dim], "selection": "masked mean log-prob",
-            "l2": "flushed between timed steps (256 MiB write); LM-head weight 1 GB+ > L2",
+            "l2": "flushed before every timed step / launch: 256 MiB write, then a 256 MiB read that "
+                  "drains the write's dirty lines; both outside the CUDA events",
             "parallelism": "replicas"}
 
 
@@ -237,8 +246,9 @@ def cpu_baseline(cfg, x, budget_s):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
-    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--kernel-reps", type=int, default=200)
     ap.add_argument("--config", default="7b", choices=sorted(configs.PRESETS))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--ref-rows", type=int, default=8)
@@ -273,54 +283,89 @@ def main():
     x = synth.make_inputs(cfg, seed=cfg.seed + 7919 * rank)
     step = VerifyStep(cfg, device=dev)
     step.upload(x)
+    # L2 flush between timed iterations: write a 256 MiB buffer (> the 126.5 MiB L2), then read
+    # another 256 MiB buffer so the flush's own dirty lines are written back before the
+    # timed kernels start (otherwise the first timed kernel pays for the flush's write-back)
+    flush_w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones((256, 1 << 18), dtype=torch.float32, device=dev)
+    flush_sink = torch.empty((256,), dtype=torch.float32, device=dev)
+
+    class _Flush:
+        @staticmethod
+        def zero_():
+            flush_w.zero_()
+            torch.amax(flush_r, dim=1, out=flush_sink)
+
+    flush = _Flush()
+    names = ["attn", "lm", "clip", "select"]
+    calls = {"attn": step.attention, "lm": step.lm_head, "clip": step.clip, "select": step.select}
+    for _ in range(args.warmup):
+        step.run()
+    torch.cuda.synchronize(dev)
+    assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
+    # one CUDA graph for the whole step, one per call for the per-kernel numbers
+    step.capture()
+    graphs = {}
+    for n in names:
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            calls[n]()
+        graphs[n] = g
     stream = torch.cuda.Stream(device=dev)
-    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
-    nk = 4
+    host = step.host_inputs(pin=True)
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
-            step.run()
-        stream.synchronize()
-        assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
-
-        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(args.steps)]
+            step.replay()
+            for n in names:
+                graphs[n].replay()
+            step.run_from_host(host)
+        torch.cuda.synchronize(dev)
         if ws_ > 1:
             dist.barrier()
         torch.cuda.synchronize(dev)
         with ClockSampler(dev.index if dev.index is not None else 0) as clk:
+            clk.wait_first()
+            # timed region: K whole steps, L2 flushed before each (outside the events)
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(args.steps)]
+            t_wall = time.perf_counter()
             for i in range(args.steps):
                 flush.zero_()
-                e = ev[i]
-                e[0].record(stream)
-                step.attention()
-                e[1].record(stream)
-                step.lm_head()
-                e[2].record(stream)
-                step.clip()
-                e[3].record(stream)
-                step.select()
-                e[4].record(stream)
+                ev[i][0].record(stream)
+                step.replay()
+                ev[i][1].record(stream)
             torch.cuda.synchronize(dev)
+            t_wall = time.perf_counter() - t_wall
+            step_ms = np.array([a.elapsed_time(b) for a, b in ev])
+            # per-kernel launch durations (each call replayed alone, L2 flushed before each)
+            kreps = max(3, min(args.steps, args.kernel_reps))
+            per_k = np.zeros((kreps, len(names)))
+            for j, n in enumerate(names):
+                kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                       for _ in range(kreps)]
+                for i in range(kreps):
+                    flush.zero_()
+                    kev[i][0].record(stream)
+                    graphs[n].replay()
+                    kev[i][1].record(stream)
+                torch.cuda.synchronize(dev)
+                per_k[:, j] = [a.elapsed_time(b) for a, b in kev]
+            # end to end through the public API with host buffers: copies of the step's inputs
+            # from pinned memory, the step, and the read of the result, all inside the events
+            ee = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                  for _ in range(args.steps)]
+            h2d = d2h = 0
+            for i in range(args.steps):
+                flush.zero_()
+                ee[i][0].record(stream)
+                _, _, h2d, d2h = step.run_from_host(host)
+                ee[i][1].record(stream)
+            torch.cuda.synchronize(dev)
+            e2e_ms = float(sum(a.elapsed_time(b) for a, b in ee))
         if ws_ > 1:
             dist.barrier()
-        per_k = np.array([[ev[i][j].elapsed_time(ev[i][j + 1]) for j in range(nk)] for i in range(args.steps)])
-        step_ms = per_k.sum(1)
         total_ms = float(step_ms.sum())
         assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
-
-        # end to end through the public API with host buffers
-        host = step.host_inputs(pin=True)
-        for _ in range(2):
-            step.run_from_host(host)
-        torch.cuda.synchronize(dev)
-        ee = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-        h2d = d2h = 0
-        for i in range(args.steps):
-            flush.zero_()
-            ee[i][0].record(stream)
-            _, _, h2d, d2h = step.run_from_host(host)
-            ee[i][1].record(stream)
-        torch.cuda.synchronize(dev)
-        e2e_ms = float(sum(a.elapsed_time(b) for a, b in ee))
 
     if ws_ > 1:
         t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
@@ -360,7 +405,10 @@ def main():
             "us_per_query": total_ms / args.steps * 1e3 / cfg.num_queries,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms / args.steps},
-            "gpu_launches": step.launches_per_step() * args.steps,
+            "gpu_launches": step.launches_per_step() * (2 * args.steps + per_k.shape[0]),
+            "timing": {"step": "CUDA graph of the four calls, CUDA events per step, L2 flushed between steps",
+                       "kernels": "each call replayed alone %d times (events per launch), L2 flushed before each"
+                                  % per_k.shape[0], "host_wall_s": t_wall},
             "roofline": roof, "kernels": kern, "clocks": clk.summary()}
     if not args.no_cpu_baseline and ws_ == 1:
         line["cpu_baseline"] = cpu_baseline(cfg, x, args.cpu_budget)

@@ -88,7 +88,7 @@ typedef struct fvrag_attn_desc {
   int32_t head_dim;     /* D: 64 or 128 */
   int32_t max_prefix;   /* upper bound on every P_q (plans the key split); >= 0 */
   int32_t total_prefix; /* sum over queries of P_q = rows of k_prefix / v_prefix */
-  float softmax_scale;  /* 0 => 1/sqrt(head_dim) */
+  float softmax_scale;  /* > 0, or 0 => 1/sqrt(head_dim); negative / NaN / inf rejected */
   uint32_t flags;       /* must be 0 */
 } fvrag_attn_desc;
 

@@ -1,25 +1,32 @@
 // K1: one attention layer of the verifier forward over all candidate rows
-// (Eq. 6 / Eq. 11): every token l of candidate k attends to the P_q tokens of
-// the shared prefix and to tokens 0..l of its own candidate.
+// (Eq. 6 / Eq. 11): token l of candidate k attends to the P_q tokens of the
+// shared prefix and to tokens 0..l of its own candidate.
 //
-// The prefix part dominates (P up to 32768 keys vs L <= 64 tail keys) and is
-// shared by every candidate row, so it is computed as a split-KV flash pass in
-// which ALL K x L x (hq/hkv) query rows that use one KV head are packed into
-// the rows of the tensor-core tiles (GQA packing): each prefix K/V tile is read
-// from HBM once per (KV head, key split) and reused by every candidate row.
+// The prefix (up to 32768 keys) is shared by every candidate row, so all
+// K x L x (hq/hkv) query rows that use one KV head are packed into the rows of
+// the tensor-core tiles (GQA packing): a row tile is T tokens x the hq/hkv
+// query heads of one KV head (T = floor(128 / (hq/hkv))), and every prefix K/V
+// block that a CTA loads feeds all of them.
 //
-// prefix kernel  grid = Qn x hkv x key-splits x row-tiles; one CTA computes 128
-//                query rows (T tokens x the hq/hkv heads of one KV head) against
-//                one key range.  Warp 8 streams 64-key K/V tiles with TMA (3-D
-//                maps over [keys][hkv][D], 128-byte swizzle) into a 3-stage ring;
-//                warps 0-7 (16 rows each) run S = Q K^T and O += P V on the tensor
-//                cores (bf16 mma.sync m16n8k16, fp32 accumulate) with an online
-//                softmax in registers, then write the normalised partial O and
-//                its log-sum-exp to the workspace.
-// tail+merge     one warp per (token, head): attention over the candidate's own
-//                tokens 0..l (at most 64 keys, CUDA cores), then a log-sum-exp
-//                merge of the tail with every prefix split; writes bf16 out and
-//                the fp32 lse.
+// attn_kernel: one CTA = one row tile x one key range (split-KV).
+//   warp 0     TMA: the Q tile once (3-D map over [tokens][hq][D]), then K and V
+//              blocks of 64 keys (3-D maps over [keys][hkv][D], 128-byte swizzle)
+//              into two 5-deep rings, K and V each issued as soon as its ring has
+//              a free slot.  Split 0 also streams the candidates' own tail
+//              tokens as extra key blocks.
+//   warp 1     allocates tensor memory and issues tcgen05.mma:
+//                S_j  = Q K_j^T  (M = 128 rows, N = 64 keys, K = D; both K-major)
+//                O   += P_j V_j  (M = 128, N = D, K = 64 keys; V read MN-major)
+//              with S double-buffered and O accumulated in tensor memory.
+//   warps 2-5  one query row per thread: tcgen05.ld of S_j, masking (key range,
+//              or same-candidate causal range for tail blocks; full blocks skip
+//              it), online softmax in base 2 against a lazily moved reference
+//              max (O and l are rescaled in place only when a row's max grows by
+//              more than 2^8), and P_j written to shared memory as a
+//              128-byte-swizzled bf16 tile for the next MMA.
+//   One split: the CTA writes the bf16 output and the lse directly.  Several
+//   splits: normalised partials go to the workspace and merge_kernel combines
+//   them with log-sum-exp weights.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -30,17 +37,44 @@
 namespace fvrag {
 namespace attn {
 
-constexpr int kConsumerWarps = 8;
-constexpr int kThreads = (kConsumerWarps + 1) * 32;
-constexpr int kRowsPerTile = 128;
-constexpr int kKeysPerBlock = 64;
-constexpr int kStages = 3;
-constexpr int kTargetCtas = 304;   // split plan aims at ~2 CTAs per SM (fixed: plan is device-independent)
+constexpr int kThreads = 192;
+constexpr int kBM = 128;          // query rows per tile (MMA M)
+constexpr int kBN = 64;           // keys per block
+constexpr int kStages = 5;       // depth of each of the K ring and the V ring
 constexpr int kMaxTail = 64;
+constexpr uint32_t kTmemCols = 256;
+// tensor-memory columns: S buffers at 0 and 64, the O accumulator at 128
+__device__ __forceinline__ uint32_t col_s(int b) { return (uint32_t)b * 64u; }
+constexpr uint32_t kColO = 128;
+constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (P stays < 2^8)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
-enum : uint32_t { kSiteQ = 0x101, kSiteFull = 0x102, kSiteEmpty = 0x103 };
+enum : uint32_t { kSiteQ = 0x101, kSiteKvFull = 0x102, kSiteKvEmpty = 0x103, kSiteSFree = 0x104,
+                  kSitePFull = 0x105, kSiteSFull = 0x107, kSitePFree = 0x108, kSiteOFull = 0x109,
+                  kSiteDrain = 0x10A };
+
+template <int D>
+struct Layout {
+  static constexpr int NH = D / 64;                 // 128-byte column halves of a row
+  static constexpr int kQ = NH * kBM * 128;         // Q tile
+  static constexpr int kKVHalf = kBN * 128;         // 64 keys x 64 elements
+  static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
+  static constexpr int kP = kBM * 128;              // 128 rows x 64 keys bf16
+  static constexpr int kBytes = kQ + 2 * kStages * kStage + 2 * kP + 1024 + 256;
+};
+
+struct Args {
+  const int32_t* offs;
+  __nv_bfloat16* out;     // final output (one split)
+  float* lse;             // final lse (one split), may be null
+  float* part_o;          // [nsplit][rows][D]  (several splits)
+  float* part_lse;        // [nsplit][rows]
+  uint32_t* status;
+  uint64_t limit_ns;
+  int Qn, K, L, KL, hq, hkv, grp, T, mtiles, nsplit, chunk;
+  float scale_log2;
+};
 
 __device__ __forceinline__ float ex2(float x) {
   float y;
@@ -48,68 +82,65 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
-__device__ __forceinline__ void ldsm_x4(uint32_t addr, uint32_t (&r)[4]) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void ldsm_x4_t(uint32_t addr, uint32_t (&r)[4]) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0, %1, %2, %3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(addr));
-}
-
-__device__ __forceinline__ void mma_bf16(float (&c)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
-  asm volatile(
-      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-      "{%8, %9}, {%0, %1, %2, %3};"
-      : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Address of 16-byte chunk c (0 .. D/8-1) of row i in a tile stored as D/64
-// column halves of `rows_per_half` rows x 128 B, each with the 128-byte swizzle
-// (chunk index XOR row mod 8, the layout TMA writes).
-__device__ __forceinline__ uint32_t sw128(uint32_t base, int rows_per_half, int i, int c) {
-  return base + (uint32_t)((c >> 3) * rows_per_half * 128 + i * 128 + (((c & 7) ^ (i & 7)) << 4));
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t d) {
+  asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+               "r"(d)
+               : "memory");
 }
 
-struct PrefixArgs {
-  const int32_t* offs;
-  float* part_o;      // [nsplit][Qn*K*L][hq][D]
-  float* part_lse;    // [nsplit][Qn*K*L][hq]
-  uint32_t* status;
-  uint64_t limit_ns;
-  int Qn, KL, hq, hkv, grp, T, mtiles, nsplit, chunk;
-  float scale_log2;
-};
+// Makes this thread's generic-proxy shared-memory writes visible to the async
+// proxy (the tensor cores read P from shared memory).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// MN-major operand with the 128-byte swizzle (V read as B of O = P V, N = D
+// contiguous in memory): 64-element MN chunks `lbo` bytes apart (leading
+// byte offset), 8-row K groups 1024 B apart (stride byte offset).
+__device__ __forceinline__ uint64_t desc_mnmajor_sw128(uint32_t smem_addr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((smem_addr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo & 0x3FFFFu) >> 4) << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1u << 46;
+  d |= (uint64_t)2u << 61;
+  return d;
+}
 
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
-    prefix_attn_kernel(const __grid_constant__ CUtensorMap tm_q,
-                       const __grid_constant__ CUtensorMap tm_k,
-                       const __grid_constant__ CUtensorMap tm_v, const PrefixArgs a) {
-  constexpr int NH = D / 64;                               // 128-byte column halves
-  constexpr int kQBytes = NH * kRowsPerTile * 128;          // Q tile
-  constexpr int kKVHalf = kKeysPerBlock * 128;              // one half of a K or V tile
-  constexpr int kStageBytes = 2 * NH * kKVHalf;             // K + V
+    attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kp,
+                const __grid_constant__ CUtensorMap tm_vp, const __grid_constant__ CUtensorMap tm_kt,
+                const __grid_constant__ CUtensorMap tm_vt, const Args a) {
+  using Lay = Layout<D>;
+  constexpr int NH = Lay::NH;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* q_s = smem;
-  uint8_t* ring = smem + kQBytes;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + kStages * kStageBytes);
-  uint64_t* full = bars;
-  uint64_t* empty = bars + kStages;
-  uint64_t* qbar = bars + 2 * kStages;
+  uint8_t* k_ring = q_s + Lay::kQ;                    // [kStages][kStage]
+  uint8_t* v_ring = k_ring + kStages * Lay::kStage;   // [kStages][kStage]
+  uint8_t* p_s = v_ring + kStages * Lay::kStage;      // [2][kP]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(p_s + 2 * Lay::kP);
+  uint64_t* k_full = bars;                        // [kStages]
+  uint64_t* k_empty = bars + kStages;             // [kStages]
+  uint64_t* v_full = bars + 2 * kStages;          // [kStages]
+  uint64_t* v_empty = bars + 3 * kStages;         // [kStages]
+  uint64_t* s_full = bars + 4 * kStages;          // [2]
+  uint64_t* s_free = s_full + 2;                  // [2]
+  uint64_t* p_full = s_full + 4;                  // [2]
+  uint64_t* p_free = s_full + 6;                  // [2]
+  uint64_t* q_full = s_full + 8;
+  uint64_t* drain = s_full + 9;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(s_full + 10);
 
+  // ---- work item
   int b = blockIdx.x;
   const int mt = b % a.mtiles;
   b /= a.mtiles;
@@ -117,331 +148,457 @@ __global__ void __launch_bounds__(kThreads, 1)
   b /= a.nsplit;
   const int g = b % a.hkv;
   const int qi = b / a.hkv;
-  const int P = a.offs[qi + 1] - a.offs[qi];
+  const int P = __ldg(&a.offs[qi + 1]) - __ldg(&a.offs[qi]);
   const int key_lo = split * a.chunk;
   const int key_hi = min(P, key_lo + a.chunk);
-  const int nblocks = key_hi > key_lo ? (key_hi - key_lo + kKeysPerBlock - 1) / kKeysPerBlock : 0;
-  const int tok0 = mt * a.T;                                // first token of this row tile
-  const int rows = min(a.T, a.KL - tok0) * a.grp;           // valid rows in the tile
+  const int nbp = key_hi > key_lo ? (key_hi - key_lo + kBN - 1) / kBN : 0;
+  const int tok0 = mt * a.T;
+  const int ntok = min(a.T, a.KL - tok0);
+  const int rows = ntok * a.grp;
+  const int c_lo = tok0 / a.L;
+  const int c_hi = (tok0 + ntok - 1) / a.L;
+  const int nbt = split == 0 ? ((c_hi - c_lo + 1) * a.L + kBN - 1) / kBN : 0;
+  const int nblk = nbp + nbt;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      mbar_init(smem_u32(&full[s]), 1);
-      mbar_init(smem_u32(&empty[s]), kConsumerWarps);
+      mbar_init(smem_u32(&k_full[s]), 1);
+      mbar_init(smem_u32(&k_empty[s]), 1);
+      mbar_init(smem_u32(&v_full[s]), 1);
+      mbar_init(smem_u32(&v_empty[s]), 1);
     }
-    mbar_init(smem_u32(qbar), 1);
+    for (int s = 0; s < 2; ++s) {
+      mbar_init(smem_u32(&s_full[s]), 1);
+      mbar_init(smem_u32(&s_free[s]), 4);
+      mbar_init(smem_u32(&p_full[s]), 4);
+      mbar_init(smem_u32(&p_free[s]), 1);
+    }
+    mbar_init(smem_u32(q_full), 1);
+    mbar_init(smem_u32(drain), 1);
     fence_barrier_init();
   }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), kTmemCols);
+    tmem_relinquish();
+  }
+  if (warp >= 2) {
+    // Rows past the T x grp rows the Q box fills are never loaded: zero them so their
+    // (discarded) scores stay finite and every lane of a warp takes the same code path.
+    const int r = (warp & 3) * 32 + lane;
+    if (r >= a.T * a.grp) {
+      for (int h = 0; h < NH; ++h)
+        for (int c = 0; c < 8; ++c)
+          st_shared_v4(smem_u32(q_s + h * kBM * 128 + r * 128 + c * 16), 0u, 0u, 0u, 0u);
+      fence_proxy_async_smem();
+    }
+  }
+  tc_fence_before();
   __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
 
-  if (warp == kConsumerWarps) {
-    // ---------------------------------------------------------- TMA producer
-    if (lane == 0 && nblocks > 0) {
+  if (warp == 0) {
+    // ------------------------------------------------------------ TMA producer
+    // Event-driven: issues the next K block or the next V block, whichever ring has
+    // a free slot (K is recycled after its S MMA, V after its PV MMA).
+    if (lane == 0 && nblk > 0) {
       const uint64_t pol_kv = policy_evict_last();   // re-read by the other row tiles
       const uint64_t pol_q = policy_evict_first();
-      const uint32_t qb = smem_u32(qbar);
+      const uint32_t qb = smem_u32(q_full);
       mbar_arrive_expect_tx(qb, NH * a.grp * a.T * 128);
       for (int h = 0; h < NH; ++h)
-        tma_load_3d(smem_u32(q_s + h * kRowsPerTile * 128), &tm_q, qb, h * 64, g * a.grp,
+        tma_load_3d(smem_u32(q_s + h * kBM * 128), &tm_q, qb, h * 64, g * a.grp,
                     qi * a.KL + tok0, pol_q);
-      int stage = 0;
-      uint32_t phase = 0;
-      const int kbase = a.offs[qi] + key_lo;
-      for (int blk = 0; blk < nblocks; ++blk) {
-        if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, a.limit_ns)) {
-          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteEmpty);
+      const int pbase = __ldg(&a.offs[qi]) + key_lo;
+      const int tbase = qi * a.KL + c_lo * a.L;
+      int nk = 0, nv = 0;
+      uint64_t t_last = globaltimer_ns();
+      while (nk < nblk || nv < nblk) {
+        bool moved = false;
+        if (nk < nblk && mbar_test(smem_u32(&k_empty[nk % kStages]), ((nk / kStages) & 1) ^ 1)) {
+          const uint32_t fb = smem_u32(&k_full[nk % kStages]);
+          mbar_arrive_expect_tx(fb, Lay::kStage);
+          uint8_t* dst = k_ring + (nk % kStages) * Lay::kStage;
+          const bool pre = nk < nbp;
+          const int key = pre ? pbase + nk * kBN : tbase + (nk - nbp) * kBN;
+          for (int h = 0; h < NH; ++h)
+            tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), pre ? &tm_kp : &tm_kt, fb, h * 64, g, key,
+                        pol_kv);
+          ++nk;
+          moved = true;
+        }
+        if (nv < nk && mbar_test(smem_u32(&v_empty[nv % kStages]), ((nv / kStages) & 1) ^ 1)) {
+          const uint32_t fb = smem_u32(&v_full[nv % kStages]);
+          mbar_arrive_expect_tx(fb, Lay::kStage);
+          uint8_t* dst = v_ring + (nv % kStages) * Lay::kStage;
+          const bool pre = nv < nbp;
+          const int key = pre ? pbase + nv * kBN : tbase + (nv - nbp) * kBN;
+          for (int h = 0; h < NH; ++h)
+            tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), pre ? &tm_vp : &tm_vt, fb, h * 64, g, key,
+                        pol_kv);
+          ++nv;
+          moved = true;
+        }
+        if (moved) {
+          t_last = globaltimer_ns();
+        } else if (globaltimer_ns() - t_last > a.limit_ns) {
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteKvEmpty);
           break;
         }
-        const uint32_t fb = smem_u32(&full[stage]);
-        mbar_arrive_expect_tx(fb, kStageBytes);
-        uint8_t* st = ring + stage * kStageBytes;
-        const int key = kbase + blk * kKeysPerBlock;
-        for (int h = 0; h < NH; ++h) {
-          tma_load_3d(smem_u32(st + h * kKVHalf), &tm_k, fb, h * 64, g, key, pol_kv);
-          tma_load_3d(smem_u32(st + (NH + h) * kKVHalf), &tm_v, fb, h * 64, g, key, pol_kv);
-        }
-        if (++stage == kStages) {
-          stage = 0;
-          phase ^= 1;
-        }
       }
-      // drain: no copy may still be in flight when the CTA exits
+      // no copy may still be in flight when the CTA exits
       mbar_wait(qb, 0, a.limit_ns);
-      const int pend = min(nblocks, kStages);
-      for (int i = 0; i < pend; ++i) {
-        if (--stage < 0) {
-          stage = kStages - 1;
-          phase ^= 1;
-        }
-        mbar_wait(smem_u32(&full[stage]), phase, a.limit_ns);
-      }
+      for (int i = max(0, nk - kStages); i < nk; ++i)
+        mbar_wait(smem_u32(&k_full[i % kStages]), (i / kStages) & 1, a.limit_ns);
+      for (int i = max(0, nv - kStages); i < nv; ++i)
+        mbar_wait(smem_u32(&v_full[i % kStages]), (i / kStages) & 1, a.limit_ns);
     }
-    return;
-  }
-
-  // ------------------------------------------------------------ consumers
-  const int r0 = warp * 16;              // first tile row of this warp
-  const int gq = lane >> 2, tq = lane & 3;
-  float o[D / 8][4];
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    // Event-driven: S_ns = Q K_ns^T as soon as K_ns is in and the S buffer is free;
+    // O += P_np V_np as soon as the softmax warps published P_np and V_np is in.
+    if (lane == 0 && nblk > 0) {
+      const uint32_t idS = idesc_bf16_f32(kBM, kBN);
+      const uint32_t idPV = idesc_bf16_f32(kBM, D) | (1u << 16);   // B (= V) MN-major
+      const uint32_t qa = smem_u32(q_s);
+      if (!mbar_wait(smem_u32(q_full), 0, a.limit_ns)) {
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
+      } else {
+        int ns = 0, np = 0;
+        uint64_t t_last = globaltimer_ns();
+        while (np < nblk) {
+          bool moved = false;
+          if (ns < nblk && mbar_test(smem_u32(&k_full[ns % kStages]), (ns / kStages) & 1) &&
+              mbar_test(smem_u32(&s_free[ns & 1]), ((ns >> 1) & 1) ^ 1)) {
+            tc_fence_after();
+            const uint32_t ks = smem_u32(k_ring + (ns % kStages) * Lay::kStage);
 #pragma unroll
-  for (int n = 0; n < D / 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
-  float mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.f, 0.f};
-
-  if (nblocks > 0) {
-    bool ok = mbar_wait(smem_u32(qbar), 0, a.limit_ns);
-    if (!ok) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
-    uint32_t qf[D / 16][4];
-    const uint32_t qbase = smem_u32(q_s);
+            for (int h = 0; h < NH; ++h)
 #pragma unroll
-    for (int ks = 0; ks < D / 16; ++ks)
-      ldsm_x4(sw128(qbase, kRowsPerTile, r0 + (lane & 15), 2 * ks + (lane >> 4)), qf[ks]);
-
-    int stage = 0;
-    uint32_t phase = 0;
-    for (int blk = 0; blk < nblocks && ok; ++blk) {
-      if (!mbar_wait(smem_u32(&full[stage]), phase, a.limit_ns)) {
-        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteFull);
+              for (int k16 = 0; k16 < 4; ++k16)
+                tc_mma_bf16(tmem_base + col_s(ns & 1),
+                            desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
+                            desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS,
+                            (h | k16) != 0);
+            tc_commit(smem_u32(&s_full[ns & 1]));
+            tc_commit(smem_u32(&k_empty[ns % kStages]));
+            ++ns;
+            moved = true;
+          }
+          if (np < ns && mbar_test(smem_u32(&p_full[np & 1]), (np >> 1) & 1) &&
+              mbar_test(smem_u32(&v_full[np % kStages]), (np / kStages) & 1)) {
+            tc_fence_after();
+            const uint32_t pa = smem_u32(p_s + (np & 1) * Lay::kP);
+            const uint32_t vs = smem_u32(v_ring + (np % kStages) * Lay::kStage);
+#pragma unroll
+            for (int k16 = 0; k16 < kBN / 16; ++k16)
+              tc_mma_bf16(tmem_base + kColO, desc_kmajor_sw128(pa + k16 * 32),
+                          desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV, (np | k16) != 0);
+            tc_commit(smem_u32(&p_free[np & 1]));   // P buffer free, and "PV_np done"
+            tc_commit(smem_u32(&v_empty[np % kStages]));
+            ++np;
+            moved = true;
+          }
+          if (moved) {
+            t_last = globaltimer_ns();
+          } else if (globaltimer_ns() - t_last > a.limit_ns) {
+            record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePFull);
+            break;
+          }
+        }
+      }
+      tc_commit(smem_u32(drain));
+      if (!mbar_wait(smem_u32(drain), 0, a.limit_ns))
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else {
+    // ------------------------------------------------------------ softmax / epilogue
+    // Online softmax in base 2 with a lazily updated reference max: P_j is taken
+    // relative to m_ref, which only moves when a row's block max exceeds it by more
+    // than kRescaleLog2 (then O in tensor memory and l are rescaled once).  P values
+    // stay below 2^kRescaleLog2, which bf16 and the fp32 accumulators hold exactly
+    // enough; the result is the same softmax.
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;                 // tile row = tensor-memory lane
+    const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
+    const bool rvalid = r < rows;
+    const int tok = tok0 + r / a.grp;
+    const int krow = tok / a.L, lrow = tok % a.L;
+    const int tlo = (krow - c_lo) * a.L;               // visible tail range [tlo, tlo + lrow]
+    const int thi = tlo + lrow + 1;
+    float m_ref = -INFINITY, l = 0.f;
+    bool ok = true;
+    const uint32_t prow = (uint32_t)r * 128u;
+    for (int j = 0; j < nblk; ++j) {
+      const int sb = j & 1;
+      if (!mbar_wait(smem_u32(&s_full[sb]), (j >> 1) & 1, a.limit_ns)) {
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteSFull);
+        ok = false;
         break;
       }
-      const uint32_t kb = smem_u32(ring + stage * kStageBytes);
-      const uint32_t vb = kb + NH * kKVHalf;
-      // S = Q K^T over 64 keys: 8 n-tiles of 8 keys
-      float s[8][4];
-#pragma unroll
-      for (int n = 0; n < 8; ++n) s[n][0] = s[n][1] = s[n][2] = s[n][3] = 0.f;
-#pragma unroll
-      for (int ks = 0; ks < D / 16; ++ks) {
-#pragma unroll
-        for (int np = 0; np < 4; ++np) {
-          uint32_t kf[4];
-          ldsm_x4(sw128(kb, kKeysPerBlock, 16 * np + (lane & 7) + ((lane >> 4) << 3),
-                        2 * ks + ((lane >> 3) & 1)),
-                  kf);
-          mma_bf16(s[2 * np], qf[ks], kf[0], kf[1]);
-          mma_bf16(s[2 * np + 1], qf[ks], kf[2], kf[3]);
-        }
-      }
-      // online softmax (base-2 domain)
-      const int kfirst = key_lo + blk * kKeysPerBlock;
-      float bmax[2] = {-INFINITY, -INFINITY};
-#pragma unroll
-      for (int n = 0; n < 8; ++n) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const int key = kfirst + 8 * n + 2 * tq + (e & 1);
-          const float v = key < key_hi ? s[n][e] * a.scale_log2 : -INFINITY;
-          s[n][e] = v;
-          bmax[e >> 1] = fmaxf(bmax[e >> 1], v);
-        }
-      }
-      float corr[2];
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        bmax[h] = fmaxf(bmax[h], __shfl_xor_sync(0xffffffffu, bmax[h], 1));
-        bmax[h] = fmaxf(bmax[h], __shfl_xor_sync(0xffffffffu, bmax[h], 2));
-        const float nm = fmaxf(mrow[h], bmax[h]);
-        corr[h] = ex2(mrow[h] - nm);
-        mrow[h] = nm;
-      }
-      float bsum[2] = {0.f, 0.f};
-#pragma unroll
-      for (int n = 0; n < 8; ++n) {
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-          const float p = ex2(s[n][e] - mrow[e >> 1]);
-          s[n][e] = p;
-          bsum[e >> 1] += p;
-        }
-      }
-#pragma unroll
-      for (int h = 0; h < 2; ++h) lrow[h] = lrow[h] * corr[h] + bsum[h];
-#pragma unroll
-      for (int n = 0; n < D / 8; ++n) {
-        o[n][0] *= corr[0];
-        o[n][1] *= corr[0];
-        o[n][2] *= corr[1];
-        o[n][3] *= corr[1];
-      }
-      // O += P V over the 64 keys (4 k-steps of 16)
-#pragma unroll
-      for (int kk = 0; kk < 4; ++kk) {
-        uint32_t pa[4];
-        pa[0] = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
-        pa[1] = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
-        pa[2] = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
-        pa[3] = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
-#pragma unroll
-        for (int dp = 0; dp < D / 16; ++dp) {
-          uint32_t vf[4];
-          ldsm_x4_t(sw128(vb, kKeysPerBlock, 16 * kk + (lane & 7) + (((lane >> 3) & 1) << 3),
-                          2 * dp + (lane >> 4)),
-                    vf);
-          mma_bf16(o[2 * dp], pa, vf[0], vf[1]);
-          mma_bf16(o[2 * dp + 1], pa, vf[2], vf[3]);
-        }
-      }
+      tc_fence_after();
+      uint32_t sr[64];
+      tmem_ld_32x32b_x32(lane_base + col_s(sb), *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
+      tmem_ld_32x32b_x32(lane_base + col_s(sb) + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+      tmem_wait_ld();
+      tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&empty[stage]));
-      if (++stage == kStages) {
-        stage = 0;
-        phase ^= 1;
+      if (lane == 0) mbar_arrive(smem_u32(&s_free[sb]));
+      int vlo, vhi;   // valid columns of this block for this row
+      if (j < nbp) {
+        vlo = 0;
+        vhi = min(kBN, key_hi - (key_lo + j * kBN));
+      } else {
+        const int base = (j - nbp) * kBN;
+        vlo = max(0, tlo - base);
+        vhi = min(kBN, thi - base);
+      }
+      // rows without output (r >= rows) are not masked: their values are finite and
+      // discarded, and masking them would split the warp between the two paths below
+      const bool full = vlo == 0 && vhi == kBN;
+      float pm[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
+      if (full) {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
+      } else {
+#pragma unroll
+        for (int c = 0; c < kBN; ++c)
+          if (c >= vlo && c < vhi) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
+      }
+      const float bmax = a.scale_log2 * fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                                              fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      const float m_old = m_ref;
+      if (bmax > m_ref + kRescaleLog2) m_ref = bmax;   // also the first finite block
+      const bool resc = m_ref != m_old && m_old != -INFINITY;
+      const float corr = resc ? ex2(m_old - m_ref) : 1.f;
+      const float ms = m_ref == -INFINITY ? 0.f : m_ref;
+      // P_j -> shared memory (row r: 64 bf16 = 128 B, 16-byte chunks swizzled by row)
+      if (!mbar_wait(smem_u32(&p_free[sb]), ((j >> 1) & 1) ^ 1, a.limit_ns)) {
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePFree);
+        ok = false;
+        break;
+      }
+      const uint32_t pbuf = smem_u32(p_s + sb * Lay::kP) + prow;
+      float rsp[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) rsp[u] = 0.f;
+      if (full) {
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) {
+          float e[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            e[u] = ex2(fmaf(__uint_as_float(sr[8 * c8 + u]), a.scale_log2, -ms));
+            rsp[u] += e[u];
+          }
+          st_shared_v4(pbuf + (uint32_t)((c8 ^ (r & 7)) << 4), pack_bf16(e[0], e[1]),
+                       pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]), pack_bf16(e[6], e[7]));
+        }
+      } else {
+#pragma unroll
+        for (int c8 = 0; c8 < 8; ++c8) {
+          float e[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) {
+            const int c = 8 * c8 + u;
+            const float x = ex2(fmaf(__uint_as_float(sr[c]), a.scale_log2, -ms));
+            e[u] = (c >= vlo && c < vhi) ? x : 0.f;
+            rsp[u] += e[u];
+          }
+          st_shared_v4(pbuf + (uint32_t)((c8 ^ (r & 7)) << 4), pack_bf16(e[0], e[1]),
+                       pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]), pack_bf16(e[6], e[7]));
+        }
+      }
+      const float rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
+      l = l * corr + rs;
+      if (__any_sync(0xffffffffu, resc)) {
+        // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale
+        const int i = j - 1;
+        if (!mbar_wait(smem_u32(&p_free[i & 1]), (i >> 1) & 1, a.limit_ns)) {
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteOFull);
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t o[32];
+          tmem_ld_32x32b_x32(lane_base + kColO + c0, o);
+          tmem_wait_ld();
+#pragma unroll
+          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
+          tmem_st_32x32b_x32(lane_base + kColO + c0, o);
+        }
+        tmem_wait_st();
+        tc_fence_before();
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&p_full[sb]));
+    }
+    // ---- epilogue: wait for the last PV, normalise O by l
+    if (ok && nblk > 0) {
+      const int i = nblk - 1;
+      if (!mbar_wait(smem_u32(&p_free[i & 1]), (i >> 1) & 1, a.limit_ns)) {
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteOFull);
+        ok = false;
+      }
+      tc_fence_after();
+    }
+    const int head = g * a.grp + r % a.grp;
+    const size_t rowid = ((size_t)qi * a.KL + tok) * a.hq + head;
+    const size_t nrows = (size_t)a.Qn * a.KL * a.hq;
+    const bool any = l > 0.f;
+    const float inv = any ? 1.f / l : 0.f;
+    const float lse = any ? kLn2 * (m_ref + __log2f(l)) : -INFINITY;
+#pragma unroll
+    for (int c0 = 0; c0 < D; c0 += 32) {
+      uint32_t o[32];
+      if (nblk > 0) {
+        tmem_ld_32x32b_x32(lane_base + kColO + c0, o);
+        tmem_wait_ld();
+      } else {
+#pragma unroll
+        for (int c = 0; c < 32; ++c) o[c] = 0u;
+      }
+      if (rvalid) {
+        if (a.nsplit == 1) {
+          uint4* dst = reinterpret_cast<uint4*>(a.out + rowid * D + c0);
+#pragma unroll
+          for (int c = 0; c < 32; c += 8)
+            dst[c / 8] = make_uint4(
+                pack_bf16(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
+                pack_bf16(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
+                pack_bf16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
+                pack_bf16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
+        } else {
+          float4* dst = reinterpret_cast<float4*>(a.part_o + ((size_t)split * nrows + rowid) * D + c0);
+#pragma unroll
+          for (int c = 0; c < 32; c += 4)
+            dst[c / 4] = make_float4(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv,
+                                     __uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv);
+        }
       }
     }
-  }
-  // finish the row sums across the quad, write the normalised partial
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    lrow[h] += __shfl_xor_sync(0xffffffffu, lrow[h], 1);
-    lrow[h] += __shfl_xor_sync(0xffffffffu, lrow[h], 2);
-  }
-#pragma unroll
-  for (int h = 0; h < 2; ++h) {
-    const int r = r0 + gq + 8 * h;
-    if (r >= rows) continue;
-    const int tok = tok0 + r / a.grp;
-    const int head = g * a.grp + r % a.grp;
-    const size_t row = ((size_t)split * a.Qn * a.KL + (size_t)qi * a.KL + tok) * a.hq + head;
-    const bool any = lrow[h] > 0.f;
-    const float inv = any ? 1.f / lrow[h] : 0.f;
-    float* dst = a.part_o + row * D;
-#pragma unroll
-    for (int n = 0; n < D / 8; ++n) {
-      float2 v = make_float2(o[n][2 * h] * inv, o[n][2 * h + 1] * inv);
-      *reinterpret_cast<float2*>(dst + 8 * n + 2 * tq) = v;
+    if (rvalid) {
+      if (a.nsplit == 1) {
+        if (a.lse) a.lse[rowid] = lse;
+      } else {
+        a.part_lse[(size_t)split * nrows + rowid] = lse;
+      }
     }
-    if (tq == 0) a.part_lse[row] = any ? kLn2 * (mrow[h] + __log2f(lrow[h])) : -INFINITY;
+    (void)ok;
   }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
 }
 
-// One warp per (query, candidate, token l, head h).  Lane j (< l+1) scores tail
-// key j; the weighted sum over tail values is split over lanes by D; then the
-// tail result is merged with every prefix split by log-sum-exp weights.
+// One warp per (token, head) row: out = sum_s exp(lse_s - LSE) * O_s, LSE = logsumexp_s lse_s.
 template <int D>
-__global__ void tail_merge_kernel(const __nv_bfloat16* __restrict__ q,
-                                  const __nv_bfloat16* __restrict__ k_tail,
-                                  const __nv_bfloat16* __restrict__ v_tail,
-                                  const float* __restrict__ part_o, const float* __restrict__ part_lse,
-                                  int nsplit, int Qn, int K, int L, int hq, int hkv, float scale,
-                                  __nv_bfloat16* __restrict__ out, float* __restrict__ lse_out) {
-  constexpr int DPL = D / 32;  // elements per lane
-  const long long rowid = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  const long long nrows = (long long)Qn * K * L * hq;
-  if (rowid >= nrows) return;
+__global__ void merge_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
+                             int nsplit, long long nrows, __nv_bfloat16* __restrict__ out,
+                             float* __restrict__ lse_out) {
+  constexpr int DPL = D / 32;
+  const long long row = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
-  const int h = (int)(rowid % hq);
-  const long long tok = rowid / hq;           // (qi*K + k)*L + l
-  const int l = (int)(tok % L);
-  const long long cand = tok / L;             // qi*K + k
-  const int g = h / (hq / hkv);
-
-  // q row in fp32, DPL elements per lane (contiguous)
-  float qv[DPL];
-  {
-    const __nv_bfloat16* qr = q + rowid * D + lane * DPL;
-#pragma unroll
-    for (int i = 0; i < DPL; i += 2) {
-      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(qr + i));
-      qv[i] = f.x;
-      qv[i + 1] = f.y;
-    }
+  if (row >= nrows) return;
+  float mx = -INFINITY;
+  for (int s = lane; s < nsplit; s += 32) mx = fmaxf(mx, part_lse[(size_t)s * nrows + row]);
+  mx = warp_max(mx);
+  float den = 0.f;
+  for (int s = lane; s < nsplit; s += 32) {
+    const float v = part_lse[(size_t)s * nrows + row];
+    if (v != -INFINITY) den += __expf(v - mx);
   }
-  // scores of tail keys 0..l: each key's dot is a warp reduction
-  float my_s[kMaxTail / 32] = {-INFINITY, -INFINITY};
-  float tmax = -INFINITY;
-  for (int j = 0; j <= l; ++j) {
-    const __nv_bfloat16* kr = k_tail + ((cand * L + j) * hkv + g) * D + lane * DPL;
-    float dot = 0.f;
-#pragma unroll
-    for (int i = 0; i < DPL; i += 2) {
-      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(kr + i));
-      dot = fmaf(qv[i], f.x, fmaf(qv[i + 1], f.y, dot));
-    }
-    dot = warp_sum(dot) * scale;
-    if ((j & 31) == lane) my_s[j >> 5] = dot;
-    tmax = fmaxf(tmax, dot);
-  }
-  float acc[DPL];
-#pragma unroll
-  for (int i = 0; i < DPL; ++i) acc[i] = 0.f;
-  float tsum = 0.f;
-  for (int j = 0; j <= l; ++j) {
-    const float sj = __shfl_sync(0xffffffffu, my_s[j >> 5], j & 31);
-    const float p = __expf(sj - tmax);
-    tsum += p;
-    const __nv_bfloat16* vr = v_tail + ((cand * L + j) * hkv + g) * D + lane * DPL;
-#pragma unroll
-    for (int i = 0; i < DPL; i += 2) {
-      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(vr + i));
-      acc[i] = fmaf(p, f.x, acc[i]);
-      acc[i + 1] = fmaf(p, f.y, acc[i + 1]);
-    }
-  }
-  const float tail_lse = tmax + __logf(tsum);
-  // merge: weights exp(lse_i - LSE)
-  float M = tail_lse;
-  for (int s = 0; s < nsplit; ++s) M = fmaxf(M, part_lse[(size_t)s * nrows + rowid]);
-  float wt = __expf(tail_lse - M);
-  float den = wt;
+  den = warp_sum(den);
   float res[DPL];
 #pragma unroll
-  for (int i = 0; i < DPL; ++i) res[i] = acc[i] / tsum * wt;
+  for (int i = 0; i < DPL; ++i) res[i] = 0.f;
+#pragma unroll 4
   for (int s = 0; s < nsplit; ++s) {
-    const float ls = part_lse[(size_t)s * nrows + rowid];
-    if (ls == -INFINITY) continue;
-    const float w = __expf(ls - M);
-    den += w;
-    const float* po = part_o + ((size_t)s * nrows + rowid) * D + lane * DPL;
+    const float v = part_lse[(size_t)s * nrows + row];
+    const float w = v == -INFINITY ? 0.f : __expf(v - mx);
+    const float* po = part_o + ((size_t)s * nrows + row) * D + lane * DPL;
+    if (DPL == 4) {
+      const float4 f = *reinterpret_cast<const float4*>(po);
+      res[0] = fmaf(w, f.x, res[0]);
+      res[1] = fmaf(w, f.y, res[1]);
+      res[2] = fmaf(w, f.z, res[2]);
+      res[3] = fmaf(w, f.w, res[3]);
+    } else {
 #pragma unroll
-    for (int i = 0; i < DPL; i += 2) {
-      const float2 f = *reinterpret_cast<const float2*>(po + i);
-      res[i] = fmaf(w, f.x, res[i]);
-      res[i + 1] = fmaf(w, f.y, res[i + 1]);
+      for (int i = 0; i < DPL; ++i) res[i] = fmaf(w, po[i], res[i]);
     }
   }
   const float inv = 1.f / den;
-  __nv_bfloat16* orow = out + rowid * D + lane * DPL;
+  __nv_bfloat16* o = out + row * D + lane * DPL;
 #pragma unroll
   for (int i = 0; i < DPL; i += 2)
-    *reinterpret_cast<__nv_bfloat162*>(orow + i) = __floats2bfloat162_rn(res[i] * inv, res[i + 1] * inv);
-  if (lane == 0 && lse_out) lse_out[rowid] = M + __logf(den);
+    *reinterpret_cast<__nv_bfloat162*>(o + i) = __floats2bfloat162_rn(res[i] * inv, res[i + 1] * inv);
+  if (lane == 0 && lse_out) lse_out[row] = mx + __logf(den);
 }
 
 struct Plan {
   int grp, T, mtiles, nsplit, chunk;
 };
 
-static Plan make_plan(const fvrag_attn_desc* d) {
+// Key-split plan: pick the number of splits that minimises an estimate of
+// waves x (blocks per CTA + fixed cost) plus the cost of writing and merging the
+// partials (one CTA per SM; a 64-key block is ~0.33 us of tensor-core time).
+static Plan make_plan(const fvrag_attn_desc* d, int sms) {
   Plan p;
   p.grp = d->hq / d->hkv;
-  p.T = std::max(1, kRowsPerTile / p.grp);
+  p.T = std::max(1, kBM / p.grp);
   const int KL = d->num_cand * d->cand_len;
   p.mtiles = (KL + p.T - 1) / p.T;
-  if (d->max_prefix <= 0) {
-    p.nsplit = 0;
-    p.chunk = 0;
-    return p;
-  }
   const long long base = (long long)d->num_queries * d->hkv * p.mtiles;
-  const int max_blocks = (d->max_prefix + kKeysPerBlock - 1) / kKeysPerBlock;
-  int ns = (int)std::min<long long>((kTargetCtas + base - 1) / base, max_blocks);
-  ns = std::max(ns, 1);
-  const int per = (max_blocks + ns - 1) / ns;   // key blocks per split
-  p.chunk = per * kKeysPerBlock;
-  p.nsplit = (max_blocks + per - 1) / per;
+  const int nb = (std::max(d->max_prefix, 0) + kBN - 1) / kBN;
+  p.nsplit = 1;
+  p.chunk = std::max(nb, 1) * kBN;
+  if (nb <= 1) return p;
+  if (sms <= 0) sms = 148;
+  const double rows = (double)d->num_queries * KL * d->hq;
+  double best = 1e30;
+  for (int ns = 1; ns <= std::min(nb, 64); ++ns) {
+    const int per = (nb + ns - 1) / ns;
+    const int nse = (nb + per - 1) / per;
+    const long long ctas = base * nse;
+    const double waves = (double)((ctas + sms - 1) / sms);
+    double t = waves * (per + 6) * 0.33;
+    if (nse > 1) t += 3.0 + nse * rows * (d->head_dim + 1) * 8.0 / 8.0e6;
+    if (t < best - 1e-9) {
+      best = t;
+      p.nsplit = nse;
+      p.chunk = per * kBN;
+    }
+  }
   return p;
 }
 
-static size_t ws_bytes(const fvrag_attn_desc* d) {
-  const Plan p = make_plan(d);
+static size_t ws_bytes(const fvrag_attn_desc* d, int sms) {
+  const Plan p = make_plan(d, sms);
   const size_t rows = (size_t)d->num_queries * d->num_cand * d->cand_len * d->hq;
-  return kWsHeaderBytes + (size_t)p.nsplit * rows * ((size_t)d->head_dim + 1) * 4;
+  return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)d->head_dim + 1) * 4 : 0);
+}
+
+static int device_sms() {
+  const int s = sm_count();
+  return s > 0 ? s : 148;
 }
 
 template <int D>
-static size_t smem_bytes() {
-  return (size_t)(D / 64) * kRowsPerTile * 128 + (size_t)kStages * 2 * (D / 64) * kKeysPerBlock * 128 +
-         1024 + 256;
+static fvrag_status launch(const CUtensorMap* maps, const Args& a, long long grid, cudaStream_t s) {
+  const int sm = Layout<D>::kBytes;
+  if (cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  attn_kernel<D><<<(unsigned)grid, kThreads, sm, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  return launch_status();
 }
 
 }  // namespace attn
@@ -453,7 +610,7 @@ extern "C" size_t fvrag_verify_attn_workspace(const fvrag_attn_desc* d) {
   if (!d || d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
       d->hq % d->hkv || (d->head_dim != 64 && d->head_dim != 128) || d->max_prefix < 0)
     return 0;
-  return attn::ws_bytes(d);
+  return attn::ws_bytes(d, attn::device_sms());
 }
 
 extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* q,
@@ -464,91 +621,82 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
   using namespace attn;
   if (!d || !q || !prefix_offsets || !k_tail || !v_tail || !out) return FVRAG_ERR_INVALID_ARG;
   if (d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
-      d->max_prefix < 0 || d->total_prefix < 0 || d->flags != 0)
+      d->max_prefix < 0 || d->total_prefix < 0 || d->flags != 0 || !(d->softmax_scale >= 0.f) ||
+      d->softmax_scale == INFINITY)
     return FVRAG_ERR_INVALID_ARG;
   if (d->total_prefix > 0 && (!k_prefix || !v_prefix)) return FVRAG_ERR_INVALID_ARG;
   if (d->hq % d->hkv != 0 || (d->head_dim != 64 && d->head_dim != 128) ||
-      d->cand_len > kMaxTail || d->hq / d->hkv > kRowsPerTile)
+      d->cand_len > kMaxTail || d->hq / d->hkv > kBM)
     return FVRAG_ERR_UNSUPPORTED;
   if (!aligned16(q) || !aligned16(k_tail) || !aligned16(v_tail) || !aligned16(out) ||
       (k_prefix && !aligned16(k_prefix)) || (v_prefix && !aligned16(v_prefix)))
     return FVRAG_ERR_MISALIGNED;
-  const size_t need = ws_bytes(d);
+  const int sms = device_sms();
+  const size_t need = ws_bytes(d, sms);
   if (!ws || ws_size < need) return FVRAG_ERR_WORKSPACE;
   if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
 
-  const Plan p = make_plan(d);
+  const Plan p = make_plan(d, sms);
   const int D = d->head_dim;
   const float scale = d->softmax_scale != 0.f ? d->softmax_scale : 1.f / sqrtf((float)D);
   const int KL = d->num_cand * d->cand_len;
+  const long long nrows = (long long)d->num_queries * KL * d->hq;
   uint8_t* base = reinterpret_cast<uint8_t*>(ws);
-  uint32_t* status = reinterpret_cast<uint32_t*>(base);
-  const size_t nrows = (size_t)d->num_queries * KL * d->hq;
-  float* part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
-  float* part_lse = part_o + (size_t)p.nsplit * nrows * D;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
-  const bool run_prefix = p.nsplit > 0 && d->total_prefix > 0;
-  if (run_prefix) {
-    CUtensorMap tq, tk, tv;
-    {
-      const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d->hq, (uint64_t)d->num_queries * KL};
-      const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d->hq * D * 2};
-      const uint32_t box[3] = {64u, (uint32_t)p.grp, (uint32_t)p.T};
-      if (!encode_tmap_bf16(&tq, q, 3, dims, strides, box, true)) return FVRAG_ERR_CUDA;
-    }
-    {
-      const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d->hkv, (uint64_t)d->total_prefix};
-      const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d->hkv * D * 2};
-      const uint32_t box[3] = {64u, 1u, (uint32_t)kKeysPerBlock};
-      if (!encode_tmap_bf16(&tk, k_prefix, 3, dims, strides, box, true)) return FVRAG_ERR_CUDA;
-      if (!encode_tmap_bf16(&tv, v_prefix, 3, dims, strides, box, true)) return FVRAG_ERR_CUDA;
-    }
-    PrefixArgs a;
-    a.offs = prefix_offsets;
-    a.part_o = part_o;
-    a.part_lse = part_lse;
-    a.status = status;
-    a.limit_ns = wait_limit_ns();
-    a.Qn = d->num_queries;
-    a.KL = KL;
-    a.hq = d->hq;
-    a.hkv = d->hkv;
-    a.grp = p.grp;
-    a.T = p.T;
-    a.mtiles = p.mtiles;
-    a.nsplit = p.nsplit;
-    a.chunk = p.chunk;
-    a.scale_log2 = scale * kLog2e;
-    const long long grid = (long long)d->num_queries * d->hkv * p.nsplit * p.mtiles;
-    if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
-    if (D == 128) {
-      const size_t sm = smem_bytes<128>();
-      if (cudaFuncSetAttribute(prefix_attn_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)sm) != cudaSuccess)
-        return FVRAG_ERR_CUDA;
-      prefix_attn_kernel<128><<<(unsigned)grid, kThreads, sm, s>>>(tq, tk, tv, a);
-    } else {
-      const size_t sm = smem_bytes<64>();
-      if (cudaFuncSetAttribute(prefix_attn_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               (int)sm) != cudaSuccess)
-        return FVRAG_ERR_CUDA;
-      prefix_attn_kernel<64><<<(unsigned)grid, kThreads, sm, s>>>(tq, tk, tv, a);
-    }
-    if (cudaGetLastError() != cudaSuccess) return FVRAG_ERR_CUDA;
+  CUtensorMap maps[5];
+  {
+    const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d->hq, (uint64_t)d->num_queries * KL};
+    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d->hq * D * 2};
+    const uint32_t box[3] = {64u, (uint32_t)p.grp, (uint32_t)p.T};
+    if (!encode_tmap_bf16(&maps[0], q, 3, dims, strides, box, true)) return FVRAG_ERR_CUDA;
   }
-  const int nsplit = run_prefix ? p.nsplit : 0;
-  const int warps_per_block = 8;
-  const long long blocks = ((long long)nrows + warps_per_block - 1) / warps_per_block;
+  {
+    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d->hkv * D * 2};
+    const uint32_t box[3] = {64u, 1u, (uint32_t)kBN};
+    const uint64_t tdims[3] = {(uint64_t)D, (uint64_t)d->hkv, (uint64_t)d->num_queries * KL};
+    if (!encode_tmap_bf16(&maps[3], k_tail, 3, tdims, strides, box, true)) return FVRAG_ERR_CUDA;
+    if (!encode_tmap_bf16(&maps[4], v_tail, 3, tdims, strides, box, true)) return FVRAG_ERR_CUDA;
+    if (d->total_prefix > 0) {
+      const uint64_t pdims[3] = {(uint64_t)D, (uint64_t)d->hkv, (uint64_t)d->total_prefix};
+      if (!encode_tmap_bf16(&maps[1], k_prefix, 3, pdims, strides, box, true)) return FVRAG_ERR_CUDA;
+      if (!encode_tmap_bf16(&maps[2], v_prefix, 3, pdims, strides, box, true)) return FVRAG_ERR_CUDA;
+    } else {
+      maps[1] = maps[3];   // never read: no query has prefix keys
+      maps[2] = maps[4];
+    }
+  }
+  Args a;
+  a.offs = prefix_offsets;
+  a.out = reinterpret_cast<__nv_bfloat16*>(out);
+  a.lse = lse;
+  a.part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
+  a.part_lse = a.part_o + (size_t)p.nsplit * nrows * D;
+  a.status = reinterpret_cast<uint32_t*>(base);
+  a.limit_ns = wait_limit_ns();
+  a.Qn = d->num_queries;
+  a.K = d->num_cand;
+  a.L = d->cand_len;
+  a.KL = KL;
+  a.hq = d->hq;
+  a.hkv = d->hkv;
+  a.grp = p.grp;
+  a.T = p.T;
+  a.mtiles = p.mtiles;
+  a.nsplit = p.nsplit;
+  a.chunk = p.chunk;
+  a.scale_log2 = scale * kLog2e;
+  const long long grid = (long long)d->num_queries * d->hkv * p.nsplit * p.mtiles;
+  if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  fvrag_status st = D == 128 ? launch<128>(maps, a, grid, s) : launch<64>(maps, a, grid, s);
+  if (st != FVRAG_OK || p.nsplit == 1) return st;
+  const int wpb = 8;
+  const long long blocks = (nrows + wpb - 1) / wpb;
   if (D == 128)
-    tail_merge_kernel<128><<<(unsigned)blocks, 32 * warps_per_block, 0, s>>>(
-        reinterpret_cast<const __nv_bfloat16*>(q), reinterpret_cast<const __nv_bfloat16*>(k_tail),
-        reinterpret_cast<const __nv_bfloat16*>(v_tail), part_o, part_lse, nsplit, d->num_queries,
-        d->num_cand, d->cand_len, d->hq, d->hkv, scale, reinterpret_cast<__nv_bfloat16*>(out), lse);
+    merge_kernel<128><<<(unsigned)blocks, 32 * wpb, 0, s>>>(a.part_o, a.part_lse, p.nsplit, nrows,
+                                                            a.out, lse);
   else
-    tail_merge_kernel<64><<<(unsigned)blocks, 32 * warps_per_block, 0, s>>>(
-        reinterpret_cast<const __nv_bfloat16*>(q), reinterpret_cast<const __nv_bfloat16*>(k_tail),
-        reinterpret_cast<const __nv_bfloat16*>(v_tail), part_o, part_lse, nsplit, d->num_queries,
-        d->num_cand, d->cand_len, d->hq, d->hkv, scale, reinterpret_cast<__nv_bfloat16*>(out), lse);
+    merge_kernel<64><<<(unsigned)blocks, 32 * wpb, 0, s>>>(a.part_o, a.part_lse, p.nsplit, nrows,
+                                                           a.out, lse);
   return launch_status();
 }

@@ -3,8 +3,8 @@
 // Eq. 12-13 and the final argmax over alignment).
 //
 // Both steps move kilobytes to a few megabytes, so they are latency-bound:
-// K3 uses one CTA per (query, candidate) with one warp per frame at a time and
-// 16-byte loads; K4 uses one CTA per query.
+// K3 uses one CTA per (query, candidate), 16 warps with four frames' 16-byte
+// loads in flight per warp; K4 uses one CTA per query.
 #include <cuda_fp16.h>
 
 #include "fvrag_common.cuh"
@@ -12,15 +12,17 @@
 
 namespace fvrag {
 
-constexpr int kClipThreads = 256;
+constexpr int kClipThreads = 512;
+constexpr int kClipUnroll = 4;   // frames in flight per warp
 constexpr int kClipMaxDim = 4096;
 
 // One CTA per (query q, candidate k).  The candidate embedding is widened to
-// fp32 in shared memory; warp w handles frames w, w + 8, ...: the 32 lanes split
-// the E dimension in 16-byte (8 x fp16) chunks, reduce <e, f> and |f|^2 with
-// shuffles, and lane 0 keeps the warp's best (cos, frame).  The 8 warp results
-// are then reduced by one warp: larger cos wins, equal cos goes to the lower
-// frame index.
+// fp32 in shared memory; warp w handles frames w, w + 16, w + 32, w + 48 together
+// (then the next 64): the 32 lanes split the E dimension in 16-byte (8 x fp16)
+// chunks with the four frames' loads in flight at once, reduce <e, f> and |f|^2
+// with shuffles, and lane 0 keeps the warp's best (cos, frame).  The 16 warp
+// results are then reduced by one warp: larger cos wins, equal cos goes to the
+// lower frame index.
 __global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
     const __half* __restrict__ cand, const __half* __restrict__ frames, int K, int F, int E,
     float tau, float* __restrict__ cos_out, float* __restrict__ max_cos, int32_t* __restrict__ argmax,
@@ -55,36 +57,54 @@ __global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
   for (int w = 0; w < kClipThreads / 32; ++w) ee += red[w];
   const float inv_e = ee > 0.f ? rsqrtf(ee) : 0.f;
 
+  constexpr int NW = kClipThreads / 32;
   float wbest = -INFINITY;
   int wbest_i = 0x7fffffff;
   const __half* fq = frames + (size_t)q * F * E;
-  for (int f = warp; f < F; f += kClipThreads / 32) {
-    const uint4* fr = reinterpret_cast<const uint4*>(fq + (size_t)f * E);
-    float dot = 0.f, ff = 0.f;
+  for (int f0 = warp; f0 < F; f0 += NW * kClipUnroll) {
+    float dot[kClipUnroll], ff[kClipUnroll];
+#pragma unroll
+    for (int u = 0; u < kClipUnroll; ++u) dot[u] = ff[u] = 0.f;
     for (int c = lane; c < nchunk; c += 32) {
-      const uint4 raw = __ldg(fr + c);
-      const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
       const float4 ea = *reinterpret_cast<const float4*>(&e_s[8 * c]);
       const float4 eb = *reinterpret_cast<const float4*>(&e_s[8 * c + 4]);
-      const float2 f0 = __half22float2(h2[0]), f1 = __half22float2(h2[1]);
-      const float2 f2 = __half22float2(h2[2]), f3 = __half22float2(h2[3]);
-      dot = fmaf(ea.x, f0.x, dot); dot = fmaf(ea.y, f0.y, dot);
-      dot = fmaf(ea.z, f1.x, dot); dot = fmaf(ea.w, f1.y, dot);
-      dot = fmaf(eb.x, f2.x, dot); dot = fmaf(eb.y, f2.y, dot);
-      dot = fmaf(eb.z, f3.x, dot); dot = fmaf(eb.w, f3.y, dot);
-      ff = fmaf(f0.x, f0.x, ff); ff = fmaf(f0.y, f0.y, ff);
-      ff = fmaf(f1.x, f1.x, ff); ff = fmaf(f1.y, f1.y, ff);
-      ff = fmaf(f2.x, f2.x, ff); ff = fmaf(f2.y, f2.y, ff);
-      ff = fmaf(f3.x, f3.x, ff); ff = fmaf(f3.y, f3.y, ff);
+      uint4 raw[kClipUnroll];
+#pragma unroll
+      for (int u = 0; u < kClipUnroll; ++u) {
+        const int f = f0 + u * NW;
+        raw[u] = f < F ? __ldg(reinterpret_cast<const uint4*>(fq + (size_t)f * E) + c)
+                       : make_uint4(0, 0, 0, 0);
+      }
+#pragma unroll
+      for (int u = 0; u < kClipUnroll; ++u) {
+        const __half2* h2 = reinterpret_cast<const __half2*>(&raw[u]);
+        const float2 f0v = __half22float2(h2[0]), f1v = __half22float2(h2[1]);
+        const float2 f2v = __half22float2(h2[2]), f3v = __half22float2(h2[3]);
+        float d = dot[u], n = ff[u];
+        d = fmaf(ea.x, f0v.x, d); d = fmaf(ea.y, f0v.y, d);
+        d = fmaf(ea.z, f1v.x, d); d = fmaf(ea.w, f1v.y, d);
+        d = fmaf(eb.x, f2v.x, d); d = fmaf(eb.y, f2v.y, d);
+        d = fmaf(eb.z, f3v.x, d); d = fmaf(eb.w, f3v.y, d);
+        n = fmaf(f0v.x, f0v.x, n); n = fmaf(f0v.y, f0v.y, n);
+        n = fmaf(f1v.x, f1v.x, n); n = fmaf(f1v.y, f1v.y, n);
+        n = fmaf(f2v.x, f2v.x, n); n = fmaf(f2v.y, f2v.y, n);
+        n = fmaf(f3v.x, f3v.x, n); n = fmaf(f3v.y, f3v.y, n);
+        dot[u] = d;
+        ff[u] = n;
+      }
     }
-    dot = warp_sum(dot);
-    ff = warp_sum(ff);
-    const float c = (ff > 0.f && inv_e > 0.f) ? dot * inv_e * rsqrtf(ff) : 0.f;
-    if (lane == 0) {
-      if (cos_out) cos_out[(size_t)qk * F + f] = c;
-      if (c > wbest) {  // frames arrive in increasing order per warp: strict > keeps the lowest
-        wbest = c;
-        wbest_i = f;
+#pragma unroll
+    for (int u = 0; u < kClipUnroll; ++u) {
+      const int f = f0 + u * NW;
+      const float dsum = warp_sum(dot[u]);
+      const float nsum = warp_sum(ff[u]);
+      if (f < F && lane == 0) {
+        const float c = (nsum > 0.f && inv_e > 0.f) ? dsum * inv_e * rsqrtf(nsum) : 0.f;
+        if (cos_out) cos_out[(size_t)qk * F + f] = c;
+        if (c > wbest) {  // a warp sees its frames in increasing order: strict > keeps the lowest
+          wbest = c;
+          wbest_i = f;
+        }
       }
     }
   }
@@ -94,8 +114,8 @@ __global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
   }
   __syncthreads();
   if (warp == 0) {
-    float v = lane < kClipThreads / 32 ? best_v[lane] : -INFINITY;
-    int i = lane < kClipThreads / 32 ? best_i[lane] : 0x7fffffff;
+    float v = lane < NW ? best_v[lane] : -INFINITY;
+    int i = lane < NW ? best_i[lane] : 0x7fffffff;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
       const float ov = __shfl_xor_sync(0xffffffffu, v, o);
@@ -130,6 +150,7 @@ __global__ void select_kernel(const float* __restrict__ logprob, const int32_t* 
       const float* lp = logprob + qk * L * G;
       if (mode == FVRAG_SEL_MASKED_MEAN_LOGPROB) {
         double acc = 0.0;
+  #pragma unroll 8
         for (int l = 0; l < n; ++l) acc += (double)lp[(size_t)l * G];
         s = acc / (double)n;
       } else {

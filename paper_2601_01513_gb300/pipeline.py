@@ -118,6 +118,24 @@ class VerifyStep:
         self.clip(stream)
         self.select(stream)
 
+    def capture(self):
+        """Captures the four calls into one CUDA graph; ``replay`` then issues the whole step
+        with a single launch.  Buffers are fixed: later uploads must copy into them in place."""
+        torch.cuda.synchronize(self.device)
+        self.run()                      # first calls set kernel attributes outside the capture
+        torch.cuda.synchronize(self.device)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, capture_error_mode="thread_local"):
+            self.run()
+        self.graph = g
+        return g
+
+    def replay(self):
+        if getattr(self, "graph", None) is not None:
+            self.graph.replay()
+        else:
+            self.run()
+
     def launches_per_step(self) -> int:
         """Kernels this library launches per step: attention prefix (if any prefix) + tail/merge,
         LM head + merge, CLIP, select."""
@@ -131,7 +149,10 @@ class VerifyStep:
         for name, x in host.items():
             self.t[name].copy_(x, non_blocking=True)
             h2d += x.numel() * x.element_size()
-        self.run(stream)
+        if stream is None:
+            self.replay()
+        else:
+            self.run(stream)
         if getattr(self, "_sel_h", None) is None:
             self._sel_h = torch.empty(self.selected.shape, dtype=self.selected.dtype, pin_memory=True)
             self._sc_h = torch.empty(self.score.shape, dtype=self.score.dtype, pin_memory=True)

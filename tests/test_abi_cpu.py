@@ -65,6 +65,8 @@ def test_attn_validation(L):
     assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 5, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
     assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 96, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
     assert _attn(L, fvrag.AttnDesc(1, 5, 65, 28, 4, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, -1.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, float("nan"), 0)) == fvrag.ERR_INVALID_ARG
     assert _attn(L, good, q=PMIS) == fvrag.ERR_MISALIGNED
     assert _attn(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE
     assert _attn(L, good, ws=None) == fvrag.ERR_WORKSPACE

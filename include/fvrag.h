@@ -114,7 +114,7 @@ fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* q, const vo
                                void* ws, size_t ws_bytes, fvrag_stream_t stream);
 
 /* ------------------------------------------------------------------------ *
- * 2. LM-head log-probabilities (Eq. 11; the verifier likelihood of Section 4.5)
+ * 2. LM-head log-probabilities (Eq. 11; the verifier likelihood of Section 4.6)
  *
  *   z[m][v]        = sum_h hidden[m][h] * weight[v][h]   (bf16 x bf16, fp32 accumulate)
  *   lse[m]         = log sum_v exp(z[m][v])              (natural log)
@@ -198,7 +198,7 @@ fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
  * 4. Candidate selection
  *
  * FVRAG_SEL_MASKED_MEAN_LOGPROB: score_k = (sum_{l < n_k} logprob[k][l][0]) / n_k
- *   (the verifier's own length-normalised likelihood, Section 4.5); selected =
+ *   (the verifier's own length-normalised likelihood, Section 4.6); selected =
  *   argmax over candidates with keep = 1, lowest index on ties, -1 if none.
  * FVRAG_SEL_TWO_STAGE (Algorithm 1): with lpY = logprob[k][n_k-1][0] and
  *   lpN = logprob[k][n_k-1][1], score_k = 1 / (1 + exp(lpN - lpY)) = pY/(pY+pN)

@@ -13,15 +13,16 @@
  * independent output rows).
  *
  * Functions and the passages they follow:
- *   oracle_verify_attn    -- the verifier forward of Eq. 6 / Eq. 11 (Section 3.1,
- *                            "Two-Stage Verification") restricted to one
- *                            attention layer: every candidate token attends to
+ *   oracle_verify_attn    -- the verifier forward of Eq. 6 (Section 3.1) and
+ *                            Eq. 11 (Section 3.2, "Two-Stage Verification")
+ *                            restricted to one attention layer: every
+ *                            candidate token attends to
  *                            the shared prefix (Q, V, retrieved passages) and to
  *                            its own candidate's tokens up to itself.
  *   oracle_score_logprobs -- the verifier's token probabilities P(token | ...):
  *                            log-softmax of the LM-head logits, gathered at the
  *                            requested token ids (Eq. 11; "self-consistent"
- *                            likelihood, Section 4.5 "Analysis of Scoring
+ *                            likelihood, Section 4.6 "Analysis of Scoring
  *                            Mechanisms").
  *   oracle_clip_align     -- Eq. 14 (cosine of CLIP embeddings) and Eq. 15 (max
  *                            over the frames), plus the keep/drop threshold.
@@ -315,7 +316,7 @@ int oracle_clip_align(int Qn, int K, int F, int E, double tau, const uint16_t* c
  *
  * mode 0 (masked mean log-prob): score_k = (sum_{l < n_k} logprob[k][l][0]) / n_k,
  *   the verifier's own likelihood of the candidate normalised by its length
- *   (Section 4.5 "self-consistent"); selected = argmax of score over candidates
+ *   (Section 4.6 "self-consistent"); selected = argmax of score over candidates
  *   with keep = 1, lowest index on ties, -1 when none is kept.
  * mode 1 (Algorithm 1): with lp_Y = logprob[k][n_k-1][0] and lp_N = logprob[k][n_k-1][1]
  *   (the first generated token after the candidate), Eq. 12 gives

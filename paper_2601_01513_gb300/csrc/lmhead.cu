@@ -1,5 +1,5 @@
 // K2: verifier LM-head log-probabilities (Eq. 11; the verifier likelihood of
-// Section 4.5) as one tcgen05 GEMM with a fused online log-sum-exp and target
+// Section 4.6) as one tcgen05 GEMM with a fused online log-sum-exp and target
 // gather, so the [rows x vocab] logits never leave the SM.
 //
 // Shape of the work: z = hidden[M x H] * W[V x H]^T with M (candidate tokens)

@@ -39,29 +39,28 @@ namespace attn {
 
 constexpr int kThreads = 192;
 constexpr int kBM = 128;          // query rows per tile (MMA M)
-constexpr int kBN = 64;           // keys per block
-constexpr int kStages = 5;       // depth of each of the K ring and the V ring
+constexpr int kBN = 128;          // keys per block (MMA N of S, K of PV)
+constexpr int kStages = 3;        // depth of each of the K ring and the V ring
 constexpr int kMaxTail = 64;
-constexpr uint32_t kTmemCols = 256;
-// tensor-memory columns: S buffers at 0 and 64, the O accumulator at 128
-__device__ __forceinline__ uint32_t col_s(int b) { return (uint32_t)b * 64u; }
-constexpr uint32_t kColO = 128;
+constexpr uint32_t kTmemCols = 512;
+// tensor-memory columns: S/P buffers at 0 and 128 (S_j as fp32 in 128 columns, then
+// P_j as packed bf16 in the first 64), the O accumulator at 256
+__device__ __forceinline__ uint32_t col_s(int b) { return (uint32_t)b * 128u; }
+constexpr uint32_t kColO = 256;
 constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (P stays < 2^8)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
-enum : uint32_t { kSiteQ = 0x101, kSiteKvFull = 0x102, kSiteKvEmpty = 0x103, kSiteSFree = 0x104,
-                  kSitePFull = 0x105, kSiteSFull = 0x107, kSitePFree = 0x108, kSiteOFull = 0x109,
-                  kSiteDrain = 0x10A };
+enum : uint32_t { kSiteQ = 0x101, kSiteMma = 0x102, kSiteProducer = 0x103, kSiteSFull = 0x107,
+                  kSitePvDone = 0x109, kSiteDrain = 0x10A };
 
 template <int D>
 struct Layout {
   static constexpr int NH = D / 64;                 // 128-byte column halves of a row
   static constexpr int kQ = NH * kBM * 128;         // Q tile
-  static constexpr int kKVHalf = kBN * 128;         // 64 keys x 64 elements
+  static constexpr int kKVHalf = kBN * 128;         // 128 keys x 64 elements
   static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
-  static constexpr int kP = kBM * 128;              // 128 rows x 64 keys bf16
-  static constexpr int kBytes = kQ + 2 * kStages * kStage + 2 * kP + 1024 + 256;
+  static constexpr int kBytes = kQ + 2 * kStages * kStage + 1024 + 256;
 };
 
 struct Args {
@@ -95,7 +94,7 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 }
 
 // Makes this thread's generic-proxy shared-memory writes visible to the async
-// proxy (the tensor cores read P from shared memory).
+// proxy (the tensor cores read Q from shared memory).
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -126,20 +125,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* q_s = smem;
   uint8_t* k_ring = q_s + Lay::kQ;                    // [kStages][kStage]
   uint8_t* v_ring = k_ring + kStages * Lay::kStage;   // [kStages][kStage]
-  uint8_t* p_s = v_ring + kStages * Lay::kStage;      // [2][kP]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(p_s + 2 * Lay::kP);
-  uint64_t* k_full = bars;                        // [kStages]
-  uint64_t* k_empty = bars + kStages;             // [kStages]
-  uint64_t* v_full = bars + 2 * kStages;          // [kStages]
-  uint64_t* v_empty = bars + 3 * kStages;         // [kStages]
-  uint64_t* s_full = bars + 4 * kStages;          // [2]
-  uint64_t* s_free = s_full + 2;                  // [2]
-  uint64_t* p_full = s_full + 4;                  // [2]
-  uint64_t* p_free = s_full + 6;                  // [2]
-  uint64_t* q_full = s_full + 8;
-  uint64_t* drain = s_full + 9;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(s_full + 10);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(v_ring + kStages * Lay::kStage);
+  uint64_t* k_full = bars;                        // [kStages]  TMA -> MMA
+  uint64_t* k_empty = bars + kStages;             // [kStages]  MMA (S done) -> TMA
+  uint64_t* v_full = bars + 2 * kStages;          // [kStages]  TMA -> MMA
+  uint64_t* v_empty = bars + 3 * kStages;         // [kStages]  MMA (PV done) -> TMA
+  uint64_t* s_full = bars + 4 * kStages;          // [2]  S_j in tensor memory
+  uint64_t* p_full = s_full + 2;                  // [2]  P_j in tensor memory (4 warps)
+  uint64_t* pv_done = s_full + 4;                 // [2]  PV_j done: S/P buffer free
+  uint64_t* q_full = s_full + 6;
+  uint64_t* drain = s_full + 7;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(s_full + 8);
 
+  griddep_wait();                 // inputs may come from the previous kernel
   // ---- work item
   int b = blockIdx.x;
   const int mt = b % a.mtiles;
@@ -170,9 +168,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
-      mbar_init(smem_u32(&s_free[s]), 4);
       mbar_init(smem_u32(&p_full[s]), 4);
-      mbar_init(smem_u32(&p_free[s]), 1);
+      mbar_init(smem_u32(&pv_done[s]), 1);
     }
     mbar_init(smem_u32(q_full), 1);
     mbar_init(smem_u32(drain), 1);
@@ -243,7 +240,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (moved) {
           t_last = globaltimer_ns();
         } else if (globaltimer_ns() - t_last > a.limit_ns) {
-          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteKvEmpty);
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteProducer);
           break;
         }
       }
@@ -256,8 +253,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    // Event-driven: S_ns = Q K_ns^T as soon as K_ns is in and the S buffer is free;
-    // O += P_np V_np as soon as the softmax warps published P_np and V_np is in.
+    //   S_ns  = Q K_ns^T         into S/P buffer ns & 1, once K_ns is in and PV_{ns-2}
+    //                            (the previous user of that buffer) is done;
+    //   O    += P_np V_np        with P_np read from tensor memory, once the softmax
+    //                            warps published P_np and V_np is in.
     if (lane == 0 && nblk > 0) {
       const uint32_t idS = idesc_bf16_f32(kBM, kBN);
       const uint32_t idPV = idesc_bf16_f32(kBM, D) | (1u << 16);   // B (= V) MN-major
@@ -269,8 +268,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint64_t t_last = globaltimer_ns();
         while (np < nblk) {
           bool moved = false;
-          if (ns < nblk && mbar_test(smem_u32(&k_full[ns % kStages]), (ns / kStages) & 1) &&
-              mbar_test(smem_u32(&s_free[ns & 1]), ((ns >> 1) & 1) ^ 1)) {
+          if (ns < nblk && ns < np + 2 &&
+              mbar_test(smem_u32(&k_full[ns % kStages]), (ns / kStages) & 1) &&
+              mbar_test(smem_u32(&pv_done[ns & 1]), ((ns >> 1) & 1) ^ 1)) {
             tc_fence_after();
             const uint32_t ks = smem_u32(k_ring + (ns % kStages) * Lay::kStage);
 #pragma unroll
@@ -289,13 +289,14 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (np < ns && mbar_test(smem_u32(&p_full[np & 1]), (np >> 1) & 1) &&
               mbar_test(smem_u32(&v_full[np % kStages]), (np / kStages) & 1)) {
             tc_fence_after();
-            const uint32_t pa = smem_u32(p_s + (np & 1) * Lay::kP);
+            const uint32_t pa = tmem_base + col_s(np & 1);
             const uint32_t vs = smem_u32(v_ring + (np % kStages) * Lay::kStage);
 #pragma unroll
             for (int k16 = 0; k16 < kBN / 16; ++k16)
-              tc_mma_bf16(tmem_base + kColO, desc_kmajor_sw128(pa + k16 * 32),
-                          desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV, (np | k16) != 0);
-            tc_commit(smem_u32(&p_free[np & 1]));   // P buffer free, and "PV_np done"
+              tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
+                             desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
+                             (np | k16) != 0);
+            tc_commit(smem_u32(&pv_done[np & 1]));
             tc_commit(smem_u32(&v_empty[np % kStages]));
             ++np;
             moved = true;
@@ -303,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1)
           if (moved) {
             t_last = globaltimer_ns();
           } else if (globaltimer_ns() - t_last > a.limit_ns) {
-            record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePFull);
+            record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
             break;
           }
         }
@@ -314,11 +315,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax / epilogue
-    // Online softmax in base 2 with a lazily updated reference max: P_j is taken
-    // relative to m_ref, which only moves when a row's block max exceeds it by more
-    // than kRescaleLog2 (then O in tensor memory and l are rescaled once).  P values
-    // stay below 2^kRescaleLog2, which bf16 and the fp32 accumulators hold exactly
-    // enough; the result is the same softmax.
+    // One row per thread.  Online softmax in base 2 with a lazily updated reference
+    // max: P_j is taken relative to m_ref, which only moves when a row's block max
+    // exceeds it by more than kRescaleLog2 (then O in tensor memory and l are rescaled
+    // once).  P values stay below 2^kRescaleLog2; the result is the same softmax.
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;                 // tile row = tensor-memory lane
     const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
@@ -329,7 +329,6 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int thi = tlo + lrow + 1;
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
-    const uint32_t prow = (uint32_t)r * 128u;
     for (int j = 0; j < nblk; ++j) {
       const int sb = j & 1;
       if (!mbar_wait(smem_u32(&s_full[sb]), (j >> 1) & 1, a.limit_ns)) {
@@ -338,13 +337,11 @@ __global__ void __launch_bounds__(kThreads, 1)
         break;
       }
       tc_fence_after();
-      uint32_t sr[64];
-      tmem_ld_32x32b_x32(lane_base + col_s(sb), *reinterpret_cast<uint32_t(*)[32]>(&sr[0]));
-      tmem_ld_32x32b_x32(lane_base + col_s(sb) + 32, *reinterpret_cast<uint32_t(*)[32]>(&sr[32]));
+      uint32_t sr[kBN];
+#pragma unroll
+      for (int c0 = 0; c0 < kBN; c0 += 32)
+        tmem_ld_32x32b_x32(lane_base + col_s(sb) + c0, *reinterpret_cast<uint32_t(*)[32]>(&sr[c0]));
       tmem_wait_ld();
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&s_free[sb]));
       int vlo, vhi;   // valid columns of this block for this row
       if (j < nbp) {
         vlo = 0;
@@ -375,50 +372,34 @@ __global__ void __launch_bounds__(kThreads, 1)
       const bool resc = m_ref != m_old && m_old != -INFINITY;
       const float corr = resc ? ex2(m_old - m_ref) : 1.f;
       const float ms = m_ref == -INFINITY ? 0.f : m_ref;
-      // P_j -> shared memory (row r: 64 bf16 = 128 B, 16-byte chunks swizzled by row)
-      if (!mbar_wait(smem_u32(&p_free[sb]), ((j >> 1) & 1) ^ 1, a.limit_ns)) {
-        record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePFree);
-        ok = false;
-        break;
-      }
-      const uint32_t pbuf = smem_u32(p_s + sb * Lay::kP) + prow;
+      // P_j (bf16 pairs) over the first 64 columns of the same buffer; S_j is in registers
       float rsp[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) rsp[u] = 0.f;
-      if (full) {
 #pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          float e[8];
+      for (int c0 = 0; c0 < kBN; c0 += 64) {
+        uint32_t pk[32];
 #pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            e[u] = ex2(fmaf(__uint_as_float(sr[8 * c8 + u]), a.scale_log2, -ms));
-            rsp[u] += e[u];
+        for (int c = 0; c < 64; c += 2) {
+          float e0 = ex2(fmaf(__uint_as_float(sr[c0 + c]), a.scale_log2, -ms));
+          float e1 = ex2(fmaf(__uint_as_float(sr[c0 + c + 1]), a.scale_log2, -ms));
+          if (!full) {
+            e0 = (c0 + c >= vlo && c0 + c < vhi) ? e0 : 0.f;
+            e1 = (c0 + c + 1 >= vlo && c0 + c + 1 < vhi) ? e1 : 0.f;
           }
-          st_shared_v4(pbuf + (uint32_t)((c8 ^ (r & 7)) << 4), pack_bf16(e[0], e[1]),
-                       pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]), pack_bf16(e[6], e[7]));
+          rsp[c & 7] += e0;
+          rsp[(c + 1) & 7] += e1;
+          pk[c / 2] = pack_bf16(e0, e1);
         }
-      } else {
-#pragma unroll
-        for (int c8 = 0; c8 < 8; ++c8) {
-          float e[8];
-#pragma unroll
-          for (int u = 0; u < 8; ++u) {
-            const int c = 8 * c8 + u;
-            const float x = ex2(fmaf(__uint_as_float(sr[c]), a.scale_log2, -ms));
-            e[u] = (c >= vlo && c < vhi) ? x : 0.f;
-            rsp[u] += e[u];
-          }
-          st_shared_v4(pbuf + (uint32_t)((c8 ^ (r & 7)) << 4), pack_bf16(e[0], e[1]),
-                       pack_bf16(e[2], e[3]), pack_bf16(e[4], e[5]), pack_bf16(e[6], e[7]));
-        }
+        tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(c0 / 2), pk);
       }
       const float rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
       l = l * corr + rs;
       if (__any_sync(0xffffffffu, resc)) {
         // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale
         const int i = j - 1;
-        if (!mbar_wait(smem_u32(&p_free[i & 1]), (i >> 1) & 1, a.limit_ns)) {
-          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteOFull);
+        if (!mbar_wait(smem_u32(&pv_done[i & 1]), (i >> 1) & 1, a.limit_ns)) {
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
           ok = false;
           break;
         }
@@ -432,20 +413,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
           tmem_st_32x32b_x32(lane_base + kColO + c0, o);
         }
-        tmem_wait_st();
-        tc_fence_before();
       }
-      fence_proxy_async_smem();
+      tmem_wait_st();
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&p_full[sb]));
     }
     // ---- epilogue: wait for the last PV, normalise O by l
     if (ok && nblk > 0) {
       const int i = nblk - 1;
-      if (!mbar_wait(smem_u32(&p_free[i & 1]), (i >> 1) & 1, a.limit_ns)) {
-        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteOFull);
-        ok = false;
-      }
+      if (!mbar_wait(smem_u32(&pv_done[i & 1]), (i >> 1) & 1, a.limit_ns))
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
       tc_fence_after();
     }
     const int head = g * a.grp + r % a.grp;
@@ -490,20 +468,21 @@ __global__ void __launch_bounds__(kThreads, 1)
         a.part_lse[(size_t)split * nrows + rowid] = lse;
       }
     }
-    (void)ok;
   }
+  griddep_launch_dependents();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
 }
 
-// One warp per (token, head) row: out = sum_s exp(lse_s - LSE) * O_s, LSE = logsumexp_s lse_s.
 template <int D>
 __global__ void merge_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
                              int nsplit, long long nrows, __nv_bfloat16* __restrict__ out,
                              float* __restrict__ lse_out) {
   constexpr int DPL = D / 32;
+  griddep_wait();
+  griddep_launch_dependents();
   const long long row = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= nrows) return;
@@ -549,7 +528,7 @@ struct Plan {
 
 // Key-split plan: pick the number of splits that minimises an estimate of
 // waves x (blocks per CTA + fixed cost) plus the cost of writing and merging the
-// partials (one CTA per SM; a 64-key block is ~0.33 us of tensor-core time).
+// partials (one CTA per SM; a 128-key block is ~0.6 us).
 static Plan make_plan(const fvrag_attn_desc* d, int sms) {
   Plan p;
   p.grp = d->hq / d->hkv;
@@ -569,7 +548,7 @@ static Plan make_plan(const fvrag_attn_desc* d, int sms) {
     const int nse = (nb + per - 1) / per;
     const long long ctas = base * nse;
     const double waves = (double)((ctas + sms - 1) / sms);
-    double t = waves * (per + 6) * 0.33;
+    double t = waves * (per + 3) * 0.6;
     if (nse > 1) t += 3.0 + nse * rows * (d->head_dim + 1) * 8.0 / 8.0e6;
     if (t < best - 1e-9) {
       best = t;
@@ -597,7 +576,9 @@ static fvrag_status launch(const CUtensorMap* maps, const Args& a, long long gri
   if (cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) !=
       cudaSuccess)
     return FVRAG_ERR_CUDA;
-  attn_kernel<D><<<(unsigned)grid, kThreads, sm, s>>>(maps[0], maps[1], maps[2], maps[3], maps[4], a);
+  if (launch_pdl(attn_kernel<D>, dim3((unsigned)grid), dim3(kThreads), (size_t)sm, s, maps[0], maps[1],
+                 maps[2], maps[3], maps[4], a) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
   return launch_status();
 }
 
@@ -692,11 +673,11 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
   if (st != FVRAG_OK || p.nsplit == 1) return st;
   const int wpb = 8;
   const long long blocks = (nrows + wpb - 1) / wpb;
-  if (D == 128)
-    merge_kernel<128><<<(unsigned)blocks, 32 * wpb, 0, s>>>(a.part_o, a.part_lse, p.nsplit, nrows,
-                                                            a.out, lse);
-  else
-    merge_kernel<64><<<(unsigned)blocks, 32 * wpb, 0, s>>>(a.part_o, a.part_lse, p.nsplit, nrows,
-                                                           a.out, lse);
+  const cudaError_t e =
+      D == 128 ? launch_pdl(merge_kernel<128>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
+                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse)
+               : launch_pdl(merge_kernel<64>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
+                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse);
+  if (e != cudaSuccess) return FVRAG_ERR_CUDA;
   return launch_status();
 }

@@ -31,6 +31,8 @@ __global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
   __shared__ float red[kClipThreads / 32];
   __shared__ float best_v[kClipThreads / 32];
   __shared__ int best_i[kClipThreads / 32];
+  griddep_wait();
+  griddep_launch_dependents();
   const int qk = blockIdx.x;
   const int q = qk / K;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -141,6 +143,8 @@ __global__ void select_kernel(const float* __restrict__ logprob, const int32_t* 
                               int K, int L, int G, int mode, double delta, float* __restrict__ score,
                               int32_t* __restrict__ selected) {
   extern __shared__ double sc[];
+  griddep_wait();
+  griddep_launch_dependents();
   const int q = blockIdx.x;
   for (int k = threadIdx.x; k < K; k += blockDim.x) {
     const size_t qk = (size_t)q * K + k;
@@ -208,9 +212,11 @@ extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* c
   if ((int64_t)d->num_queries * d->num_cand > 0x7fffffff) return FVRAG_ERR_UNSUPPORTED;
   if (!aligned16(cand_emb) || !aligned16(frame_emb)) return FVRAG_ERR_MISALIGNED;
   const int blocks = d->num_queries * d->num_cand;
-  clip_align_kernel<<<blocks, kClipThreads, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
-      reinterpret_cast<const __half*>(cand_emb), reinterpret_cast<const __half*>(frame_emb),
-      d->num_cand, d->num_frames, d->dim, d->threshold, cos, max_cos, argmax, keep);
+  if (launch_pdl(clip_align_kernel, dim3(blocks), dim3(kClipThreads), 0,
+                 reinterpret_cast<cudaStream_t>(stream), reinterpret_cast<const __half*>(cand_emb),
+                 reinterpret_cast<const __half*>(frame_emb), d->num_cand, d->num_frames, d->dim,
+                 d->threshold, cos, max_cos, argmax, keep) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
   return launch_status();
 }
 
@@ -227,9 +233,10 @@ extern "C" fvrag_status fvrag_select_candidate(const fvrag_select_desc* d, const
   if (d->mode == FVRAG_SEL_TWO_STAGE && (!max_cos || d->gathers < 2)) return FVRAG_ERR_INVALID_ARG;
   if (d->num_cand > 1024) return FVRAG_ERR_UNSUPPORTED;
   const int threads = ((d->num_cand + 31) / 32) * 32;
-  select_kernel<<<d->num_queries, threads, sizeof(double) * d->num_cand,
-                  reinterpret_cast<cudaStream_t>(stream)>>>(
-      logprob, lengths, keep, max_cos, d->num_cand, d->cand_len, d->gathers, d->mode,
-      (double)d->delta, score, selected);
+  if (launch_pdl(select_kernel, dim3(d->num_queries), dim3(threads), sizeof(double) * d->num_cand,
+                 reinterpret_cast<cudaStream_t>(stream), logprob, lengths, keep, max_cos,
+                 d->num_cand, d->cand_len, d->gathers, d->mode, (double)d->delta, score,
+                 selected) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
   return launch_status();
 }

@@ -25,6 +25,25 @@ bool encode_tmap_bf16(CUtensorMap* map, const void* base, int rank, const uint64
 
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Launches `kernel` with programmatic stream serialization: its launch and
+// prologue may overlap the tail of the previous kernel on the stream; the kernel
+// itself calls griddep_wait() before touching global memory.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
+
 inline fvrag_status launch_status() {
   return cudaGetLastError() == cudaSuccess ? FVRAG_OK : FVRAG_ERR_CUDA;
 }

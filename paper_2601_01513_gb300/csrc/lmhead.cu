@@ -76,7 +76,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     lm_head_kernel(const __grid_constant__ CUtensorMap tm_hidden,
                    const __grid_constant__ CUtensorMap tm_w64,
                    const __grid_constant__ CUtensorMap tm_w16, const int32_t* __restrict__ targets,
-                   int M, int H, int V, int G, float* __restrict__ part_max,
+                   int M, int H, int V, int G, int hrows, float* __restrict__ part_max,
                    float* __restrict__ part_sum, float* __restrict__ tgt_logit, uint32_t* status,
                    uint64_t limit_ns) {
   using C = Cfg<BN, MG>;
@@ -129,6 +129,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     st_max[i] = -INFINITY;
     st_sum[i] = 0.f;
   }
+  if (hrows < kBM) {
+    // A-tile rows the hidden box never fills: zero them once so the (discarded)
+    // accumulator rows they produce stay finite
+    for (int i = threadIdx.x; i < kStages * MG * (kBM - hrows) * 8; i += kThreads) {
+      const int chunk = i & 7, rr = (i >> 3) % (kBM - hrows) + hrows, tile = (i >> 3) / (kBM - hrows);
+      uint4* dst = reinterpret_cast<uint4*>(ring + (tile / MG) * C::kStageBytes +
+                                            (tile % MG) * C::kABytes + rr * 128 + chunk * 16);
+      *dst = make_uint4(0u, 0u, 0u, 0u);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
   if (warp == 1) {
     tmem_alloc(smem_u32(tmem_holder), C::kTmemCols);
     tmem_relinquish();
@@ -137,6 +148,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  griddep_wait();                 // the prologue above touched no global memory
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -152,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int v0 = v_lo + t * BN;
         const int rows16 = (min(BN, v_hi - v0) + 15) & ~15;
         const int mcount = min(MG, mtiles - grp * MG);
-        const uint32_t bytes = mcount * C::kABytes + rows16 * kBK * 2;
+        const uint32_t bytes = mcount * hrows * kBK * 2 + rows16 * kBK * 2;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
             record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
@@ -312,6 +324,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
   }
+  griddep_launch_dependents();    // the merge kernel may start launching
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -324,6 +337,8 @@ __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float*
                                 const float* __restrict__ tgt_logit,
                                 const int32_t* __restrict__ targets, int M, int V, int G, int nparts,
                                 float* __restrict__ logprob, float* __restrict__ lse_out) {
+  griddep_wait();
+  griddep_launch_dependents();
   const int m = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (m >= M) return;
@@ -368,16 +383,17 @@ static size_t ws_bytes(const fvrag_lm_desc* d) {
 template <int BN, int MG>
 static fvrag_status launch(const Plan& p, const CUtensorMap& th, const CUtensorMap& tw64,
                            const CUtensorMap& tw16, const int32_t* targets, const fvrag_lm_desc* d,
-                           float* pmax, float* psum, float* ptgt, uint32_t* status,
+                           int hrows, float* pmax, float* psum, float* ptgt, uint32_t* status,
                            cudaStream_t s) {
   using C = Cfg<BN, MG>;
   auto kern = lm_head_kernel<BN, MG>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
       cudaSuccess)
     return FVRAG_ERR_CUDA;
-  kern<<<p.ctas, kThreads, C::kSmemBytes, s>>>(th, tw64, tw16, targets, d->rows, d->hidden,
-                                               d->vocab, d->gathers, pmax, psum, ptgt, status,
-                                               wait_limit_ns());
+  if (launch_pdl(kern, dim3(p.ctas), dim3(kThreads), (size_t)C::kSmemBytes, s, th, tw64, tw16, targets,
+                 d->rows, d->hidden, d->vocab, d->gathers, hrows, pmax, psum, ptgt, status,
+                 wait_limit_ns()) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
   return launch_status();
 }
 
@@ -408,9 +424,11 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   const Plan p = make_plan(d, sm_count());
   const uint64_t H = (uint64_t)d->hidden, M = (uint64_t)d->rows, V = (uint64_t)d->vocab;
   CUtensorMap th, tw64, tw16;
+  // one M-tile: load only the rows that exist (rounded to 16), not all 128
+  const int hrows = M <= (uint64_t)kBM ? (int)((M + 15) / 16 * 16) : kBM;
   {
     const uint64_t dims[2] = {H, M}, strides[1] = {H * 2};
-    const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)kBM};
+    const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)hrows};
     if (!encode_tmap_bf16(&th, hidden, 2, dims, strides, box, true)) return FVRAG_ERR_CUDA;
   }
   {
@@ -428,13 +446,16 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
 
   fvrag_status st;
   if (p.bn == 256)
-    st = launch<256, 1>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
+    st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else
-    st = launch<128, 2>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
+    st = launch<128, 2>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   if (st != FVRAG_OK) return st;
   const int rows_per_block = 8;
-  lm_merge_kernel<<<(d->rows + rows_per_block - 1) / rows_per_block, 32 * rows_per_block, 0, s>>>(
-      pmax, psum, ptgt, targets, d->rows, d->vocab, d->gathers, p.ctas, logprob, lse);
+  if (launch_pdl(lm_merge_kernel, dim3((d->rows + rows_per_block - 1) / rows_per_block),
+                 dim3(32 * rows_per_block), 0, s, (const float*)pmax, (const float*)psum,
+                 (const float*)ptgt, targets, d->rows, d->vocab, d->gathers, p.ctas, logprob,
+                 lse) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
   return launch_status();
 }
 

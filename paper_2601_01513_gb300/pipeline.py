@@ -57,6 +57,7 @@ class VerifyStep:
         lmd = fvrag.LmDesc(M, cfg.hidden, cfg.vocab, cfg.gathers, 0)
         self.lm_ws = torch.zeros(fvrag.lm_workspace_bytes(lmd), dtype=torch.uint8, device=dev)
         self.attn_ws = None
+        self._side = None
 
     # ---------------------------------------------------------------- inputs
     def upload(self, inputs: dict) -> None:
@@ -112,11 +113,25 @@ class VerifyStep:
                                delta=c.delta, stream=stream)
 
     def run(self, stream=None):
-        """All four calls of one verify step, enqueued on `stream` (default: current)."""
-        self.attention(stream)
-        self.lm_head(stream)
-        self.clip(stream)
-        self.select(stream)
+        """All four calls of one verify step, enqueued on `stream` (default: current).
+
+        The CLIP alignment score does not depend on the verifier forward (Algorithm 1
+        combines the two only at selection), so it runs on a forked side stream while
+        attention and the LM head run on the main stream; selection waits for both."""
+        main = stream if stream is not None else torch.cuda.current_stream(self.device)
+        if self._side is None:
+            self._side = torch.cuda.Stream(device=self.device)
+        fork, join = torch.cuda.Event(), torch.cuda.Event()
+        fork.record(main)
+        self._side.wait_event(fork)
+        with torch.cuda.stream(self._side):
+            self.clip()
+        join.record(self._side)
+        with torch.cuda.stream(main):
+            self.attention()
+            self.lm_head()
+            main.wait_event(join)
+            self.select()
 
     def capture(self):
         """Captures the four calls into one CUDA graph; ``replay`` then issues the whole step

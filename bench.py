@@ -146,6 +146,26 @@ class ClockSampler:
                 "samples": len(sm)}
 
 
+def replica_seed(cfg, rank):
+    """Seed of rank `rank`'s independent replica (each rank verifies its own queries)."""
+    return cfg.seed + 7919 * rank
+
+
+def max_over_ranks(values, device):
+    """Element-wise max of per-rank timings over all ranks (the job time is the slowest rank)."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor(values, dtype=torch.float64, device=device)
+    if dist.is_available() and dist.is_initialized() and dist.get_world_size() > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_throughput(tokens_per_step, steps, world, max_ms):
+    """Whole-job tokens/s: every rank's tokens over the slowest rank's time."""
+    return tokens_per_step * steps * world / (max_ms / 1e3)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -280,7 +300,7 @@ def main():
     fvrag.lib()
 
     # each rank verifies its own queries (independent replica, rank-dependent seed)
-    x = synth.make_inputs(cfg, seed=cfg.seed + 7919 * rank)
+    x = synth.make_inputs(cfg, seed=replica_seed(cfg, rank))
     step = VerifyStep(cfg, device=dev)
     step.upload(x)
     # L2 flush between timed iterations: write a 256 MiB buffer (> the 126.5 MiB L2), then read
@@ -367,14 +387,9 @@ def main():
         total_ms = float(step_ms.sum())
         assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
 
-    if ws_ > 1:
-        t = torch.tensor([total_ms, e2e_ms], dtype=torch.float64, device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms, e2e_ms = float(t[0]), float(t[1])
-
-    tokens = cfg.rows * args.steps * ws_
-    value = tokens / (total_ms / 1e3)
-    e2e_value = tokens / (e2e_ms / 1e3)
+    total_ms, e2e_ms = max_over_ranks([total_ms, e2e_ms], dev)
+    value = job_throughput(cfg.rows, args.steps, ws_, total_ms)
+    e2e_value = job_throughput(cfg.rows, args.steps, ws_, e2e_ms)
     pk, pk_src = peaks()
     alg = algorithmic(cfg)
     names = ["attn", "lm", "clip", "select"]

@@ -47,7 +47,7 @@
 extern "C" {
 #endif
 
-#define FVRAG_ABI_VERSION 1
+#define FVRAG_ABI_VERSION 2
 
 /* cudaStream_t without including the CUDA headers. */
 typedef struct CUstream_st* fvrag_stream_t;
@@ -204,27 +204,48 @@ fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
  *   lpN = logprob[k][n_k-1][1], score_k = 1 / (1 + exp(lpN - lpY)) = pY/(pY+pN)
  *   (Eq. 12); A_H = {k : score_k >= max_j score_j - delta} (Eq. 13); selected =
  *   the k in A_H with the largest max_cos, lowest index on ties.
+ * The other strategies the paper compares share the reliability r_k of Eq. 12 (the
+ * TWO_STAGE score) and the alignment a_k = max_cos of Eq. 15:
+ * FVRAG_SEL_ADDITION ("addition", Section 4.6, Table 3): score_k = r_k + a_k;
+ *   selected = argmax over all candidates.
+ * FVRAG_SEL_INVERT ("invert", Section 4.6, Table 3): filter by alignment first
+ *   (keep_k = 1), then rank by reliability: score_k = r_k, argmax over kept, -1 if none.
+ * FVRAG_SEL_RELIABILITY_ONLY ("w/o ett", Section 4.5, Table 2): score_k = r_k,
+ *   argmax over all candidates.
+ * FVRAG_SEL_ALIGNMENT_ONLY ("w/o rel", Table 2): score_k = a_k, argmax over all.
+ * FVRAG_SEL_RANDOM ("Random", Table 2): selected[q] = floor(u_q * K) with
+ *   u_q = (x_q >> 32) / 2^32 and x_q the q-th output of SplitMix64 seeded with
+ *   `seed` (x_q = mix(seed + (q + 1) * 0x9E3779B97F4A7C15)); score_k = 0.
  * n_k = lengths[q][k] (or L when lengths is NULL); a candidate with n_k outside
  * [1, L] or a NaN score gets score NaN and is never selected.  Sums and the
  * comparisons run in fp64; score is rounded to fp32 on output.
  * ------------------------------------------------------------------------ */
-typedef enum { FVRAG_SEL_MASKED_MEAN_LOGPROB = 0, FVRAG_SEL_TWO_STAGE = 1 } fvrag_sel_mode;
+typedef enum {
+  FVRAG_SEL_MASKED_MEAN_LOGPROB = 0,
+  FVRAG_SEL_TWO_STAGE = 1,
+  FVRAG_SEL_ADDITION = 2,
+  FVRAG_SEL_INVERT = 3,
+  FVRAG_SEL_RELIABILITY_ONLY = 4,
+  FVRAG_SEL_ALIGNMENT_ONLY = 5,
+  FVRAG_SEL_RANDOM = 6
+} fvrag_sel_mode;
 
 typedef struct fvrag_select_desc {
   int32_t num_queries; /* Qn >= 1 */
   int32_t num_cand;    /* K, 1..1024 */
   int32_t cand_len;    /* L >= 1 */
-  int32_t gathers;     /* G: innermost extent of logprob (>= 2 for TWO_STAGE) */
+  int32_t gathers;     /* G: innermost extent of logprob (>= 2 for the reliability modes) */
   int32_t mode;        /* fvrag_sel_mode */
   float delta;         /* Eq. 13 margin (the paper uses 0.05) */
   uint32_t flags;      /* must be 0 */
+  uint64_t seed;       /* FVRAG_SEL_RANDOM only */
 } fvrag_select_desc;
 
 /*
  *   logprob  [Qn][K][L][G] fp32
  *   lengths  [Qn][K] int32, or NULL
- *   keep     [Qn][K] uint8  (required for MASKED_MEAN_LOGPROB)
- *   max_cos  [Qn][K] fp32   (required for TWO_STAGE)
+ *   keep     [Qn][K] uint8  (required for MASKED_MEAN_LOGPROB and INVERT)
+ *   max_cos  [Qn][K] fp32   (required for TWO_STAGE, ADDITION, ALIGNMENT_ONLY)
  *   score    [Qn][K] fp32   written
  *   selected [Qn]    int32  written
  */

@@ -304,64 +304,80 @@ int oracle_clip_align(int Qn, int K, int F, int E, double tau, const uint16_t* c
   return 0;
 }
 
+/* SplitMix64 (Steele, Lea & Flood, OOPSLA 2014), counter form: output n of the
+ * generator seeded with s is mix(s + (n+1) * 0x9E3779B97F4A7C15), mix being the
+ * published finaliser.  Used for the Random selection baseline. */
+static uint64_t oracle_splitmix64(uint64_t s, uint64_t n) {
+  uint64_t z = s + (n + 1ULL) * 0x9E3779B97F4A7C15ULL;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ULL;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBULL;
+  return z ^ (z >> 31);
+}
+
 /*
  * Candidate selection.
  *
  *   logprob [Qn][K][L][G] fp64   per-token log-probabilities (gather g)
  *   lengths [Qn][K] int32 or NULL  valid tokens n_k per candidate (default L)
- *   keep    [Qn][K] uint8          CLIP filter decision          (mode 0)
- *   max_cos [Qn][K] fp64           alignment score of Eq. 15     (mode 1)
- *   score   [Qn][K] fp64           mode 0: mean log-prob; mode 1: reliability
+ *   keep    [Qn][K] uint8          CLIP filter decision          (modes 0, 3)
+ *   max_cos [Qn][K] fp64           alignment score of Eq. 15     (modes 1, 2, 5)
+ *   score   [Qn][K] fp64           the per-candidate score of the mode
  *   selected[Qn]    int32          chosen candidate, or -1
  *
+ * r_k = p_Y / (p_Y + p_N) = 1 / (1 + exp(lp_N - lp_Y)) is the reliability of Eq. 12,
+ * with lp_Y = logprob[k][n_k-1][0] and lp_N = logprob[k][n_k-1][1] (the first
+ * generated token after the candidate); a_k = max_cos[k] is the alignment of Eq. 15.
  * mode 0 (masked mean log-prob): score_k = (sum_{l < n_k} logprob[k][l][0]) / n_k,
- *   the verifier's own likelihood of the candidate normalised by its length
- *   (Section 4.6 "self-consistent"); selected = argmax of score over candidates
- *   with keep = 1, lowest index on ties, -1 when none is kept.
- * mode 1 (Algorithm 1): with lp_Y = logprob[k][n_k-1][0] and lp_N = logprob[k][n_k-1][1]
- *   (the first generated token after the candidate), Eq. 12 gives
- *   score_k = p_Y / (p_Y + p_N) = 1 / (1 + exp(lp_N - lp_Y));
- *   Eq. 13 keeps A_H = { k : score_k >= max_j score_j - delta };
- *   the answer is the k in A_H with the largest max_cos (lowest index on ties).
- * A candidate whose n_k is outside [1, L] or whose score is NaN is never selected.
+ *   the verifier's own likelihood normalised by length (Section 4.6
+ *   "self-consistent"); argmax over candidates with keep = 1, -1 if none.
+ * mode 1 (Algorithm 1): score_k = r_k; Eq. 13 keeps A_H = { k : r_k >= max_j r_j - delta };
+ *   the answer is the k in A_H with the largest a_k.
+ * mode 2 (Section 4.6 "addition"): score_k = r_k + a_k, argmax over all.
+ * mode 3 (Section 4.6 "invert"): filter by alignment (keep = 1), rank by reliability:
+ *   score_k = r_k, argmax over kept, -1 if none.
+ * mode 4 (Section 4.5 ablation "w/o ett"): score_k = r_k, argmax over all.
+ * mode 5 (ablation "w/o rel"): score_k = a_k, argmax over all.
+ * mode 6 (ablation "Random"): selected = floor(((x >> 32) * K) / 2^32) with x the q-th
+ *   SplitMix64 output of `seed`; score_k = 0.
+ * Ties go to the lowest index.  A candidate whose n_k is outside [1, L] or whose
+ * score is NaN is never selected (modes 0-5).
  */
 int oracle_select(int Qn, int K, int L, int G, int mode, double delta, const double* logprob,
                   const int32_t* lengths, const uint8_t* keep, const double* max_cos,
-                  double* score, int32_t* selected) {
+                  double* score, int32_t* selected, uint64_t seed) {
   if (Qn <= 0 || K <= 0 || L <= 0 || G <= 0 || !logprob || !score || !selected) return -1;
-  if (mode == 0 && !keep) return -1;
-  if (mode == 1 && (G < 2 || !max_cos)) return -1;
-  if (mode != 0 && mode != 1) return -1;
+  if (mode < 0 || mode > 6) return -1;
+  if ((mode == 0 || mode == 3) && !keep) return -1;
+  if ((mode == 1 || mode == 2 || mode == 5) && !max_cos) return -1;
+  if ((mode >= 1 && mode <= 4) && G < 2) return -1;
   for (int qi = 0; qi < Qn; ++qi) {
     for (int k = 0; k < K; ++k) {
       const int64_t qk = (int64_t)qi * K + k;
       const int n = lengths ? lengths[qk] : L;
       double sc = NAN;
-      if (n >= 1 && n <= L) {
+      if (mode == 6) {
+        sc = 0.0;
+      } else if (n >= 1 && n <= L) {
         if (mode == 0) {
           double s = 0.0;
           for (int l = 0; l < n; ++l) s += logprob[(qk * L + l) * G + 0];
           sc = s / (double)n;
+        } else if (mode == 5) {
+          sc = max_cos[qk];
         } else {
           const double lpY = logprob[(qk * L + (n - 1)) * G + 0];
           const double lpN = logprob[(qk * L + (n - 1)) * G + 1];
           sc = 1.0 / (1.0 + exp(lpN - lpY));
+          if (mode == 2) sc += max_cos[qk];
         }
       }
       score[qk] = sc;
     }
     int sel = -1;
-    if (mode == 0) {
-      double best = -INFINITY;
-      for (int k = 0; k < K; ++k) {
-        const int64_t qk = (int64_t)qi * K + k;
-        if (!keep[qk] || isnan(score[qk])) continue;
-        if (sel < 0 || score[qk] > best) {
-          best = score[qk];
-          sel = k;
-        }
-      }
-    } else {
+    if (mode == 6) {
+      const uint64_t x = oracle_splitmix64(seed, (uint64_t)qi);
+      sel = (int)(((x >> 32) * (uint64_t)K) >> 32);
+    } else if (mode == 1) {
       double top = -INFINITY;
       for (int k = 0; k < K; ++k) {
         const double s = score[(int64_t)qi * K + k];
@@ -374,6 +390,17 @@ int oracle_select(int Qn, int K, int L, int G, int mode, double delta, const dou
         if (isnan(s) || !(s >= top - delta)) continue; /* Eq. 13 */
         if (sel < 0 || max_cos[qk] > best) {
           best = max_cos[qk];
+          sel = k;
+        }
+      }
+    } else {
+      double best = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const int64_t qk = (int64_t)qi * K + k;
+        if (isnan(score[qk])) continue;
+        if ((mode == 0 || mode == 3) && !keep[qk]) continue;
+        if (sel < 0 || score[qk] > best) {
+          best = score[qk];
           sel = k;
         }
       }

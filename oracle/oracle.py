@@ -18,6 +18,11 @@ _lib = None
 
 SEL_MASKED_MEAN_LOGPROB = 0
 SEL_TWO_STAGE = 1
+SEL_ADDITION = 2
+SEL_INVERT = 3
+SEL_RELIABILITY_ONLY = 4
+SEL_ALIGNMENT_ONLY = 5
+SEL_RANDOM = 6
 
 
 def build(force: bool = False) -> str:
@@ -43,7 +48,7 @@ def _L():
         lib.oracle_score_logprobs.restype = ci
         lib.oracle_clip_align.argtypes = [ci] * 4 + [cd] + [vp] * 6
         lib.oracle_clip_align.restype = ci
-        lib.oracle_select.argtypes = [ci] * 5 + [cd] + [vp] * 6
+        lib.oracle_select.argtypes = [ci] * 5 + [cd] + [vp] * 6 + [ctypes.c_uint64]
         lib.oracle_select.restype = ci
         lib.oracle_decode_bf16.argtypes = [vp, vp, ctypes.c_int64]
         lib.oracle_decode_f16.argtypes = [vp, vp, ctypes.c_int64]
@@ -137,7 +142,8 @@ def clip_align(cand, frames, tau):
     return cosm, mc, am, keep
 
 
-def select(logprob, mode=SEL_MASKED_MEAN_LOGPROB, lengths=None, keep=None, max_cos=None, delta=0.05):
+def select(logprob, mode=SEL_MASKED_MEAN_LOGPROB, lengths=None, keep=None, max_cos=None, delta=0.05,
+           seed=0):
     """logprob [Qn][K][L][G] (any float dtype, widened exactly to fp64).  Returns (score, selected)."""
     lp = _c(logprob, np.float64)
     Qn, K, L, G = lp.shape
@@ -147,7 +153,7 @@ def select(logprob, mode=SEL_MASKED_MEAN_LOGPROB, lengths=None, keep=None, max_c
     score = np.empty((Qn, K), np.float64)
     sel = np.empty(Qn, np.int32)
     rc = _L().oracle_select(Qn, K, L, G, int(mode), float(delta), _p(lp), _p(lengths), _p(keep),
-                            _p(max_cos), _p(score), _p(sel))
+                            _p(max_cos), _p(score), _p(sel), int(seed) & (2**64 - 1))
     if rc != 0:
         raise ValueError("oracle_select: bad arguments")
     return score, sel

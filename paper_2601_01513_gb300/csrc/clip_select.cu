@@ -135,32 +135,46 @@ __global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
   }
 }
 
+// SplitMix64 (Steele, Lea & Flood 2014): output n of the generator seeded with s.
+__device__ __forceinline__ uint64_t splitmix64_at(uint64_t s, uint64_t n) {
+  uint64_t z = s + (n + 1ull) * 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
 // One CTA per query; thread k scores candidate k in fp64 (fixed summation
 // order l = 0 .. n_k-1), then thread 0 runs the selection rule serially
 // (K <= 1024 candidates).
 __global__ void select_kernel(const float* __restrict__ logprob, const int32_t* __restrict__ lengths,
                               const uint8_t* __restrict__ keep, const float* __restrict__ max_cos,
-                              int K, int L, int G, int mode, double delta, float* __restrict__ score,
-                              int32_t* __restrict__ selected) {
+                              int K, int L, int G, int mode, double delta, uint64_t seed,
+                              float* __restrict__ score, int32_t* __restrict__ selected) {
   extern __shared__ double sc[];
   griddep_wait();
   griddep_launch_dependents();
   const int q = blockIdx.x;
+  const double nan = __longlong_as_double(0x7ff8000000000000ll);
   for (int k = threadIdx.x; k < K; k += blockDim.x) {
     const size_t qk = (size_t)q * K + k;
     const int n = lengths ? lengths[qk] : L;
-    double s = __longlong_as_double(0x7ff8000000000000ll);  // NaN
-    if (n >= 1 && n <= L) {
+    double s = nan;
+    if (mode == FVRAG_SEL_RANDOM) {
+      s = 0.0;
+    } else if (n >= 1 && n <= L) {
       const float* lp = logprob + qk * L * G;
       if (mode == FVRAG_SEL_MASKED_MEAN_LOGPROB) {
         double acc = 0.0;
-  #pragma unroll 8
+#pragma unroll 8
         for (int l = 0; l < n; ++l) acc += (double)lp[(size_t)l * G];
         s = acc / (double)n;
+      } else if (mode == FVRAG_SEL_ALIGNMENT_ONLY) {
+        s = (double)max_cos[qk];
       } else {
         const double lpY = lp[(size_t)(n - 1) * G + 0];
         const double lpN = lp[(size_t)(n - 1) * G + 1];
-        s = 1.0 / (1.0 + exp(lpN - lpY));
+        s = 1.0 / (1.0 + exp(lpN - lpY));   // Eq. 12
+        if (mode == FVRAG_SEL_ADDITION) s += (double)max_cos[qk];
       }
     }
     sc[k] = s;
@@ -169,27 +183,31 @@ __global__ void select_kernel(const float* __restrict__ logprob, const int32_t* 
   __syncthreads();
   if (threadIdx.x == 0) {
     int sel = -1;
-    if (mode == FVRAG_SEL_MASKED_MEAN_LOGPROB) {
-      double best = -INFINITY;
-      for (int k = 0; k < K; ++k) {
-        const double s = sc[k];
-        if (!keep[(size_t)q * K + k] || isnan(s)) continue;
-        if (sel < 0 || s > best) {
-          best = s;
-          sel = k;
-        }
-      }
-    } else {
+    if (mode == FVRAG_SEL_RANDOM) {
+      const uint64_t x = splitmix64_at(seed, (uint64_t)q);
+      sel = (int)(((x >> 32) * (uint64_t)K) >> 32);
+    } else if (mode == FVRAG_SEL_TWO_STAGE) {
       double top = -INFINITY;
       for (int k = 0; k < K; ++k)
         if (!isnan(sc[k]) && sc[k] > top) top = sc[k];
       float best = -INFINITY;
       for (int k = 0; k < K; ++k) {
         const double s = sc[k];
-        if (isnan(s) || !(s >= top - delta)) continue;
+        if (isnan(s) || !(s >= top - delta)) continue;   // Eq. 13
         const float a = max_cos[(size_t)q * K + k];
         if (sel < 0 || a > best) {
           best = a;
+          sel = k;
+        }
+      }
+    } else {
+      const bool masked = mode == FVRAG_SEL_MASKED_MEAN_LOGPROB || mode == FVRAG_SEL_INVERT;
+      double best = -INFINITY;
+      for (int k = 0; k < K; ++k) {
+        const double s = sc[k];
+        if (isnan(s) || (masked && !keep[(size_t)q * K + k])) continue;
+        if (sel < 0 || s > best) {
+          best = s;
           sel = k;
         }
       }
@@ -227,15 +245,20 @@ extern "C" fvrag_status fvrag_select_candidate(const fvrag_select_desc* d, const
   if (!d || !logprob || !score || !selected) return FVRAG_ERR_INVALID_ARG;
   if (d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->gathers < 1 || d->flags != 0)
     return FVRAG_ERR_INVALID_ARG;
-  if (d->mode != FVRAG_SEL_MASKED_MEAN_LOGPROB && d->mode != FVRAG_SEL_TWO_STAGE)
+  const int m = d->mode;
+  if (m < FVRAG_SEL_MASKED_MEAN_LOGPROB || m > FVRAG_SEL_RANDOM) return FVRAG_ERR_INVALID_ARG;
+  const bool needs_keep = m == FVRAG_SEL_MASKED_MEAN_LOGPROB || m == FVRAG_SEL_INVERT;
+  const bool needs_cos = m == FVRAG_SEL_TWO_STAGE || m == FVRAG_SEL_ADDITION ||
+                         m == FVRAG_SEL_ALIGNMENT_ONLY;
+  const bool needs_rel = m == FVRAG_SEL_TWO_STAGE || m == FVRAG_SEL_ADDITION ||
+                         m == FVRAG_SEL_INVERT || m == FVRAG_SEL_RELIABILITY_ONLY;
+  if ((needs_keep && !keep) || (needs_cos && !max_cos) || (needs_rel && d->gathers < 2))
     return FVRAG_ERR_INVALID_ARG;
-  if (d->mode == FVRAG_SEL_MASKED_MEAN_LOGPROB && !keep) return FVRAG_ERR_INVALID_ARG;
-  if (d->mode == FVRAG_SEL_TWO_STAGE && (!max_cos || d->gathers < 2)) return FVRAG_ERR_INVALID_ARG;
   if (d->num_cand > 1024) return FVRAG_ERR_UNSUPPORTED;
   const int threads = ((d->num_cand + 31) / 32) * 32;
   if (launch_pdl(select_kernel, dim3(d->num_queries), dim3(threads), sizeof(double) * d->num_cand,
                  reinterpret_cast<cudaStream_t>(stream), logprob, lengths, keep, max_cos,
-                 d->num_cand, d->cand_len, d->gathers, d->mode, (double)d->delta, score,
+                 d->num_cand, d->cand_len, d->gathers, d->mode, (double)d->delta, d->seed, score,
                  selected) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();

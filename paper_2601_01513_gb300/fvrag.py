@@ -14,6 +14,11 @@ LIB_PATH = os.path.join(HERE, "libfvrag.so")
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_MISALIGNED, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT = range(7)
 SEL_MASKED_MEAN_LOGPROB = 0
 SEL_TWO_STAGE = 1
+SEL_ADDITION = 2
+SEL_INVERT = 3
+SEL_RELIABILITY_ONLY = 4
+SEL_ALIGNMENT_ONLY = 5
+SEL_RANDOM = 6
 WS_HEADER_BYTES = 256
 
 EXPORTED = (
@@ -54,7 +59,8 @@ class ClipDesc(ctypes.Structure):
 class SelectDesc(ctypes.Structure):
     _fields_ = [("num_queries", ctypes.c_int32), ("num_cand", ctypes.c_int32),
                 ("cand_len", ctypes.c_int32), ("gathers", ctypes.c_int32),
-                ("mode", ctypes.c_int32), ("delta", ctypes.c_float), ("flags", ctypes.c_uint32)]
+                ("mode", ctypes.c_int32), ("delta", ctypes.c_float), ("flags", ctypes.c_uint32),
+                ("seed", ctypes.c_uint64)]
 
 
 _lib = None
@@ -173,10 +179,10 @@ def clip_align(cand_emb, frame_emb, threshold, max_cos, argmax, keep, cos=None, 
 
 
 def select_candidate(logprob, score, selected, mode=SEL_MASKED_MEAN_LOGPROB, keep=None, max_cos=None,
-                     lengths=None, delta=0.05, stream=None):
+                     lengths=None, delta=0.05, seed=0, stream=None):
     """logprob [Qn][K][L][G] fp32 -> score [Qn][K] fp32, selected [Qn] int32."""
     Qn, K, L, G = logprob.shape
-    d = SelectDesc(Qn, K, L, G, int(mode), float(delta), 0)
+    d = SelectDesc(Qn, K, L, G, int(mode), float(delta), 0, int(seed) & (2**64 - 1))
     s = lib().fvrag_select_candidate(ctypes.byref(d), _ptr(logprob), _ptr(lengths), _ptr(keep),
                                      _ptr(max_cos), _ptr(score), _ptr(selected), _stream(stream))
     _check(s, "fvrag_select_candidate")

@@ -72,7 +72,7 @@ def run_clip(cand, frames, tau, with_cos=True):
             keep.cpu().numpy())
 
 
-def run_select(lp, mode, keep=None, max_cos=None, lengths=None, delta=0.05):
+def run_select(lp, mode, keep=None, max_cos=None, lengths=None, delta=0.05, seed=0):
     Qn, K, L, G = lp.shape
     score = torch.full((Qn, K), float("nan"), device="cuda")
     sel = torch.full((Qn,), -7, dtype=torch.int32, device="cuda")
@@ -80,7 +80,7 @@ def run_select(lp, mode, keep=None, max_cos=None, lengths=None, delta=0.05):
                            keep=None if keep is None else dev(keep.astype(np.uint8)),
                            max_cos=None if max_cos is None else dev(max_cos.astype(np.float32)),
                            lengths=None if lengths is None else dev(lengths.astype(np.int32)),
-                           delta=delta)
+                           delta=delta, seed=seed)
     torch.cuda.synchronize()
     return score.cpu().numpy(), sel.cpu().numpy()
 

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert L.fvrag_abi_version() == 1
+    assert L.fvrag_abi_version() == 2
     for s in range(7):
         assert fvrag.status_string(s)
     assert fvrag.status_string(99) == "unknown status"
@@ -110,6 +110,14 @@ def test_clip_and_select_validation(L):
     assert L.fvrag_select_candidate(ctypes.byref(s3), P, None, P, P, P, P, None) == fvrag.ERR_INVALID_ARG
     s4 = fvrag.SelectDesc(1, 2000, 16, 1, 0, 0.05, 0)
     assert L.fvrag_select_candidate(ctypes.byref(s4), P, None, P, P, P, P, None) == fvrag.ERR_UNSUPPORTED
+    sel = lambda mode, G, keep, mc: L.fvrag_select_candidate(
+        ctypes.byref(fvrag.SelectDesc(1, 5, 16, G, mode, 0.05, 0, 7)), P, None, keep, mc, P, P, None)
+    assert sel(fvrag.SEL_INVERT, 2, None, P) == fvrag.ERR_INVALID_ARG        # needs keep
+    assert sel(fvrag.SEL_ADDITION, 2, P, None) == fvrag.ERR_INVALID_ARG      # needs max_cos
+    assert sel(fvrag.SEL_ADDITION, 1, P, P) == fvrag.ERR_INVALID_ARG        # needs Yes/No gathers
+    assert sel(fvrag.SEL_ALIGNMENT_ONLY, 1, None, None) == fvrag.ERR_INVALID_ARG
+    assert sel(fvrag.SEL_RANDOM + 1, 2, P, P) == fvrag.ERR_INVALID_ARG       # unknown mode
+    assert ctypes.sizeof(fvrag.SelectDesc) == 40
 
 
 def test_status_calls_reject_null(L):

@@ -195,15 +195,21 @@ def test_clip_edges():
 
 
 # ============================================================ selection
-@pytest.mark.parametrize("mode", [fvrag.SEL_MASKED_MEAN_LOGPROB, fvrag.SEL_TWO_STAGE])
-@pytest.mark.parametrize("Qn,K,L", [(1, 1, 1), (3, 7, 5), (16, 5, 16), (2, 1000, 3)])
+ALL_MODES = [fvrag.SEL_MASKED_MEAN_LOGPROB, fvrag.SEL_TWO_STAGE, fvrag.SEL_ADDITION, fvrag.SEL_INVERT,
+             fvrag.SEL_RELIABILITY_ONLY, fvrag.SEL_ALIGNMENT_ONLY, fvrag.SEL_RANDOM]
+
+
+@pytest.mark.parametrize("mode", ALL_MODES)
+@pytest.mark.parametrize("Qn,K,L", [(1, 1, 1), (3, 7, 5), (16, 5, 16), (2, 1000, 3), (600, 10, 2)])
 def test_select_matches_oracle(mode, Qn, K, L):
     lp, keep, mc = synth.selection_inputs(Qn, K, L, 2, seed=Qn * 31 + K)
     lengths = synth.uniform_i32((Qn, K), 77, 1, 0, L + 2)   # includes invalid 0 and L+1
     delta = float(np.float32(0.05))
+    seed = 0xD1B54A32D192ED03 + Qn
     for lens in (None, lengths):
-        score, sel = run_select(lp, mode, keep=keep, max_cos=mc, lengths=lens, delta=delta)
-        rscore, rsel = oracle.select(lp, mode=mode, lengths=lens, keep=keep, max_cos=mc, delta=delta)
+        score, sel = run_select(lp, mode, keep=keep, max_cos=mc, lengths=lens, delta=delta, seed=seed)
+        rscore, rsel = oracle.select(lp, mode=mode, lengths=lens, keep=keep, max_cos=mc, delta=delta,
+                                     seed=seed)
         assert np.array_equal(np.isnan(score), np.isnan(rscore))
         ok = ~np.isnan(rscore)
         assert np.array_equal(score[ok], rscore[ok].astype(np.float32))   # fp64 on both sides

@@ -366,3 +366,52 @@ def test_selection_permutation_invariance():
                 assert sel2[qi] == -1
             else:
                 assert perm[sel2[qi]] == sel[qi]
+
+
+# ---------------------------------------------------------------- other selection strategies
+def test_selection_strategies_by_hand():
+    rel = [0.9, 0.5, 0.7]
+    cos = np.array([[0.1, 0.6, 0.35]])
+    lp = _two_stage_logprobs(rel)
+    # addition (Section 4.6): r + a = [1.0, 1.1, 1.05]
+    score, sel = oracle.select(lp, mode=oracle.SEL_ADDITION, max_cos=cos)
+    np.testing.assert_allclose(score[0], [1.0, 1.1, 1.05], rtol=0, atol=1e-14)
+    assert sel[0] == 1
+    # invert (Section 4.6): filter by alignment keep, rank by reliability
+    _, sel = oracle.select(lp, mode=oracle.SEL_INVERT, keep=np.array([[0, 1, 1]], np.uint8))
+    assert sel[0] == 2
+    _, sel = oracle.select(lp, mode=oracle.SEL_INVERT, keep=np.zeros((1, 3), np.uint8))
+    assert sel[0] == -1
+    # ablations (Section 4.5, Table 2): reliability only / alignment only
+    score, sel = oracle.select(lp, mode=oracle.SEL_RELIABILITY_ONLY)
+    np.testing.assert_allclose(score[0], rel, rtol=0, atol=1e-14)
+    assert sel[0] == 0
+    score, sel = oracle.select(lp, mode=oracle.SEL_ALIGNMENT_ONLY, max_cos=cos)
+    np.testing.assert_array_equal(score[0], cos[0])
+    assert sel[0] == 1
+    # the case studies under the other rules: alignment alone picks the wrong draft
+    # for the penguin, reliability alone for the cuttlefish (why both stages exist)
+    with open(os.path.join(GOLDEN, "case_penguin.json")) as f:
+        pen = json.load(f)
+    _, sel = oracle.select(_two_stage_logprobs(pen["reliability"]), mode=oracle.SEL_ALIGNMENT_ONLY,
+                           max_cos=np.array([pen["max_cos"]]))
+    assert sel[0] != pen["expected_selected"]
+    with open(os.path.join(GOLDEN, "case_cuttlefish.json")) as f:
+        cut = json.load(f)
+    _, sel = oracle.select(_two_stage_logprobs(cut["reliability"]), mode=oracle.SEL_RELIABILITY_ONLY)
+    assert sel[0] != cut["expected_selected"]
+
+
+def test_random_selection_follows_published_splitmix64():
+    # Vigna's splitmix64.c seeded with 1234567 produces these first three outputs
+    outputs = [6457827717110365317, 3203168211198807973, 9817491932198370423]
+    K = 7
+    lp = np.zeros((3, K, 1, 1))
+    score, sel = oracle.select(lp, mode=oracle.SEL_RANDOM, seed=1234567)
+    assert np.all(score == 0.0)
+    assert list(sel) == [((x >> 32) * K) >> 32 for x in outputs]
+    # roughly uniform over many queries
+    lp = np.zeros((7000, K, 1, 1))
+    _, sel = oracle.select(lp, mode=oracle.SEL_RANDOM, seed=99)
+    counts = np.bincount(sel, minlength=K)
+    assert counts.min() > 850 and counts.max() < 1150

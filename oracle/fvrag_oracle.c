@@ -29,7 +29,13 @@
  *   oracle_select         -- selection: length-normalised likelihood masked by
  *                            keep (mode 0), or Algorithm 1's two stages:
  *                            Eq. 12 reliability, Eq. 13 high-reliability set,
- *                            argmax alignment over it (mode 1).
+ *                            argmax alignment over it (mode 1), and the
+ *                            other strategies of Sections 4.5-4.6 (modes 2-6).
+ *   oracle_frame_topk     -- Eq. 2: each keyframe's most similar corpus texts.
+ *   oracle_aggregate_topk -- Eq. 3: the union of a query's per-keyframe lists
+ *                            and its K best texts.
+ *   oracle_keyframes      -- Eq. 1: colour-histogram similarity of consecutive
+ *                            frames and the keyframe set.
  * Readings where the paper is silent are stated beside each function.
  *
  * Build: gcc -O2 -fopenmp -shared -fPIC fvrag_oracle.c -o libfvrag_oracle.so -lm
@@ -407,5 +413,175 @@ int oracle_select(int Qn, int K, int L, int G, int mode, double delta, const dou
     }
     selected[qi] = sel;
   }
+  return 0;
+}
+
+/*
+ * Video-to-text retrieval, per keyframe (Eq. 2 and the retrieval loop of
+ * Algorithm 1): for every keyframe f, the kf corpus texts t of largest
+ * sim(f, t) = cos(CLIP(f), CLIP(t)).
+ *
+ *   frames  [Fr][E] fp16     CLIP image embeddings of the keyframes
+ *   texts   [Nt][E] fp16     CLIP text embeddings of the document corpus
+ *   top_idx [Fr][kf] int32   text ids, best first; -1 past the Nt-th entry
+ *   top_sim [Fr][kf] fp64    their similarities; -inf where the id is -1
+ * Order: larger similarity first, the smaller text id first among equal
+ * similarities.  cos is 0 when either vector is zero.
+ * Reading: the paper fixes K = 3 retrieved documents per query (Section 4.3)
+ * but not the per-keyframe list length; kf is a parameter.
+ */
+int oracle_frame_topk(int Fr, int Nt, int E, int kf, const uint16_t* frames,
+                      const uint16_t* texts, int32_t* top_idx, double* top_sim) {
+  if (Fr < 0 || Nt <= 0 || E <= 0 || kf <= 0 || (Fr > 0 && (!frames || !top_idx || !top_sim)) ||
+      !texts)
+    return -1;
+  double* tnorm = (double*)malloc(sizeof(double) * (size_t)Nt);
+  if (!tnorm) return -2;
+#pragma omp parallel for schedule(static)
+  for (int64_t t = 0; t < Nt; ++t) {
+    double s = 0.0;
+    for (int i = 0; i < E; ++i) s += dec_f16(texts[t * E + i]) * dec_f16(texts[t * E + i]);
+    tnorm[t] = sqrt(s);
+  }
+  int err = 0;
+#pragma omp parallel
+  {
+    double* sim = (double*)malloc(sizeof(double) * (size_t)Nt);
+    if (!sim) {
+#pragma omp atomic write
+      err = -2;
+    }
+#pragma omp for schedule(dynamic, 1)
+    for (int f = 0; f < Fr; ++f) {
+      if (!sim) continue;
+      const uint16_t* x = frames + (int64_t)f * E;
+      double xx = 0.0;
+      for (int i = 0; i < E; ++i) xx += dec_f16(x[i]) * dec_f16(x[i]);
+      const double xn = sqrt(xx);
+      for (int64_t t = 0; t < Nt; ++t) {
+        const uint16_t* y = texts + t * E;
+        double d = 0.0;
+        for (int i = 0; i < E; ++i) d += dec_f16(x[i]) * dec_f16(y[i]);
+        sim[t] = (xn > 0.0 && tnorm[t] > 0.0) ? d / (xn * tnorm[t]) : 0.0;
+      }
+      /* kf rounds of "best not yet taken"; scanning ids upwards with a strict >
+       * keeps the smallest id among equal similarities */
+      for (int r = 0; r < kf; ++r) {
+        int32_t best = -1;
+        for (int64_t t = 0; t < Nt; ++t) {
+          int taken = 0;
+          for (int p = 0; p < r; ++p)
+            if (top_idx[(int64_t)f * kf + p] == (int32_t)t) taken = 1;
+          if (taken) continue;
+          if (best < 0 || sim[t] > sim[best]) best = (int32_t)t;
+        }
+        top_idx[(int64_t)f * kf + r] = best;
+        top_sim[(int64_t)f * kf + r] = best >= 0 ? sim[best] : -INFINITY;
+      }
+    }
+    free(sim);
+  }
+  free(tnorm);
+  return err;
+}
+
+/*
+ * Video-to-text retrieval, per query (Eq. 3): the texts the query's keyframes
+ * retrieved form the set T; each text of T is scored by the largest similarity
+ * with which one of those keyframes retrieved it, and the Kq best texts of T are
+ * the query's external knowledge T*.
+ *
+ *   frame_offsets [Qn+1]  keyframes of query q: rows frame_offsets[q] .. frame_offsets[q+1]-1
+ *   top_idx, top_sim [Fr][kf]  per-keyframe lists (oracle_frame_topk's layout;
+ *                         entries with id -1 are ignored)
+ *   out_idx [Qn][Kq] int32, out_sim [Qn][Kq] fp64: best first, the smaller id
+ *                         first among equal scores; -1 / -inf past |T|
+ * Reading: Eq. 3 writes sim(f, t) with f free; the f taken is the keyframe
+ * that retrieved t (the best such keyframe when several did).
+ */
+int oracle_aggregate_topk(int Qn, int kf, int Kq, const int32_t* frame_offsets,
+                          const int32_t* top_idx, const double* top_sim, int32_t* out_idx,
+                          double* out_sim) {
+  if (Qn <= 0 || kf <= 0 || Kq <= 0 || !frame_offsets || !out_idx || !out_sim) return -1;
+  for (int q = 0; q < Qn; ++q)
+    if (frame_offsets[q] < 0 || frame_offsets[q + 1] < frame_offsets[q]) return -1;
+  for (int q = 0; q < Qn; ++q) {
+    const int64_t e0 = (int64_t)frame_offsets[q] * kf, e1 = (int64_t)frame_offsets[q + 1] * kf;
+    for (int r = 0; r < Kq; ++r) {
+      int64_t best = -1;
+      for (int64_t e = e0; e < e1; ++e) {
+        const int32_t t = top_idx[e];
+        if (t < 0) continue;
+        int taken = 0;
+        for (int p = 0; p < r; ++p)
+          if (out_idx[(int64_t)q * Kq + p] == t) taken = 1;
+        if (taken) continue;
+        if (best < 0 || top_sim[e] > top_sim[best] ||
+            (top_sim[e] == top_sim[best] && t < top_idx[best]))
+          best = e;
+      }
+      out_idx[(int64_t)q * Kq + r] = best >= 0 ? top_idx[best] : -1;
+      out_sim[(int64_t)q * Kq + r] = best >= 0 ? top_sim[best] : -INFINITY;
+    }
+  }
+  return 0;
+}
+
+/*
+ * Keyframe extraction (Eq. 1 and the first loop of Algorithm 1), with colour
+ * histograms as the inter-frame similarity (Section 3.1).
+ *
+ *   pixels  [T][npix][3] uint8   RGB frames of Nv videos stored back to back
+ *   video_offsets [Nv+1]         frames of video v: video_offsets[v] .. video_offsets[v+1]-1
+ *   hist    [T][512] int32 or NULL  joint colour histogram with 8 levels per
+ *                                channel: bin = 64 * (r / 32) + 8 * (g / 32) + b / 32
+ *   sim     [T] fp64             sim(f_i, f_{i-1}) = sum_b min(h_i[b], h_{i-1}[b]) / npix
+ *   is_key  [T] uint8            sim < theta (Eq. 1)
+ *   key_index [T] int32          ids of the keyframes in frame order, video by video
+ *   key_offsets [Nv+1] int32     keyframes of video v: key_index[key_offsets[v] ..]
+ * Readings: the histogram is the joint RGB histogram above and the similarity is
+ * its normalised intersection (1 for equal colour distributions, 0 for disjoint
+ * ones); the previous frame of a video's first frame is empty, so its
+ * similarity is 0 and it is always a keyframe (theta > 0); the comparison is
+ * the strict < of Eq. 1, taken on the fp64 quotient.
+ */
+int oracle_keyframes(int Nv, int64_t npix, double theta, const int32_t* video_offsets,
+                     const uint8_t* pixels, int32_t* hist, double* sim, uint8_t* is_key,
+                     int32_t* key_index, int32_t* key_offsets) {
+  if (Nv <= 0 || npix <= 0 || !video_offsets || !pixels || !sim || !is_key || !key_index ||
+      !key_offsets || !(theta > 0.0))
+    return -1;
+  for (int v = 0; v < Nv; ++v)
+    if (video_offsets[v] < 0 || video_offsets[v + 1] < video_offsets[v]) return -1;
+  const int T = video_offsets[Nv];
+  int32_t* h = hist ? hist : (int32_t*)malloc(sizeof(int32_t) * 512 * (size_t)(T > 0 ? T : 1));
+  if (!h) return -2;
+#pragma omp parallel for schedule(static)
+  for (int i = 0; i < T; ++i) {
+    int32_t* hi = h + (int64_t)i * 512;
+    for (int b = 0; b < 512; ++b) hi[b] = 0;
+    const uint8_t* p = pixels + (int64_t)i * npix * 3;
+    for (int64_t x = 0; x < npix; ++x) {
+      const int r = p[3 * x] / 32, g = p[3 * x + 1] / 32, b = p[3 * x + 2] / 32;
+      hi[64 * r + 8 * g + b] += 1;
+    }
+  }
+  int32_t nk = 0;
+  for (int v = 0; v < Nv; ++v) {
+    key_offsets[v] = nk;
+    for (int i = video_offsets[v]; i < video_offsets[v + 1]; ++i) {
+      int64_t inter = 0;
+      if (i > video_offsets[v])
+        for (int b = 0; b < 512; ++b) {
+          const int32_t a = h[(int64_t)i * 512 + b], c = h[(int64_t)(i - 1) * 512 + b];
+          inter += a < c ? a : c;
+        }
+      sim[i] = (double)inter / (double)npix;
+      is_key[i] = sim[i] < theta ? 1 : 0;
+      if (is_key[i]) key_index[nk++] = i;
+    }
+  }
+  key_offsets[Nv] = nk;
+  if (!hist) free(h);
   return 0;
 }

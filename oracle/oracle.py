@@ -50,6 +50,12 @@ def _L():
         lib.oracle_clip_align.restype = ci
         lib.oracle_select.argtypes = [ci] * 5 + [cd] + [vp] * 6 + [ctypes.c_uint64]
         lib.oracle_select.restype = ci
+        lib.oracle_frame_topk.argtypes = [ci] * 4 + [vp] * 4
+        lib.oracle_frame_topk.restype = ci
+        lib.oracle_aggregate_topk.argtypes = [ci] * 3 + [vp] * 5
+        lib.oracle_aggregate_topk.restype = ci
+        lib.oracle_keyframes.argtypes = [ci, ctypes.c_int64, cd] + [vp] * 7
+        lib.oracle_keyframes.restype = ci
         lib.oracle_decode_bf16.argtypes = [vp, vp, ctypes.c_int64]
         lib.oracle_decode_f16.argtypes = [vp, vp, ctypes.c_int64]
         _lib = lib
@@ -157,3 +163,59 @@ def select(logprob, mode=SEL_MASKED_MEAN_LOGPROB, lengths=None, keep=None, max_c
     if rc != 0:
         raise ValueError("oracle_select: bad arguments")
     return score, sel
+
+
+def frame_topk(frames, texts, kf):
+    """Eq. 2 per keyframe: returns (top_idx [Fr][kf] int32, top_sim [Fr][kf] fp64)."""
+    frames, texts = _c(frames, np.uint16), _c(texts, np.uint16)
+    Fr, E = frames.shape
+    Nt = texts.shape[0]
+    idx = np.empty((Fr, kf), np.int32)
+    sim = np.empty((Fr, kf), np.float64)
+    rc = _L().oracle_frame_topk(Fr, Nt, E, kf, _p(frames), _p(texts), _p(idx), _p(sim))
+    if rc != 0:
+        raise ValueError("oracle_frame_topk: bad arguments or out of memory")
+    return idx, sim
+
+
+def aggregate_topk(frame_offsets, top_idx, top_sim, Kq):
+    """Eq. 3 per query: returns (idx [Qn][Kq] int32, sim [Qn][Kq] fp64)."""
+    offs = _c(frame_offsets, np.int32)
+    top_idx, top_sim = _c(top_idx, np.int32), _c(top_sim, np.float64)
+    Qn = offs.shape[0] - 1
+    kf = top_idx.shape[1]
+    idx = np.empty((Qn, Kq), np.int32)
+    sim = np.empty((Qn, Kq), np.float64)
+    rc = _L().oracle_aggregate_topk(Qn, kf, Kq, _p(offs), _p(top_idx), _p(top_sim), _p(idx), _p(sim))
+    if rc != 0:
+        raise ValueError("oracle_aggregate_topk: bad arguments")
+    return idx, sim
+
+
+def retrieve(frames, frame_offsets, texts, kf, Kq):
+    """Eq. 2-3 end to end: (frame lists, query lists) as (idx, sim) pairs."""
+    fi, fs = frame_topk(frames, texts, kf)
+    qi, qs = aggregate_topk(frame_offsets, fi, fs, Kq)
+    return fi, fs, qi, qs
+
+
+def keyframes(pixels, video_offsets, theta):
+    """Eq. 1.  pixels [T][npix][3] (or [T][H][W][3]) uint8.
+
+    Returns (hist [T][512] int32, sim [T] fp64, is_key [T] uint8, key_index [n] int32,
+    key_offsets [Nv+1] int32)."""
+    px = _c(pixels, np.uint8)
+    T = px.shape[0]
+    npix = px[0].size // 3 if T > 0 else 1
+    offs = _c(video_offsets, np.int32)
+    Nv = offs.shape[0] - 1
+    hist = np.empty((T, 512), np.int32)
+    sim = np.empty(T, np.float64)
+    key = np.empty(T, np.uint8)
+    kidx = np.empty(max(T, 1), np.int32)
+    koffs = np.empty(Nv + 1, np.int32)
+    rc = _L().oracle_keyframes(Nv, npix, float(theta), _p(offs), _p(px), _p(hist), _p(sim), _p(key),
+                               _p(kidx), _p(koffs))
+    if rc != 0:
+        raise ValueError("oracle_keyframes: bad arguments")
+    return hist, sim, key, kidx[:koffs[-1]].copy(), koffs

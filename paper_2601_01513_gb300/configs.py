@@ -75,3 +75,76 @@ V72B = VerifyConfig(
                 "V=152064, CLIP 10x256x1024")
 
 PRESETS = {c.name: c for c in (TINY, V7B, LONG, BATCH16, V72B)}
+
+
+@dataclass(frozen=True)
+class RetrievalConfig:
+    """Video-to-text retrieval (Section 3.1, Eq. 2-3): ``num_queries`` videos, each
+    with a ragged number of keyframes drawn from ``keyframes_range``, against a
+    corpus of ``num_texts`` CLIP text embeddings of ``dim``; each keyframe keeps
+    its ``k_frame`` most similar texts and each query its ``k_query`` best texts
+    of their union.  ``relevant`` texts per query are planted with similarity
+    c ~ U(0.25, 0.5) to about half of the query's keyframes."""
+    name: str
+    num_queries: int
+    keyframes_range: tuple          # (lo, hi) inclusive keyframes per query
+    num_texts: int
+    dim: int
+    k_frame: int = 3
+    k_query: int = 3                # Section 4.3: k = 3 documents per query
+    relevant: int = 4
+    seed: int = 20260102
+    description: str = ""
+
+    def with_(self, **kw) -> "RetrievalConfig":
+        return replace(self, **kw)
+
+
+RT_TINY = RetrievalConfig(
+    name="retrieve-tiny", num_queries=3, keyframes_range=(1, 6), num_texts=2000, dim=512,
+    description="3 queries x 1-6 keyframes against 2000 texts of dim 512")
+
+RT_16Q_1M = RetrievalConfig(
+    name="retrieve-16q-1m", num_queries=16, keyframes_range=(4, 32), num_texts=1 << 20, dim=768,
+    description="16 queries x 4-32 keyframes against 1,048,576 CLIP ViT-L/14 text embeddings "
+                "(dim 768, fp16)")
+
+RETRIEVAL_PRESETS = {c.name: c for c in (RT_TINY, RT_16Q_1M)}
+
+
+@dataclass(frozen=True)
+class KeyframeConfig:
+    """Keyframe extraction (Section 3.1, Eq. 1): ``num_videos`` RGB videos of
+    ``height`` x ``width`` with a number of frames drawn from ``frames_range``;
+    scenes last an exponential number of frames (mean ``scene_mean`` frames,
+    at least 8), and a scene change is a fade of 8-15 frames with probability
+    ``fade_prob`` (a hard cut otherwise)."""
+    name: str
+    num_videos: int
+    frames_range: tuple             # (lo, hi) inclusive frames per video
+    height: int
+    width: int
+    theta: float = 0.6              # keyframe threshold of Eq. 1
+    scene_mean: float = 75.0        # 2.5 s at 30 frames/s
+    fade_prob: float = 0.3
+    seed: int = 20260103
+    description: str = ""
+
+    @property
+    def npix(self) -> int:
+        return self.height * self.width
+
+    def with_(self, **kw) -> "KeyframeConfig":
+        return replace(self, **kw)
+
+
+KF_TINY = KeyframeConfig(
+    name="keyframe-tiny", num_videos=3, frames_range=(5, 40), height=16, width=24, scene_mean=6.0,
+    description="3 videos of 5-40 frames at 24x16")
+
+KF_720P = KeyframeConfig(
+    name="keyframe-8x720p", num_videos=8, frames_range=(500, 840), height=720, width=1280,
+    description="8 videos of 500-840 frames (16.7-28 s at 30 frames/s, mean 22.3 s) at 1280x720 "
+                "RGB uint8")
+
+KEYFRAME_PRESETS = {c.name: c for c in (KF_TINY, KF_720P)}

@@ -110,3 +110,100 @@ void synth_round_bf16(const double* in, uint16_t* out, int64_t n) {
 #pragma omp parallel for schedule(static)
   for (int64_t i = 0; i < n; ++i) out[i] = f32_to_bf16_rne((float)in[i]);
 }
+
+/* Rows of unit-length vectors: element (r, i) starts as normal variate r*E+i of
+ * the stream, each row is divided by its Euclidean length, then rounded to fp16
+ * (round-to-nearest-even).  Used for CLIP-like text embeddings of a corpus. */
+void synth_fill_unit_rows_f16(uint16_t* out, int64_t rows, int E, uint64_t key) {
+#pragma omp parallel
+  {
+    double* buf = (double*)__builtin_alloca(sizeof(double) * (size_t)E);
+#pragma omp for schedule(static)
+    for (int64_t r = 0; r < rows; ++r) {
+      double ss = 0.0;
+      for (int i = 0; i < E; ++i) {
+        buf[i] = synth_normal_at(key, (uint64_t)(r * E + i));
+        ss += buf[i] * buf[i];
+      }
+      const double inv = ss > 0.0 ? 1.0 / sqrt(ss) : 0.0;
+      for (int i = 0; i < E; ++i) {
+        _Float16 h = (_Float16)(buf[i] * inv);
+        memcpy(&out[r * E + i], &h, 2);
+      }
+    }
+  }
+}
+
+/* Synthetic RGB video frames, out[T][H][W][3] uint8.
+ * A scene is a smooth two-colour gradient (angle, drift per frame) with a disc of
+ * a third colour moving across it; frame t shows scene fa[t] at time ftau[t]
+ * (frames since the scene began), blended with scene fb[t] by weight fw[t]
+ * (a fade), plus uniform noise of amplitude sigma (of scene fa[t]).  The noise of
+ * pixel p of frame t comes from output t * H * W + p of the stream: its bits
+ * 21c .. 21c+20 give channel c a uniform u in [0, 1) and the noise is
+ * sigma * (2u - 1).
+ * scene parameters, 17 doubles each:
+ *   c0[3] c1[3] c2[3] angle drift cx cy vx vy radius sigma
+ * (cx, cy, radius in fractions of the frame; vx, vy in fractions per frame). */
+typedef struct {
+  double ca, sa, ph, cx, cy, rr;
+  const double* sp;
+} scene_state;
+
+static void scene_at(const double* sp, double tau, double H, scene_state* st) {
+  st->sp = sp;
+  st->ca = cos(sp[9]);
+  st->sa = sin(sp[9]);
+  st->ph = sp[10] * tau;
+  st->cx = sp[11] + sp[13] * tau;
+  st->cy = sp[12] + sp[14] * tau;
+  st->cx -= floor(st->cx);
+  st->cy -= floor(st->cy);
+  st->rr = sp[15] * H;
+}
+
+static inline void scene_colour(const scene_state* st, double xn, double yn, double W, double H,
+                                double col[3]) {
+  const double u = xn * st->ca + yn * st->sa + st->ph;
+  double g = u - floor(u);
+  g = g < 0.5 ? 2.0 * g : 2.0 - 2.0 * g;
+  const double dx = (xn - st->cx) * W, dy = (yn - st->cy) * H;
+  const double* sp = st->sp;
+  if (dx * dx + dy * dy < st->rr * st->rr) {
+    col[0] = sp[6]; col[1] = sp[7]; col[2] = sp[8];
+  } else {
+    for (int c = 0; c < 3; ++c) col[c] = sp[c] + (sp[3 + c] - sp[c]) * g;
+  }
+}
+
+void synth_video_frames(uint8_t* out, int T, int H, int W, uint64_t key, const int32_t* fa,
+                        const int32_t* fb, const double* fw, const double* ftau,
+                        const double* scenes) {
+  const int64_t npix = (int64_t)H * W;
+  const double two_m21 = 1.0 / 2097152.0;
+#pragma omp parallel for collapse(2) schedule(static)
+  for (int t = 0; t < T; ++t) {
+    for (int y = 0; y < H; ++y) {
+      scene_state A, B;
+      scene_at(scenes + 17 * (int64_t)fa[t], ftau[t], H, &A);
+      scene_at(scenes + 17 * (int64_t)fb[t], ftau[t], H, &B);
+      const double w = fw[t], sigma = A.sp[16];
+      const double yn = (y + 0.5) / H;
+      for (int x = 0; x < W; ++x) {
+        const double xn = (x + 0.5) / W;
+        double ca[3], cb[3];
+        scene_colour(&A, xn, yn, W, H, ca);
+        if (w > 0.0) scene_colour(&B, xn, yn, W, H, cb);
+        const int64_t p = (int64_t)y * W + x;
+        const uint64_t r = sm64_at(key, (uint64_t)((int64_t)t * npix + p));
+        for (int c = 0; c < 3; ++c) {
+          const double base = w > 0.0 ? (1.0 - w) * ca[c] + w * cb[c] : ca[c];
+          const double u = (double)((r >> (21 * c)) & 0x1FFFFFu) * two_m21;
+          double v = floor(base + sigma * (2.0 * u - 1.0) + 0.5);
+          v = v < 0.0 ? 0.0 : (v > 255.0 ? 255.0 : v);
+          out[(t * npix + p) * 3 + c] = (uint8_t)v;
+        }
+      }
+    }
+  }
+}

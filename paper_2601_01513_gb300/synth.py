@@ -37,7 +37,7 @@ import os
 
 import numpy as np
 
-from .configs import VerifyConfig
+from .configs import KeyframeConfig, RetrievalConfig, VerifyConfig
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 SYNTH_SO = os.path.join(_HERE, "libfvrag_synth.so")
@@ -46,6 +46,8 @@ SYNTH_SO = os.path.join(_HERE, "libfvrag_synth.so")
 S_Q, S_KP, S_VP, S_KT, S_VT, S_HID, S_W, S_TGT = 1, 2, 3, 4, 5, 6, 7, 8
 S_CAND, S_FRAME, S_PLEN, S_PERM, S_PFRAME, S_PC = 9, 10, 11, 12, 13, 14
 S_LOGPROB, S_KEEP, S_MAXCOS, S_LEN = 20, 21, 22, 23
+S_RT_NKF, S_RT_TEXT, S_RT_FRAME, S_RT_REL, S_RT_PICK, S_RT_C = 30, 31, 32, 33, 34, 35
+S_KF_LEN, S_KF_SCENE, S_KF_CUT, S_KF_FADE, S_KF_PARAM, S_KF_NOISE = 40, 41, 42, 43, 44, 45
 
 _lib = None
 
@@ -85,6 +87,10 @@ def _L():
         lib.synth_round_f16.restype = None
         lib.synth_round_bf16.argtypes = [vp, vp, i64]
         lib.synth_round_bf16.restype = None
+        lib.synth_fill_unit_rows_f16.argtypes = [vp, i64, ctypes.c_int, u64]
+        lib.synth_fill_unit_rows_f16.restype = None
+        lib.synth_video_frames.argtypes = [vp] + [ctypes.c_int] * 3 + [u64] + [vp] * 5
+        lib.synth_video_frames.restype = None
         _lib = lib
     return _lib
 
@@ -215,6 +221,119 @@ def selection_inputs(num_queries, num_cand, cand_len, gathers, seed, std=1.0):
     keep = (uniform_f64((num_queries, num_cand), seed, S_KEEP) < 0.6).astype(np.uint8)
     mc = uniform_f64((num_queries, num_cand), seed, S_MAXCOS, -0.2, 0.8)
     return lp.astype(np.float32), keep, mc.astype(np.float32)
+
+
+def unit_rows_f16(rows, dim, seed, stream) -> np.ndarray:
+    """[rows][dim] fp16 bit patterns of unit-length Gaussian directions."""
+    out = np.empty((rows, dim), dtype=np.uint16)
+    _L().synth_fill_unit_rows_f16(out.ctypes.data, rows, dim, stream_key(seed, stream))
+    return out
+
+
+def retrieval_inputs(cfg: RetrievalConfig, seed=None) -> dict:
+    """Keyframe and corpus embeddings for video-to-text retrieval (Eq. 2-3).
+
+    texts [Nt][E] fp16 unit vectors; frames [Fr][E] fp16 unit vectors with
+    frame_offsets [Qn+1].  Each query gets ``cfg.relevant`` relevant text ids; each
+    of its keyframes, with probability 1/2, is replaced by
+    c*t_hat + sqrt(1-c^2)*n_hat with t_hat one of those texts (decoded from fp16),
+    c ~ U(0.25, 0.5) and n_hat the keyframe's own draw made orthogonal to t_hat.
+    Unplanted pairs have cosines of about N(0, 1/sqrt(E)), so a keyframe's best
+    background text over a million sits near 0.18.
+    """
+    seed = cfg.seed if seed is None else seed
+    Qn, E = cfg.num_queries, cfg.dim
+    lo, hi = cfg.keyframes_range
+    nkf = uniform_i32((Qn,), seed, S_RT_NKF, lo, hi + 1)
+    offs = np.zeros(Qn + 1, dtype=np.int32)
+    offs[1:] = np.cumsum(nkf)
+    Fr = int(offs[-1])
+    texts = unit_rows_f16(cfg.num_texts, E, seed, S_RT_TEXT)
+    frames = normal_f64((Fr, E), seed, S_RT_FRAME)
+    rel = uniform_i32((Qn, cfg.relevant), seed, S_RT_REL, 0, cfg.num_texts)
+    pick = uniform_f64((Fr,), seed, S_RT_PICK)
+    cs = uniform_f64((Fr,), seed, S_RT_C, 0.25, 0.5)
+    for q in range(Qn):
+        for f in range(int(offs[q]), int(offs[q + 1])):
+            if pick[f] >= 0.5:
+                continue
+            t = int(rel[q, int(pick[f] * 2 * cfg.relevant) % cfg.relevant])
+            t_hat = texts[t].view(np.float16).astype(np.float64)
+            t_hat = t_hat / np.linalg.norm(t_hat)
+            n = frames[f] - np.dot(frames[f], t_hat) * t_hat
+            c = cs[f]
+            frames[f] = c * t_hat + math.sqrt(1.0 - c * c) * n / np.linalg.norm(n)
+    frames = frames / np.linalg.norm(frames, axis=-1, keepdims=True)
+    return {"frames": round_f16(frames), "frame_offsets": offs, "texts": texts, "relevant": rel}
+
+
+def video_timeline(cfg: KeyframeConfig, seed=None):
+    """Per-frame scene schedule of ``cfg.num_videos`` videos.
+
+    Returns (video_offsets [Nv+1], fa [T], fb [T], fw [T], ftau [T], scenes [S][17]).
+    Scene lengths are max(8, round(-scene_mean * ln u)); at each scene change a
+    fade of 8-15 frames (with probability fade_prob) blends the old scene into the
+    new one linearly, otherwise the cut is hard.
+    """
+    seed = cfg.seed if seed is None else seed
+    lo, hi = cfg.frames_range
+    nfr = uniform_i32((cfg.num_videos,), seed, S_KF_LEN, lo, hi + 1)
+    voffs = np.zeros(cfg.num_videos + 1, dtype=np.int32)
+    voffs[1:] = np.cumsum(nfr)
+    T = int(voffs[-1])
+    ucut = uniform_f64((T + 1,), seed, S_KF_CUT)
+    ufade = uniform_f64((T + 1, 2), seed, S_KF_FADE)
+    fa = np.zeros(T, np.int32)
+    fb = np.zeros(T, np.int32)
+    fw = np.zeros(T, np.float64)
+    ftau = np.zeros(T, np.float64)
+    scene = -1
+    draws = 0
+    for v in range(cfg.num_videos):
+        t = int(voffs[v])
+        end = int(voffs[v + 1])
+        prev = -1
+        while t < end:
+            scene += 1
+            n = max(8, int(round(-cfg.scene_mean * math.log(max(ucut[draws], 1e-300)))))
+            fade = prev >= 0 and ufade[draws, 0] < cfg.fade_prob
+            nf = 8 + int(ufade[draws, 1] * 8) if fade else 0
+            draws += 1
+            for i in range(n):
+                if t >= end:
+                    break
+                fa[t], ftau[t] = scene, float(i)
+                if i < nf:
+                    # fade from the previous scene (continuing its clock) into this one
+                    fa[t], fb[t], fw[t] = prev, scene, (i + 1) / (nf + 1)
+                    ftau[t] = float(i)
+                t += 1
+            prev = scene
+    S = scene + 1
+    u = uniform_f64((S, 17), seed, S_KF_PARAM)
+    scenes = np.empty((S, 17), np.float64)
+    scenes[:, 0:9] = u[:, 0:9] * 255.0                       # c0, c1, c2
+    scenes[:, 9] = u[:, 9] * 2.0 * math.pi                   # gradient angle
+    scenes[:, 10] = (u[:, 10] - 0.5) * 0.02                  # drift, cycles per frame
+    scenes[:, 11:13] = u[:, 11:13]                           # disc centre
+    scenes[:, 13:15] = (u[:, 13:15] - 0.5) * 0.01            # disc velocity per frame
+    scenes[:, 15] = 0.05 + 0.2 * u[:, 15]                    # disc radius (fraction of height)
+    scenes[:, 16] = 2.0 + 8.0 * u[:, 16]                     # noise amplitude
+    return voffs, fa, fb, fw, ftau, scenes
+
+
+def video_frames(cfg: KeyframeConfig, seed=None, out=None):
+    """RGB frames [T][H][W][3] uint8 of the videos of ``video_timeline`` and the offsets."""
+    seed = cfg.seed if seed is None else seed
+    voffs, fa, fb, fw, ftau, scenes = video_timeline(cfg, seed)
+    T = int(voffs[-1])
+    if out is None:
+        out = np.empty((T, cfg.height, cfg.width, 3), dtype=np.uint8)
+    assert out.shape == (T, cfg.height, cfg.width, 3) and out.dtype == np.uint8 and out.flags.c_contiguous
+    _L().synth_video_frames(out.ctypes.data, T, cfg.height, cfg.width, stream_key(seed, S_KF_NOISE),
+                            fa.ctypes.data, fb.ctypes.data, fw.ctypes.data, ftau.ctypes.data,
+                            np.ascontiguousarray(scenes).ctypes.data)
+    return out, voffs
 
 
 def bf16_bits_to_f32(x: np.ndarray) -> np.ndarray:

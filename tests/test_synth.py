@@ -82,3 +82,35 @@ def test_ragged_prefix_lengths():
     p = synth.prefix_lengths(cfg)
     assert p.shape == (16,) and p.min() >= 4096 and p.max() <= 16384
     assert len(set(p.tolist())) > 8
+
+
+def test_unit_rows_and_retrieval_inputs():
+    from paper_2601_01513_gb300 import configs
+    rows = synth.unit_rows_f16(64, 96, 5, 31)
+    norms = np.linalg.norm(rows.view(np.float16).astype(np.float64), axis=1)
+    assert np.all(np.abs(norms - 1.0) < 2e-3)
+    assert np.array_equal(rows, synth.unit_rows_f16(64, 96, 5, 31))
+    cfg = configs.RT_TINY
+    r = synth.retrieval_inputs(cfg)
+    offs = r["frame_offsets"]
+    nkf = np.diff(offs)
+    assert offs[0] == 0 and np.all(nkf >= cfg.keyframes_range[0]) and np.all(nkf <= cfg.keyframes_range[1])
+    assert r["frames"].shape == (offs[-1], cfg.dim) and r["texts"].shape == (cfg.num_texts, cfg.dim)
+    r2 = synth.retrieval_inputs(cfg)
+    assert all(np.array_equal(r[k], r2[k]) for k in r)
+
+
+def test_video_frames_are_seeded_and_follow_the_timeline():
+    from paper_2601_01513_gb300 import configs
+    cfg = configs.KF_TINY
+    voffs, fa, fb, fw, ftau, scenes = synth.video_timeline(cfg)
+    n = np.diff(voffs)
+    assert np.all(n >= cfg.frames_range[0]) and np.all(n <= cfg.frames_range[1])
+    assert np.all((fw >= 0) & (fw < 1)) and scenes.shape[1] == 17
+    for v in range(cfg.num_videos):                  # a video starts on a fresh scene, no fade
+        assert fw[voffs[v]] == 0 and (v == 0 or fa[voffs[v]] != fa[voffs[v] - 1])
+    px, vo = synth.video_frames(cfg)
+    px2, _ = synth.video_frames(cfg)
+    assert px.shape == (voffs[-1], cfg.height, cfg.width, 3) and np.array_equal(px, px2)
+    px3, _ = synth.video_frames(cfg, seed=cfg.seed + 1)
+    assert not np.array_equal(px, px3)

@@ -263,6 +263,203 @@ def cpu_baseline(cfg, x, budget_s):
                       % (reps, nrows, M, cfg.hq, dt)}
 
 
+def _time_calls(fn, stream, steps, dev):
+    """CUDA-event time of `steps` back-to-back calls of fn on `stream` (ms per call, and the list)."""
+    import torch
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(steps)]
+    for i in range(steps):
+        ev[i][0].record(stream)
+        fn()
+        ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    ms = np.array([a.elapsed_time(b) for a, b in ev])
+    return float(ms.mean()), ms
+
+
+def bench_row(args):
+    """One JSON line for the retrieval or keyframe step (1 GPU; other ranks replicate)."""
+    import torch
+    import torch.distributed as dist
+
+    from paper_2601_01513_gb300 import fvrag
+    from paper_2601_01513_gb300.build import build_all
+    from oracle import oracle
+
+    ws_, rank, local = dist_env()
+    if ws_ > 1:
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local if ws_ > 1 else 0)
+    if rank == 0:
+        build_all()
+    if ws_ > 1:
+        dist.barrier()
+    fvrag.lib()
+    pk, pk_src = peaks()
+    stream = torch.cuda.Stream(device=dev)
+    steps = max(3, min(args.steps, 200))
+
+    if args.row == "retrieve":
+        cfg = configs.RT_16Q_1M
+        r = synth.retrieval_inputs(cfg, seed=cfg.seed + 7919 * rank)
+        Fr, E, Nt = r["frames"].shape[0], cfg.dim, cfg.num_texts
+        texts = torch.from_numpy(r["texts"].view(np.int16)).view(torch.float16).to(dev)
+        frames = torch.from_numpy(r["frames"].view(np.int16)).view(torch.float16).to(dev)
+        offs = torch.from_numpy(r["frame_offsets"]).to(dev)
+        inv = torch.empty(Nt, dtype=torch.float32, device=dev)
+        d = fvrag.retrieve_desc(cfg.num_queries, frames, texts, cfg.k_frame, cfg.k_query)
+        ws = torch.zeros(fvrag.retrieve_workspace_bytes(d), dtype=torch.uint8, device=dev)
+        oi = torch.empty((cfg.num_queries, cfg.k_query), dtype=torch.int32, device=dev)
+        os_ = torch.empty((cfg.num_queries, cfg.k_query), dtype=torch.float32, device=dev)
+        h_frames = torch.from_numpy(r["frames"].view(np.int16)).view(torch.float16).pin_memory()
+        h_offs = torch.from_numpy(r["frame_offsets"]).pin_memory()
+        h_oi = torch.empty_like(oi, device="cpu").pin_memory()
+        h_os = torch.empty_like(os_, device="cpu").pin_memory()
+
+        def call():
+            fvrag.retrieve(frames, offs, texts, cfg.k_frame, oi, os_, ws, text_inv_norm=inv,
+                           stream=stream)
+
+        def call_host():
+            frames.copy_(h_frames, non_blocking=True)
+            offs.copy_(h_offs, non_blocking=True)
+            call()
+            h_oi.copy_(oi, non_blocking=True)
+            h_os.copy_(os_, non_blocking=True)
+
+        with torch.cuda.stream(stream):
+            fvrag.embed_inv_norms(texts, inv, stream=stream)      # index build, once per corpus
+            inv_ms, _ = _time_calls(lambda: fvrag.embed_inv_norms(texts, inv, stream=stream),
+                                    stream, 5, dev)
+            for _ in range(args.warmup):
+                call()
+                call_host()
+            torch.cuda.synchronize(dev)
+            with ClockSampler(dev.index or 0) as clk:
+                clk.wait_first()
+                t_ms, _ = _time_calls(call, stream, steps, dev)
+                e_ms, _ = _time_calls(call_host, stream, steps, dev)
+        assert fvrag.read_status(ws) == fvrag.OK
+        units = Fr
+        metric, unit = "keyframes retrieved/s", "keyframes/s"
+        flops = 2.0 * Fr * Nt * E
+        nbytes = Nt * E * 2 + Nt * 4 + Fr * E * 2
+        t_tc = flops / (pk["bf16_tflops_sustained"] * 1e12)
+        t_hbm = nbytes / (pk["hbm_gbs"] * 1e9)
+        if t_tc >= t_hbm:
+            roof = {"bound": "tensor", "achieved": flops / (t_ms * 1e-3) / 1e12,
+                    "peak": pk["bf16_tflops_sustained"], "unit": "TFLOP/s"}
+        else:
+            roof = {"bound": "hbm", "achieved": nbytes / (t_ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"],
+                    "unit": "GB/s"}
+        roof.update({"frac": roof["achieved"] / roof["peak"], "traffic": None,
+                     "kernel": "fvrag retrieve (tcgen05 fp16 GEMM + per-keyframe top-k), timed "
+                               "with its two small merge kernels",
+                     "peak_source": pk_src + (" (fp16 tensor peak = the measured bf16 peak; same "
+                                              "nominal rate)" if t_tc >= t_hbm else ""),
+                     "other_roof_frac": (nbytes / (t_ms * 1e-3) / 1e9) / pk["hbm_gbs"] if t_tc >= t_hbm
+                     else (flops / (t_ms * 1e-3) / 1e12) / pk["bf16_tflops_sustained"]})
+        h2d = Fr * E * 2 + (cfg.num_queries + 1) * 4
+        d2h = cfg.num_queries * cfg.k_query * 8
+        config = {"workload": cfg.description, "name": cfg.name, "keyframes": Fr, "texts": Nt,
+                  "dim": E, "k_frame": cfg.k_frame, "k_query": cfg.k_query,
+                  "l2": "inputs larger than L2 (the 1.6 GB corpus is streamed every call)",
+                  "inv_norm_index_build_ms": inv_ms, "parallelism": "replicas"}
+        dtype = "f16"
+        launches = 3
+        cpu = None
+        if not args.no_cpu_baseline and ws_ == 1:
+            oracle.build()
+            sample = np.arange(0, Fr, max(1, Fr // 4))[:4]
+            t0 = time.perf_counter()
+            fi, fs = oracle.frame_topk(r["frames"][sample], r["texts"], cfg.k_frame)
+            oracle.aggregate_topk(np.array([0, len(sample)], np.int32), fi, fs, cfg.k_query)
+            dt = time.perf_counter() - t0
+            cpu = {"value": len(sample) / dt, "unit": unit, "cores": oracle.max_threads(),
+                   "kind": "oracle", "sample": "%d of %d keyframes scanned against the whole corpus "
+                   "and aggregated, %.1f s" % (len(sample), Fr, dt)}
+    else:
+        cfg = configs.KF_720P
+        px, voffs = synth.video_frames(cfg, seed=cfg.seed + 7919 * rank)
+        T = int(voffs[-1])
+        pixels = torch.from_numpy(px).to(dev)
+        vo = torch.from_numpy(voffs).to(dev)
+        d = fvrag.keyframe_desc(cfg.num_videos, pixels, cfg.theta)
+        ws = torch.zeros(fvrag.keyframes_workspace_bytes(d), dtype=torch.uint8, device=dev)
+        sim = torch.empty(T, dtype=torch.float32, device=dev)
+        key = torch.empty(T, dtype=torch.uint8, device=dev)
+        kidx = torch.empty(T, dtype=torch.int32, device=dev)
+        koffs = torch.empty(cfg.num_videos + 1, dtype=torch.int32, device=dev)
+        h_px = torch.from_numpy(px).pin_memory()
+        h_vo = torch.from_numpy(voffs).pin_memory()
+        h_kidx = torch.empty(T, dtype=torch.int32).pin_memory()
+        h_koffs = torch.empty(cfg.num_videos + 1, dtype=torch.int32).pin_memory()
+
+        def call():
+            fvrag.keyframes(pixels, vo, cfg.theta, sim, key, kidx, koffs, ws, stream=stream)
+
+        def call_host():
+            pixels.copy_(h_px, non_blocking=True)
+            vo.copy_(h_vo, non_blocking=True)
+            call()
+            h_koffs.copy_(koffs, non_blocking=True)
+            h_kidx.copy_(kidx, non_blocking=True)
+
+        steps = max(3, min(steps, 50))
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                call()
+            call_host()
+            torch.cuda.synchronize(dev)
+            with ClockSampler(dev.index or 0) as clk:
+                clk.wait_first()
+                t_ms, _ = _time_calls(call, stream, steps, dev)
+                e_ms, _ = _time_calls(call_host, stream, max(3, steps // 5), dev)
+        assert fvrag.read_status(ws) == fvrag.OK
+        units = T
+        metric, unit = "video frames processed/s", "frames/s"
+        nbytes = T * cfg.npix * 3 + T * 512 * 4
+        roof = {"bound": "hbm", "achieved": nbytes / (t_ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "traffic": None, "peak_source": pk_src,
+                "kernel": "fvrag keyframe histogram (bulk-copy ring + shared-memory histograms), "
+                          "timed with its similarity and compaction kernels"}
+        roof["frac"] = roof["achieved"] / roof["peak"]
+        h2d = T * cfg.npix * 3 + (cfg.num_videos + 1) * 4
+        d2h = T * 4 + (cfg.num_videos + 1) * 4
+        config = {"workload": cfg.description, "name": cfg.name, "frames": T,
+                  "resolution": [cfg.width, cfg.height], "theta": cfg.theta,
+                  "l2": "inputs larger than L2 (14.8 GB of frames per call)", "parallelism": "replicas"}
+        dtype = "u8"
+        launches = 3
+        cpu = None
+        if not args.no_cpu_baseline and ws_ == 1:
+            oracle.build()
+            n = min(T, 90)
+            t0 = time.perf_counter()
+            oracle.keyframes(px[:n], np.array([0, n], np.int32), cfg.theta)
+            dt = time.perf_counter() - t0
+            cpu = {"value": n / dt, "unit": unit, "cores": oracle.max_threads(), "kind": "oracle",
+                   "sample": "the first %d frames of video 0, %.1f s" % (n, dt)}
+
+    t_ms, e_ms = max_over_ranks([t_ms, e_ms], dev)
+    if rank == 0:
+        line = {"metric": metric, "value": units * ws_ / (t_ms * 1e-3), "unit": unit, "n_gpus": ws_,
+                "steps": steps, "warmup": args.warmup, "ms_per_step": t_ms, "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": dtype, "data": "synthetic",
+                "config": config,
+                "e2e": {"value": units * ws_ / (e_ms * 1e-3), "unit": unit, "h2d_bytes_per_step": int(h2d),
+                        "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms},
+                "gpu_launches": launches * (steps * 2 + args.warmup + 1),
+                "roofline": roof, "clocks": clk.summary()}
+        if cpu:
+            line["cpu_baseline"] = cpu
+        print(json.dumps(line), flush=True)
+    if ws_ > 1:
+        dist.destroy_process_group()
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -274,8 +471,13 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=8)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--row", default="verify", choices=["verify", "retrieve", "keyframes"],
+                    help="verify: the verify step (default); retrieve / keyframes: the retrieval "
+                         "(Eq. 2-3) or keyframe (Eq. 1) step on its own workload")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.row != "verify":
+        return bench_row(args)
     cfg = configs.PRESETS[args.config]
 
     if args.impl == "reference":

@@ -20,6 +20,14 @@
  *                           frame embedding, max/argmax over frames, keep flag;
  *   fvrag_select_candidate  the per-query selection reduction.
  *
+ * and the two data-parallel steps before the drafts (Section 3.1, "Multimodal
+ * Retrieval"; Algorithm 1's first two loops):
+ *
+ *   fvrag_keyframes         colour histograms of the video frames, similarity
+ *                           with the previous frame, keyframe set (Eq. 1);
+ *   fvrag_retrieve          CLIP cosine of every keyframe with every corpus text,
+ *                           per-keyframe top-k and per-query top-K (Eq. 2-3).
+ *
  * Conventions shared by every call
  *   - All tensor pointers are DEVICE pointers owned by the caller; the library
  *     never allocates, frees or synchronises (except fvrag_read_status), and
@@ -47,7 +55,7 @@
 extern "C" {
 #endif
 
-#define FVRAG_ABI_VERSION 2
+#define FVRAG_ABI_VERSION 3
 
 /* cudaStream_t without including the CUDA headers. */
 typedef struct CUstream_st* fvrag_stream_t;
@@ -253,6 +261,98 @@ fvrag_status fvrag_select_candidate(const fvrag_select_desc* d, const float* log
                                     const int32_t* lengths, const uint8_t* keep,
                                     const float* max_cos, float* score, int32_t* selected,
                                     fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * 5. Video-to-text retrieval (Eq. 2-3; the retrieval loop of Algorithm 1)
+ *
+ *   sim(f, t)        = <f, t> / (|f| |t|)   CLIP cosine (Eq. 2), 0 when either is 0
+ *   frame list of f  = the k_frame texts of largest sim(f, t), best first, the
+ *                      smaller text id first among equal similarities
+ *   T_q              = the texts in the lists of query q's keyframes, each scored by
+ *                      the largest similarity with which one of them retrieved it
+ *   query list of q  = the k_query best texts of T_q (Eq. 3), same order; id -1 and
+ *                      similarity -inf past |T_q|
+ * The [keyframes x texts] similarity matrix is never written to memory.
+ * ------------------------------------------------------------------------ */
+typedef struct fvrag_retrieve_desc {
+  int32_t num_queries;   /* Qn >= 1 */
+  int32_t num_keyframes; /* Fr = frame_offsets[Qn], 0..2048, with
+                            ceil(Fr / 128) * 128 * k_frame <= 4096 */
+  int32_t num_texts;     /* Nt >= 1 */
+  int32_t dim;           /* E >= 8, multiple of 8 (16-byte rows) */
+  int32_t k_frame;       /* texts kept per keyframe, 1..8 */
+  int32_t k_query;       /* texts kept per query, 1..64 (the paper retrieves 3) */
+  uint32_t flags;        /* must be 0 */
+} fvrag_retrieve_desc;
+
+size_t fvrag_retrieve_workspace(const fvrag_retrieve_desc* d);
+
+/*
+ * inv_norm[r] = 1 / |x_r| (0 for a zero row) for an fp16 matrix x [rows][dim]
+ * (dim a multiple of 8).  Computing the corpus norms is an index-build step: run
+ * it once per corpus and pass the result to every fvrag_retrieve call.
+ */
+fvrag_status fvrag_embed_inv_norms(const void* x, int32_t rows, int32_t dim, float* inv_norm,
+                                   fvrag_stream_t stream);
+
+/*
+ *   frame_emb      [Fr][E] fp16   keyframe CLIP image embeddings, query by query
+ *   frame_offsets  [Qn+1]  int32  device; keyframes of query q are rows
+ *                                 frame_offsets[q] .. frame_offsets[q+1]-1 (non-decreasing,
+ *                                 offsets[0] = 0, offsets[Qn] = Fr; a query whose offsets
+ *                                 fall outside [0, Fr] is treated as empty)
+ *   text_emb       [Nt][E] fp16   corpus CLIP text embeddings
+ *   text_inv_norm  [Nt]    fp32   from fvrag_embed_inv_norms, or NULL (then computed
+ *                                 in the workspace on every call: one more corpus pass)
+ *   frame_topk     [Fr][k_frame] int32, frame_topk_sim [Fr][k_frame] fp32: the
+ *                                 per-keyframe lists, written when not NULL
+ *   out_idx        [Qn][k_query] int32, out_sim [Qn][k_query] fp32: written
+ * Similarities are fp32 from an fp32-accumulated fp16 dot product.
+ */
+fvrag_status fvrag_retrieve(const fvrag_retrieve_desc* d, const void* frame_emb,
+                            const int32_t* frame_offsets, const void* text_emb,
+                            const float* text_inv_norm, int32_t* frame_topk,
+                            float* frame_topk_sim, int32_t* out_idx, float* out_sim, void* ws,
+                            size_t ws_bytes, fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * 6. Keyframe extraction (Eq. 1; the first loop of Algorithm 1)
+ *
+ *   hist[i][b] = number of pixels of frame i in bin b of the joint RGB histogram
+ *                with 8 levels per channel: b = 64 (r / 32) + 8 (g / 32) + b / 32
+ *   sim[i]     = sum_b min(hist[i][b], hist[i-1][b]) / (height * width)
+ *                (histogram intersection with the previous frame of the same video;
+ *                0 for a video's first frame, which has no previous frame)
+ *   is_key[i]  = sim[i] < theta (Eq. 1), the quotient and the comparison in fp64
+ *   key_index  = ids of the frames with is_key = 1 in increasing order; the keyframes
+ *                of video v are key_index[key_offsets[v] .. key_offsets[v+1]-1]
+ * ------------------------------------------------------------------------ */
+typedef struct fvrag_keyframe_desc {
+  int32_t num_videos;   /* Nv >= 1 */
+  int32_t total_frames; /* T = video_offsets[Nv] >= 0 */
+  int32_t height;       /* >= 1 */
+  int32_t width;        /* >= 1; height * width a multiple of 16 (frames start on 16 B) */
+  double theta;         /* > 0 */
+  uint32_t flags;       /* must be 0 */
+} fvrag_keyframe_desc;
+
+size_t fvrag_keyframes_workspace(const fvrag_keyframe_desc* d);
+
+/*
+ *   pixels        [T][height][width][3] uint8  RGB, videos back to back
+ *   video_offsets [Nv+1] int32  device; frames of video v are video_offsets[v] ..
+ *                               video_offsets[v+1]-1 (non-decreasing, offsets[0] = 0,
+ *                               offsets[Nv] = T; not checked on the device)
+ *   hist          [T][512] int32  written when not NULL (else kept in the workspace)
+ *   sim           [T] fp32   written (the fp64 quotient rounded to fp32)
+ *   is_key        [T] uint8  written
+ *   key_index     [T] int32  the first key_offsets[Nv] entries written
+ *   key_offsets   [Nv+1] int32  written
+ */
+fvrag_status fvrag_keyframes(const fvrag_keyframe_desc* d, const uint8_t* pixels,
+                             const int32_t* video_offsets, int32_t* hist, float* sim,
+                             uint8_t* is_key, int32_t* key_index, int32_t* key_offsets, void* ws,
+                             size_t ws_bytes, fvrag_stream_t stream);
 
 /* ------------------------------------------------------------------------ *
  * Device status (failure detection without faulting the GPU)

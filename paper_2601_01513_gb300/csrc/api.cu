@@ -43,8 +43,9 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
-bool encode_tmap_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
-                      const uint64_t* strides_bytes, const uint32_t* box, bool swizzle128) {
+static bool encode_tmap_16bit(CUtensorMap* map, CUtensorMapDataType dtype, const void* base,
+                              int rank, const uint64_t* dims, const uint64_t* strides_bytes,
+                              const uint32_t* box, bool swizzle128) {
   auto fn = encode_fn();
   if (!fn || rank < 1 || rank > 5) return false;
   cuuint64_t gdim[5], gstride[4];
@@ -55,11 +56,23 @@ bool encode_tmap_bf16(CUtensorMap* map, const void* base, int rank, const uint64
     estride[i] = 1;
     if (i > 0) gstride[i - 1] = strides_bytes[i - 1];
   }
-  CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(base),
-                  gdim, gstride, bdim, estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
+  CUresult r = fn(map, dtype, (cuuint32_t)rank, const_cast<void*>(base), gdim, gstride, bdim,
+                  estride, CU_TENSOR_MAP_INTERLEAVE_NONE,
                   swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                   CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
+}
+
+bool encode_tmap_bf16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
+                      const uint64_t* strides_bytes, const uint32_t* box, bool swizzle128) {
+  return encode_tmap_16bit(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, base, rank, dims, strides_bytes,
+                           box, swizzle128);
+}
+
+bool encode_tmap_f16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
+                     const uint64_t* strides_bytes, const uint32_t* box, bool swizzle128) {
+  return encode_tmap_16bit(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, base, rank, dims, strides_bytes,
+                           box, swizzle128);
 }
 
 // One CTA, one thread: waits on a barrier whose phase never completes (its

@@ -1,0 +1,642 @@
+// Video-to-text retrieval (Eq. 2-3, the retrieval loop of Algorithm 1): every
+// keyframe's k_frame most similar corpus texts by CLIP cosine, then per query the
+// k_query best texts of the union of its keyframes' lists.
+//
+// Shape of the work: sim = frames[Fr x E] * texts[Nt x E]^T with Fr (keyframes of
+// a batch of queries) small (1 .. 2048) and the corpus large (1,048,576 x 768
+// fp16 = 1.6 GB).  It is the LM head's shape with a different epilogue, so the
+// kernel has the same structure: a persistent grid, one CTA per SM, each CTA
+// owning a contiguous range of texts (16-row units) and walking it in tiles of
+// BN texts; per tile a tcgen05 GEMM accumulates D[128 x BN] = frames_tile *
+// texts_tile^T in tensor memory (fp16 inputs, fp32 accumulate), K-loop over E
+// in 64-element blocks (one 128-byte swizzled row per operand row).
+//
+// Warp roles (192 threads):
+//   warp 0     TMA producer (frame tiles 64 x 128, text tiles 64 x 64 / 64 x 16)
+//              into a 4-deep shared-memory ring;
+//   warp 1     tensor-memory allocation and the single MMA-issuing lane;
+//   warps 2-5  epilogue: tcgen05.ld of 32 columns (one keyframe per thread),
+//              scale by the text's inverse norm, keep a running top-k_frame list
+//              per keyframe (in shared memory between tiles).  Columns arrive in
+//              increasing text id, so a strict > keeps the smaller id on ties.
+// Two accumulator slots in tensor memory let the epilogue of one tile overlap the
+// MMAs of the next.
+//
+// Two small kernels follow: one merges the per-CTA lists of each keyframe and
+// applies the keyframe's inverse norm (cos = <f, t> / |f| / |t|); one forms each
+// query's union (a text scored by its best retrieving keyframe) and its top
+// k_query.  A fourth, optional kernel computes the corpus inverse norms when the
+// caller does not pass them (fvrag_embed_inv_norms is the same kernel on its own).
+#include <cuda_fp16.h>
+
+#include <algorithm>
+
+#include "fvrag_common.cuh"
+#include "fvrag_internal.h"
+
+namespace fvrag {
+namespace rt {
+
+constexpr int kThreads = 192;
+constexpr int kBK = 64;            // fp16 elements per 128-byte swizzled row
+constexpr int kBM = 128;           // keyframes per M-tile (MMA M)
+constexpr int kStages = 4;
+constexpr int kMaxCtas = 256;
+constexpr int kMaxMTiles = 16;     // keyframes <= 2048
+constexpr int kMaxKf = 8;          // k_frame <= 8
+constexpr int kMaxState = 4096;    // ceil(keyframes / 128) * 128 * k_frame <= 4096 (32 KB of lists)
+constexpr int kMaxKq = 64;
+
+enum : uint32_t { kSiteProdEmpty = 0x601, kSiteMmaTmem = 0x602, kSiteMmaFull = 0x603,
+                  kSiteEpiFull = 0x604, kSiteDrain = 0x605 };
+
+template <int BN, int MG>
+struct Cfg {
+  static constexpr int kABytes = kBM * kBK * 2;
+  static constexpr int kBBytes = BN * kBK * 2;
+  static constexpr int kStageBytes = MG * kABytes + kBBytes;
+  static constexpr int kSlots = 2;
+  static constexpr int kTmemCols = kSlots * MG * BN;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + kMaxState * 8;
+  static_assert(kTmemCols == 512, "tensor memory plan uses all 512 columns");
+  static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+};
+
+// (s, i) ranks before (t, j): larger similarity first, smaller id first on ties.
+__device__ __forceinline__ bool better(float s, int i, float t, int j) {
+  return s > t || (s == t && (unsigned)i < (unsigned)j);  // id -1 ranks last among equals
+}
+
+template <int BN, int MG>
+__global__ void __launch_bounds__(kThreads, 1)
+    retrieve_kernel(const __grid_constant__ CUtensorMap tm_frames,
+                    const __grid_constant__ CUtensorMap tm_t64,
+                    const __grid_constant__ CUtensorMap tm_t16,
+                    const float* __restrict__ text_inv_norm, int M, int E, int Nt, int kf,
+                    int hrows, float* __restrict__ part_sim, int32_t* __restrict__ part_idx,
+                    uint32_t* status, uint64_t limit_ns) {
+  using C = Cfg<BN, MG>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* ring = smem;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + kStages * C::kStageBytes);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + kStages;
+  uint64_t* tfull = bars + 2 * kStages;
+  uint64_t* tempty = tfull + C::kSlots;
+  uint64_t* drain = tempty + C::kSlots;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* st_sim = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);
+  int32_t* st_idx = reinterpret_cast<int32_t*>(st_sim + kMaxState);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  const int nunits = (Nt + 15) >> 4;
+  const int u_lo = (int)(((long long)blockIdx.x * nunits) / gridDim.x);
+  const int u_hi = (int)(((long long)(blockIdx.x + 1) * nunits) / gridDim.x);
+  const int v_lo = u_lo * 16;
+  const int v_hi = min(u_hi * 16, Nt);
+  const int ntiles = (v_hi - v_lo + BN - 1) / BN;
+  const int mtiles = (M + kBM - 1) / kBM;
+  const int ngroups = (mtiles + MG - 1) / MG;
+  const int nitems = ntiles * ngroups;
+  const int kblocks = (E + kBK - 1) / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int s = 0; s < C::kSlots; ++s) {
+      mbar_init(smem_u32(&tfull[s]), 1);
+      mbar_init(smem_u32(&tempty[s]), 4);
+    }
+    mbar_init(smem_u32(drain), 1);
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_frames);
+    tma_prefetch_desc(&tm_t64);
+    tma_prefetch_desc(&tm_t16);
+  }
+  for (int i = threadIdx.x; i < mtiles * kBM * kf; i += kThreads) {
+    st_sim[i] = -INFINITY;
+    st_idx[i] = -1;
+  }
+  if (hrows < kBM) {
+    for (int i = threadIdx.x; i < kStages * MG * (kBM - hrows) * 8; i += kThreads) {
+      const int chunk = i & 7, rr = (i >> 3) % (kBM - hrows) + hrows, tile = (i >> 3) / (kBM - hrows);
+      uint4* dst = reinterpret_cast<uint4*>(ring + (tile / MG) * C::kStageBytes +
+                                            (tile % MG) * C::kABytes + rr * 128 + chunk * 16);
+      *dst = make_uint4(0u, 0u, 0u, 0u);
+    }
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  }
+  if (warp == 1) {
+    tmem_alloc(smem_u32(tmem_holder), C::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  griddep_wait();
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      const uint64_t pol_t = policy_evict_first();
+      const uint64_t pol_f = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int t = it / ngroups, grp = it % ngroups;
+        const int v0 = v_lo + t * BN;
+        const int rows16 = (min(BN, v_hi - v0) + 15) & ~15;
+        const int mcount = min(MG, mtiles - grp * MG);
+        const uint32_t bytes = mcount * hrows * kBK * 2 + rows16 * kBK * 2;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
+            ok = false;
+            break;
+          }
+          const uint32_t fb = smem_u32(&full[stage]);
+          mbar_arrive_expect_tx(fb, bytes);
+          uint8_t* st = ring + stage * C::kStageBytes;
+          for (int j = 0; j < mcount; ++j)
+            tma_load_2d(smem_u32(st + j * C::kABytes), &tm_frames, fb, kb * kBK,
+                        (grp * MG + j) * kBM, pol_f);
+          uint8_t* bsm = st + MG * C::kABytes;
+          int r = 0;
+          for (; r + 64 <= rows16; r += 64)
+            tma_load_2d(smem_u32(bsm + r * 128), &tm_t64, fb, kb * kBK, v0 + r, pol_t);
+          for (; r < rows16; r += 16)
+            tma_load_2d(smem_u32(bsm + r * 128), &tm_t16, fb, kb * kBK, v0 + r, pol_t);
+          ++issued;
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      const int pend = issued < kStages ? (int)issued : kStages;
+      for (int i = 0; i < pend; ++i) {
+        if (--stage < 0) {
+          stage = kStages - 1;
+          phase ^= 1;
+        }
+        mbar_wait(smem_u32(&full[stage]), phase, limit_ns);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int slot = it % C::kSlots;
+        const uint32_t use = it / C::kSlots;
+        const int t = it / ngroups, grp = it % ngroups;
+        const int v0 = v_lo + t * BN;
+        const int rows16 = (min(BN, v_hi - v0) + 15) & ~15;
+        const int mcount = min(MG, mtiles - grp * MG);
+        const uint32_t idesc = idesc_f16_f32(kBM, rows16);
+        if (!mbar_wait(smem_u32(&tempty[slot]), (use & 1) ^ 1, limit_ns)) {
+          record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaTmem);
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait(smem_u32(&full[stage]), phase, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaFull);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(ring + stage * C::kStageBytes);
+          const uint32_t bsm = st + MG * C::kABytes;
+          for (int j = 0; j < mcount; ++j) {
+            const uint32_t d = tmem_base + (uint32_t)((slot * MG + j) * BN);
+#pragma unroll
+            for (int k16 = 0; k16 < kBK / 16; ++k16) {
+              const uint64_t a = desc_kmajor_sw128(st + j * C::kABytes + k16 * 32);
+              const uint64_t b = desc_kmajor_sw128(bsm + k16 * 32);
+              tc_mma_bf16(d, a, b, idesc, (kb | k16) != 0);
+            }
+          }
+          tc_commit(smem_u32(&empty[stage]));
+          if (++stage == kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit(smem_u32(&tfull[slot]));
+      }
+      tc_commit(smem_u32(drain));
+      if (!mbar_wait(smem_u32(drain), 0, limit_ns))
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;
+    for (int it = 0; it < nitems; ++it) {
+      const int slot = it % C::kSlots;
+      const uint32_t use = it / C::kSlots;
+      const int t = it / ngroups, grp = it % ngroups;
+      const int v0 = v_lo + t * BN;
+      const int ncols = min(BN, v_hi - v0);
+      const int rows16 = (ncols + 15) & ~15;
+      const int mcount = min(MG, mtiles - grp * MG);
+      if (!mbar_wait(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
+        break;
+      }
+      tc_fence_after();
+      for (int j = 0; j < mcount; ++j) {
+        const int mt = grp * MG + j;
+        const bool live = mt * kBM + row < M;
+        float* ss = st_sim + (mt * kBM + row) * kf;
+        int32_t* si = st_idx + (mt * kBM + row) * kf;
+        float ls[kMaxKf];
+        int li[kMaxKf];
+#pragma unroll
+        for (int p = 0; p < kMaxKf; ++p) {
+          ls[p] = p < kf ? ss[p] : -INFINITY;
+          li[p] = p < kf ? si[p] : -1;
+        }
+        float thr = ss[kf - 1];
+        const uint32_t tbase =
+            tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * MG + j) * BN);
+        for (int c0 = 0; c0 < rows16; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + c0, r);
+          tmem_wait_ld();
+          const int nvalid = min(32, ncols - c0);
+          if (!live) continue;
+          const float* invp = text_inv_norm + v0 + c0;    // 64-byte aligned: v0 % 16 == 0
+#pragma unroll
+          for (int q4 = 0; q4 < 8; ++q4) {
+            float inv[4];
+            if (q4 * 4 + 4 <= nvalid) {
+              const float4 in4 = __ldg(reinterpret_cast<const float4*>(invp) + q4);
+              inv[0] = in4.x;
+              inv[1] = in4.y;
+              inv[2] = in4.z;
+              inv[3] = in4.w;
+            } else {
+#pragma unroll
+              for (int e = 0; e < 4; ++e) inv[e] = q4 * 4 + e < nvalid ? __ldg(invp + q4 * 4 + e) : 0.f;
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int i = q4 * 4 + e;
+              const float v = __uint_as_float(r[i]) * inv[e];
+              if (i < nvalid && v > thr) {
+                float nv = v;
+                int ni = v0 + c0 + i;
+#pragma unroll
+                for (int p = 0; p < kMaxKf; ++p) {
+                  if (p < kf && better(nv, ni, ls[p], li[p])) {
+                    const float ts = ls[p];
+                    const int ti = li[p];
+                    ls[p] = nv;
+                    li[p] = ni;
+                    nv = ts;
+                    ni = ti;
+                  }
+                }
+#pragma unroll
+                for (int p = 0; p < kMaxKf; ++p)
+                  if (p == kf - 1) thr = ls[p];
+              }
+            }
+          }
+        }
+        if (live) {
+#pragma unroll
+          for (int p = 0; p < kMaxKf; ++p)
+            if (p < kf) {
+              ss[p] = ls[p];
+              si[p] = li[p];
+            }
+        }
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(smem_u32(&tempty[slot]));
+    }
+    for (int mt = 0; mt < mtiles; ++mt) {
+      const int m = mt * kBM + row;
+      if (m < M)
+        for (int p = 0; p < kf; ++p) {
+          part_sim[((size_t)blockIdx.x * M + m) * kf + p] = st_sim[(mt * kBM + row) * kf + p];
+          part_idx[((size_t)blockIdx.x * M + m) * kf + p] = st_idx[(mt * kBM + row) * kf + p];
+        }
+    }
+  }
+  griddep_launch_dependents();
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
+}
+
+// inv_norm[r] = 1 / |x_r| (0 for a zero row); one warp per row, 16-byte loads.
+__global__ void inv_norm_kernel(const __half* __restrict__ x, int rows, int E,
+                                float* __restrict__ inv_norm) {
+  griddep_wait();
+  const int lane = threadIdx.x & 31;
+  const int nw = gridDim.x * (blockDim.x >> 5);
+  for (int r = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5); r < rows; r += nw) {
+    const uint4* p = reinterpret_cast<const uint4*>(x + (size_t)r * E);
+    float s = 0.f;
+    for (int c = lane; c < E / 8; c += 32) {
+      const uint4 u = __ldcs(p + c);
+      const __half2* h = reinterpret_cast<const __half2*>(&u);
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const float2 f = __half22float2(h[k]);
+        s = fmaf(f.x, f.x, s);
+        s = fmaf(f.y, f.y, s);
+      }
+    }
+    s = warp_sum(s);
+    if (lane == 0) inv_norm[r] = s > 0.f ? rsqrtf(s) : 0.f;
+  }
+  griddep_launch_dependents();
+}
+
+// Per keyframe: merge the per-CTA lists (each sorted, ids unique across CTAs)
+// into the keyframe's top k_frame and scale by the keyframe's inverse norm.
+// One warp per keyframe.
+__global__ void frame_merge_kernel(const float* __restrict__ part_sim,
+                                   const int32_t* __restrict__ part_idx,
+                                   const __half* __restrict__ frames, int M, int E, int kf,
+                                   int nparts, int32_t* __restrict__ out_idx,
+                                   float* __restrict__ out_sim) {
+  griddep_wait();
+  griddep_launch_dependents();
+  const int m = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  const int lane = threadIdx.x & 31;
+  if (m >= M) return;
+  const uint4* p = reinterpret_cast<const uint4*>(frames + (size_t)m * E);
+  float s = 0.f;
+  for (int c = lane; c < E / 8; c += 32) {
+    const uint4 u = p[c];
+    const __half2* h = reinterpret_cast<const __half2*>(&u);
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 f = __half22float2(h[k]);
+      s = fmaf(f.x, f.x, s);
+      s = fmaf(f.y, f.y, s);
+    }
+  }
+  s = warp_sum(s);
+  const float inv = s > 0.f ? rsqrtf(s) : 0.f;
+  const int n = nparts * kf;          // entries of this keyframe: n <= 256 * 8
+  uint64_t taken = 0;                 // bit j: entry lane + 32 j already chosen
+  for (int r = 0; r < kf; ++r) {
+    float bs = -INFINITY;
+    int bi = -1, bpos = -1;
+    for (int j = 0, e = lane; e < n; ++j, e += 32) {
+      if ((taken >> j) & 1ull) continue;
+      const int b = e / kf, pidx = e % kf;
+      const size_t a = ((size_t)b * M + m) * kf + pidx;
+      const int id = part_idx[a];
+      if (id < 0) continue;
+      const float v = part_sim[a];
+      if (bi < 0 || better(v, id, bs, bi)) {
+        bs = v;
+        bi = id;
+        bpos = e;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      const int op = __shfl_xor_sync(0xffffffffu, bpos, o);
+      if (oi >= 0 && (bi < 0 || better(os, oi, bs, bi))) {
+        bs = os;
+        bi = oi;
+        bpos = op;
+      }
+    }
+    if (bpos >= 0 && (bpos & 31) == lane) taken |= 1ull << (bpos >> 5);
+    if (lane == 0) {
+      out_idx[(size_t)m * kf + r] = bi;
+      out_sim[(size_t)m * kf + r] = bi >= 0 ? bs * inv : -INFINITY;
+    }
+  }
+}
+
+// Per query: T = the texts its keyframes retrieved, each scored by its best
+// retrieving keyframe; out = the k_query best of T.  One warp per query; a text
+// chosen in one round marks all its entries dead.
+__global__ void query_merge_kernel(const int32_t* __restrict__ fidx, const float* __restrict__ fsim,
+                                   const int32_t* __restrict__ frame_offsets, int Qn, int M, int kf,
+                                   int Kq, int32_t* __restrict__ out_idx,
+                                   float* __restrict__ out_sim) {
+  __shared__ uint8_t dead[kMaxState];
+  griddep_wait();
+  griddep_launch_dependents();
+  const int q = blockIdx.x;
+  const int lane = threadIdx.x;
+  if (q >= Qn) return;
+  const int f0 = frame_offsets[q], f1 = frame_offsets[q + 1];
+  // offsets outside [0, M] or decreasing (a caller error) read as an empty query
+  const bool sane = f0 >= 0 && f1 >= f0 && f1 <= M;
+  const int e0 = sane ? f0 * kf : 0;
+  const int n = sane ? (f1 - f0) * kf : 0;
+  for (int e = lane; e < n; e += 32) dead[e] = fidx[e0 + e] < 0;
+  __syncwarp();
+  for (int r = 0; r < Kq; ++r) {
+    float bs = -INFINITY;
+    int bi = -1;
+    for (int e = lane; e < n; e += 32) {
+      if (dead[e]) continue;
+      const float v = fsim[e0 + e];
+      const int id = fidx[e0 + e];
+      if (bi < 0 || better(v, id, bs, bi)) {
+        bs = v;
+        bi = id;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float os = __shfl_xor_sync(0xffffffffu, bs, o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi, o);
+      if (oi >= 0 && (bi < 0 || better(os, oi, bs, bi))) {
+        bs = os;
+        bi = oi;
+      }
+    }
+    if (lane == 0) {
+      out_idx[(size_t)q * Kq + r] = bi;
+      out_sim[(size_t)q * Kq + r] = bi >= 0 ? bs : -INFINITY;
+    }
+    if (bi >= 0)
+      for (int e = lane; e < n; e += 32)
+        if (fidx[e0 + e] == bi) dead[e] = 1;
+    __syncwarp();
+  }
+}
+
+struct Plan {
+  int ctas, bn, mg;
+};
+
+static Plan make_plan(const fvrag_retrieve_desc* d, int sms) {
+  Plan p;
+  const int mtiles = (d->num_keyframes + kBM - 1) / kBM;
+  p.bn = mtiles <= 1 ? 256 : 128;
+  p.mg = mtiles <= 1 ? 1 : 2;
+  const int nunits = (d->num_texts + 15) / 16;
+  p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
+  return p;
+}
+
+struct WsLayout {
+  size_t part_sim, part_idx, frame_idx, frame_sim, inv_norm, total;
+};
+
+static WsLayout ws_layout(const fvrag_retrieve_desc* d) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  const size_t lists = (size_t)kMaxCtas * d->num_keyframes * d->k_frame;
+  const size_t fl = (size_t)d->num_keyframes * d->k_frame;
+  WsLayout w;
+  w.part_sim = kWsHeaderBytes;
+  w.part_idx = w.part_sim + up(lists * 4);
+  w.frame_idx = w.part_idx + up(lists * 4);
+  w.frame_sim = w.frame_idx + up(fl * 4);
+  w.inv_norm = w.frame_sim + up(fl * 4);
+  w.total = w.inv_norm + up((size_t)d->num_texts * 4);
+  return w;
+}
+
+static bool desc_ok(const fvrag_retrieve_desc* d) {
+  return d && d->num_queries >= 1 && d->num_keyframes >= 0 && d->num_texts >= 1 && d->dim >= 8 &&
+         d->k_frame >= 1 && d->k_query >= 1 && d->flags == 0;
+}
+
+template <int BN, int MG>
+static fvrag_status launch(const Plan& p, const CUtensorMap& tf, const CUtensorMap& t64,
+                           const CUtensorMap& t16, const float* inv_norm,
+                           const fvrag_retrieve_desc* d, int hrows, float* psim, int32_t* pidx,
+                           uint32_t* status, cudaStream_t s) {
+  using C = Cfg<BN, MG>;
+  auto kern = retrieve_kernel<BN, MG>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  if (launch_pdl(kern, dim3(p.ctas), dim3(kThreads), (size_t)C::kSmemBytes, s, tf, t64, t16,
+                 inv_norm, d->num_keyframes, d->dim, d->num_texts, d->k_frame, hrows, psim, pidx,
+                 status, wait_limit_ns()) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return launch_status();
+}
+
+static fvrag_status launch_inv_norms(const void* x, int rows, int dim, float* inv, cudaStream_t s) {
+  const int sms = sm_count() > 0 ? sm_count() : 148;
+  const int blocks = std::max(1, std::min((rows + 7) / 8, sms * 8));
+  if (launch_pdl(inv_norm_kernel, dim3(blocks), dim3(256), 0, s, (const __half*)x, rows, dim, inv) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return launch_status();
+}
+
+}  // namespace rt
+}  // namespace fvrag
+
+using namespace fvrag;
+
+extern "C" fvrag_status fvrag_embed_inv_norms(const void* x, int32_t rows, int32_t dim,
+                                              float* inv_norm, fvrag_stream_t stream) {
+  if (!x || !inv_norm || rows < 1 || dim < 8) return FVRAG_ERR_INVALID_ARG;
+  if (dim % 8 != 0 || !aligned16(x)) return FVRAG_ERR_MISALIGNED;
+  return rt::launch_inv_norms(x, rows, dim, inv_norm, reinterpret_cast<cudaStream_t>(stream));
+}
+
+extern "C" size_t fvrag_retrieve_workspace(const fvrag_retrieve_desc* d) {
+  if (!rt::desc_ok(d)) return 0;
+  return rt::ws_layout(d).total;
+}
+
+extern "C" fvrag_status fvrag_retrieve(const fvrag_retrieve_desc* d, const void* frame_emb,
+                                       const int32_t* frame_offsets, const void* text_emb,
+                                       const float* text_inv_norm, int32_t* frame_topk,
+                                       float* frame_topk_sim, int32_t* out_idx, float* out_sim,
+                                       void* ws, size_t ws_size, fvrag_stream_t stream) {
+  using namespace rt;
+  if (!desc_ok(d) || !frame_offsets || !text_emb || !out_idx || !out_sim)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->num_keyframes > 0 && !frame_emb) return FVRAG_ERR_INVALID_ARG;
+  if (d->num_keyframes > kMaxMTiles * kBM || d->k_frame > kMaxKf ||
+      (long long)((d->num_keyframes + kBM - 1) / kBM) * kBM * d->k_frame > kMaxState ||
+      d->k_query > kMaxKq)
+    return FVRAG_ERR_UNSUPPORTED;
+  if (d->dim % 8 != 0) return FVRAG_ERR_MISALIGNED;
+  if ((frame_emb && !aligned16(frame_emb)) || !aligned16(text_emb) ||
+      (text_inv_norm && !aligned16(text_inv_norm)))
+    return FVRAG_ERR_MISALIGNED;
+  const WsLayout w = ws_layout(d);
+  if (!ws || ws_size < w.total) return FVRAG_ERR_WORKSPACE;
+  if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
+
+  uint8_t* base = reinterpret_cast<uint8_t*>(ws);
+  uint32_t* status = reinterpret_cast<uint32_t*>(base);
+  float* psim = reinterpret_cast<float*>(base + w.part_sim);
+  int32_t* pidx = reinterpret_cast<int32_t*>(base + w.part_idx);
+  int32_t* fidx = frame_topk ? frame_topk : reinterpret_cast<int32_t*>(base + w.frame_idx);
+  float* fsim = frame_topk_sim ? frame_topk_sim : reinterpret_cast<float*>(base + w.frame_sim);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  const int M = d->num_keyframes;
+
+  if (M > 0) {
+    const float* inv = text_inv_norm;
+    if (!inv) {
+      float* tmp = reinterpret_cast<float*>(base + w.inv_norm);
+      const fvrag_status st = launch_inv_norms(text_emb, d->num_texts, d->dim, tmp, s);
+      if (st != FVRAG_OK) return st;
+      inv = tmp;
+    }
+    const Plan p = make_plan(d, sm_count());
+    const uint64_t E = (uint64_t)d->dim, Nt = (uint64_t)d->num_texts;
+    const int hrows = M <= kBM ? (M + 15) / 16 * 16 : kBM;
+    CUtensorMap tf, t64, t16;
+    {
+      const uint64_t dims[2] = {E, (uint64_t)M}, strides[1] = {E * 2};
+      const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)hrows};
+      if (!encode_tmap_f16(&tf, frame_emb, 2, dims, strides, box, true)) return FVRAG_ERR_CUDA;
+    }
+    {
+      const uint64_t dims[2] = {E, Nt}, strides[1] = {E * 2};
+      const uint32_t b64[2] = {(uint32_t)kBK, 64u}, b16[2] = {(uint32_t)kBK, 16u};
+      if (!encode_tmap_f16(&t64, text_emb, 2, dims, strides, b64, true)) return FVRAG_ERR_CUDA;
+      if (!encode_tmap_f16(&t16, text_emb, 2, dims, strides, b16, true)) return FVRAG_ERR_CUDA;
+    }
+    fvrag_status st;
+    if (p.bn == 256)
+      st = launch<256, 1>(p, tf, t64, t16, inv, d, hrows, psim, pidx, status, s);
+    else
+      st = launch<128, 2>(p, tf, t64, t16, inv, d, hrows, psim, pidx, status, s);
+    if (st != FVRAG_OK) return st;
+    if (launch_pdl(frame_merge_kernel, dim3((M + 7) / 8), dim3(256), 0, s, (const float*)psim,
+                   (const int32_t*)pidx, (const __half*)frame_emb, M, d->dim, d->k_frame, p.ctas,
+                   fidx, fsim) != cudaSuccess)
+      return FVRAG_ERR_CUDA;
+  }
+  if (launch_pdl(query_merge_kernel, dim3(d->num_queries), dim3(32), 0, s, (const int32_t*)fidx,
+                 (const float*)fsim, frame_offsets, d->num_queries, M, d->k_frame, d->k_query,
+                 out_idx, out_sim) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return launch_status();
+}

@@ -26,6 +26,8 @@ EXPORTED = (
     "fvrag_verify_attn_workspace", "fvrag_verify_attn",
     "fvrag_score_logprobs_workspace", "fvrag_score_logprobs", "fvrag_score_logprobs_noalloc",
     "fvrag_clip_align", "fvrag_select_candidate",
+    "fvrag_embed_inv_norms", "fvrag_retrieve_workspace", "fvrag_retrieve",
+    "fvrag_keyframes_workspace", "fvrag_keyframes",
     "fvrag_read_status", "fvrag_clear_status",
     "fvrag_set_wait_limit_ns", "fvrag_get_wait_limit_ns", "fvrag_selftest_wait_timeout",
 )
@@ -63,6 +65,18 @@ class SelectDesc(ctypes.Structure):
                 ("seed", ctypes.c_uint64)]
 
 
+class RetrieveDesc(ctypes.Structure):
+    _fields_ = [("num_queries", ctypes.c_int32), ("num_keyframes", ctypes.c_int32),
+                ("num_texts", ctypes.c_int32), ("dim", ctypes.c_int32), ("k_frame", ctypes.c_int32),
+                ("k_query", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+
+
+class KeyframeDesc(ctypes.Structure):
+    _fields_ = [("num_videos", ctypes.c_int32), ("total_frames", ctypes.c_int32),
+                ("height", ctypes.c_int32), ("width", ctypes.c_int32), ("theta", ctypes.c_double),
+                ("flags", ctypes.c_uint32)]
+
+
 _lib = None
 
 
@@ -91,6 +105,16 @@ def lib():
         L.fvrag_clip_align.argtypes = [ctypes.POINTER(ClipDesc)] + [vp] * 6 + [vp]
         L.fvrag_select_candidate.restype = i32
         L.fvrag_select_candidate.argtypes = [ctypes.POINTER(SelectDesc)] + [vp] * 6 + [vp]
+        L.fvrag_embed_inv_norms.restype = i32
+        L.fvrag_embed_inv_norms.argtypes = [vp, ctypes.c_int32, ctypes.c_int32, vp, vp]
+        L.fvrag_retrieve_workspace.restype = sz
+        L.fvrag_retrieve_workspace.argtypes = [ctypes.POINTER(RetrieveDesc)]
+        L.fvrag_retrieve.restype = i32
+        L.fvrag_retrieve.argtypes = [ctypes.POINTER(RetrieveDesc)] + [vp] * 9 + [sz, vp]
+        L.fvrag_keyframes_workspace.restype = sz
+        L.fvrag_keyframes_workspace.argtypes = [ctypes.POINTER(KeyframeDesc)]
+        L.fvrag_keyframes.restype = i32
+        L.fvrag_keyframes.argtypes = [ctypes.POINTER(KeyframeDesc)] + [vp] * 8 + [sz, vp]
         L.fvrag_read_status.restype = i32
         L.fvrag_read_status.argtypes = [vp, vp]
         L.fvrag_clear_status.restype = i32
@@ -186,6 +210,56 @@ def select_candidate(logprob, score, selected, mode=SEL_MASKED_MEAN_LOGPROB, kee
     s = lib().fvrag_select_candidate(ctypes.byref(d), _ptr(logprob), _ptr(lengths), _ptr(keep),
                                      _ptr(max_cos), _ptr(score), _ptr(selected), _stream(stream))
     _check(s, "fvrag_select_candidate")
+
+
+def embed_inv_norms(x, inv_norm, stream=None):
+    """x [rows][dim] fp16 -> inv_norm [rows] fp32 (1/|row|, 0 for a zero row)."""
+    s = lib().fvrag_embed_inv_norms(_ptr(x), int(x.shape[0]), int(x.shape[1]), _ptr(inv_norm),
+                                    _stream(stream))
+    _check(s, "fvrag_embed_inv_norms")
+
+
+def retrieve_desc(num_queries, frame_emb, text_emb, k_frame, k_query) -> RetrieveDesc:
+    return RetrieveDesc(int(num_queries), int(frame_emb.shape[0]), int(text_emb.shape[0]),
+                        int(text_emb.shape[1]), int(k_frame), int(k_query), 0)
+
+
+def retrieve_workspace_bytes(desc: RetrieveDesc) -> int:
+    return int(lib().fvrag_retrieve_workspace(ctypes.byref(desc)))
+
+
+def retrieve(frame_emb, frame_offsets, text_emb, k_frame, out_idx, out_sim, ws, text_inv_norm=None,
+             frame_topk=None, frame_topk_sim=None, stream=None):
+    """frame_emb [Fr][E] fp16, frame_offsets [Qn+1] int32 (device), text_emb [Nt][E] fp16 ->
+    out_idx [Qn][Kq] int32, out_sim [Qn][Kq] fp32; frame_topk / frame_topk_sim [Fr][k_frame]
+    are written when given; text_inv_norm [Nt] fp32 from embed_inv_norms, or None."""
+    Qn, Kq = out_idx.shape
+    d = retrieve_desc(Qn, frame_emb, text_emb, k_frame, Kq)
+    s = lib().fvrag_retrieve(ctypes.byref(d), _ptr(frame_emb), _ptr(frame_offsets), _ptr(text_emb),
+                             _ptr(text_inv_norm), _ptr(frame_topk), _ptr(frame_topk_sim),
+                             _ptr(out_idx), _ptr(out_sim), _ptr(ws), ws.numel() * ws.element_size(),
+                             _stream(stream))
+    _check(s, "fvrag_retrieve")
+
+
+def keyframe_desc(num_videos, pixels, theta) -> KeyframeDesc:
+    return KeyframeDesc(int(num_videos), int(pixels.shape[0]), int(pixels.shape[1]),
+                        int(pixels.shape[2]), float(theta), 0)
+
+
+def keyframes_workspace_bytes(desc: KeyframeDesc) -> int:
+    return int(lib().fvrag_keyframes_workspace(ctypes.byref(desc)))
+
+
+def keyframes(pixels, video_offsets, theta, sim, is_key, key_index, key_offsets, ws, hist=None,
+              stream=None):
+    """pixels [T][H][W][3] uint8, video_offsets [Nv+1] int32 (device) -> sim [T] fp32,
+    is_key [T] uint8, key_index [T] int32, key_offsets [Nv+1] int32 (and hist [T][512])."""
+    d = keyframe_desc(int(video_offsets.shape[0]) - 1, pixels, theta)
+    s = lib().fvrag_keyframes(ctypes.byref(d), _ptr(pixels), _ptr(video_offsets), _ptr(hist),
+                              _ptr(sim), _ptr(is_key), _ptr(key_index), _ptr(key_offsets), _ptr(ws),
+                              ws.numel() * ws.element_size(), _stream(stream))
+    _check(s, "fvrag_keyframes")
 
 
 # --------------------------------------------------------------------- status

@@ -121,3 +121,78 @@ def check_selection_masked(gpu_sel, oracle_score, oracle_maxcos, tau, tol_score=
         assert maybe[s]
         best_sure = oracle_score[q][sure].max() if sure.any() else -np.inf
         assert oracle_score[q, s] >= best_sure - tol_score
+
+
+def run_keyframes(pixels, video_offsets, theta, with_hist=True):
+    """fvrag_keyframes on numpy inputs; returns (hist, sim, is_key, key_index, key_offsets, status)."""
+    T = pixels.shape[0]
+    Nv = len(video_offsets) - 1
+    px = torch.from_numpy(np.ascontiguousarray(pixels)).cuda() if T > 0 else \
+        torch.empty((0,) + tuple(pixels.shape[1:]), dtype=torch.uint8, device="cuda")
+    vo = dev(np.asarray(video_offsets, np.int32))
+    d = fvrag.keyframe_desc(Nv, px, theta)
+    ws = torch.zeros(fvrag.keyframes_workspace_bytes(d), dtype=torch.uint8, device="cuda")
+    hist = torch.full((T, 512), -7, dtype=torch.int32, device="cuda") if with_hist else None
+    sim = torch.full((max(T, 1),), float("nan"), device="cuda")
+    key = torch.full((max(T, 1),), 9, dtype=torch.uint8, device="cuda")
+    kidx = torch.full((max(T, 1),), -7, dtype=torch.int32, device="cuda")
+    koffs = torch.full((Nv + 1,), -7, dtype=torch.int32, device="cuda")
+    fvrag.keyframes(px, vo, theta, sim, key, kidx, koffs, ws, hist=hist)
+    st = fvrag.read_status(ws)
+    ko = koffs.cpu().numpy()
+    return ((hist.cpu().numpy() if with_hist else None), sim.cpu().numpy()[:T], key.cpu().numpy()[:T],
+            kidx.cpu().numpy()[:ko[-1]], ko, st)
+
+
+def run_retrieve(frames, frame_offsets, texts, k_frame, k_query, precompute_norms=True):
+    """fvrag_retrieve on numpy inputs; returns (frame_idx, frame_sim, idx, sim, status)."""
+    Fr = frames.shape[0]
+    Qn = len(frame_offsets) - 1
+    tf = dev_f16(frames) if Fr > 0 else torch.empty((0, texts.shape[1]), dtype=torch.float16, device="cuda")
+    tt = dev_f16(texts)
+    fo = dev(np.asarray(frame_offsets, np.int32))
+    inv = None
+    if precompute_norms:
+        inv = torch.empty(texts.shape[0], dtype=torch.float32, device="cuda")
+        fvrag.embed_inv_norms(tt, inv)
+    d = fvrag.retrieve_desc(Qn, tf, tt, k_frame, k_query)
+    ws = torch.zeros(fvrag.retrieve_workspace_bytes(d), dtype=torch.uint8, device="cuda")
+    fi = torch.full((max(Fr, 1), k_frame), -7, dtype=torch.int32, device="cuda")
+    fs = torch.full((max(Fr, 1), k_frame), float("nan"), device="cuda")
+    oi = torch.full((Qn, k_query), -7, dtype=torch.int32, device="cuda")
+    os_ = torch.full((Qn, k_query), float("nan"), device="cuda")
+    fvrag.retrieve(tf, fo, tt, k_frame, oi, os_, ws, text_inv_norm=inv, frame_topk=fi,
+                   frame_topk_sim=fs)
+    st = fvrag.read_status(ws)
+    return (fi.cpu().numpy()[:Fr], fs.cpu().numpy()[:Fr], oi.cpu().numpy(), os_.cpu().numpy(), st)
+
+
+def check_frame_lists(gpu_idx, gpu_sim, texts, frames, oracle_frame_topk_all, tol=COS_ATOL):
+    """Per-keyframe lists: each GPU entry is a real similarity of that text (within tol), the
+    list is sorted, ids are unique, and it agrees with the oracle's full ordering: the j-th
+    GPU similarity is within tol of the oracle's j-th, every text whose oracle similarity
+    beats the oracle's k-th by more than tol is present, and ids match exactly wherever the
+    oracle's neighbours are more than tol apart.  ``oracle_frame_topk_all(f)`` returns the
+    oracle's (ids, sims) of keyframe f over the whole corpus, best first."""
+    Fr, kf = gpu_idx.shape
+    for f in range(Fr):
+        oi, osim = oracle_frame_topk_all(f)
+        n = min(kf, len(oi))
+        gi, gs = gpu_idx[f], gpu_sim[f]
+        assert np.all(gi[n:] == -1) and np.all(np.isneginf(gs[n:]))
+        gi, gs = gi[:n], gs[:n]
+        assert len(set(gi.tolist())) == n and np.all(gi >= 0)
+        assert np.all(np.diff(gs) <= 0)
+        sim_of = dict(zip(oi.tolist(), osim.tolist()))
+        for j in range(n):
+            assert abs(gs[j] - osim[j]) <= tol, (f, j, gs[j], osim[j])
+            if int(gi[j]) in sim_of:
+                assert abs(gs[j] - sim_of[int(gi[j])]) <= tol
+        kth = osim[n - 1]
+        sure = oi[osim > kth + tol]
+        assert set(sure.tolist()) <= set(gi.tolist())
+        for j in range(n):
+            lo = osim[j - 1] - osim[j] if j > 0 else np.inf
+            hi = osim[j] - osim[j + 1] if j + 1 < len(osim) else np.inf
+            if lo > tol and hi > tol:
+                assert gi[j] == oi[j], (f, j, gi[j], oi[j])

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert L.fvrag_abi_version() == 2
+    assert L.fvrag_abi_version() == 3
     for s in range(7):
         assert fvrag.status_string(s)
     assert fvrag.status_string(99) == "unknown status"
@@ -131,3 +131,57 @@ def test_binding_raises_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(fvrag, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(OSError):
         fvrag.lib()
+
+
+def _rt(L, d, ws_bytes=1 << 30, fe=P, fo=P, te=P, inv=P, oi=P, os_=P, ws=P):
+    return L.fvrag_retrieve(ctypes.byref(d), fe, fo, te, inv, None, None, oi, os_, ws, ws_bytes, None)
+
+
+def test_retrieve_validation(L):
+    assert ctypes.sizeof(fvrag.RetrieveDesc) == 28
+    good = fvrag.RetrieveDesc(16, 300, 1 << 20, 768, 3, 3, 0)
+    ws = L.fvrag_retrieve_workspace(ctypes.byref(good))
+    assert ws >= 256 + 2 * 256 * 300 * 3 * 4 + (1 << 20) * 4
+    assert _rt(L, fvrag.RetrieveDesc(0, 300, 1 << 20, 768, 3, 3, 0)) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, fvrag.RetrieveDesc(16, 300, 0, 768, 3, 3, 0)) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, fvrag.RetrieveDesc(16, 300, 1 << 20, 768, 0, 3, 0)) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, fvrag.RetrieveDesc(16, 300, 1 << 20, 768, 3, 3, 2)) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, good, te=None) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, good, fe=None) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, good, oi=None) == fvrag.ERR_INVALID_ARG
+    assert _rt(L, fvrag.RetrieveDesc(16, 2049, 1 << 20, 768, 1, 3, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _rt(L, fvrag.RetrieveDesc(16, 300, 1 << 20, 768, 9, 3, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _rt(L, fvrag.RetrieveDesc(16, 1281, 1 << 20, 768, 3, 3, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _rt(L, fvrag.RetrieveDesc(16, 513, 1 << 20, 768, 8, 3, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _rt(L, fvrag.RetrieveDesc(16, 300, 1 << 20, 768, 3, 65, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _rt(L, fvrag.RetrieveDesc(16, 300, 1 << 20, 764, 3, 3, 0)) == fvrag.ERR_MISALIGNED
+    assert _rt(L, good, te=PMIS) == fvrag.ERR_MISALIGNED
+    assert _rt(L, good, inv=PMIS) == fvrag.ERR_MISALIGNED
+    assert _rt(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE
+    assert L.fvrag_embed_inv_norms(None, 10, 768, P, None) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_embed_inv_norms(P, 0, 768, P, None) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_embed_inv_norms(P, 10, 764, P, None) == fvrag.ERR_MISALIGNED
+    assert L.fvrag_embed_inv_norms(PMIS, 10, 768, P, None) == fvrag.ERR_MISALIGNED
+
+
+def _kf(L, d, ws_bytes=1 << 30, px=P, vo=P, sim=P, key=P, ki=P, ko=P, ws=P):
+    return L.fvrag_keyframes(ctypes.byref(d), px, vo, None, sim, key, ki, ko, ws, ws_bytes, None)
+
+
+def test_keyframes_validation(L):
+    assert ctypes.sizeof(fvrag.KeyframeDesc) == 32
+    good = fvrag.KeyframeDesc(8, 5000, 720, 1280, 0.6, 0)
+    ws = L.fvrag_keyframes_workspace(ctypes.byref(good))
+    assert ws == 256 + 5000 * 512 * 4
+    assert _kf(L, fvrag.KeyframeDesc(0, 5000, 720, 1280, 0.6, 0)) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, fvrag.KeyframeDesc(8, -1, 720, 1280, 0.6, 0)) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, fvrag.KeyframeDesc(8, 5000, 720, 1280, 0.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, fvrag.KeyframeDesc(8, 5000, 720, 1280, float("nan"), 0)) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, fvrag.KeyframeDesc(8, 5000, 720, 1280, 0.6, 1)) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, good, px=None) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, good, vo=None) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, good, ki=None) == fvrag.ERR_INVALID_ARG
+    assert _kf(L, fvrag.KeyframeDesc(8, 5000, 3, 5, 0.6, 0)) == fvrag.ERR_MISALIGNED
+    assert _kf(L, good, px=PMIS) == fvrag.ERR_MISALIGNED
+    assert _kf(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE
+    assert _kf(L, good, ws=None) == fvrag.ERR_WORKSPACE

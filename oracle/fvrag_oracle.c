@@ -31,6 +31,9 @@
  *                            Eq. 12 reliability, Eq. 13 high-reliability set,
  *                            argmax alignment over it (mode 1), and the
  *                            other strategies of Sections 4.5-4.6 (modes 2-6).
+ *   oracle_decode_attn    -- one decode step of the K drafts (Eq. 5, Eq. 8-10):
+ *                            each draft's newest token over the shared prefix
+ *                            and its own tokens.
  *   oracle_frame_topk     -- Eq. 2: each keyframe's most similar corpus texts.
  *   oracle_aggregate_topk -- Eq. 3: the union of a query's per-keyframe lists
  *                            and its K best texts.
@@ -184,6 +187,106 @@ int oracle_verify_attn(int Qn, int K, int L, int Hq, int Hkv, int D, double scal
       for (int t = 0; t <= l; ++t, ++j) {
         const double p = exp(s[j] - m) / Z;
         const uint16_t* vr = v_tail + ((((int64_t)qi * K + k) * L + t) * Hkv + g) * D;
+        for (int d = 0; d < D; ++d) acc[d] += p * dec_bf16(vr[d]);
+      }
+      for (int d = 0; d < D; ++d) out[r * D + d] = acc[d];
+      if (lse) lse[r] = m + log(Z);
+    }
+    free(s);
+    free(qv);
+    free(acc);
+  }
+  return bad ? -1 : 0;
+}
+
+/*
+ * One decode step of the drafter (Eq. 5; the generation of e_i, r_i and a_i in
+ * Eq. 8-10): the K drafts of a query are generated in parallel, each from the
+ * shared prefix (video tokens and question) followed by its own tokens (its
+ * retrieved text t_i and what it has generated so far).  Each draft's newest
+ * token attends to the whole prefix and to its own tokens up to itself.
+ *
+ *   q        [Qn][K][Hq][D]     bf16   query of each draft's newest token
+ *   k_pre    [sum P][Hkv][D]    bf16   shared prefix keys / values; query qi owns
+ *   v_pre    [sum P][Hkv][D]    bf16     rows offs[qi] .. offs[qi+1]-1
+ *   offs     [Qn+1]             int32
+ *   k_cache  [Qn][K][C][Hkv][D] bf16   each draft's own keys / values; the newest
+ *   v_cache  [Qn][K][C][Hkv][D] bf16     token is at position n_k - 1
+ *   cache_len[Qn][K]            int32  n_k, 1 <= n_k <= C
+ *   out      [Qn][K][Hq][D]     fp64
+ *   lse      [Qn][K][Hq]        fp64 or NULL
+ * For query qi, draft k, head h with kv head g = h / (Hq / Hkv):
+ *   keys  S = { prefix j : 0 <= j < P_qi }  U  { own (k, t) : 0 <= t < n_k }
+ *   out   = softmax(scale * q K_S^T) V_S,  lse as in oracle_verify_attn.
+ * Readings: drafts never see one another's tokens (each a_i is drafted from its own
+ * t_i, Eq. 5); cache positions at or past n_k are not read.
+ * Returns 0, or -1 on bad arguments (including n_k outside [1, C]).
+ */
+int oracle_decode_attn(int Qn, int K, int C, int Hq, int Hkv, int D, double scale,
+                       const uint16_t* q, const uint16_t* k_pre, const uint16_t* v_pre,
+                       const int32_t* offs, const uint16_t* k_cache, const uint16_t* v_cache,
+                       const int32_t* cache_len, double* out, double* lse) {
+  if (Qn <= 0 || K <= 0 || C <= 0 || Hq <= 0 || Hkv <= 0 || D <= 0 || Hq % Hkv) return -1;
+  if (!q || !offs || !k_cache || !v_cache || !cache_len || !out) return -1;
+  if (scale == 0.0) scale = 1.0 / sqrt((double)D);
+  const int grp = Hq / Hkv;
+  int maxP = 0;
+  for (int qi = 0; qi < Qn; ++qi) {
+    const int p = offs[qi + 1] - offs[qi];
+    if (p < 0) return -1;
+    if (p > maxP) maxP = p;
+  }
+  for (int64_t i = 0; i < (int64_t)Qn * K; ++i)
+    if (cache_len[i] < 1 || cache_len[i] > C) return -1;
+  if (maxP > 0 && (!k_pre || !v_pre)) return -1;
+  const int64_t nrows = (int64_t)Qn * K * Hq;
+  int bad = 0;
+#pragma omp parallel
+  {
+    double* s = (double*)malloc(sizeof(double) * (size_t)(maxP + C));
+    double* qv = (double*)malloc(sizeof(double) * (size_t)D);
+    double* acc = (double*)malloc(sizeof(double) * (size_t)D);
+    if (!s || !qv || !acc) {
+#pragma omp atomic write
+      bad = 1;
+    }
+#pragma omp for schedule(dynamic, 4)
+    for (int64_t r = 0; r < nrows; ++r) {
+      if (bad) continue;
+      const int h = (int)(r % Hq);
+      const int64_t qk = r / Hq; /* qi*K + k */
+      const int qi = (int)(qk / K);
+      const int g = h / grp;
+      const int P = offs[qi + 1] - offs[qi];
+      const int n_own = cache_len[qk];
+      for (int d = 0; d < D; ++d) qv[d] = dec_bf16(q[r * D + d]);
+      int n = 0;
+      for (int j = 0; j < P; ++j) {
+        const uint16_t* kr = k_pre + ((int64_t)(offs[qi] + j) * Hkv + g) * D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d) dot += qv[d] * dec_bf16(kr[d]);
+        s[n++] = scale * dot;
+      }
+      for (int t = 0; t < n_own; ++t) {
+        const uint16_t* kr = k_cache + ((qk * C + t) * Hkv + g) * D;
+        double dot = 0.0;
+        for (int d = 0; d < D; ++d) dot += qv[d] * dec_bf16(kr[d]);
+        s[n++] = scale * dot;
+      }
+      double m = -INFINITY;
+      for (int j = 0; j < n; ++j) if (s[j] > m) m = s[j];
+      double Z = 0.0;
+      for (int j = 0; j < n; ++j) Z += exp(s[j] - m);
+      for (int d = 0; d < D; ++d) acc[d] = 0.0;
+      int j = 0;
+      for (; j < P; ++j) {
+        const double p = exp(s[j] - m) / Z;
+        const uint16_t* vr = v_pre + ((int64_t)(offs[qi] + j) * Hkv + g) * D;
+        for (int d = 0; d < D; ++d) acc[d] += p * dec_bf16(vr[d]);
+      }
+      for (int t = 0; t < n_own; ++t, ++j) {
+        const double p = exp(s[j] - m) / Z;
+        const uint16_t* vr = v_cache + ((qk * C + t) * Hkv + g) * D;
         for (int d = 0; d < D; ++d) acc[d] += p * dec_bf16(vr[d]);
       }
       for (int d = 0; d < D; ++d) out[r * D + d] = acc[d];

@@ -50,6 +50,8 @@ def _L():
         lib.oracle_clip_align.restype = ci
         lib.oracle_select.argtypes = [ci] * 5 + [cd] + [vp] * 6 + [ctypes.c_uint64]
         lib.oracle_select.restype = ci
+        lib.oracle_decode_attn.argtypes = [ci] * 6 + [cd] + [vp] * 9
+        lib.oracle_decode_attn.restype = ci
         lib.oracle_frame_topk.argtypes = [ci] * 4 + [vp] * 4
         lib.oracle_frame_topk.restype = ci
         lib.oracle_aggregate_topk.argtypes = [ci] * 3 + [vp] * 5
@@ -112,6 +114,25 @@ def verify_attn(q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, scale=0.0
                                  _p(offs), _p(kt), _p(vt), _p(sel), _p(out), _p(lse))
     if rc != 0:
         raise ValueError("oracle_verify_attn: bad arguments")
+    return out, lse
+
+
+def decode_attn(q, k_prefix, v_prefix, prefix_offsets, k_cache, v_cache, cache_len, scale=0.0):
+    """One drafter decode step.  q [Qn][K][Hq][D]; caches [Qn][K][C][Hkv][D] (bf16 bits);
+    cache_len [Qn][K].  Returns (out [Qn][K][Hq][D] fp64, lse [Qn][K][Hq] fp64)."""
+    Qn, K, Hq, D = q.shape
+    C, Hkv = k_cache.shape[2], k_cache.shape[3]
+    q, kc, vc = _c(q, np.uint16), _c(k_cache, np.uint16), _c(v_cache, np.uint16)
+    kp, vp_ = _c(k_prefix, np.uint16), _c(v_prefix, np.uint16)
+    offs, n = _c(prefix_offsets, np.int32), _c(cache_len, np.int32)
+    out = np.full(q.shape, np.nan)
+    lse = np.full(q.shape[:-1], np.nan)
+    rc = _L().oracle_decode_attn(Qn, K, C, Hq, Hkv, D, float(scale), _p(q),
+                                 _p(kp) if kp is not None and kp.size else None,
+                                 _p(vp_) if vp_ is not None and vp_.size else None,
+                                 _p(offs), _p(kc), _p(vc), _p(n), _p(out), _p(lse))
+    if rc != 0:
+        raise ValueError("oracle_decode_attn: bad arguments")
     return out, lse
 
 

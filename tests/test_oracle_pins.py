@@ -415,3 +415,89 @@ def test_random_selection_follows_published_splitmix64():
     _, sel = oracle.select(lp, mode=oracle.SEL_RANDOM, seed=99)
     counts = np.bincount(sel, minlength=K)
     assert counts.min() > 850 and counts.max() < 1150
+
+
+# --------------------------------------------------------------------------- drafter decode step
+
+def _decode_case(Qn, K, C, Hq, Hkv, D, plens, seed):
+    offs = np.zeros(Qn + 1, np.int32)
+    offs[1:] = np.cumsum(plens)
+    tot = int(offs[-1])
+    q = rand_bf16((Qn, K, Hq, D), seed, 1)
+    kp = rand_bf16((tot, Hkv, D), seed, 2)
+    vp = rand_bf16((tot, Hkv, D), seed, 3)
+    kc = rand_bf16((Qn, K, C, Hkv, D), seed, 4)
+    vc = rand_bf16((Qn, K, C, Hkv, D), seed, 5)
+    n = synth.uniform_i32((Qn, K), seed, 6, 1, C + 1)
+    return q, kp, vp, offs, kc, vc, n
+
+
+@pytest.mark.parametrize("Qn,K,C,Hq,Hkv,D,plens", [
+    (1, 3, 6, 4, 2, 16, [7]),
+    (2, 2, 9, 6, 3, 8, [5, 0]),       # ragged prefix, one query without prefix
+    (2, 4, 1, 8, 1, 16, [3, 9]),      # one-token caches, MQA
+])
+def test_decode_matches_sdpa(Qn, K, C, Hq, Hkv, D, plens):
+    """Library reference: torch SDPA (fp64) per draft over [prefix | own cache], with a mask
+    that hides the cache positions at or past n_k; lse via torch.logsumexp."""
+    q, kp, vp, offs, kc, vc, n = _decode_case(Qn, K, C, Hq, Hkv, D, plens, seed=21 + C)
+    scale = 1.0 / math.sqrt(D)
+    out, lse = oracle.decode_attn(q, kp, vp, offs, kc, vc, n)
+    for qi in range(Qn):
+        P = int(offs[qi + 1] - offs[qi])
+        for k in range(K):
+            keys = np.concatenate([bf16_vals(kp[offs[qi]:offs[qi + 1]]), bf16_vals(kc[qi, k])], 0)
+            vals = np.concatenate([bf16_vals(vp[offs[qi]:offs[qi + 1]]), bf16_vals(vc[qi, k])], 0)
+            Q = torch.from_numpy(bf16_vals(q[qi, k]))[None, :, None, :]         # [1,Hq,1,D]
+            Kt = torch.from_numpy(keys).permute(1, 0, 2)[None]                 # [1,Hkv,P+C,D]
+            Vt = torch.from_numpy(vals).permute(1, 0, 2)[None]
+            mask = torch.zeros(1, P + C, dtype=torch.bool)
+            mask[0, :P + int(n[qi, k])] = True
+            o = torch.nn.functional.scaled_dot_product_attention(Q, Kt, Vt, attn_mask=mask, scale=scale,
+                                                                 enable_gqa=True)
+            np.testing.assert_allclose(out[qi, k], o[0, :, 0].numpy(), rtol=0, atol=1e-12)
+            s = torch.einsum("bhld,bhjd->bhlj", Q, Kt.repeat_interleave(Hq // Hkv, dim=1)) * scale
+            s = s.masked_fill(~mask, float("-inf"))
+            np.testing.assert_allclose(lse[qi, k], torch.logsumexp(s, -1)[0, :, 0].numpy(), rtol=0,
+                                       atol=1e-12)
+
+
+def test_decode_zero_query_averages_the_visible_keys_and_ignores_the_rest():
+    """q = 0: out = mean of V over prefix U own cache[0 .. n_k-1], lse = ln(P + n_k).
+    Changing cache entries at or past n_k, or another draft's cache, changes nothing."""
+    Qn, K, C, Hq, Hkv, D = 2, 3, 5, 6, 2, 8
+    plens = [4, 2]
+    q, kp, vp, offs, kc, vc, n = _decode_case(Qn, K, C, Hq, Hkv, D, plens, seed=4)
+    q = np.zeros_like(q)
+    out, lse = oracle.decode_attn(q, kp, vp, offs, kc, vc, n)
+    vpd, vcd = bf16_vals(vp), bf16_vals(vc)
+    for qi in range(Qn):
+        for k in range(K):
+            for h in range(Hq):
+                g = h // (Hq // Hkv)
+                vis = np.concatenate([vpd[offs[qi]:offs[qi + 1], g], vcd[qi, k, :n[qi, k], g]], 0)
+                np.testing.assert_allclose(out[qi, k, h], vis.mean(0), rtol=0, atol=1e-14)
+                assert abs(lse[qi, k, h] - math.log(plens[qi] + n[qi, k])) < 1e-14
+    q, kp, vp, offs, kc, vc, n = _decode_case(Qn, K, C, Hq, Hkv, D, plens, seed=9)
+    out, lse = oracle.decode_attn(q, kp, vp, offs, kc, vc, n)
+    kc2, vc2 = kc.copy(), vc.copy()
+    for qi in range(Qn):
+        for k in range(K):
+            kc2[qi, k, n[qi, k]:] = rand_bf16(kc2[qi, k, n[qi, k]:].shape, 99, 1)
+            vc2[qi, k, n[qi, k]:] = rand_bf16(vc2[qi, k, n[qi, k]:].shape, 99, 2)
+    out2, lse2 = oracle.decode_attn(q, kp, vp, offs, kc2, vc2, n)
+    assert np.array_equal(out, out2) and np.array_equal(lse, lse2)
+    kc3 = kc.copy()
+    kc3[0, 1] = rand_bf16(kc3[0, 1].shape, 98, 1)            # draft 1's cache only
+    out3, _ = oracle.decode_attn(q, kp, vp, offs, kc3, vc, n)
+    assert np.array_equal(out3[0, [0, 2]], out[0, [0, 2]]) and np.array_equal(out3[1], out[1])
+    assert not np.array_equal(out3[0, 1], out[0, 1])
+
+
+def test_decode_rejects_bad_lengths():
+    q, kp, vp, offs, kc, vc, n = _decode_case(1, 2, 4, 2, 1, 8, [3], seed=2)
+    for bad in (0, 5):
+        n2 = n.copy()
+        n2[0, 1] = bad
+        with pytest.raises(ValueError):
+            oracle.decode_attn(q, kp, vp, offs, kc, vc, n2)

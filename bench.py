@@ -263,12 +263,15 @@ def cpu_baseline(cfg, x, budget_s):
                       % (reps, nrows, M, cfg.hq, dt)}
 
 
-def _time_calls(fn, stream, steps, dev):
-    """CUDA-event time of `steps` back-to-back calls of fn on `stream` (ms per call, and the list)."""
+def _time_calls(fn, stream, steps, dev, between=None):
+    """CUDA-event time of `steps` calls of fn on `stream` (ms per call, and the list);
+    `between` (outside the events) runs before each call."""
     import torch
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps)]
     for i in range(steps):
+        if between is not None:
+            between()
         ev[i][0].record(stream)
         fn()
         ev[i][1].record(stream)
@@ -301,7 +304,7 @@ def bench_row(args):
     steps = max(3, min(args.steps, 200))
 
     if args.row == "retrieve":
-        cfg = configs.RT_16Q_1M
+        cfg = configs.RETRIEVAL_PRESETS[args.row_config or "retrieve-16q-1m"]
         r = synth.retrieval_inputs(cfg, seed=cfg.seed + 7919 * rank)
         Fr, E, Nt = r["frames"].shape[0], cfg.dim, cfg.num_texts
         texts = torch.from_numpy(r["texts"].view(np.int16)).view(torch.float16).to(dev)
@@ -364,14 +367,15 @@ def bench_row(args):
         d2h = cfg.num_queries * cfg.k_query * 8
         config = {"workload": cfg.description, "name": cfg.name, "keyframes": Fr, "texts": Nt,
                   "dim": E, "k_frame": cfg.k_frame, "k_query": cfg.k_query,
-                  "l2": "inputs larger than L2 (the 1.6 GB corpus is streamed every call)",
+                  "l2": "inputs larger than L2 (the %.2f GB corpus is streamed every call)"
+                        % (Nt * E * 2 / 1e9),
                   "inv_norm_index_build_ms": inv_ms, "parallelism": "replicas"}
         dtype = "f16"
         launches = 3
         cpu = None
         if not args.no_cpu_baseline and ws_ == 1:
             oracle.build()
-            sample = np.arange(0, Fr, max(1, Fr // 4))[:4]
+            sample = np.arange(0, Fr, max(1, Fr // 8))[:8]
             t0 = time.perf_counter()
             fi, fs = oracle.frame_topk(r["frames"][sample], r["texts"], cfg.k_frame)
             oracle.aggregate_topk(np.array([0, len(sample)], np.int32), fi, fs, cfg.k_query)
@@ -379,8 +383,83 @@ def bench_row(args):
             cpu = {"value": len(sample) / dt, "unit": unit, "cores": oracle.max_threads(),
                    "kind": "oracle", "sample": "%d of %d keyframes scanned against the whole corpus "
                    "and aggregated, %.1f s" % (len(sample), Fr, dt)}
+    elif args.row == "decode":
+        cfg = configs.DECODE_PRESETS[args.row_config or "decode-3b-16q"]
+        x = synth.decode_inputs(cfg, seed=cfg.seed + 7919 * rank)
+
+        def up(a):
+            t = torch.from_numpy(np.ascontiguousarray(a).view(np.int16) if a.dtype == np.uint16 else a)
+            return (t.view(torch.bfloat16) if a.dtype == np.uint16 else t).to(dev)
+
+        q, kp, vp = up(x["q"]), up(x["k_prefix"]), up(x["v_prefix"])
+        kc, vc = up(x["k_cache"]), up(x["v_cache"])
+        offs, n = up(x["prefix_offsets"]), up(x["cache_len"])
+        maxp = int(np.max(np.diff(x["prefix_offsets"])))
+        d = fvrag.decode_desc(q, kp, kc, maxp)
+        ws = torch.zeros(fvrag.decode_workspace_bytes(d), dtype=torch.uint8, device=dev)
+        out = torch.empty_like(q)
+        h_q = torch.from_numpy(x["q"].view(np.int16)).view(torch.bfloat16).pin_memory()
+        h_n = torch.from_numpy(x["cache_len"]).pin_memory()
+        h_out = torch.empty(q.shape, dtype=torch.bfloat16).pin_memory()
+        flush_w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+        def call():
+            fvrag.decode_attn(q, kp, vp, offs, kc, vc, n, out, ws, maxp, stream=stream)
+
+        def call_host():
+            q.copy_(h_q, non_blocking=True)
+            n.copy_(h_n, non_blocking=True)
+            call()
+            h_out.copy_(out, non_blocking=True)
+
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                call()
+                call_host()
+            torch.cuda.synchronize(dev)
+            with ClockSampler(dev.index or 0) as clk:
+                clk.wait_first()
+                t_ms, _ = _time_calls(call, stream, steps, dev, between=flush_w.zero_)
+                e_ms, _ = _time_calls(call_host, stream, steps, dev, between=flush_w.zero_)
+        assert fvrag.read_status(ws) == fvrag.OK
+        Qn, K, hkv, D = cfg.num_queries, cfg.num_drafts, cfg.hkv, cfg.head_dim
+        units = Qn * K
+        metric, unit = "draft tokens decoded/s (one attention layer)", "tokens/s"
+        sumP = int(x["prefix_offsets"][-1])
+        sumN = int(x["cache_len"].sum())
+        nbytes = (sumP + sumN) * hkv * D * 2 * 2 + 2 * q.numel() * 2
+        roof = {"bound": "hbm", "achieved": nbytes / (t_ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "traffic": None, "peak_source": pk_src,
+                "kernel": "fvrag shared-prefix attention in decode form (Lq = 1), timed with its "
+                          "merge kernel"}
+        roof["frac"] = roof["achieved"] / roof["peak"]
+        h2d = q.numel() * 2 + n.numel() * 4
+        d2h = out.numel() * 2
+        config = {"workload": cfg.description, "name": cfg.name, "drafts": units,
+                  "prefix_tokens": sumP, "cache_tokens": sumN, "heads": [cfg.hq, hkv, D],
+                  "l2": "flushed before every timed call (256 MiB write, outside the events)",
+                  "parallelism": "replicas"}
+        dtype = "bf16"
+        launches = 2
+        cpu = None
+        if not args.no_cpu_baseline and ws_ == 1:
+            oracle.build()
+            a, b = int(x["prefix_offsets"][0]), int(x["prefix_offsets"][1])
+            t0 = time.perf_counter()
+            reps = 0
+            while True:
+                oracle.decode_attn(x["q"][:1], x["k_prefix"][a:b], x["v_prefix"][a:b],
+                                   np.array([0, b - a], np.int32), x["k_cache"][:1], x["v_cache"][:1],
+                                   x["cache_len"][:1])
+                reps += 1
+                if time.perf_counter() - t0 > args.cpu_budget:
+                    break
+            dt = time.perf_counter() - t0
+            cpu = {"value": reps * K / dt, "unit": unit, "cores": oracle.max_threads(),
+                   "kind": "oracle", "sample": "%d passes over query 0 (%d drafts, all heads), %.1f s"
+                   % (reps, K, dt)}
     else:
-        cfg = configs.KF_720P
+        cfg = configs.KEYFRAME_PRESETS[args.row_config or "keyframe-8x720p"]
         px, voffs = synth.video_frames(cfg, seed=cfg.seed + 7919 * rank)
         T = int(voffs[-1])
         pixels = torch.from_numpy(px).to(dev)
@@ -429,18 +508,24 @@ def bench_row(args):
         d2h = T * 4 + (cfg.num_videos + 1) * 4
         config = {"workload": cfg.description, "name": cfg.name, "frames": T,
                   "resolution": [cfg.width, cfg.height], "theta": cfg.theta,
-                  "l2": "inputs larger than L2 (14.8 GB of frames per call)", "parallelism": "replicas"}
+                  "l2": "inputs larger than L2 (%.2f GB of frames per call)" % (T * cfg.npix * 3 / 1e9),
+                  "parallelism": "replicas"}
         dtype = "u8"
         launches = 3
         cpu = None
         if not args.no_cpu_baseline and ws_ == 1:
             oracle.build()
-            n = min(T, 90)
+            n = int(voffs[1])
             t0 = time.perf_counter()
-            oracle.keyframes(px[:n], np.array([0, n], np.int32), cfg.theta)
+            reps = 0
+            while True:
+                oracle.keyframes(px[:n], np.array([0, n], np.int32), cfg.theta)
+                reps += 1
+                if time.perf_counter() - t0 > args.cpu_budget:
+                    break
             dt = time.perf_counter() - t0
-            cpu = {"value": n / dt, "unit": unit, "cores": oracle.max_threads(), "kind": "oracle",
-                   "sample": "the first %d frames of video 0, %.1f s" % (n, dt)}
+            cpu = {"value": reps * n / dt, "unit": unit, "cores": oracle.max_threads(), "kind": "oracle",
+                   "sample": "%d passes over video 0 (%d frames), %.1f s" % (reps, n, dt)}
 
     t_ms, e_ms = max_over_ranks([t_ms, e_ms], dev)
     if rank == 0:
@@ -471,9 +556,13 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=8)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--row", default="verify", choices=["verify", "retrieve", "keyframes"],
-                    help="verify: the verify step (default); retrieve / keyframes: the retrieval "
-                         "(Eq. 2-3) or keyframe (Eq. 1) step on its own workload")
+    ap.add_argument("--row", default="verify", choices=["verify", "retrieve", "keyframes", "decode"],
+                    help="verify: the verify step (default); retrieve / keyframes / decode: the "
+                         "retrieval (Eq. 2-3), keyframe (Eq. 1) or drafter decode-attention "
+                         "(Eq. 5) step on its own workload")
+    ap.add_argument("--row-config", default=None,
+                    help="workload preset of --row (default: retrieve-16q-1m / keyframe-8x720p / "
+                         "decode-3b-16q)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     if args.row != "verify":

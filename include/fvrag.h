@@ -20,6 +20,11 @@
  *                           frame embedding, max/argmax over frames, keep flag;
  *   fvrag_select_candidate  the per-query selection reduction.
  *
+ * the drafts' own decode step (Eq. 5, Eq. 8-10):
+ *
+ *   fvrag_decode_attn       each draft's newest token over the shared prefix and
+ *                           its own cached tokens (the same kernel as above);
+ *
  * and the two data-parallel steps before the drafts (Section 3.1, "Multimodal
  * Retrieval"; Algorithm 1's first two loops):
  *
@@ -55,7 +60,7 @@
 extern "C" {
 #endif
 
-#define FVRAG_ABI_VERSION 3
+#define FVRAG_ABI_VERSION 4
 
 /* cudaStream_t without including the CUDA headers. */
 typedef struct CUstream_st* fvrag_stream_t;
@@ -120,6 +125,52 @@ fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* q, const vo
                                const void* v_prefix, const int32_t* prefix_offsets,
                                const void* k_tail, const void* v_tail, void* out, float* lse,
                                void* ws, size_t ws_bytes, fvrag_stream_t stream);
+
+/* ------------------------------------------------------------------------ *
+ * 1b. Drafter decode step (Eq. 5; the generation of e_i, r_i, a_i in Eq. 8-10)
+ *
+ * The K drafts of a query are generated in parallel from the shared prefix
+ * (video tokens and question) followed by each draft's own tokens (its retrieved
+ * text t_i, then what it has generated so far).  One call is one decode step:
+ * for query q, draft k and query head h (KV head g = h / (hq / hkv)),
+ *   keys   = the P_q prefix tokens of query q, then own slots 0 .. n_k - 1 of draft k
+ *            (the newest token, whose K/V is already in slot n_k - 1, included;
+ *            drafts never see one another's tokens)
+ *   out    = softmax(scale * q . K^T) V,  lse as in fvrag_verify_attn.
+ * Same kernel as fvrag_verify_attn: the prefix is read once for all drafts.
+ * ------------------------------------------------------------------------ */
+typedef struct fvrag_decode_desc {
+  int32_t num_queries;  /* Qn >= 1 */
+  int32_t num_drafts;   /* K >= 1 */
+  int32_t cache_cap;    /* C >= 1: own-token slots per draft */
+  int32_t hq;           /* query heads, multiple of hkv, hq / hkv <= 128 */
+  int32_t hkv;          /* KV heads >= 1 */
+  int32_t head_dim;     /* D: 64 or 128 */
+  int32_t max_prefix;   /* upper bound on every P_q; >= 0 */
+  int32_t total_prefix; /* sum over queries of P_q */
+  float softmax_scale;  /* > 0, or 0 => 1/sqrt(head_dim) */
+  uint32_t flags;       /* must be 0 */
+} fvrag_decode_desc;
+
+size_t fvrag_decode_attn_workspace(const fvrag_decode_desc* d);
+
+/*
+ *   q              [Qn][K][hq][D]        bf16   the newest token of each draft
+ *   k_prefix, v_prefix, prefix_offsets   as in fvrag_verify_attn
+ *   k_cache        [Qn][K][C][hkv][D]    bf16   each draft's own keys / values
+ *   v_cache        [Qn][K][C][hkv][D]    bf16
+ *   cache_len      [Qn][K]               int32  device; n_k in [1, C] (values outside are
+ *                                               clamped to [0, C], not reported)
+ *   out            [Qn][K][hq][D]        bf16   written
+ *   lse            [Qn][K][hq]           fp32   written when not NULL
+ *   ws / ws_bytes  workspace of at least fvrag_decode_attn_workspace(d) bytes
+ * Slots at or past n_k are never read into the result (they may hold anything).
+ */
+fvrag_status fvrag_decode_attn(const fvrag_decode_desc* d, const void* q, const void* k_prefix,
+                               const void* v_prefix, const int32_t* prefix_offsets,
+                               const void* k_cache, const void* v_cache, const int32_t* cache_len,
+                               void* out, float* lse, void* ws, size_t ws_bytes,
+                               fvrag_stream_t stream);
 
 /* ------------------------------------------------------------------------ *
  * 2. LM-head log-probabilities (Eq. 11; the verifier likelihood of Section 4.6)

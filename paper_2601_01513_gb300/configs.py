@@ -109,7 +109,12 @@ RT_16Q_1M = RetrievalConfig(
     description="16 queries x 4-32 keyframes against 1,048,576 CLIP ViT-L/14 text embeddings "
                 "(dim 768, fp16)")
 
-RETRIEVAL_PRESETS = {c.name: c for c in (RT_TINY, RT_16Q_1M)}
+RT_16Q_256K = RT_16Q_1M.with_(
+    name="retrieve-16q-256k", num_texts=1 << 18,
+    description="16 queries x 4-32 keyframes against 262,144 text embeddings (dim 768, fp16; "
+                "the profiling size)")
+
+RETRIEVAL_PRESETS = {c.name: c for c in (RT_TINY, RT_16Q_1M, RT_16Q_256K)}
 
 
 @dataclass(frozen=True)
@@ -147,4 +152,46 @@ KF_720P = KeyframeConfig(
     description="8 videos of 500-840 frames (16.7-28 s at 30 frames/s, mean 22.3 s) at 1280x720 "
                 "RGB uint8")
 
-KEYFRAME_PRESETS = {c.name: c for c in (KF_TINY, KF_720P)}
+KF_720P_1V = KF_720P.with_(
+    name="keyframe-1x720p", num_videos=1, frames_range=(300, 300),
+    description="1 video of 300 frames at 1280x720 RGB uint8 (the profiling size)")
+
+KEYFRAME_PRESETS = {c.name: c for c in (KF_TINY, KF_720P, KF_720P_1V)}
+
+
+@dataclass(frozen=True)
+class DecodeConfig:
+    """One decode step of the drafter (Eq. 5, Eq. 8-10): ``num_queries`` queries,
+    each with ``num_drafts`` drafts generated in parallel from one shared prefix
+    (video tokens and question) of ``prefix_len`` tokens (or ragged in
+    ``prefix_range``) and an own-token cache of ``cache_cap`` slots per draft, of
+    which n_k ~ U[cache_range] are filled (retrieved text plus generated tokens)."""
+    name: str
+    num_queries: int
+    num_drafts: int
+    hq: int
+    hkv: int
+    head_dim: int
+    prefix_len: int
+    cache_cap: int
+    cache_range: tuple              # (lo, hi) inclusive filled slots per draft
+    prefix_range: tuple = None
+    seed: int = 20260104
+    description: str = ""
+
+    def with_(self, **kw) -> "DecodeConfig":
+        return replace(self, **kw)
+
+
+DEC_TINY = DecodeConfig(
+    name="decode-tiny", num_queries=2, num_drafts=3, hq=4, hkv=2, head_dim=64, prefix_len=0,
+    prefix_range=(40, 300), cache_cap=150, cache_range=(1, 150),
+    description="2 queries x 3 drafts, 4/2 heads of 64, ragged prefix 40-300, caches of 1-150 of 150")
+
+DEC_3B_16Q = DecodeConfig(
+    name="decode-3b-16q", num_queries=16, num_drafts=5, hq=16, hkv=2, head_dim=128, prefix_len=0,
+    prefix_range=(4096, 16384), cache_cap=1024, cache_range=(256, 1024),
+    description="3B-class drafter (Qwen2.5-VL-3B shapes: 16/2 heads of 128), 16 queries x 5 drafts, "
+                "ragged shared prefix U[4096,16384], own caches of U[256,1024] of 1024 slots")
+
+DECODE_PRESETS = {c.name: c for c in (DEC_TINY, DEC_3B_16Q)}

@@ -1,32 +1,41 @@
 // K1: one attention layer of the verifier forward over all candidate rows
 // (Eq. 6 / Eq. 11): token l of candidate k attends to the P_q tokens of the
-// shared prefix and to tokens 0..l of its own candidate.
+// shared prefix and to tokens 0..l of its own candidate.  The same kernel runs
+// one decode step of the drafts (Eq. 5, Eq. 8-10): the newest token of each
+// draft attends to the shared prefix and to the draft's own cached tokens.
+//
+// General form: every candidate owns C own-token slots of which the first n_k
+// are valid, and its Lq query tokens are the last Lq of those n_k (query l sits
+// at slot n_k - Lq + l and sees own slots 0 .. n_k - Lq + l).  Verification is
+// Lq = C = n_k = L; a decode step is Lq = 1 with n_k read from the device.
 //
 // The prefix (up to 32768 keys) is shared by every candidate row, so all
-// K x L x (hq/hkv) query rows that use one KV head are packed into the rows of
-// the tensor-core tiles (GQA packing): a row tile is T tokens x the hq/hkv
-// query heads of one KV head (T = floor(128 / (hq/hkv))), and every prefix K/V
-// block that a CTA loads feeds all of them.
+// query rows that use one KV head are packed into the rows of the tensor-core
+// tiles (GQA packing): a row tile is T query tokens x the hq/hkv query heads of
+// one KV head (T = floor(128 / (hq/hkv))), and every prefix K/V block that a
+// CTA loads feeds all of them.
 //
-// attn_kernel: one CTA = one row tile x one key range (split-KV).
+// Key blocks of 128: the query's prefix blocks, then the blocks of the tile's
+// candidates' own slots (concatenated) that hold at least one valid slot.  The
+// list is cut into equal runs of blocks, one run per CTA (split-KV).
+//
+// attn_kernel: one CTA = one row tile x one run of key blocks.
 //   warp 0     TMA: the Q tile once (3-D map over [tokens][hq][D]), then K and V
-//              blocks of 64 keys (3-D maps over [keys][hkv][D], 128-byte swizzle)
-//              into two 5-deep rings, K and V each issued as soon as its ring has
-//              a free slot.  Split 0 also streams the candidates' own tail
-//              tokens as extra key blocks.
+//              blocks (3-D maps over [keys][hkv][D], 128-byte swizzle) into two
+//              3-deep rings, K and V each issued as soon as its ring has a free slot.
 //   warp 1     allocates tensor memory and issues tcgen05.mma:
-//                S_j  = Q K_j^T  (M = 128 rows, N = 64 keys, K = D; both K-major)
-//                O   += P_j V_j  (M = 128, N = D, K = 64 keys; V read MN-major)
-//              with S double-buffered and O accumulated in tensor memory.
-//   warps 2-5  one query row per thread: tcgen05.ld of S_j, masking (key range,
-//              or same-candidate causal range for tail blocks; full blocks skip
-//              it), online softmax in base 2 against a lazily moved reference
-//              max (O and l are rescaled in place only when a row's max grows by
-//              more than 2^8), and P_j written to shared memory as a
-//              128-byte-swizzled bf16 tile for the next MMA.
-//   One split: the CTA writes the bf16 output and the lse directly.  Several
-//   splits: normalised partials go to the workspace and merge_kernel combines
-//   them with log-sum-exp weights.
+//                S_j  = Q K_j^T   (M = 128 rows, N = 128 keys, K = D; both K-major)
+//                O   += P_j V_j   (M = 128, N = D, K = 128 keys; P_j read from tensor
+//                                  memory, V MN-major from shared memory)
+//              with S/P double-buffered and O accumulated in tensor memory.
+//   warps 2-5  one query row per thread: tcgen05.ld of S_j, masking (prefix length,
+//              or the row's own visible slots; full blocks skip it), online softmax
+//              in base 2 against a lazily moved reference max (O and l are rescaled
+//              in place only when a row's max grows by more than 2^8), and P_j
+//              written back as bf16 pairs over S_j in tensor memory.
+//   One run: the CTA writes the bf16 output and the lse directly.  Several runs:
+//   normalised partials go to the workspace and merge_kernel combines them with
+//   log-sum-exp weights.
 #include <cuda_bf16.h>
 
 #include <algorithm>
@@ -41,7 +50,8 @@ constexpr int kThreads = 192;
 constexpr int kBM = 128;          // query rows per tile (MMA M)
 constexpr int kBN = 128;          // keys per block (MMA N of S, K of PV)
 constexpr int kStages = 3;        // depth of each of the K ring and the V ring
-constexpr int kMaxTail = 64;
+constexpr int kMaxTail = 64;            // verification: tokens per candidate
+constexpr int kMaxCand = kBM + 1;       // candidates a row tile can touch
 constexpr uint32_t kTmemCols = 512;
 // tensor-memory columns: S/P buffers at 0 and 128 (S_j as fp32 in 128 columns, then
 // P_j as packed bf16 in the first 64), the O accumulator at 256
@@ -60,18 +70,20 @@ struct Layout {
   static constexpr int kQ = NH * kBM * 128;         // Q tile
   static constexpr int kKVHalf = kBN * 128;         // 128 keys x 64 elements
   static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
-  static constexpr int kBytes = kQ + 2 * kStages * kStage + 1024 + 256;
+  static constexpr int kBytes = kQ + 2 * kStages * kStage + 1024 + 256 + kMaxCand * 4;
+  static_assert(kBytes <= 232448, "shared memory per CTA");
 };
 
 struct Args {
   const int32_t* offs;
+  const int32_t* own_len;  // [Qn][K] valid own slots n_k, or null (n_k = C)
   __nv_bfloat16* out;     // final output (one split)
   float* lse;             // final lse (one split), may be null
   float* part_o;          // [nsplit][rows][D]  (several splits)
   float* part_lse;        // [nsplit][rows]
   uint32_t* status;
   uint64_t limit_ns;
-  int Qn, K, L, KL, hq, hkv, grp, T, mtiles, nsplit, chunk;
+  int Qn, K, Lq, C, KL, hq, hkv, grp, T, mtiles, nsplit, bps;
   float scale_log2;
 };
 
@@ -147,17 +159,19 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int g = b % a.hkv;
   const int qi = b / a.hkv;
   const int P = __ldg(&a.offs[qi + 1]) - __ldg(&a.offs[qi]);
-  const int key_lo = split * a.chunk;
-  const int key_hi = min(P, key_lo + a.chunk);
-  const int nbp = key_hi > key_lo ? (key_hi - key_lo + kBN - 1) / kBN : 0;
+  const int nbp = (P + kBN - 1) / kBN;                 // prefix blocks of this query
   const int tok0 = mt * a.T;
   const int ntok = min(a.T, a.KL - tok0);
   const int rows = ntok * a.grp;
-  const int c_lo = tok0 / a.L;
-  const int c_hi = (tok0 + ntok - 1) / a.L;
-  const int nbt = split == 0 ? ((c_hi - c_lo + 1) * a.L + kBN - 1) / kBN : 0;
-  const int nblk = nbp + nbt;
-
+  const int c_lo = tok0 / a.Lq;
+  const int ncand = (tok0 + ntok - 1) / a.Lq - c_lo + 1;
+  const int ntb = (ncand * a.C + kBN - 1) / kBN;       // blocks over the candidates' own slots
+  // valid own slots of the tile's candidates (the own blocks with none are skipped)
+  int* n_own = reinterpret_cast<int*>(s_full + 8) + 4;
+  for (int c = threadIdx.x; c < ncand; c += kThreads) {
+    int n = a.own_len ? __ldg(&a.own_len[qi * a.K + c_lo + c]) : a.C;
+    n_own[c] = n < 0 ? 0 : (n > a.C ? a.C : n);
+  }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
@@ -194,6 +208,44 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
+  // own block tb holds a valid slot when some candidate c it overlaps has
+  // c * C + n_c > tb * kBN (each candidate's valid slots are its first n_c)
+  auto own_valid = [&](int tb) {
+    const int s0 = tb * kBN;
+    const int s1 = min(s0 + kBN, ncand * a.C);
+    for (int c = s0 / a.C; c * a.C < s1; ++c)
+      if (c * a.C + n_own[c] > s0) return true;
+    return false;
+  };
+  auto own_next = [&](int tb) {                      // first valid own block >= tb
+    while (tb < ntb && !own_valid(tb)) ++tb;
+    return tb;
+  };
+  // count the valid own blocks and find the first one this run uses, 32 blocks per
+  // step of the warp (every warp computes the same values)
+  const int blk_lo = split * a.bps;
+  int nvt = 0, tb_first = -1;
+  {
+    int skip = max(0, blk_lo - nbp);               // valid own blocks before this run's first
+    for (int base = 0; base < ntb; base += 32) {
+      const int tb = base + lane;
+      const uint32_t m = __ballot_sync(0xffffffffu, tb < ntb && own_valid(tb));
+      const int cnt = __popc(m);
+      if (tb_first < 0) {
+        if (skip < cnt) {
+          uint32_t mm = m;
+          for (int i = 0; i < skip; ++i) mm &= mm - 1u;
+          tb_first = base + __ffs(mm) - 1;
+        } else {
+          skip -= cnt;
+        }
+      }
+      nvt += cnt;
+    }
+    if (tb_first < 0) tb_first = ntb;
+  }
+  const int nb = nbp + nvt;
+  const int nblk = max(0, min(nb, blk_lo + a.bps) - blk_lo);
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -207,9 +259,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int h = 0; h < NH; ++h)
         tma_load_3d(smem_u32(q_s + h * kBM * 128), &tm_q, qb, h * 64, g * a.grp,
                     qi * a.KL + tok0, pol_q);
-      const int pbase = __ldg(&a.offs[qi]) + key_lo;
-      const int tbase = qi * a.KL + c_lo * a.L;
+      const int pbase = __ldg(&a.offs[qi]);
+      const int tbase = (qi * a.K + c_lo) * a.C;       // own slot 0 of candidate c_lo
       int nk = 0, nv = 0;
+      int tbk = tb_first, tbv = tb_first;               // own-block cursors of the two rings
       uint64_t t_last = globaltimer_ns();
       while (nk < nblk || nv < nblk) {
         bool moved = false;
@@ -217,8 +270,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t fb = smem_u32(&k_full[nk % kStages]);
           mbar_arrive_expect_tx(fb, Lay::kStage);
           uint8_t* dst = k_ring + (nk % kStages) * Lay::kStage;
-          const bool pre = nk < nbp;
-          const int key = pre ? pbase + nk * kBN : tbase + (nk - nbp) * kBN;
+          const int bi = blk_lo + nk;
+          const bool pre = bi < nbp;
+          int key;
+          if (pre) {
+            key = pbase + bi * kBN;
+          } else {
+            tbk = own_next(tbk);
+            key = tbase + tbk * kBN;
+            ++tbk;
+          }
           for (int h = 0; h < NH; ++h)
             tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), pre ? &tm_kp : &tm_kt, fb, h * 64, g, key,
                         pol_kv);
@@ -229,8 +290,16 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t fb = smem_u32(&v_full[nv % kStages]);
           mbar_arrive_expect_tx(fb, Lay::kStage);
           uint8_t* dst = v_ring + (nv % kStages) * Lay::kStage;
-          const bool pre = nv < nbp;
-          const int key = pre ? pbase + nv * kBN : tbase + (nv - nbp) * kBN;
+          const int bi = blk_lo + nv;
+          const bool pre = bi < nbp;
+          int key;
+          if (pre) {
+            key = pbase + bi * kBN;
+          } else {
+            tbv = own_next(tbv);
+            key = tbase + tbv * kBN;
+            ++tbv;
+          }
           for (int h = 0; h < NH; ++h)
             tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), pre ? &tm_vp : &tm_vt, fb, h * 64, g, key,
                         pol_kv);
@@ -324,9 +393,12 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
     const bool rvalid = r < rows;
     const int tok = tok0 + r / a.grp;
-    const int krow = tok / a.L, lrow = tok % a.L;
-    const int tlo = (krow - c_lo) * a.L;               // visible tail range [tlo, tlo + lrow]
-    const int thi = tlo + lrow + 1;
+    const int crow = min(tok / a.Lq - c_lo, ncand - 1);  // rows past the tile: any candidate
+    const int lrow = tok % a.Lq;
+    // visible own slots of this row, in the tile's concatenated own-slot space
+    const int tlo = crow * a.C;
+    const int thi = tlo + max(0, n_own[crow] - a.Lq + lrow + 1);
+    int tbs = tb_first;                                // own-block cursor
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
@@ -343,11 +415,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         tmem_ld_32x32b_x32(lane_base + col_s(sb) + c0, *reinterpret_cast<uint32_t(*)[32]>(&sr[c0]));
       tmem_wait_ld();
       int vlo, vhi;   // valid columns of this block for this row
-      if (j < nbp) {
+      if (blk_lo + j < nbp) {
         vlo = 0;
-        vhi = min(kBN, key_hi - (key_lo + j * kBN));
+        vhi = min(kBN, P - (blk_lo + j) * kBN);
       } else {
-        const int base = (j - nbp) * kBN;
+        tbs = own_next(tbs);
+        const int base = tbs * kBN;
+        ++tbs;
         vlo = max(0, tlo - base);
         vhi = min(kBN, thi - base);
       }
@@ -522,26 +596,37 @@ __global__ void merge_kernel(const float* __restrict__ part_o, const float* __re
   if (lane == 0 && lse_out) lse_out[row] = mx + __logf(den);
 }
 
-struct Plan {
-  int grp, T, mtiles, nsplit, chunk;
+// One attention problem in the general form of the kernel (see the top of the file).
+struct Problem {
+  int Qn, K, Lq, C, hq, hkv, D, max_prefix, total_prefix;
+  float scale;                 // 0 => 1/sqrt(D)
+  const int32_t* own_len;      // device [Qn][K] or null (every candidate has C valid slots)
 };
 
-// Key-split plan: pick the number of splits that minimises an estimate of
-// waves x (blocks per CTA + fixed cost) plus the cost of writing and merging the
-// partials (one CTA per SM; a 128-key block is ~0.6 us).
-static Plan make_plan(const fvrag_attn_desc* d, int sms) {
+struct Plan {
+  int grp, T, mtiles, nsplit, bps;
+};
+
+// Key-split plan: the longest block list a row tile can have (the longest prefix
+// plus every own block of the candidates a tile can touch) is cut into runs of
+// `bps` blocks; pick the run count that minimises an estimate of waves x (blocks
+// per CTA + fixed cost) plus the cost of writing and merging the partials (one CTA
+// per SM; a 128-key block is ~0.6 us).
+static Plan make_plan(const Problem& pr, int sms) {
   Plan p;
-  p.grp = d->hq / d->hkv;
+  p.grp = pr.hq / pr.hkv;
   p.T = std::max(1, kBM / p.grp);
-  const int KL = d->num_cand * d->cand_len;
+  const int KL = pr.K * pr.Lq;
   p.mtiles = (KL + p.T - 1) / p.T;
-  const long long base = (long long)d->num_queries * d->hkv * p.mtiles;
-  const int nb = (std::max(d->max_prefix, 0) + kBN - 1) / kBN;
+  const long long base = (long long)pr.Qn * pr.hkv * p.mtiles;
+  const int ncand = std::min(pr.K, (p.T + pr.Lq - 1) / pr.Lq + 1);
+  const int nb = (std::max(pr.max_prefix, 0) + kBN - 1) / kBN +
+                 (int)(((long long)ncand * pr.C + kBN - 1) / kBN);
   p.nsplit = 1;
-  p.chunk = std::max(nb, 1) * kBN;
+  p.bps = std::max(nb, 1);
   if (nb <= 1) return p;
   if (sms <= 0) sms = 148;
-  const double rows = (double)d->num_queries * KL * d->hq;
+  const double rows = (double)pr.Qn * KL * pr.hq;
   double best = 1e30;
   for (int ns = 1; ns <= std::min(nb, 64); ++ns) {
     const int per = (nb + ns - 1) / ns;
@@ -549,20 +634,20 @@ static Plan make_plan(const fvrag_attn_desc* d, int sms) {
     const long long ctas = base * nse;
     const double waves = (double)((ctas + sms - 1) / sms);
     double t = waves * (per + 3) * 0.6;
-    if (nse > 1) t += 3.0 + nse * rows * (d->head_dim + 1) * 8.0 / 8.0e6;
+    if (nse > 1) t += 3.0 + nse * rows * (pr.D + 1) * 8.0 / 8.0e6;
     if (t < best - 1e-9) {
       best = t;
       p.nsplit = nse;
-      p.chunk = per * kBN;
+      p.bps = per;
     }
   }
   return p;
 }
 
-static size_t ws_bytes(const fvrag_attn_desc* d, int sms) {
-  const Plan p = make_plan(d, sms);
-  const size_t rows = (size_t)d->num_queries * d->num_cand * d->cand_len * d->hq;
-  return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)d->head_dim + 1) * 4 : 0);
+static size_t ws_bytes(const Problem& pr, int sms) {
+  const Plan p = make_plan(pr, sms);
+  const size_t rows = (size_t)pr.Qn * pr.K * pr.Lq * pr.hq;
+  return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)pr.D + 1) * 4 : 0);
 }
 
 static int device_sms() {
@@ -582,6 +667,101 @@ static fvrag_status launch(const CUtensorMap* maps, const Args& a, long long gri
   return launch_status();
 }
 
+// Shape checks shared by both entry points (after their own argument checks).
+static fvrag_status check_problem(const Problem& pr) {
+  if (pr.hq % pr.hkv != 0 || (pr.D != 64 && pr.D != 128) || pr.hq / pr.hkv > kBM)
+    return FVRAG_ERR_UNSUPPORTED;
+  if ((long long)pr.Qn * pr.K * pr.C >= (1LL << 31) || (long long)pr.Qn * pr.K * pr.Lq >= (1LL << 31) ||
+      (long long)pr.total_prefix + kBN >= (1LL << 31))
+    return FVRAG_ERR_UNSUPPORTED;
+  return FVRAG_OK;
+}
+
+// q [Qn][K][Lq][hq][D]; own K/V [Qn][K][C][hkv][D]; out like q.
+static fvrag_status run(const Problem& pr, const void* q, const void* k_prefix, const void* v_prefix,
+                        const int32_t* prefix_offsets, const void* k_own, const void* v_own,
+                        void* out, float* lse, void* ws, size_t ws_size, cudaStream_t s) {
+  const int sms = device_sms();
+  const size_t need = ws_bytes(pr, sms);
+  if (!ws || ws_size < need) return FVRAG_ERR_WORKSPACE;
+  if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
+
+  const Plan p = make_plan(pr, sms);
+  const int D = pr.D;
+  const float scale = pr.scale != 0.f ? pr.scale : 1.f / sqrtf((float)D);
+  const int KL = pr.K * pr.Lq;
+  const long long nrows = (long long)pr.Qn * KL * pr.hq;
+  uint8_t* base = reinterpret_cast<uint8_t*>(ws);
+
+  CUtensorMap maps[5];
+  {
+    const uint64_t dims[3] = {(uint64_t)D, (uint64_t)pr.hq, (uint64_t)pr.Qn * KL};
+    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)pr.hq * D * 2};
+    const uint32_t box[3] = {64u, (uint32_t)p.grp, (uint32_t)p.T};
+    if (!encode_tmap_bf16(&maps[0], q, 3, dims, strides, box, true)) return FVRAG_ERR_CUDA;
+  }
+  {
+    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)pr.hkv * D * 2};
+    const uint32_t box[3] = {64u, 1u, (uint32_t)kBN};
+    const uint64_t tdims[3] = {(uint64_t)D, (uint64_t)pr.hkv, (uint64_t)pr.Qn * pr.K * pr.C};
+    if (!encode_tmap_bf16(&maps[3], k_own, 3, tdims, strides, box, true)) return FVRAG_ERR_CUDA;
+    if (!encode_tmap_bf16(&maps[4], v_own, 3, tdims, strides, box, true)) return FVRAG_ERR_CUDA;
+    if (pr.total_prefix > 0) {
+      const uint64_t pdims[3] = {(uint64_t)D, (uint64_t)pr.hkv, (uint64_t)pr.total_prefix};
+      if (!encode_tmap_bf16(&maps[1], k_prefix, 3, pdims, strides, box, true)) return FVRAG_ERR_CUDA;
+      if (!encode_tmap_bf16(&maps[2], v_prefix, 3, pdims, strides, box, true)) return FVRAG_ERR_CUDA;
+    } else {
+      maps[1] = maps[3];   // never read: no query has prefix keys
+      maps[2] = maps[4];
+    }
+  }
+  Args a;
+  a.offs = prefix_offsets;
+  a.own_len = pr.own_len;
+  a.out = reinterpret_cast<__nv_bfloat16*>(out);
+  a.lse = lse;
+  a.part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
+  a.part_lse = a.part_o + (size_t)p.nsplit * nrows * D;
+  a.status = reinterpret_cast<uint32_t*>(base);
+  a.limit_ns = wait_limit_ns();
+  a.Qn = pr.Qn;
+  a.K = pr.K;
+  a.Lq = pr.Lq;
+  a.C = pr.C;
+  a.KL = KL;
+  a.hq = pr.hq;
+  a.hkv = pr.hkv;
+  a.grp = p.grp;
+  a.T = p.T;
+  a.mtiles = p.mtiles;
+  a.nsplit = p.nsplit;
+  a.bps = p.bps;
+  a.scale_log2 = scale * kLog2e;
+  const long long grid = (long long)pr.Qn * pr.hkv * p.nsplit * p.mtiles;
+  if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
+  fvrag_status st = D == 128 ? launch<128>(maps, a, grid, s) : launch<64>(maps, a, grid, s);
+  if (st != FVRAG_OK || p.nsplit == 1) return st;
+  const int wpb = 8;
+  const long long blocks = (nrows + wpb - 1) / wpb;
+  const cudaError_t e =
+      D == 128 ? launch_pdl(merge_kernel<128>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
+                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse)
+               : launch_pdl(merge_kernel<64>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
+                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse);
+  if (e != cudaSuccess) return FVRAG_ERR_CUDA;
+  return launch_status();
+}
+
+static Problem verify_problem(const fvrag_attn_desc* d) {
+  return Problem{d->num_queries, d->num_cand, d->cand_len, d->cand_len, d->hq, d->hkv,
+                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, nullptr};
+}
+
+static Problem decode_problem(const fvrag_decode_desc* d, const int32_t* cache_len) {
+  return Problem{d->num_queries, d->num_drafts, 1, d->cache_cap, d->hq, d->hkv,
+                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, cache_len};
+}
+
 }  // namespace attn
 }  // namespace fvrag
 
@@ -591,7 +771,7 @@ extern "C" size_t fvrag_verify_attn_workspace(const fvrag_attn_desc* d) {
   if (!d || d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
       d->hq % d->hkv || (d->head_dim != 64 && d->head_dim != 128) || d->max_prefix < 0)
     return 0;
-  return attn::ws_bytes(d, attn::device_sms());
+  return attn::ws_bytes(attn::verify_problem(d), attn::device_sms());
 }
 
 extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* q,
@@ -606,78 +786,44 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
       d->softmax_scale == INFINITY)
     return FVRAG_ERR_INVALID_ARG;
   if (d->total_prefix > 0 && (!k_prefix || !v_prefix)) return FVRAG_ERR_INVALID_ARG;
-  if (d->hq % d->hkv != 0 || (d->head_dim != 64 && d->head_dim != 128) ||
-      d->cand_len > kMaxTail || d->hq / d->hkv > kBM)
-    return FVRAG_ERR_UNSUPPORTED;
+  if (d->cand_len > kMaxTail) return FVRAG_ERR_UNSUPPORTED;
+  const Problem pr = verify_problem(d);
+  const fvrag_status cs = check_problem(pr);
+  if (cs != FVRAG_OK) return cs;
   if (!aligned16(q) || !aligned16(k_tail) || !aligned16(v_tail) || !aligned16(out) ||
       (k_prefix && !aligned16(k_prefix)) || (v_prefix && !aligned16(v_prefix)))
     return FVRAG_ERR_MISALIGNED;
-  const int sms = device_sms();
-  const size_t need = ws_bytes(d, sms);
-  if (!ws || ws_size < need) return FVRAG_ERR_WORKSPACE;
-  if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
+  return run(pr, q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, out, lse, ws, ws_size,
+             reinterpret_cast<cudaStream_t>(stream));
+}
 
-  const Plan p = make_plan(d, sms);
-  const int D = d->head_dim;
-  const float scale = d->softmax_scale != 0.f ? d->softmax_scale : 1.f / sqrtf((float)D);
-  const int KL = d->num_cand * d->cand_len;
-  const long long nrows = (long long)d->num_queries * KL * d->hq;
-  uint8_t* base = reinterpret_cast<uint8_t*>(ws);
+extern "C" size_t fvrag_decode_attn_workspace(const fvrag_decode_desc* d) {
+  if (!d || d->num_queries < 1 || d->num_drafts < 1 || d->cache_cap < 1 || d->hq < 1 ||
+      d->hkv < 1 || d->hq % d->hkv || (d->head_dim != 64 && d->head_dim != 128) || d->max_prefix < 0)
+    return 0;
+  return attn::ws_bytes(attn::decode_problem(d, nullptr), attn::device_sms());
+}
 
-  CUtensorMap maps[5];
-  {
-    const uint64_t dims[3] = {(uint64_t)D, (uint64_t)d->hq, (uint64_t)d->num_queries * KL};
-    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d->hq * D * 2};
-    const uint32_t box[3] = {64u, (uint32_t)p.grp, (uint32_t)p.T};
-    if (!encode_tmap_bf16(&maps[0], q, 3, dims, strides, box, true)) return FVRAG_ERR_CUDA;
-  }
-  {
-    const uint64_t strides[2] = {(uint64_t)D * 2, (uint64_t)d->hkv * D * 2};
-    const uint32_t box[3] = {64u, 1u, (uint32_t)kBN};
-    const uint64_t tdims[3] = {(uint64_t)D, (uint64_t)d->hkv, (uint64_t)d->num_queries * KL};
-    if (!encode_tmap_bf16(&maps[3], k_tail, 3, tdims, strides, box, true)) return FVRAG_ERR_CUDA;
-    if (!encode_tmap_bf16(&maps[4], v_tail, 3, tdims, strides, box, true)) return FVRAG_ERR_CUDA;
-    if (d->total_prefix > 0) {
-      const uint64_t pdims[3] = {(uint64_t)D, (uint64_t)d->hkv, (uint64_t)d->total_prefix};
-      if (!encode_tmap_bf16(&maps[1], k_prefix, 3, pdims, strides, box, true)) return FVRAG_ERR_CUDA;
-      if (!encode_tmap_bf16(&maps[2], v_prefix, 3, pdims, strides, box, true)) return FVRAG_ERR_CUDA;
-    } else {
-      maps[1] = maps[3];   // never read: no query has prefix keys
-      maps[2] = maps[4];
-    }
-  }
-  Args a;
-  a.offs = prefix_offsets;
-  a.out = reinterpret_cast<__nv_bfloat16*>(out);
-  a.lse = lse;
-  a.part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
-  a.part_lse = a.part_o + (size_t)p.nsplit * nrows * D;
-  a.status = reinterpret_cast<uint32_t*>(base);
-  a.limit_ns = wait_limit_ns();
-  a.Qn = d->num_queries;
-  a.K = d->num_cand;
-  a.L = d->cand_len;
-  a.KL = KL;
-  a.hq = d->hq;
-  a.hkv = d->hkv;
-  a.grp = p.grp;
-  a.T = p.T;
-  a.mtiles = p.mtiles;
-  a.nsplit = p.nsplit;
-  a.chunk = p.chunk;
-  a.scale_log2 = scale * kLog2e;
-  const long long grid = (long long)d->num_queries * d->hkv * p.nsplit * p.mtiles;
-  if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  fvrag_status st = D == 128 ? launch<128>(maps, a, grid, s) : launch<64>(maps, a, grid, s);
-  if (st != FVRAG_OK || p.nsplit == 1) return st;
-  const int wpb = 8;
-  const long long blocks = (nrows + wpb - 1) / wpb;
-  const cudaError_t e =
-      D == 128 ? launch_pdl(merge_kernel<128>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
-                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse)
-               : launch_pdl(merge_kernel<64>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
-                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse);
-  if (e != cudaSuccess) return FVRAG_ERR_CUDA;
-  return launch_status();
+extern "C" fvrag_status fvrag_decode_attn(const fvrag_decode_desc* d, const void* q,
+                                          const void* k_prefix, const void* v_prefix,
+                                          const int32_t* prefix_offsets, const void* k_cache,
+                                          const void* v_cache, const int32_t* cache_len, void* out,
+                                          float* lse, void* ws, size_t ws_size,
+                                          fvrag_stream_t stream) {
+  using namespace attn;
+  if (!d || !q || !prefix_offsets || !k_cache || !v_cache || !cache_len || !out)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->num_queries < 1 || d->num_drafts < 1 || d->cache_cap < 1 || d->hq < 1 || d->hkv < 1 ||
+      d->max_prefix < 0 || d->total_prefix < 0 || d->flags != 0 || !(d->softmax_scale >= 0.f) ||
+      d->softmax_scale == INFINITY)
+    return FVRAG_ERR_INVALID_ARG;
+  if (d->total_prefix > 0 && (!k_prefix || !v_prefix)) return FVRAG_ERR_INVALID_ARG;
+  const Problem pr = decode_problem(d, cache_len);
+  const fvrag_status cs = check_problem(pr);
+  if (cs != FVRAG_OK) return cs;
+  if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out) ||
+      (k_prefix && !aligned16(k_prefix)) || (v_prefix && !aligned16(v_prefix)))
+    return FVRAG_ERR_MISALIGNED;
+  return run(pr, q, k_prefix, v_prefix, prefix_offsets, k_cache, v_cache, out, lse, ws, ws_size,
+             reinterpret_cast<cudaStream_t>(stream));
 }

@@ -253,8 +253,15 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int t = it / ngroups, grp = it % ngroups;
       const int v0 = v_lo + t * BN;
       const int ncols = min(BN, v_hi - v0);
-      const int rows16 = (ncols + 15) & ~15;
       const int mcount = min(MG, mtiles - grp * MG);
+      // the tile's inverse text norms, lane i holding column 32 c + i of chunk c; loaded
+      // before the accumulator wait so their latency hides behind the MMAs
+      float invr[BN / 32];
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        const int col = c * 32 + lane;
+        invr[c] = col < ncols ? __ldg(text_inv_norm + v0 + col) : 0.f;
+      }
       if (!mbar_wait(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
         record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
         break;
@@ -263,70 +270,54 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < mcount; ++j) {
         const int mt = grp * MG + j;
         const bool live = mt * kBM + row < M;
+        // this keyframe's running list, best first, in shared memory (row-private)
         float* ss = st_sim + (mt * kBM + row) * kf;
         int32_t* si = st_idx + (mt * kBM + row) * kf;
-        float ls[kMaxKf];
-        int li[kMaxKf];
-#pragma unroll
-        for (int p = 0; p < kMaxKf; ++p) {
-          ls[p] = p < kf ? ss[p] : -INFINITY;
-          li[p] = p < kf ? si[p] : -1;
-        }
         float thr = ss[kf - 1];
         const uint32_t tbase =
             tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * MG + j) * BN);
-        for (int c0 = 0; c0 < rows16; c0 += 32) {
+        const int nch = (ncols + 31) / 32;
+#pragma unroll 1
+        for (int c = 0; c < nch; ++c) {
+          float invc = invr[0];
+#pragma unroll
+          for (int cc = 1; cc < BN / 32; ++cc)
+            if (cc == c) invc = invr[cc];
           uint32_t r[32];
-          tmem_ld_32x32b_x32(tbase + c0, r);
+          tmem_ld_32x32b_x32(tbase + c * 32, r);
           tmem_wait_ld();
-          const int nvalid = min(32, ncols - c0);
-          if (!live) continue;
-          const float* invp = text_inv_norm + v0 + c0;    // 64-byte aligned: v0 % 16 == 0
+          const int nvalid = min(32, ncols - c * 32);
+          // fast filter: scaled similarities in place, bit i set when column i beats the list
+          uint32_t hits = 0;
 #pragma unroll
-          for (int q4 = 0; q4 < 8; ++q4) {
-            float inv[4];
-            if (q4 * 4 + 4 <= nvalid) {
-              const float4 in4 = __ldg(reinterpret_cast<const float4*>(invp) + q4);
-              inv[0] = in4.x;
-              inv[1] = in4.y;
-              inv[2] = in4.z;
-              inv[3] = in4.w;
-            } else {
-#pragma unroll
-              for (int e = 0; e < 4; ++e) inv[e] = q4 * 4 + e < nvalid ? __ldg(invp + q4 * 4 + e) : 0.f;
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int i = q4 * 4 + e;
-              const float v = __uint_as_float(r[i]) * inv[e];
-              if (i < nvalid && v > thr) {
-                float nv = v;
-                int ni = v0 + c0 + i;
-#pragma unroll
-                for (int p = 0; p < kMaxKf; ++p) {
-                  if (p < kf && better(nv, ni, ls[p], li[p])) {
-                    const float ts = ls[p];
-                    const int ti = li[p];
-                    ls[p] = nv;
-                    li[p] = ni;
-                    nv = ts;
-                    ni = ti;
-                  }
-                }
-#pragma unroll
-                for (int p = 0; p < kMaxKf; ++p)
-                  if (p == kf - 1) thr = ls[p];
-              }
-            }
+          for (int i = 0; i < 32; ++i) {
+            const float v = __uint_as_float(r[i]) * __shfl_sync(0xffffffffu, invc, i);
+            r[i] = __float_as_uint(v);
+            hits |= (v > thr ? 1u : 0u) << i;
           }
-        }
-        if (live) {
+          if (!live) hits = 0;
+          if (nvalid < 32) hits &= (1u << nvalid) - 1u;
+          // rare path: insert the hits in column order (ids ascend, so a strict >
+          // against the list keeps the smaller id first among equal similarities)
+          while (hits) {
+            const int i = __ffs(hits) - 1;
+            hits &= hits - 1u;
+            float v = 0.f;
 #pragma unroll
-          for (int p = 0; p < kMaxKf; ++p)
-            if (p < kf) {
-              ss[p] = ls[p];
-              si[p] = li[p];
+            for (int k = 0; k < 32; ++k)
+              if (k == i) v = __uint_as_float(r[k]);
+            if (!(v > thr)) continue;
+            const int id = v0 + c * 32 + i;
+            int p = kf - 1;
+            while (p > 0 && better(v, id, ss[p - 1], si[p - 1])) {
+              ss[p] = ss[p - 1];
+              si[p] = si[p - 1];
+              --p;
             }
+            ss[p] = v;
+            si[p] = id;
+            thr = ss[kf - 1];
+          }
         }
       }
       tc_fence_before();

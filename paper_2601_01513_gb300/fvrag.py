@@ -24,6 +24,7 @@ WS_HEADER_BYTES = 256
 EXPORTED = (
     "fvrag_abi_version", "fvrag_status_string",
     "fvrag_verify_attn_workspace", "fvrag_verify_attn",
+    "fvrag_decode_attn_workspace", "fvrag_decode_attn",
     "fvrag_score_logprobs_workspace", "fvrag_score_logprobs", "fvrag_score_logprobs_noalloc",
     "fvrag_clip_align", "fvrag_select_candidate",
     "fvrag_embed_inv_norms", "fvrag_retrieve_workspace", "fvrag_retrieve",
@@ -42,6 +43,14 @@ class FvragError(RuntimeError):
 class AttnDesc(ctypes.Structure):
     _fields_ = [("num_queries", ctypes.c_int32), ("num_cand", ctypes.c_int32),
                 ("cand_len", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("max_prefix", ctypes.c_int32),
+                ("total_prefix", ctypes.c_int32), ("softmax_scale", ctypes.c_float),
+                ("flags", ctypes.c_uint32)]
+
+
+class DecodeDesc(ctypes.Structure):
+    _fields_ = [("num_queries", ctypes.c_int32), ("num_drafts", ctypes.c_int32),
+                ("cache_cap", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("max_prefix", ctypes.c_int32),
                 ("total_prefix", ctypes.c_int32), ("softmax_scale", ctypes.c_float),
                 ("flags", ctypes.c_uint32)]
@@ -95,6 +104,10 @@ def lib():
         L.fvrag_verify_attn_workspace.argtypes = [ctypes.POINTER(AttnDesc)]
         L.fvrag_verify_attn.restype = i32
         L.fvrag_verify_attn.argtypes = [ctypes.POINTER(AttnDesc)] + [vp] * 8 + [vp, sz, vp]
+        L.fvrag_decode_attn_workspace.restype = sz
+        L.fvrag_decode_attn_workspace.argtypes = [ctypes.POINTER(DecodeDesc)]
+        L.fvrag_decode_attn.restype = i32
+        L.fvrag_decode_attn.argtypes = [ctypes.POINTER(DecodeDesc)] + [vp] * 9 + [vp, sz, vp]
         L.fvrag_score_logprobs_workspace.restype = sz
         L.fvrag_score_logprobs_workspace.argtypes = [ctypes.POINTER(LmDesc)]
         L.fvrag_score_logprobs.restype = i32
@@ -174,6 +187,29 @@ def verify_attn(q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, out, ws, 
                                 _ptr(prefix_offsets), _ptr(k_tail), _ptr(v_tail), _ptr(out),
                                 _ptr(lse), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream))
     _check(s, "fvrag_verify_attn")
+
+
+def decode_desc(q, k_prefix, k_cache, max_prefix, softmax_scale=0.0) -> DecodeDesc:
+    return DecodeDesc(int(q.shape[0]), int(q.shape[1]), int(k_cache.shape[2]), int(q.shape[2]),
+                      int(k_cache.shape[3]), int(q.shape[3]), int(max_prefix),
+                      0 if k_prefix is None else int(k_prefix.shape[0]), float(softmax_scale), 0)
+
+
+def decode_workspace_bytes(desc: DecodeDesc) -> int:
+    return int(lib().fvrag_decode_attn_workspace(ctypes.byref(desc)))
+
+
+def decode_attn(q, k_prefix, v_prefix, prefix_offsets, k_cache, v_cache, cache_len, out, ws,
+                max_prefix, lse=None, softmax_scale=0.0, stream=None):
+    """q [Qn][K][hq][D] bf16; k/v_prefix [sum P][hkv][D]; prefix_offsets [Qn+1] int32 (device);
+    k/v_cache [Qn][K][C][hkv][D]; cache_len [Qn][K] int32 (device); out like q;
+    lse [Qn][K][hq] fp32 or None."""
+    d = decode_desc(q, k_prefix, k_cache, max_prefix, softmax_scale)
+    s = lib().fvrag_decode_attn(ctypes.byref(d), _ptr(q), _ptr(k_prefix), _ptr(v_prefix),
+                                _ptr(prefix_offsets), _ptr(k_cache), _ptr(v_cache), _ptr(cache_len),
+                                _ptr(out), _ptr(lse), _ptr(ws), ws.numel() * ws.element_size(),
+                                _stream(stream))
+    _check(s, "fvrag_decode_attn")
 
 
 def score_logprobs(hidden, weight, targets, logprob, ws, lse=None, stream=None):

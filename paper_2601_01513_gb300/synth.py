@@ -37,7 +37,7 @@ import os
 
 import numpy as np
 
-from .configs import KeyframeConfig, RetrievalConfig, VerifyConfig
+from .configs import DecodeConfig, KeyframeConfig, RetrievalConfig, VerifyConfig
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 SYNTH_SO = os.path.join(_HERE, "libfvrag_synth.so")
@@ -47,6 +47,7 @@ S_Q, S_KP, S_VP, S_KT, S_VT, S_HID, S_W, S_TGT = 1, 2, 3, 4, 5, 6, 7, 8
 S_CAND, S_FRAME, S_PLEN, S_PERM, S_PFRAME, S_PC = 9, 10, 11, 12, 13, 14
 S_LOGPROB, S_KEEP, S_MAXCOS, S_LEN = 20, 21, 22, 23
 S_RT_NKF, S_RT_TEXT, S_RT_FRAME, S_RT_REL, S_RT_PICK, S_RT_C = 30, 31, 32, 33, 34, 35
+S_DC_Q, S_DC_KP, S_DC_VP, S_DC_KC, S_DC_VC, S_DC_LEN, S_DC_PLEN = 50, 51, 52, 53, 54, 55, 56
 S_KF_LEN, S_KF_SCENE, S_KF_CUT, S_KF_FADE, S_KF_PARAM, S_KF_NOISE = 40, 41, 42, 43, 44, 45
 
 _lib = None
@@ -221,6 +222,31 @@ def selection_inputs(num_queries, num_cand, cand_len, gathers, seed, std=1.0):
     keep = (uniform_f64((num_queries, num_cand), seed, S_KEEP) < 0.6).astype(np.uint8)
     mc = uniform_f64((num_queries, num_cand), seed, S_MAXCOS, -0.2, 0.8)
     return lp.astype(np.float32), keep, mc.astype(np.float32)
+
+
+def decode_inputs(cfg: DecodeConfig, seed=None) -> dict:
+    """One drafter decode step: q [Qn][K][hq][D], prefix K/V [sum P][hkv][D] with
+    prefix_offsets [Qn+1], own caches [Qn][K][C][hkv][D] (all N(0,1) bf16) and
+    cache_len [Qn][K] ~ U[cache_range]."""
+    seed = cfg.seed if seed is None else seed
+    Qn, K, C = cfg.num_queries, cfg.num_drafts, cfg.cache_cap
+    if cfg.prefix_range is None:
+        plen = np.full(Qn, cfg.prefix_len, dtype=np.int32)
+    else:
+        plen = uniform_i32((Qn,), seed, S_DC_PLEN, cfg.prefix_range[0], cfg.prefix_range[1] + 1)
+    offs = np.zeros(Qn + 1, dtype=np.int32)
+    offs[1:] = np.cumsum(plen)
+    tot = int(offs[-1])
+    lo, hi = cfg.cache_range
+    return {
+        "q": normal_bf16((Qn, K, cfg.hq, cfg.head_dim), seed, S_DC_Q),
+        "k_prefix": normal_bf16((tot, cfg.hkv, cfg.head_dim), seed, S_DC_KP),
+        "v_prefix": normal_bf16((tot, cfg.hkv, cfg.head_dim), seed, S_DC_VP),
+        "prefix_offsets": offs,
+        "k_cache": normal_bf16((Qn, K, C, cfg.hkv, cfg.head_dim), seed, S_DC_KC),
+        "v_cache": normal_bf16((Qn, K, C, cfg.hkv, cfg.head_dim), seed, S_DC_VC),
+        "cache_len": uniform_i32((Qn, K), seed, S_DC_LEN, lo, hi + 1),
+    }
 
 
 def unit_rows_f16(rows, dim, seed, stream) -> np.ndarray:

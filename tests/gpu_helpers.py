@@ -196,3 +196,20 @@ def check_frame_lists(gpu_idx, gpu_sim, texts, frames, oracle_frame_topk_all, to
             hi = osim[j] - osim[j + 1] if j + 1 < len(osim) else np.inf
             if lo > tol and hi > tol:
                 assert gi[j] == oi[j], (f, j, gi[j], oi[j])
+
+
+def run_decode(q, kp, vp, offs, kc, vc, n, with_lse=True, scale=0.0):
+    """fvrag_decode_attn on numpy inputs; returns (out fp32 numpy, lse numpy, status)."""
+    tq, tkc, tvc = dev_bf16(q), dev_bf16(kc), dev_bf16(vc)
+    tkp = dev_bf16(kp) if kp.shape[0] > 0 else None
+    tvp = dev_bf16(vp) if vp.shape[0] > 0 else None
+    toffs = dev(np.asarray(offs, np.int32))
+    tn = dev(np.asarray(n, np.int32))
+    maxp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
+    d = fvrag.decode_desc(tq, tkp, tkc, maxp, scale)
+    ws = torch.zeros(fvrag.decode_workspace_bytes(d), dtype=torch.uint8, device="cuda")
+    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device="cuda")
+    lse = torch.full(q.shape[:-1], float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
+    fvrag.decode_attn(tq, tkp, tvp, toffs, tkc, tvc, tn, out, ws, maxp, lse=lse, softmax_scale=scale)
+    st = fvrag.read_status(ws)
+    return out.float().cpu().numpy(), (lse.cpu().numpy() if with_lse else None), st

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert L.fvrag_abi_version() == 3
+    assert L.fvrag_abi_version() == 4
     for s in range(7):
         assert fvrag.status_string(s)
     assert fvrag.status_string(99) == "unknown status"
@@ -185,3 +185,27 @@ def test_keyframes_validation(L):
     assert _kf(L, good, px=PMIS) == fvrag.ERR_MISALIGNED
     assert _kf(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE
     assert _kf(L, good, ws=None) == fvrag.ERR_WORKSPACE
+
+
+def _dec(L, d, ws_bytes=1 << 30, q=P, kp=P, vp=P, offs=P, kc=P, vc=P, n=P, out=P, ws=P):
+    return L.fvrag_decode_attn(ctypes.byref(d), q, kp, vp, offs, kc, vc, n, out, None, ws, ws_bytes, None)
+
+
+def test_decode_validation(L):
+    assert ctypes.sizeof(fvrag.DecodeDesc) == 40
+    good = fvrag.DecodeDesc(16, 5, 1024, 16, 2, 128, 16384, 160000, 0.0, 0)
+    ws = L.fvrag_decode_attn_workspace(ctypes.byref(good))
+    assert ws >= 256
+    assert _dec(L, fvrag.DecodeDesc(0, 5, 1024, 16, 2, 128, 16384, 160000, 0.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, fvrag.DecodeDesc(16, 5, 0, 16, 2, 128, 16384, 160000, 0.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, fvrag.DecodeDesc(16, 5, 1024, 16, 2, 128, 16384, 160000, -1.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, fvrag.DecodeDesc(16, 5, 1024, 16, 2, 128, 16384, 160000, 0.0, 4)) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, good, n=None) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, good, kc=None) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, good, kp=None) == fvrag.ERR_INVALID_ARG
+    assert _dec(L, fvrag.DecodeDesc(16, 5, 1024, 16, 3, 128, 16384, 160000, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _dec(L, fvrag.DecodeDesc(16, 5, 1024, 16, 2, 96, 16384, 160000, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _dec(L, fvrag.DecodeDesc(1 << 16, 64, 1024, 16, 2, 128, 0, 0, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
+    assert _dec(L, good, q=PMIS) == fvrag.ERR_MISALIGNED
+    assert _dec(L, good, kc=PMIS) == fvrag.ERR_MISALIGNED
+    assert _dec(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE

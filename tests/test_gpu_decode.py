@@ -1,0 +1,74 @@
+"""GPU parity of the drafter decode step (Eq. 5, Eq. 8-10) against the fp64 oracle,
+through the C ABI."""
+import numpy as np
+import pytest
+
+from oracle import oracle
+from paper_2601_01513_gb300 import configs, fvrag, synth
+
+from gpu_helpers import ATTN_ATOL, ATTN_LSE_ATOL, ensure_built, run_decode
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    ensure_built()
+
+
+def _check(x, scale=0.0):
+    out, lse, st = run_decode(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_cache"],
+                              x["v_cache"], x["cache_len"], scale=scale)
+    assert st == fvrag.OK
+    ro, rl = oracle.decode_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"],
+                                x["k_cache"], x["v_cache"], x["cache_len"], scale=scale)
+    assert np.max(np.abs(out - ro)) <= ATTN_ATOL
+    assert np.max(np.abs(lse - rl)) <= ATTN_LSE_ATOL
+    return out
+
+
+def test_decode_tiny_matches_oracle():
+    _check(synth.decode_inputs(configs.DEC_TINY))
+
+
+@pytest.mark.parametrize("Qn,K,hq,hkv,D,pr,C,cr", [
+    (1, 5, 28, 4, 128, (8192, 8192), 200, (1, 200)),     # 7B-class heads, C not a block multiple
+    (2, 20, 16, 2, 128, (0, 700), 64, (64, 64)),         # two row tiles; full caches; P may be 0
+    (3, 4, 8, 1, 64, (100, 900), 300, (1, 1)),           # MQA, D = 64, only the newest token
+    (1, 7, 2, 2, 128, (5000, 5000), 2048, (1500, 2048)), # long caches spread over many runs
+])
+def test_decode_shapes(Qn, K, hq, hkv, D, pr, C, cr):
+    cfg = configs.DEC_TINY.with_(num_queries=Qn, num_drafts=K, hq=hq, hkv=hkv, head_dim=D,
+                                 prefix_range=pr, cache_cap=C, cache_range=cr, seed=17 + K)
+    _check(synth.decode_inputs(cfg))
+
+
+def test_decode_ignores_slots_past_the_cache_length_and_scale():
+    x = synth.decode_inputs(configs.DEC_TINY)
+    big = synth.round_bf16(np.full((1,), 3.0e4))[0]
+    for qi in range(x["q"].shape[0]):
+        for k in range(x["q"].shape[1]):
+            n = x["cache_len"][qi, k]
+            x["k_cache"][qi, k, n:] = big
+            x["v_cache"][qi, k, n:] = big
+    _check(x)
+    _check(x, scale=0.05)
+
+
+@pytest.mark.slow
+def test_decode_full_size_sampled_queries():
+    """16 queries x 5 drafts of the 3B-class drafter with ragged 4K-16K prefixes; the
+    oracle checks the first and the last query on their own."""
+    cfg = configs.DEC_3B_16Q
+    x = synth.decode_inputs(cfg)
+    out, lse, st = run_decode(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_cache"],
+                              x["v_cache"], x["cache_len"])
+    assert st == fvrag.OK
+    offs = x["prefix_offsets"]
+    for qi in (0, cfg.num_queries - 1):
+        a, b = int(offs[qi]), int(offs[qi + 1])
+        ro, rl = oracle.decode_attn(x["q"][qi:qi + 1], x["k_prefix"][a:b], x["v_prefix"][a:b],
+                                    np.array([0, b - a], np.int32), x["k_cache"][qi:qi + 1],
+                                    x["v_cache"][qi:qi + 1], x["cache_len"][qi:qi + 1])
+        assert np.max(np.abs(out[qi:qi + 1] - ro)) <= ATTN_ATOL
+        assert np.max(np.abs(lse[qi:qi + 1] - rl)) <= ATTN_LSE_ATOL

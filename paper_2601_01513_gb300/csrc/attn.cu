@@ -39,6 +39,7 @@
 #include <cuda_bf16.h>
 
 #include <algorithm>
+#include <cmath>
 
 #include "fvrag_common.cuh"
 #include "fvrag_internal.h"
@@ -83,7 +84,7 @@ struct Args {
   float* part_lse;        // [nsplit][rows]
   uint32_t* status;
   uint64_t limit_ns;
-  int Qn, K, Lq, C, KL, hq, hkv, grp, T, mtiles, nsplit, bps;
+  int Qn, K, Lq, C, KL, hq, hkv, grp, T, mtiles, nsplit;
   float scale_log2;
 };
 
@@ -221,31 +222,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     while (tb < ntb && !own_valid(tb)) ++tb;
     return tb;
   };
-  // count the valid own blocks and find the first one this run uses, 32 blocks per
-  // step of the warp (every warp computes the same values)
-  const int blk_lo = split * a.bps;
-  int nvt = 0, tb_first = -1;
-  {
-    int skip = max(0, blk_lo - nbp);               // valid own blocks before this run's first
-    for (int base = 0; base < ntb; base += 32) {
-      const int tb = base + lane;
-      const uint32_t m = __ballot_sync(0xffffffffu, tb < ntb && own_valid(tb));
-      const int cnt = __popc(m);
-      if (tb_first < 0) {
-        if (skip < cnt) {
-          uint32_t mm = m;
-          for (int i = 0; i < skip; ++i) mm &= mm - 1u;
-          tb_first = base + __ffs(mm) - 1;
-        } else {
-          skip -= cnt;
-        }
-      }
-      nvt += cnt;
-    }
-    if (tb_first < 0) tb_first = ntb;
-  }
+  // count the valid own blocks, 32 per step of the warp (every warp computes the
+  // same values); this tile's list of nb blocks is cut into nsplit equal runs
+  int nvt = 0;
+  for (int base = 0; base < ntb; base += 32)
+    nvt += __popc(__ballot_sync(0xffffffffu, base + lane < ntb && own_valid(base + lane)));
   const int nb = nbp + nvt;
-  const int nblk = max(0, min(nb, blk_lo + a.bps) - blk_lo);
+  const int bps = (nb + a.nsplit - 1) / a.nsplit;
+  const int blk_lo = split * bps;
+  const int nblk = max(0, min(nb, blk_lo + bps) - blk_lo);
+  // the first own block this run uses: skip the valid own blocks of earlier runs
+  int tb_first = ntb;
+  {
+    int skip = max(0, blk_lo - nbp);
+    for (int base = 0; base < ntb; base += 32) {
+      const uint32_t m = __ballot_sync(0xffffffffu, base + lane < ntb && own_valid(base + lane));
+      const int cnt = __popc(m);
+      if (skip < cnt) {
+        uint32_t mm = m;
+        for (int i = 0; i < skip; ++i) mm &= mm - 1u;
+        tb_first = base + __ffs(mm) - 1;
+        break;
+      }
+      skip -= cnt;
+    }
+  }
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -604,14 +605,15 @@ struct Problem {
 };
 
 struct Plan {
-  int grp, T, mtiles, nsplit, bps;
+  int grp, T, mtiles, nsplit;
 };
 
-// Key-split plan: the longest block list a row tile can have (the longest prefix
-// plus every own block of the candidates a tile can touch) is cut into runs of
-// `bps` blocks; pick the run count that minimises an estimate of waves x (blocks
-// per CTA + fixed cost) plus the cost of writing and merging the partials (one CTA
-// per SM; a 128-key block is ~0.6 us).
+// Key-split plan: every row tile's block list (its query's prefix blocks plus the
+// own blocks of its candidates) is cut on the device into nsplit equal runs, one
+// CTA each, so a short ragged prefix gives short CTAs that the block scheduler
+// backfills.  Pick nsplit to minimise an estimate of the time: the larger of the
+// mean work per SM (waves x mean run) and the longest run, plus the cost of
+// writing and merging the partials (a 128-key block is ~0.6 us).
 static Plan make_plan(const Problem& pr, int sms) {
   Plan p;
   p.grp = pr.hq / pr.hkv;
@@ -620,25 +622,24 @@ static Plan make_plan(const Problem& pr, int sms) {
   p.mtiles = (KL + p.T - 1) / p.T;
   const long long base = (long long)pr.Qn * pr.hkv * p.mtiles;
   const int ncand = std::min(pr.K, (p.T + pr.Lq - 1) / pr.Lq + 1);
-  const int nb = (std::max(pr.max_prefix, 0) + kBN - 1) / kBN +
-                 (int)(((long long)ncand * pr.C + kBN - 1) / kBN);
+  const int nb_own = (int)(((long long)ncand * pr.C + kBN - 1) / kBN);
+  const int nb = (std::max(pr.max_prefix, 0) + kBN - 1) / kBN + nb_own;
+  const double nb_mean = std::ceil((double)std::max(pr.total_prefix, 0) / pr.Qn / kBN) + nb_own;
   p.nsplit = 1;
-  p.bps = std::max(nb, 1);
   if (nb <= 1) return p;
   if (sms <= 0) sms = 148;
   const double rows = (double)pr.Qn * KL * pr.hq;
   double best = 1e30;
   for (int ns = 1; ns <= std::min(nb, 64); ++ns) {
-    const int per = (nb + ns - 1) / ns;
-    const int nse = (nb + per - 1) / per;
-    const long long ctas = base * nse;
+    const long long ctas = base * ns;
     const double waves = (double)((ctas + sms - 1) / sms);
-    double t = waves * (per + 3) * 0.6;
-    if (nse > 1) t += 3.0 + nse * rows * (pr.D + 1) * 8.0 / 8.0e6;
+    const double t_mean = waves * (std::ceil(nb_mean / ns) + 3);
+    const double t_max = std::ceil((double)nb / ns) + 3;
+    double t = std::max(t_mean, t_max) * 0.6;
+    if (ns > 1) t += 3.0 + ns * rows * (pr.D + 1) * 8.0 / 8.0e6;
     if (t < best - 1e-9) {
       best = t;
-      p.nsplit = nse;
-      p.bps = per;
+      p.nsplit = ns;
     }
   }
   return p;
@@ -735,7 +736,6 @@ static fvrag_status run(const Problem& pr, const void* q, const void* k_prefix, 
   a.T = p.T;
   a.mtiles = p.mtiles;
   a.nsplit = p.nsplit;
-  a.bps = p.bps;
   a.scale_log2 = scale * kLog2e;
   const long long grid = (long long)pr.Qn * pr.hkv * p.nsplit * p.mtiles;
   if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;

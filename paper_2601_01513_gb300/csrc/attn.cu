@@ -27,7 +27,7 @@
 //                S_j  = Q K_j^T   (M = 128 rows, N = 128 keys, K = D; both K-major)
 //                O   += P_j V_j   (M = 128, N = D, K = 128 keys; P_j read from tensor
 //                                  memory, V MN-major from shared memory)
-//              with S/P double-buffered and O accumulated in tensor memory.
+//              with three S/P buffers and O accumulated in tensor memory.
 //   warps 2-5  one query row per thread: tcgen05.ld of S_j, masking (prefix length,
 //              or the row's own visible slots; full blocks skip it), online softmax
 //              in base 2 against a lazily moved reference max (O and l are rescaled
@@ -54,10 +54,13 @@ constexpr int kStages = 3;        // depth of each of the K ring and the V ring
 constexpr int kMaxTail = 64;            // verification: tokens per candidate
 constexpr int kMaxCand = kBM + 1;       // candidates a row tile can touch
 constexpr uint32_t kTmemCols = 512;
-// tensor-memory columns: S/P buffers at 0 and 128 (S_j as fp32 in 128 columns, then
-// P_j as packed bf16 in the first 64), the O accumulator at 256
+// tensor-memory columns: kSP S/P buffers of 128 columns (S_j as fp32 in 128 columns, then
+// P_j as packed bf16 in the first 64), the O accumulator after them.  Three buffers let
+// S_{j+2} be computed while PV_j still reads P_j.
+constexpr int kSP = 3;
 __device__ __forceinline__ uint32_t col_s(int b) { return (uint32_t)b * 128u; }
-constexpr uint32_t kColO = 256;
+constexpr uint32_t kColO = kSP * 128;
+static_assert(kColO + 128 <= kTmemCols, "S/P buffers and O must fit in tensor memory");
 constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (P stays < 2^8)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
@@ -143,12 +146,12 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* k_empty = bars + kStages;             // [kStages]  MMA (S done) -> TMA
   uint64_t* v_full = bars + 2 * kStages;          // [kStages]  TMA -> MMA
   uint64_t* v_empty = bars + 3 * kStages;         // [kStages]  MMA (PV done) -> TMA
-  uint64_t* s_full = bars + 4 * kStages;          // [2]  S_j in tensor memory
-  uint64_t* p_full = s_full + 2;                  // [2]  P_j in tensor memory (4 warps)
-  uint64_t* pv_done = s_full + 4;                 // [2]  PV_j done: S/P buffer free
-  uint64_t* q_full = s_full + 6;
-  uint64_t* drain = s_full + 7;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(s_full + 8);
+  uint64_t* s_full = bars + 4 * kStages;          // [kSP]  S_j in tensor memory
+  uint64_t* p_full = s_full + kSP;                // [kSP]  P_j in tensor memory (4 warps)
+  uint64_t* pv_done = s_full + 2 * kSP;           // [kSP]  PV_j done: S/P buffer free
+  uint64_t* q_full = s_full + 3 * kSP;
+  uint64_t* drain = q_full + 1;
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
 
   griddep_wait();                 // inputs may come from the previous kernel
   // ---- work item
@@ -168,7 +171,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ncand = (tok0 + ntok - 1) / a.Lq - c_lo + 1;
   const int ntb = (ncand * a.C + kBN - 1) / kBN;       // blocks over the candidates' own slots
   // valid own slots of the tile's candidates (the own blocks with none are skipped)
-  int* n_own = reinterpret_cast<int*>(s_full + 8) + 4;
+  int* n_own = reinterpret_cast<int*>(drain + 1) + 4;
   for (int c = threadIdx.x; c < ncand; c += kThreads) {
     int n = a.own_len ? __ldg(&a.own_len[qi * a.K + c_lo + c]) : a.C;
     n_own[c] = n < 0 ? 0 : (n > a.C ? a.C : n);
@@ -181,7 +184,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       mbar_init(smem_u32(&v_full[s]), 1);
       mbar_init(smem_u32(&v_empty[s]), 1);
     }
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < kSP; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
       mbar_init(smem_u32(&p_full[s]), 4);
       mbar_init(smem_u32(&pv_done[s]), 1);
@@ -323,7 +326,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    //   S_ns  = Q K_ns^T         into S/P buffer ns & 1, once K_ns is in and PV_{ns-2}
+    //   S_ns  = Q K_ns^T         into S/P buffer ns % kSP, once K_ns is in and PV_{ns-kSP}
     //                            (the previous user of that buffer) is done;
     //   O    += P_np V_np        with P_np read from tensor memory, once the softmax
     //                            warps published P_np and V_np is in.
@@ -338,35 +341,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         uint64_t t_last = globaltimer_ns();
         while (np < nblk) {
           bool moved = false;
-          if (ns < nblk && ns < np + 2 &&
+          if (ns < nblk && ns < np + kSP &&
               mbar_test(smem_u32(&k_full[ns % kStages]), (ns / kStages) & 1) &&
-              mbar_test(smem_u32(&pv_done[ns & 1]), ((ns >> 1) & 1) ^ 1)) {
+              mbar_test(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1)) {
             tc_fence_after();
             const uint32_t ks = smem_u32(k_ring + (ns % kStages) * Lay::kStage);
 #pragma unroll
             for (int h = 0; h < NH; ++h)
 #pragma unroll
               for (int k16 = 0; k16 < 4; ++k16)
-                tc_mma_bf16(tmem_base + col_s(ns & 1),
+                tc_mma_bf16(tmem_base + col_s(ns % kSP),
                             desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
                             desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS,
                             (h | k16) != 0);
-            tc_commit(smem_u32(&s_full[ns & 1]));
+            tc_commit(smem_u32(&s_full[ns % kSP]));
             tc_commit(smem_u32(&k_empty[ns % kStages]));
             ++ns;
             moved = true;
           }
-          if (np < ns && mbar_test(smem_u32(&p_full[np & 1]), (np >> 1) & 1) &&
+          if (np < ns && mbar_test(smem_u32(&p_full[np % kSP]), (np / kSP) & 1) &&
               mbar_test(smem_u32(&v_full[np % kStages]), (np / kStages) & 1)) {
             tc_fence_after();
-            const uint32_t pa = tmem_base + col_s(np & 1);
+            const uint32_t pa = tmem_base + col_s(np % kSP);
             const uint32_t vs = smem_u32(v_ring + (np % kStages) * Lay::kStage);
 #pragma unroll
             for (int k16 = 0; k16 < kBN / 16; ++k16)
               tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
                              desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
                              (np | k16) != 0);
-            tc_commit(smem_u32(&pv_done[np & 1]));
+            tc_commit(smem_u32(&pv_done[np % kSP]));
             tc_commit(smem_u32(&v_empty[np % kStages]));
             ++np;
             moved = true;
@@ -403,8 +406,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
     for (int j = 0; j < nblk; ++j) {
-      const int sb = j & 1;
-      if (!mbar_wait(smem_u32(&s_full[sb]), (j >> 1) & 1, a.limit_ns)) {
+      const int sb = j % kSP;
+      if (!mbar_wait(smem_u32(&s_full[sb]), (j / kSP) & 1, a.limit_ns)) {
         record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteSFull);
         ok = false;
         break;
@@ -473,7 +476,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (__any_sync(0xffffffffu, resc)) {
         // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale
         const int i = j - 1;
-        if (!mbar_wait(smem_u32(&pv_done[i & 1]), (i >> 1) & 1, a.limit_ns)) {
+        if (!mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns)) {
           record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
           ok = false;
           break;
@@ -497,7 +500,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---- epilogue: wait for the last PV, normalise O by l
     if (ok && nblk > 0) {
       const int i = nblk - 1;
-      if (!mbar_wait(smem_u32(&pv_done[i & 1]), (i >> 1) & 1, a.limit_ns))
+      if (!mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))
         record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
       tc_fence_after();
     }
@@ -551,6 +554,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
 }
 
+// One warp per output row: out = sum_s w_s o_s / sum_s w_s with w_s = exp(lse_s - max lse),
+// lse = max + log(sum_s w_s).  Lane s holds split s's weight (and s + 32); all partial
+// loads of a group of 8 splits are issued before any is used.
 template <int D>
 __global__ void merge_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
                              int nsplit, long long nrows, __nv_bfloat16* __restrict__ out,
@@ -561,40 +567,50 @@ __global__ void merge_kernel(const float* __restrict__ part_o, const float* __re
   const long long row = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= nrows) return;
-  float mx = -INFINITY;
-  for (int s = lane; s < nsplit; s += 32) mx = fmaxf(mx, part_lse[(size_t)s * nrows + row]);
-  mx = warp_max(mx);
-  float den = 0.f;
-  for (int s = lane; s < nsplit; s += 32) {
-    const float v = part_lse[(size_t)s * nrows + row];
-    if (v != -INFINITY) den += __expf(v - mx);
-  }
-  den = warp_sum(den);
+  const float l0 = lane < nsplit ? part_lse[(size_t)lane * nrows + row] : -INFINITY;
+  const float l1 = lane + 32 < nsplit ? part_lse[(size_t)(lane + 32) * nrows + row] : -INFINITY;
+  const float mx = warp_max(fmaxf(l0, l1));
+  const float w0 = l0 == -INFINITY ? 0.f : __expf(l0 - mx);
+  const float w1 = l1 == -INFINITY ? 0.f : __expf(l1 - mx);
+  const float den = warp_sum(w0 + w1);
   float res[DPL];
 #pragma unroll
   for (int i = 0; i < DPL; ++i) res[i] = 0.f;
-#pragma unroll 4
-  for (int s = 0; s < nsplit; ++s) {
-    const float v = part_lse[(size_t)s * nrows + row];
-    const float w = v == -INFINITY ? 0.f : __expf(v - mx);
-    const float* po = part_o + ((size_t)s * nrows + row) * D + lane * DPL;
-    if (DPL == 4) {
-      const float4 f = *reinterpret_cast<const float4*>(po);
-      res[0] = fmaf(w, f.x, res[0]);
-      res[1] = fmaf(w, f.y, res[1]);
-      res[2] = fmaf(w, f.z, res[2]);
-      res[3] = fmaf(w, f.w, res[3]);
-    } else {
+  const float* base = part_o + (size_t)row * D + lane * DPL;
+  for (int s0 = 0; s0 < nsplit; s0 += 8) {
+    float v[8][DPL];
 #pragma unroll
-      for (int i = 0; i < DPL; ++i) res[i] = fmaf(w, po[i], res[i]);
+    for (int u = 0; u < 8; ++u) {
+      if (s0 + u < nsplit) {
+        const float* po = base + (size_t)(s0 + u) * nrows * D;
+        if constexpr (DPL == 4) {
+          const float4 f = *reinterpret_cast<const float4*>(po);
+          v[u][0] = f.x;
+          v[u][1] = f.y;
+          v[u][2] = f.z;
+          v[u][3] = f.w;
+        } else {
+#pragma unroll
+          for (int i = 0; i < DPL; ++i) v[u][i] = po[i];
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int sp = s0 + u;
+      if (sp < nsplit) {
+        const float w = __shfl_sync(0xffffffffu, sp < 32 ? w0 : w1, sp & 31);
+#pragma unroll
+        for (int i = 0; i < DPL; ++i) res[i] = fmaf(w, v[u][i], res[i]);
+      }
     }
   }
-  const float inv = 1.f / den;
+  const float inv = den > 0.f ? 1.f / den : 0.f;
   __nv_bfloat16* o = out + row * D + lane * DPL;
 #pragma unroll
   for (int i = 0; i < DPL; i += 2)
     *reinterpret_cast<__nv_bfloat162*>(o + i) = __floats2bfloat162_rn(res[i] * inv, res[i + 1] * inv);
-  if (lane == 0 && lse_out) lse_out[row] = mx + __logf(den);
+  if (lane == 0 && lse_out) lse_out[row] = den > 0.f ? mx + __logf(den) : -INFINITY;
 }
 
 // One attention problem in the general form of the kernel (see the top of the file).

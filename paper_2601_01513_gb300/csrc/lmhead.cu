@@ -332,7 +332,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 }
 
 // One warp per row: lse = ln 2 * (M2 + log2 S) with M2 = max_b max_b and
-// S = sum_b sum_b * 2^(max_b - M2); logprob = z_target - lse.
+// S = sum_b sum_b * 2^(max_b - M2) (partials in the log2 domain); logprob = z_target - lse.
 __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float* __restrict__ part_sum,
                                 const float* __restrict__ tgt_logit,
                                 const int32_t* __restrict__ targets, int M, int V, int G, int nparts,
@@ -342,15 +342,28 @@ __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float*
   const int m = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (m >= M) return;
-  float mx = -INFINITY;
-  for (int b = lane; b < nparts; b += 32) mx = fmaxf(mx, part_max[(size_t)b * M + m]);
-  mx = warp_max(mx);
-  float s = 0.f;
+  // one pass over the partials: each lane folds its (max, sum) pairs online, then the
+  // warp combines the 32 lane states
+  float mx = -INFINITY, s = 0.f;
+#pragma unroll 4
   for (int b = lane; b < nparts; b += 32) {
     const float pm = part_max[(size_t)b * M + m];
-    if (pm != -INFINITY) s += part_sum[(size_t)b * M + m] * ex2(pm - mx);
+    const float ps = part_sum[(size_t)b * M + m];
+    if (pm > mx) {
+      s = s * ex2(mx - pm) + ps;
+      mx = pm;
+    } else if (pm != -INFINITY) {
+      s += ps * ex2(pm - mx);
+    }
   }
-  s = warp_sum(s);
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float om = __shfl_xor_sync(0xffffffffu, mx, o);
+    const float os = __shfl_xor_sync(0xffffffffu, s, o);
+    const float nm = fmaxf(mx, om);
+    s = (mx == -INFINITY ? 0.f : s * ex2(mx - nm)) + (om == -INFINITY ? 0.f : os * ex2(om - nm));
+    mx = nm;
+  }
   const float l = kLn2 * (mx + __log2f(s));
   if (lane == 0 && lse_out) lse_out[m] = l;
   for (int g = lane; g < G; g += 32) {

@@ -21,18 +21,20 @@
 //
 // attn_kernel: one CTA = one row tile x one run of key blocks.
 //   warp 0     TMA: the Q tile once (3-D map over [tokens][hq][D]), then K and V
-//              blocks (3-D maps over [keys][hkv][D], 128-byte swizzle) into two
-//              3-deep rings, K and V each issued as soon as its ring has a free slot.
+//              blocks (3-D maps over [keys][hkv][D], 128-byte swizzle) into a 2-deep
+//              K ring and a 3-deep V ring, each issued as soon as its ring has a free slot.
 //   warp 1     allocates tensor memory and issues tcgen05.mma:
 //                S_j  = Q K_j^T   (M = 128 rows, N = 128 keys, K = D; both K-major)
 //                O   += P_j V_j   (M = 128, N = D, K = 128 keys; P_j read from tensor
 //                                  memory, V MN-major from shared memory)
 //              with three S/P buffers and O accumulated in tensor memory.
-//   warps 2-5  one query row per thread: tcgen05.ld of S_j, masking (prefix length,
-//              or the row's own visible slots; full blocks skip it), online softmax
-//              in base 2 against a lazily moved reference max (O and l are rescaled
-//              in place only when a row's max grows by more than 2^8), and P_j
-//              written back as bf16 pairs over S_j in tensor memory.
+//   warps 2-9  two warps per tensor-memory lane quarter, one query row per thread and
+//              half of the block's keys per warp: tcgen05.ld of S_j, masking (prefix
+//              length, or the row's own visible slots; full blocks skip it), the block
+//              max shared by the two halves through shared memory, online softmax in
+//              base 2 against a lazily moved reference max (O and l are rescaled in
+//              place only when a row's max grows by more than 2^8), and P_j written
+//              back as bf16 pairs over S_j in tensor memory.
 //   One run: the CTA writes the bf16 output and the lse directly.  Several runs:
 //   normalised partials go to the workspace and merge_kernel combines them with
 //   log-sum-exp weights.
@@ -47,10 +49,11 @@
 namespace fvrag {
 namespace attn {
 
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;      // producer, MMA issuer, 8 softmax warps
 constexpr int kBM = 128;          // query rows per tile (MMA M)
 constexpr int kBN = 128;          // keys per block (MMA N of S, K of PV)
-constexpr int kStages = 3;        // depth of each of the K ring and the V ring
+constexpr int kKStages = 2;       // depth of the K ring (K_j is consumed early, by S_j)
+constexpr int kVStages = 3;       // depth of the V ring (V_j is read by PV_j, after softmax_j)
 constexpr int kMaxTail = 64;            // verification: tokens per candidate
 constexpr int kMaxCand = kBM + 1;       // candidates a row tile can touch
 constexpr uint32_t kTmemCols = 512;
@@ -74,7 +77,9 @@ struct Layout {
   static constexpr int kQ = NH * kBM * 128;         // Q tile
   static constexpr int kKVHalf = kBN * 128;         // 128 keys x 64 elements
   static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
-  static constexpr int kBytes = kQ + 2 * kStages * kStage + 1024 + 256 + kMaxCand * 4;
+  // + row-max exchange [2 slots][2 halves][128 rows] and row-sum exchange [2][128] floats
+  static constexpr int kBytes =
+      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4;
   static_assert(kBytes <= 232448, "shared memory per CTA");
 };
 
@@ -139,14 +144,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* q_s = smem;
-  uint8_t* k_ring = q_s + Lay::kQ;                    // [kStages][kStage]
-  uint8_t* v_ring = k_ring + kStages * Lay::kStage;   // [kStages][kStage]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(v_ring + kStages * Lay::kStage);
-  uint64_t* k_full = bars;                        // [kStages]  TMA -> MMA
-  uint64_t* k_empty = bars + kStages;             // [kStages]  MMA (S done) -> TMA
-  uint64_t* v_full = bars + 2 * kStages;          // [kStages]  TMA -> MMA
-  uint64_t* v_empty = bars + 3 * kStages;         // [kStages]  MMA (PV done) -> TMA
-  uint64_t* s_full = bars + 4 * kStages;          // [kSP]  S_j in tensor memory
+  uint8_t* k_ring = q_s + Lay::kQ;                     // [kKStages][kStage]
+  uint8_t* v_ring = k_ring + kKStages * Lay::kStage;   // [kVStages][kStage]
+  float* xmax = reinterpret_cast<float*>(v_ring + kVStages * Lay::kStage);  // [2][2][kBM]
+  float* xsum = xmax + 4 * kBM;                                             // [2][kBM]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xsum + 2 * kBM);
+  uint64_t* k_full = bars;                        // [kKStages]  TMA -> MMA
+  uint64_t* k_empty = bars + kKStages;            // [kKStages]  MMA (S done) -> TMA
+  uint64_t* v_full = k_empty + kKStages;          // [kVStages]  TMA -> MMA
+  uint64_t* v_empty = v_full + kVStages;          // [kVStages]  MMA (PV done) -> TMA
+  uint64_t* s_full = v_empty + kVStages;          // [kSP]  S_j in tensor memory
   uint64_t* p_full = s_full + kSP;                // [kSP]  P_j in tensor memory (4 warps)
   uint64_t* pv_done = s_full + 2 * kSP;           // [kSP]  PV_j done: S/P buffer free
   uint64_t* q_full = s_full + 3 * kSP;
@@ -178,15 +185,17 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < kKStages; ++s) {
       mbar_init(smem_u32(&k_full[s]), 1);
       mbar_init(smem_u32(&k_empty[s]), 1);
+    }
+    for (int s = 0; s < kVStages; ++s) {
       mbar_init(smem_u32(&v_full[s]), 1);
       mbar_init(smem_u32(&v_empty[s]), 1);
     }
     for (int s = 0; s < kSP; ++s) {
       mbar_init(smem_u32(&s_full[s]), 1);
-      mbar_init(smem_u32(&p_full[s]), 4);
+      mbar_init(smem_u32(&p_full[s]), 8);   // one arrival per softmax warp
       mbar_init(smem_u32(&pv_done[s]), 1);
     }
     mbar_init(smem_u32(q_full), 1);
@@ -197,7 +206,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     tmem_alloc(smem_u32(tmem_holder), kTmemCols);
     tmem_relinquish();
   }
-  if (warp >= 2) {
+  if (warp >= 2 && warp < 6) {
     // Rows past the T x grp rows the Q box fills are never loaded: zero them so their
     // (discarded) scores stay finite and every lane of a warp takes the same code path.
     const int r = (warp & 3) * 32 + lane;
@@ -270,10 +279,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       uint64_t t_last = globaltimer_ns();
       while (nk < nblk || nv < nblk) {
         bool moved = false;
-        if (nk < nblk && mbar_test(smem_u32(&k_empty[nk % kStages]), ((nk / kStages) & 1) ^ 1)) {
-          const uint32_t fb = smem_u32(&k_full[nk % kStages]);
+        if (nk < nblk && mbar_test(smem_u32(&k_empty[nk % kKStages]), ((nk / kKStages) & 1) ^ 1)) {
+          const uint32_t fb = smem_u32(&k_full[nk % kKStages]);
           mbar_arrive_expect_tx(fb, Lay::kStage);
-          uint8_t* dst = k_ring + (nk % kStages) * Lay::kStage;
+          uint8_t* dst = k_ring + (nk % kKStages) * Lay::kStage;
           const int bi = blk_lo + nk;
           const bool pre = bi < nbp;
           int key;
@@ -290,10 +299,10 @@ __global__ void __launch_bounds__(kThreads, 1)
           ++nk;
           moved = true;
         }
-        if (nv < nk && mbar_test(smem_u32(&v_empty[nv % kStages]), ((nv / kStages) & 1) ^ 1)) {
-          const uint32_t fb = smem_u32(&v_full[nv % kStages]);
+        if (nv < nk && mbar_test(smem_u32(&v_empty[nv % kVStages]), ((nv / kVStages) & 1) ^ 1)) {
+          const uint32_t fb = smem_u32(&v_full[nv % kVStages]);
           mbar_arrive_expect_tx(fb, Lay::kStage);
-          uint8_t* dst = v_ring + (nv % kStages) * Lay::kStage;
+          uint8_t* dst = v_ring + (nv % kVStages) * Lay::kStage;
           const int bi = blk_lo + nv;
           const bool pre = bi < nbp;
           int key;
@@ -319,10 +328,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       // no copy may still be in flight when the CTA exits
       mbar_wait(qb, 0, a.limit_ns);
-      for (int i = max(0, nk - kStages); i < nk; ++i)
-        mbar_wait(smem_u32(&k_full[i % kStages]), (i / kStages) & 1, a.limit_ns);
-      for (int i = max(0, nv - kStages); i < nv; ++i)
-        mbar_wait(smem_u32(&v_full[i % kStages]), (i / kStages) & 1, a.limit_ns);
+      for (int i = max(0, nk - kKStages); i < nk; ++i)
+        mbar_wait(smem_u32(&k_full[i % kKStages]), (i / kKStages) & 1, a.limit_ns);
+      for (int i = max(0, nv - kVStages); i < nv; ++i)
+        mbar_wait(smem_u32(&v_full[i % kVStages]), (i / kVStages) & 1, a.limit_ns);
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
@@ -342,10 +351,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         while (np < nblk) {
           bool moved = false;
           if (ns < nblk && ns < np + kSP &&
-              mbar_test(smem_u32(&k_full[ns % kStages]), (ns / kStages) & 1) &&
+              mbar_test(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1) &&
               mbar_test(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1)) {
             tc_fence_after();
-            const uint32_t ks = smem_u32(k_ring + (ns % kStages) * Lay::kStage);
+            const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
 #pragma unroll
             for (int h = 0; h < NH; ++h)
 #pragma unroll
@@ -355,22 +364,22 @@ __global__ void __launch_bounds__(kThreads, 1)
                             desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS,
                             (h | k16) != 0);
             tc_commit(smem_u32(&s_full[ns % kSP]));
-            tc_commit(smem_u32(&k_empty[ns % kStages]));
+            tc_commit(smem_u32(&k_empty[ns % kKStages]));
             ++ns;
             moved = true;
           }
           if (np < ns && mbar_test(smem_u32(&p_full[np % kSP]), (np / kSP) & 1) &&
-              mbar_test(smem_u32(&v_full[np % kStages]), (np / kStages) & 1)) {
+              mbar_test(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1)) {
             tc_fence_after();
             const uint32_t pa = tmem_base + col_s(np % kSP);
-            const uint32_t vs = smem_u32(v_ring + (np % kStages) * Lay::kStage);
+            const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
 #pragma unroll
             for (int k16 = 0; k16 < kBN / 16; ++k16)
               tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
                              desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
                              (np | k16) != 0);
             tc_commit(smem_u32(&pv_done[np % kSP]));
-            tc_commit(smem_u32(&v_empty[np % kStages]));
+            tc_commit(smem_u32(&v_empty[np % kVStages]));
             ++np;
             moved = true;
           }
@@ -388,11 +397,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
   } else {
     // ------------------------------------------------------------ softmax / epilogue
-    // One row per thread.  Online softmax in base 2 with a lazily updated reference
-    // max: P_j is taken relative to m_ref, which only moves when a row's block max
-    // exceeds it by more than kRescaleLog2 (then O in tensor memory and l are rescaled
-    // once).  P values stay below 2^kRescaleLog2; the result is the same softmax.
+    // Two warps per tensor-memory lane quarter: warp w (2..9) serves rows 32 (w % 4) ..
+    // +31 and the key half `half` = (w - 2) / 4 of every block (64 keys, written back as
+    // 32 columns of packed bf16 P), and the same half of O's columns.  The two halves
+    // of a row agree on the block max through shared memory (a named barrier per
+    // quarter) and keep separate partial sums, added at the end.
+    // Online softmax in base 2 with a lazily updated reference max: P_j is taken
+    // relative to m_ref, which only moves when a row's block max exceeds it by more than
+    // kRescaleLog2 (then O in tensor memory and l are rescaled once).  P values stay below
+    // 2^kRescaleLog2; the result is the same softmax.
+    constexpr int kHalf = kBN / 2;                     // keys per warp and block
+    constexpr int kOHalf = D / 2;                      // O columns per warp
     const int quarter = warp & 3;
+    const int half = (warp - 2) >> 2;
     const int r = quarter * 32 + lane;                 // tile row = tensor-memory lane
     const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
     const bool rvalid = r < rows;
@@ -405,19 +422,29 @@ __global__ void __launch_bounds__(kThreads, 1)
     int tbs = tb_first;                                // own-block cursor
     float m_ref = -INFINITY, l = 0.f;
     bool ok = true;
+    auto pair_sync = [&]() {                           // the two warps of this quarter
+      asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");
+    };
     for (int j = 0; j < nblk; ++j) {
       const int sb = j % kSP;
-      if (!mbar_wait(smem_u32(&s_full[sb]), (j / kSP) & 1, a.limit_ns)) {
+      // `ok` stays warp-uniform (the warp votes on every bounded wait), so a timed-out
+      // warp still meets its partner at every barrier below and the kernel drains
+      if (ok && !__all_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[sb]), (j / kSP) & 1, a.limit_ns))) {
         record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteSFull);
         ok = false;
-        break;
       }
       tc_fence_after();
-      uint32_t sr[kBN];
+      uint32_t sr[kHalf];
+      if (ok) {
 #pragma unroll
-      for (int c0 = 0; c0 < kBN; c0 += 32)
-        tmem_ld_32x32b_x32(lane_base + col_s(sb) + c0, *reinterpret_cast<uint32_t(*)[32]>(&sr[c0]));
-      tmem_wait_ld();
+        for (int c0 = 0; c0 < kHalf; c0 += 32)
+          tmem_ld_32x32b_x32(lane_base + col_s(sb) + half * kHalf + c0,
+                             *reinterpret_cast<uint32_t(*)[32]>(&sr[c0]));
+        tmem_wait_ld();
+      } else {
+#pragma unroll
+        for (int c = 0; c < kHalf; ++c) sr[c] = 0u;
+      }
       int vlo, vhi;   // valid columns of this block for this row
       if (blk_lo + j < nbp) {
         vlo = 0;
@@ -429,22 +456,35 @@ __global__ void __launch_bounds__(kThreads, 1)
         vlo = max(0, tlo - base);
         vhi = min(kBN, thi - base);
       }
+      // this warp's columns are [c_off, c_off + kHalf) of the block
+      const int c_off = half * kHalf;
+      vlo -= c_off;
+      vhi -= c_off;
       // rows without output (r >= rows) are not masked: their values are finite and
       // discarded, and masking them would split the warp between the two paths below
-      const bool full = vlo == 0 && vhi == kBN;
+      const bool full = vlo <= 0 && vhi >= kHalf;
       float pm[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
       if (full) {
 #pragma unroll
-        for (int c = 0; c < kBN; ++c) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
+        for (int c = 0; c < kHalf; ++c) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
       } else {
 #pragma unroll
-        for (int c = 0; c < kBN; ++c)
+        for (int c = 0; c < kHalf; ++c)
           if (c >= vlo && c < vhi) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
       }
-      const float bmax = a.scale_log2 * fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                                              fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                         fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+      // block max over both halves (double-buffered slots: the partner may still be
+      // reading the previous block's value)
+      float* xs = xmax + (j & 1) * 2 * kBM;
+      xs[half * kBM + r] = hmax;
+      tc_fence_before();          // this warp's S loads are complete before the partner
+      pair_sync();                // writes its P over them
+      tc_fence_after();
+      hmax = fmaxf(hmax, xs[(half ^ 1) * kBM + r]);
+      const float bmax = a.scale_log2 * hmax;
       const float m_old = m_ref;
       if (bmax > m_ref + kRescaleLog2) m_ref = bmax;   // also the first finite block
       const bool resc = m_ref != m_old && m_old != -INFINITY;
@@ -454,42 +494,39 @@ __global__ void __launch_bounds__(kThreads, 1)
       float rsp[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) rsp[u] = 0.f;
+      uint32_t pk[32];
 #pragma unroll
-      for (int c0 = 0; c0 < kBN; c0 += 64) {
-        uint32_t pk[32];
-#pragma unroll
-        for (int c = 0; c < 64; c += 2) {
-          float e0 = ex2(fmaf(__uint_as_float(sr[c0 + c]), a.scale_log2, -ms));
-          float e1 = ex2(fmaf(__uint_as_float(sr[c0 + c + 1]), a.scale_log2, -ms));
-          if (!full) {
-            e0 = (c0 + c >= vlo && c0 + c < vhi) ? e0 : 0.f;
-            e1 = (c0 + c + 1 >= vlo && c0 + c + 1 < vhi) ? e1 : 0.f;
-          }
-          rsp[c & 7] += e0;
-          rsp[(c + 1) & 7] += e1;
-          pk[c / 2] = pack_bf16(e0, e1);
+      for (int c = 0; c < kHalf; c += 2) {
+        float e0 = ex2(fmaf(__uint_as_float(sr[c]), a.scale_log2, -ms));
+        float e1 = ex2(fmaf(__uint_as_float(sr[c + 1]), a.scale_log2, -ms));
+        if (!full) {
+          e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
+          e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
         }
-        tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(c0 / 2), pk);
+        rsp[c & 7] += e0;
+        rsp[(c + 1) & 7] += e1;
+        pk[c / 2] = pack_bf16(e0, e1);
       }
+      if (ok) tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(half * kHalf / 2), pk);
       const float rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
       l = l * corr + rs;
-      if (__any_sync(0xffffffffu, resc)) {
+      if (ok && __any_sync(0xffffffffu, resc)) {
         // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale
         const int i = j - 1;
-        if (!mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns)) {
+        if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))) {
           record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
           ok = false;
-          break;
-        }
-        tc_fence_after();
+        } else {
+          tc_fence_after();
 #pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
-          uint32_t o[32];
-          tmem_ld_32x32b_x32(lane_base + kColO + c0, o);
-          tmem_wait_ld();
+          for (int c0 = 0; c0 < kOHalf; c0 += 32) {
+            uint32_t o[32];
+            tmem_ld_32x32b_x32(lane_base + kColO + half * kOHalf + c0, o);
+            tmem_wait_ld();
 #pragma unroll
-          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
-          tmem_st_32x32b_x32(lane_base + kColO + c0, o);
+            for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
+            tmem_st_32x32b_x32(lane_base + kColO + half * kOHalf + c0, o);
+          }
         }
       }
       tmem_wait_st();
@@ -497,13 +534,16 @@ __global__ void __launch_bounds__(kThreads, 1)
       __syncwarp();
       if (lane == 0) mbar_arrive(smem_u32(&p_full[sb]));
     }
-    // ---- epilogue: wait for the last PV, normalise O by l
+    // ---- epilogue: wait for the last PV, add the two halves' sums, normalise O by l
     if (ok && nblk > 0) {
       const int i = nblk - 1;
       if (!mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))
         record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
       tc_fence_after();
     }
+    xsum[half * kBM + r] = l;
+    pair_sync();
+    l += xsum[(half ^ 1) * kBM + r];
     const int head = g * a.grp + r % a.grp;
     const size_t rowid = ((size_t)qi * a.KL + tok) * a.hq + head;
     const size_t nrows = (size_t)a.Qn * a.KL * a.hq;
@@ -511,10 +551,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     const float inv = any ? 1.f / l : 0.f;
     const float lse = any ? kLn2 * (m_ref + __log2f(l)) : -INFINITY;
 #pragma unroll
-    for (int c0 = 0; c0 < D; c0 += 32) {
+    for (int c0 = 0; c0 < kOHalf; c0 += 32) {
+      const int oc = half * kOHalf + c0;               // O column of this chunk
       uint32_t o[32];
       if (nblk > 0) {
-        tmem_ld_32x32b_x32(lane_base + kColO + c0, o);
+        tmem_ld_32x32b_x32(lane_base + kColO + oc, o);
         tmem_wait_ld();
       } else {
 #pragma unroll
@@ -522,7 +563,7 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
       if (rvalid) {
         if (a.nsplit == 1) {
-          uint4* dst = reinterpret_cast<uint4*>(a.out + rowid * D + c0);
+          uint4* dst = reinterpret_cast<uint4*>(a.out + rowid * D + oc);
 #pragma unroll
           for (int c = 0; c < 32; c += 8)
             dst[c / 8] = make_uint4(
@@ -531,7 +572,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pack_bf16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
                 pack_bf16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
         } else {
-          float4* dst = reinterpret_cast<float4*>(a.part_o + ((size_t)split * nrows + rowid) * D + c0);
+          float4* dst = reinterpret_cast<float4*>(a.part_o + ((size_t)split * nrows + rowid) * D + oc);
 #pragma unroll
           for (int c = 0; c < 32; c += 4)
             dst[c / 4] = make_float4(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv,
@@ -539,7 +580,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
       }
     }
-    if (rvalid) {
+    if (rvalid && half == 0) {
       if (a.nsplit == 1) {
         if (a.lse) a.lse[rowid] = lse;
       } else {

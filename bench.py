@@ -383,6 +383,72 @@ def bench_row(args):
             cpu = {"value": len(sample) / dt, "unit": unit, "cores": oracle.max_threads(),
                    "kind": "oracle", "sample": "%d of %d keyframes scanned against the whole corpus "
                    "and aggregated, %.1f s" % (len(sample), Fr, dt)}
+    elif args.row == "clip-sweep":
+        # the CLIP alignment of Eq. 14-15 alone on a large case, to show its bandwidth
+        cfg = configs.V7B.with_(name="clip-16x10x4096x768", num_queries=16, num_cand=10,
+                                num_frames=4096, clip_dim=768,
+                                description="CLIP alignment alone: 16 queries x 10 candidates x 4096 "
+                                            "frames x 768 (fp16)")
+        cand, frames = synth.clip_embeddings(cfg, seed=cfg.seed + 7919 * rank)
+        tc = torch.from_numpy(cand.view(np.int16)).view(torch.float16).to(dev)
+        tf = torch.from_numpy(frames.view(np.int16)).view(torch.float16).to(dev)
+        Qn, K = cfg.num_queries, cfg.num_cand
+        mc = torch.empty((Qn, K), dtype=torch.float32, device=dev)
+        am = torch.empty((Qn, K), dtype=torch.int32, device=dev)
+        keep = torch.empty((Qn, K), dtype=torch.uint8, device=dev)
+        h_c = torch.from_numpy(cand.view(np.int16)).view(torch.float16).pin_memory()
+        h_f = torch.from_numpy(frames.view(np.int16)).view(torch.float16).pin_memory()
+        h_keep = torch.empty((Qn, K), dtype=torch.uint8).pin_memory()
+        flush_w = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+
+        def call():
+            fvrag.clip_align(tc, tf, cfg.threshold, mc, am, keep, stream=stream)
+
+        def call_host():
+            tc.copy_(h_c, non_blocking=True)
+            tf.copy_(h_f, non_blocking=True)
+            call()
+            h_keep.copy_(keep, non_blocking=True)
+
+        with torch.cuda.stream(stream):
+            for _ in range(args.warmup):
+                call()
+                call_host()
+            torch.cuda.synchronize(dev)
+            with ClockSampler(dev.index or 0) as clk:
+                clk.wait_first()
+                t_ms, _ = _time_calls(call, stream, steps, dev, between=flush_w.zero_)
+                e_ms, _ = _time_calls(call_host, stream, steps, dev, between=flush_w.zero_)
+        units = Qn * K * cfg.num_frames
+        metric, unit = "candidate-frame cosines/s", "cosines/s"
+        nbytes = Qn * (K + cfg.num_frames) * cfg.clip_dim * 2 + Qn * K * 9
+        roof = {"bound": "hbm", "achieved": nbytes / (t_ms * 1e-3) / 1e9, "peak": pk["hbm_gbs"],
+                "unit": "GB/s", "traffic": None, "peak_source": pk_src,
+                "kernel": "fvrag CLIP alignment (clip_align_kernel)"}
+        roof["frac"] = roof["achieved"] / roof["peak"]
+        h2d = (tc.numel() + tf.numel()) * 2
+        d2h = Qn * K
+        config = {"workload": cfg.description, "name": cfg.name,
+                  "clip": [Qn, K, cfg.num_frames, cfg.clip_dim],
+                  "l2": "flushed before every timed call (256 MiB write, outside the events); "
+                        "the %.0f MB of frames also exceed L2" % (tf.numel() * 2 / 1e6),
+                  "parallelism": "replicas"}
+        dtype = "f16"
+        launches = 1
+        cpu = None
+        if not args.no_cpu_baseline and ws_ == 1:
+            oracle.build()
+            t0 = time.perf_counter()
+            reps = 0
+            while True:
+                oracle.clip_align(cand[:1], frames[:1], cfg.threshold)
+                reps += 1
+                if time.perf_counter() - t0 > args.cpu_budget:
+                    break
+            dt = time.perf_counter() - t0
+            cpu = {"value": reps * K * cfg.num_frames / dt, "unit": unit, "cores": oracle.max_threads(),
+                   "kind": "oracle", "sample": "%d passes over query 0 (%d candidates x %d frames), %.1f s"
+                   % (reps, K, cfg.num_frames, dt)}
     elif args.row == "decode":
         cfg = configs.DECODE_PRESETS[args.row_config or "decode-3b-16q"]
         x = synth.decode_inputs(cfg, seed=cfg.seed + 7919 * rank)
@@ -556,10 +622,12 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=8)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--row", default="verify", choices=["verify", "retrieve", "keyframes", "decode"],
+    ap.add_argument("--row", default="verify",
+                    choices=["verify", "retrieve", "keyframes", "decode", "clip-sweep"],
                     help="verify: the verify step (default); retrieve / keyframes / decode: the "
                          "retrieval (Eq. 2-3), keyframe (Eq. 1) or drafter decode-attention "
-                         "(Eq. 5) step on its own workload")
+                         "(Eq. 5) step on its own workload; clip-sweep: the CLIP alignment call "
+                         "alone at 16 queries x 10 candidates x 4096 frames x 768 (its bandwidth)")
     ap.add_argument("--row-config", default=None,
                     help="workload preset of --row (default: retrieve-16q-1m / keyframe-8x720p / "
                          "decode-3b-16q)")
@@ -714,7 +782,9 @@ def main():
             "gpu_launches": step.launches_per_step() * (2 * args.steps + per_k.shape[0]),
             "timing": {"step": "CUDA graph of the four calls, CUDA events per step, L2 flushed between steps",
                        "kernels": "each call replayed alone %d times (events per launch), L2 flushed before each"
-                                  % per_k.shape[0], "host_wall_s": t_wall},
+                                  % per_k.shape[0], "host_wall_s": t_wall,
+                       "step_us_p10_p50_p90": [float(np.percentile(step_ms, q)) * 1e3 for q in (10, 50, 90)],
+                       "sum_of_call_medians_us": float(sum(k["us_median"] for k in kern.values()))},
             "roofline": roof, "kernels": kern, "clocks": clk.summary()}
     if not args.no_cpu_baseline and ws_ == 1:
         line["cpu_baseline"] = cpu_baseline(cfg, x, args.cpu_budget)

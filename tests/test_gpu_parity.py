@@ -52,6 +52,7 @@ ATTN_CASES = [
     (1, 5, 16, 28, 4, 128, [1000]),        # 7b-style GQA: 5 row tiles of 18 tokens x 7 heads
     (2, 3, 9, 16, 2, 128, [700, 2049]),    # 8 heads per KV head, several key splits
     (1, 2, 64, 8, 8, 64, [300]),           # longest supported tail
+    (1, 2, 3, 128, 1, 64, [200]),          # hq / hkv = 128: one token per row tile
 ]
 
 
@@ -111,6 +112,7 @@ LM_CASES = [
     (129, 256, 4103, 1),      # two M-tiles (second with one row)
     (300, 192, 3001, 2),      # three M-tiles: two groups
     (80, 3584, 9000, 1),      # 7b hidden size, small vocabulary
+    (2048, 64, 1000, 1),      # the most rows supported: 16 M-tiles in 8 groups
 ]
 
 
@@ -200,7 +202,8 @@ ALL_MODES = [fvrag.SEL_MASKED_MEAN_LOGPROB, fvrag.SEL_TWO_STAGE, fvrag.SEL_ADDIT
 
 
 @pytest.mark.parametrize("mode", ALL_MODES)
-@pytest.mark.parametrize("Qn,K,L", [(1, 1, 1), (3, 7, 5), (16, 5, 16), (2, 1000, 3), (600, 10, 2)])
+@pytest.mark.parametrize("Qn,K,L", [(1, 1, 1), (3, 7, 5), (16, 5, 16), (2, 1000, 3), (600, 10, 2),
+                                    (1, 1024, 2)])
 def test_select_matches_oracle(mode, Qn, K, L):
     lp, keep, mc = synth.selection_inputs(Qn, K, L, 2, seed=Qn * 31 + K)
     lengths = synth.uniform_i32((Qn, K), 77, 1, 0, L + 2)   # includes invalid 0 and L+1

@@ -124,6 +124,8 @@ def test_retrieve_tiny_matches_oracle():
     ([40, 50, 60], 4099, 96, 2, 5), # 150 keyframes: two M-tiles in one group
     ([200, 150, 120], 3001, 64, 1, 64),  # 470 keyframes: two M-tile groups; k_frame = 1
     ([100, 28], 1 << 14, 768, 8, 8),     # k_frame = 8, M = 128 exactly
+    ([1024, 1024], 600, 64, 2, 16),      # the most keyframes at k_frame = 2 (16 M-tiles)
+    ([300, 212], 2000, 128, 8, 64),      # the most keyframes at k_frame = 8; k_query = 64
 ])
 def test_retrieve_shapes(nkf, Nt, E, kf, Kq):
     offs = np.zeros(len(nkf) + 1, np.int32)

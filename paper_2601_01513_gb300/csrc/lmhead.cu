@@ -8,8 +8,8 @@
 // every CTA.
 //
 // Persistent grid, one CTA per SM.  CTA b owns a contiguous vocabulary range
-// (multiples of 16 rows, balanced to within 16 rows) and walks it in tiles of BN
-// rows.  Per tile it accumulates, for a group of MG M-tiles of 128 hidden rows,
+// (multiples of 16 rows, balanced to within 16 rows) and walks it in tiles of
+// BN = 256 rows.  Per tile it accumulates, for a group of MG M-tiles of 128 hidden rows,
 // D[128 x BN] = hidden_tile * W_tile^T in tensor memory (fp32), K-loop over H
 // in blocks of 64 (one 128-byte swizzled row per operand row).
 //
@@ -22,8 +22,11 @@
 //   warps 2-5  epilogue: tcgen05.ld of 32 columns at a time (one hidden row per
 //              thread), online max / sum of exp over the CTA's vocabulary slice,
 //              and the gather of target logits that fall in the slice.
-// SLOTS accumulator sets in tensor memory let the epilogue of tile t overlap the
-// MMAs of tile t+1.
+// With one M-tile, two accumulator sets in tensor memory let the epilogue of tile
+// t overlap the MMAs of tile t+1.  With two M-tiles the 512 columns hold a single
+// set: the N = 256 MMAs run at the full tensor rate (N = 128 ones issue at about
+// 80% of it) and each W byte feeds twice the hidden rows, which outweighs the lost
+// overlap while the epilogue is this light.
 //
 // A second small kernel merges the per-CTA (max, sum) partials of every row into
 // lse and writes logprob = z_target - lse (NaN for ids outside [0, V)).
@@ -41,7 +44,6 @@ namespace lm {
 constexpr int kThreads = 192;
 constexpr int kBK = 64;            // bf16 elements per 128-byte swizzled row
 constexpr int kBM = 128;           // hidden rows per M-tile (MMA M)
-constexpr int kStages = 4;
 constexpr int kMaxCtas = 256;      // workspace is sized for this many partials
 constexpr int kMaxMTiles = 16;     // rows <= 2048
 constexpr int kMaxGathers = 8;
@@ -52,17 +54,24 @@ constexpr float kLn2 = 0.6931471805599453f;
 enum : uint32_t { kSiteProdEmpty = 0x201, kSiteMmaTmem = 0x202, kSiteMmaFull = 0x203,
                   kSiteEpiFull = 0x204, kSiteDrain = 0x205 };
 
+// BN vocabulary rows per tile and MG M-tiles per pass; the accumulators of one item take
+// MG * BN tensor-memory columns, so <256, 1> double-buffers them (two slots) and
+// <256, 2> has a single slot (its epilogue then waits for the MMAs, a small share when H
+// is large).  N = 256 MMAs run at the full tensor rate; two M-tiles per W tile halve the
+// hidden bytes fetched per W byte compared with one.
 template <int BN, int MG>
 struct Cfg {
   static constexpr int kABytes = kBM * kBK * 2;           // 16 KB per M-tile
   static constexpr int kBBytes = BN * kBK * 2;            // BN rows x 128 B
   static constexpr int kStageBytes = MG * kABytes + kBBytes;
-  static constexpr int kSlots = 2;
+  static constexpr int kSlots = 512 / (MG * BN);
+  static constexpr int kStages = MG * BN > 256 ? 3 : 4;  // ring depth within shared memory
   static constexpr int kTmemCols = kSlots * MG * BN;      // 512
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/ +
                                     2 * kMaxMTiles * kBM * 4 /*row state*/;
   static_assert(kTmemCols == 512, "tensor memory plan uses all 512 columns");
   static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -84,10 +93,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                              ~uintptr_t(1023));
   uint8_t* ring = smem;
-  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + kStages * C::kStageBytes);
-  uint64_t* full = bars;                    // [kStages]
-  uint64_t* empty = bars + kStages;         // [kStages]
-  uint64_t* tfull = bars + 2 * kStages;     // [kSlots]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStageBytes);
+  uint64_t* full = bars;                    // [C::kStages]
+  uint64_t* empty = bars + C::kStages;         // [C::kStages]
+  uint64_t* tfull = bars + 2 * C::kStages;     // [kSlots]
   uint64_t* tempty = tfull + C::kSlots;     // [kSlots]
   uint64_t* drain = tempty + C::kSlots;     // [1]
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
@@ -109,7 +118,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int kblocks = (H + kBK - 1) / kBK;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < C::kStages; ++s) {
       mbar_init(smem_u32(&full[s]), 1);
       mbar_init(smem_u32(&empty[s]), 1);
     }
@@ -132,7 +141,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (hrows < kBM) {
     // A-tile rows the hidden box never fills: zero them once so the (discarded)
     // accumulator rows they produce stay finite
-    for (int i = threadIdx.x; i < kStages * MG * (kBM - hrows) * 8; i += kThreads) {
+    for (int i = threadIdx.x; i < C::kStages * MG * (kBM - hrows) * 8; i += kThreads) {
       const int chunk = i & 7, rr = (i >> 3) % (kBM - hrows) + hrows, tile = (i >> 3) / (kBM - hrows);
       uint4* dst = reinterpret_cast<uint4*>(ring + (tile / MG) * C::kStageBytes +
                                             (tile % MG) * C::kABytes + rr * 128 + chunk * 16);
@@ -184,17 +193,17 @@ __global__ void __launch_bounds__(kThreads, 1)
           for (; r < rows16; r += 16)
             tma_load_2d(smem_u32(bsm + r * 128), &tm_w16, fb, kb * kBK, v0 + r, pol_w);
           ++issued;
-          if (++stage == kStages) {
+          if (++stage == C::kStages) {
             stage = 0;
             phase ^= 1;
           }
         }
       }
-      // leave no copy in flight: wait for the last (up to kStages) loads issued
-      const int pend = issued < kStages ? (int)issued : kStages;
+      // leave no copy in flight: wait for the last (up to C::kStages) loads issued
+      const int pend = issued < C::kStages ? (int)issued : C::kStages;
       for (int i = 0; i < pend; ++i) {
         if (--stage < 0) {
-          stage = kStages - 1;
+          stage = C::kStages - 1;
           phase ^= 1;
         }
         mbar_wait(smem_u32(&full[stage]), phase, limit_ns);
@@ -238,7 +247,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
           }
           tc_commit(smem_u32(&empty[stage]));
-          if (++stage == kStages) {
+          if (++stage == C::kStages) {
             stage = 0;
             phase ^= 1;
           }
@@ -381,7 +390,7 @@ struct Plan {
 static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->rows + kBM - 1) / kBM;
-  p.bn = mtiles == 1 ? 256 : 128;
+  p.bn = 256;
   p.mg = mtiles == 1 ? 1 : 2;
   const int nunits = (d->vocab + 15) / 16;
   p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
@@ -458,10 +467,10 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   fvrag_status st;
-  if (p.bn == 256)
+  if (p.mg == 1)
     st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else
-    st = launch<128, 2>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
+    st = launch<256, 2>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   if (st != FVRAG_OK) return st;
   const int rows_per_block = 8;
   if (launch_pdl(lm_merge_kernel, dim3((d->rows + rows_per_block - 1) / rows_per_block),

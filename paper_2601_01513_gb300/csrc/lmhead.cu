@@ -58,7 +58,10 @@ enum : uint32_t { kSiteProdEmpty = 0x201, kSiteMmaTmem = 0x202, kSiteMmaFull = 0
 // MG * BN tensor-memory columns, so <256, 1> double-buffers them (two slots) and
 // <256, 2> has a single slot (its epilogue then waits for the MMAs, a small share when H
 // is large).  N = 256 MMAs run at the full tensor rate; two M-tiles per W tile halve the
-// hidden bytes fetched per W byte compared with one.
+// hidden bytes fetched per W byte compared with one.  <160, 3> serves exactly three
+// M-tiles (129-384 rows) in one pass over W (480 of the 512 columns): with <256, 2> the
+// third M-tile would need a second pass, and a CTA's 256-row W tile (2H * 256 bytes, 4 MB
+// at H = 8192) is long gone from L2 by the time the second pass comes back to it.
 template <int BN, int MG>
 struct Cfg {
   static constexpr int kABytes = kBM * kBK * 2;           // 16 KB per M-tile
@@ -66,10 +69,11 @@ struct Cfg {
   static constexpr int kStageBytes = MG * kABytes + kBBytes;
   static constexpr int kSlots = 512 / (MG * BN);
   static constexpr int kStages = MG * BN > 256 ? 3 : 4;  // ring depth within shared memory
-  static constexpr int kTmemCols = kSlots * MG * BN;      // 512
+  static constexpr int kTmemCols = 512;                   // allocation: a power of two
   static constexpr int kSmemBytes = kStages * kStageBytes + 1024 /*align*/ + 256 /*barriers*/ +
                                     2 * kMaxMTiles * kBM * 4 /*row state*/;
-  static_assert(kTmemCols == 512, "tensor memory plan uses all 512 columns");
+  static_assert(kSlots >= 1 && kSlots * MG * BN <= kTmemCols, "accumulators fit tensor memory");
+  static_assert(BN % 32 == 0 && BN <= 256, "epilogue reads 32-column chunks; MMA N <= 256");
   static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
   static_assert(kSmemBytes <= 232448, "shared memory per CTA");
 };
@@ -390,8 +394,8 @@ struct Plan {
 static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->rows + kBM - 1) / kBM;
-  p.bn = 256;
-  p.mg = mtiles == 1 ? 1 : 2;
+  p.bn = mtiles == 3 ? 160 : 256;
+  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : 2;
   const int nunits = (d->vocab + 15) / 16;
   p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
   return p;
@@ -469,6 +473,8 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   fvrag_status st;
   if (p.mg == 1)
     st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
+  else if (p.mg == 3)
+    st = launch<160, 3>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else
     st = launch<256, 2>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   if (st != FVRAG_OK) return st;

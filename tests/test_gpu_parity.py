@@ -110,7 +110,9 @@ LM_CASES = [
     (33, 72, 1007, 2),        # H not a multiple of 64; V not a multiple of 16
     (128, 128, 5000, 8),      # one full M-tile, 8 gathers
     (129, 256, 4103, 1),      # two M-tiles (second with one row)
-    (300, 192, 3001, 2),      # three M-tiles: two groups
+    (300, 192, 3001, 2),      # three M-tiles: one pass of 160-row vocabulary tiles
+    (257, 64, 50021, 1),      # three M-tiles, the third with one row; ~3 vocabulary tiles per CTA
+    (512, 96, 7777, 3),       # four M-tiles: two passes of two
     (80, 3584, 9000, 1),      # 7b hidden size, small vocabulary
     (2048, 64, 1000, 1),      # the most rows supported: 16 M-tiles in 8 groups
 ]

@@ -17,7 +17,11 @@
 //
 // Key blocks of 128: the query's prefix blocks, then the blocks of the tile's
 // candidates' own slots (concatenated) that hold at least one valid slot.  The
-// list is cut into equal runs of blocks, one run per CTA (split-KV).
+// list is cut into equal runs of blocks, one run per CTA (split-KV): the same
+// number of runs for every tile when the tiles' lists are alike (verification),
+// or, when their lengths differ with data known only on the device (decode: n_k),
+// runs of one length R for all tiles, chosen so that all runs fit one grid of CTAs;
+// every CTA makes that plan in its prologue and takes its own (tile, run).
 //
 // attn_kernel: one CTA = one row tile x one run of key blocks.
 //   warp 0     TMA: the Q tile once (3-D map over [tokens][hq][D]), then K and V
@@ -68,6 +72,14 @@ constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (P stays < 2^8)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
+// balanced plan (see plan_run): shared-memory capacity
+constexpr int kMaxPlanTiles = 1024;   // tiles the plan holds in shared memory
+constexpr int kMaxPlanQueries = 1024; // queries whose offsets it stages
+constexpr int kMaxPlanOwn = 2048;     // Qn * K own lengths it stages
+constexpr int kMaxRuns = 64;          // runs of one tile that merge_kernel combines
+constexpr int kPlanScratch = 256;     // reduction and control words
+constexpr int kPlanInts = kPlanScratch + kMaxPlanTiles + kMaxPlanQueries + 4 + kMaxPlanOwn;
+
 enum : uint32_t { kSiteQ = 0x101, kSiteMma = 0x102, kSiteProducer = 0x103, kSiteSFull = 0x107,
                   kSitePvDone = 0x109, kSiteDrain = 0x10A };
 
@@ -79,11 +91,13 @@ struct Layout {
   static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
   // + row-max exchange [2 slots][2 halves][128 rows] and row-sum exchange [2][128] floats
   static constexpr int kBytes =
-      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4;
+      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4 + 16 +
+      kPlanInts * 4;
   static_assert(kBytes <= 232448, "shared memory per CTA");
 };
 
 struct Args {
+  int2* tile_runs;         // balanced plan: [tiles] {first slot, runs}, written here; or null
   const int32_t* offs;
   const int32_t* own_len;  // [Qn][K] valid own slots n_k, or null (n_k = C)
   __nv_bfloat16* out;     // final output (one split)
@@ -93,6 +107,7 @@ struct Args {
   uint32_t* status;
   uint64_t limit_ns;
   int Qn, K, Lq, C, KL, hq, hkv, grp, T, mtiles, nsplit;
+  int slot_rows;           // balanced plan: rows per partial slot (T * grp)
   float scale_log2;
 };
 
@@ -133,6 +148,159 @@ __device__ __forceinline__ uint64_t desc_mnmajor_sw128(uint32_t smem_addr, uint3
   return d;
 }
 
+// ---------------------------------------------------------------------------
+// Balanced plan, for tiles whose block lists differ in length by data on the device
+// (decode: n_k).  Every CTA of the grid makes the same plan from the same inputs in its
+// prologue: the smallest run length R (in blocks) such that the runs of all tiles,
+// ns_t = max(1, ceil(nb_t / R)) each, fit in the grid (and ns_t <= kMaxRuns); tile t's
+// list is cut into ns_t equal runs held by consecutive CTAs.
+
+// Length of tile t's block list: its query's prefix blocks plus the own blocks that hold a
+// valid slot, i.e. the union over its candidates c with n_c > 0 of the blocks
+// [c C / 128, (c C + n_c - 1) / 128] (the count the kernel makes with own_valid).
+// offs_s and own_s are the prefix offsets and own lengths staged in shared memory.
+__device__ int tile_blocks(const Args& a, const int* offs_s, const int* own_s, int t) {
+  const int mt = t % a.mtiles;
+  const int qi = t / a.mtiles / a.hkv;
+  const int P = max(0, offs_s[qi + 1] - offs_s[qi]);
+  int nb = (P + kBN - 1) / kBN;
+  const int tok0 = mt * a.T;
+  const int ntok = min(a.T, a.KL - tok0);
+  const int c_lo = tok0 / a.Lq;
+  const int ncand = (tok0 + ntok - 1) / a.Lq - c_lo + 1;
+  int last = -1;                                  // highest own block counted so far
+  for (int c = 0; c < ncand; ++c) {
+    int n = a.own_len ? own_s[qi * a.K + c_lo + c] : a.C;
+    n = n < 0 ? 0 : (n > a.C ? a.C : n);
+    if (n == 0) continue;
+    const int lo = (c * a.C) / kBN, hi = (c * a.C + n - 1) / kBN;
+    if (hi > last) {
+      nb += hi - max(lo, last + 1) + 1;
+      last = hi;
+    }
+  }
+  return nb;
+}
+
+// Called by all NT threads of the CTA.  Returns this CTA's run {tile, first block, blocks,
+// 1 if the tile has a single run}, or tile -1 when the plan leaves the CTA idle; the CTA
+// holding a tile's first run records {first slot (CTA), runs} of the tile for the merge.
+template <int NT>
+__device__ int4 plan_run(const Args& a, int* ps) {
+  constexpr int NW = NT / 32;
+  long long* red_sum = reinterpret_cast<long long*>(ps);   // [NW]
+  int* red_max = ps + 64;
+  int* red_r = ps + 96;
+  int* red_ok = ps + 128;
+  int* scan_s = ps + 160;
+  int* ctl = ps + 192;             // [0], [1] search range of R; [2..5] this CTA's run
+  int* nb_s = ps + kPlanScratch;
+  int* offs_s = nb_s + kMaxPlanTiles;
+  int* own_s = offs_s + kMaxPlanQueries + 4;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int ntiles = a.Qn * a.hkv * a.mtiles;
+  for (int i = tid; i <= a.Qn; i += NT) offs_s[i] = __ldg(&a.offs[i]);
+  if (a.own_len)
+    for (int i = tid; i < a.Qn * a.K; i += NT) own_s[i] = __ldg(&a.own_len[i]);
+  if (tid == 0) ctl[2] = -1;
+  __syncthreads();
+  long long sum = 0;
+  int mx = 0;
+  for (int t = tid; t < ntiles; t += NT) {
+    const int nb = tile_blocks(a, offs_s, own_s, t);
+    nb_s[t] = nb;
+    sum += nb;
+    mx = max(mx, nb);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    mx = max(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  if (lane == 0) {
+    red_sum[warp] = sum;
+    red_max[warp] = mx;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    long long total = 0;
+    int m = 0;
+    for (int w = 0; w < NW; ++w) {
+      total += red_sum[w];
+      m = max(m, red_max[w]);
+    }
+    // any R >= total / (grid - tiles) fits: the run count is at most total / R + tiles
+    const int rmin = max(1, (m + kMaxRuns - 1) / kMaxRuns);
+    const long long slack = (long long)gridDim.x - ntiles;
+    ctl[0] = rmin;
+    ctl[1] = (int)max((long long)rmin, (total + slack - 1) / slack);
+  }
+  __syncthreads();
+  // NW-ary search: warp w tests R_w = lo + (hi - lo) w / (NW - 1) (R_{NW-1} = hi fits)
+  while (ctl[0] < ctl[1]) {
+    const int lo = ctl[0], hi = ctl[1];
+    const int rw = lo + (int)((long long)(hi - lo) * warp / (NW - 1));
+    long long cnt = 0;
+    for (int t = lane; t < ntiles; t += 32) cnt += max(1, (nb_s[t] + rw - 1) / rw);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cnt += __shfl_xor_sync(0xffffffffu, cnt, o);
+    if (lane == 0) {
+      red_r[warp] = rw;
+      red_ok[warp] = cnt <= (long long)gridDim.x;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      int w = 0;
+      while (!red_ok[w]) ++w;
+      ctl[0] = w > 0 ? red_r[w - 1] + 1 : lo;
+      ctl[1] = red_r[w];
+    }
+    __syncthreads();
+  }
+  const int R = ctl[1];
+  // runs per tile over a contiguous chunk of tiles per thread; exclusive scan of the counts
+  const int per = (ntiles + NT - 1) / NT;
+  const int t0 = min(ntiles, tid * per), t1 = min(ntiles, t0 + per);
+  int local = 0;
+  for (int t = t0; t < t1; ++t) local += max(1, (nb_s[t] + R - 1) / R);
+  int incl = local;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) scan_s[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int v = lane < NW ? scan_s[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int u = __shfl_up_sync(0xffffffffu, v, o);
+      if (lane >= o) v += u;
+    }
+    if (lane < NW) scan_s[lane] = v;   // inclusive over warps
+  }
+  __syncthreads();
+  int start = incl - local + (warp > 0 ? scan_s[warp - 1] : 0);
+  const int b = blockIdx.x;
+  for (int t = t0; t < t1; ++t) {
+    const int nb = nb_s[t];
+    const int ns = max(1, (nb + R - 1) / R);
+    if (b >= start && b < start + ns) {
+      const int bps = (nb + ns - 1) / ns;
+      const int lo = (b - start) * bps;
+      ctl[2] = t;
+      ctl[3] = lo;
+      ctl[4] = max(0, min(nb, lo + bps) - lo);
+      ctl[5] = ns == 1 ? 1 : 0;
+      if (b == start) a.tile_runs[t] = make_int2(start, ns);
+    }
+    start += ns;
+  }
+  __syncthreads();
+  return make_int4(ctl[2], ctl[3], ctl[4], ctl[5]);
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kp,
@@ -162,14 +330,24 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   griddep_wait();                 // inputs may come from the previous kernel
   // ---- work item
-  int b = blockIdx.x;
-  const int mt = b % a.mtiles;
-  b /= a.mtiles;
-  const int split = b % a.nsplit;
-  b /= a.nsplit;
-  const int g = b % a.hkv;
-  const int qi = b / a.hkv;
-  const int P = __ldg(&a.offs[qi + 1]) - __ldg(&a.offs[qi]);
+  int mt, split = 0, g, qi;
+  int4 wk = make_int4(0, 0, 0, 0);
+  if (a.tile_runs) {
+    wk = plan_run<kThreads>(a, reinterpret_cast<int*>(drain + 1) + 4 + ((kMaxCand + 3) & ~3));
+    if (wk.x < 0) return;         // the plan left this CTA without a run
+    mt = wk.x % a.mtiles;
+    g = (wk.x / a.mtiles) % a.hkv;
+    qi = wk.x / a.mtiles / a.hkv;
+  } else {
+    int b = blockIdx.x;
+    mt = b % a.mtiles;
+    b /= a.mtiles;
+    split = b % a.nsplit;
+    b /= a.nsplit;
+    g = b % a.hkv;
+    qi = b / a.hkv;
+  }
+  const int P = max(0, __ldg(&a.offs[qi + 1]) - __ldg(&a.offs[qi]));
   const int nbp = (P + kBN - 1) / kBN;                 // prefix blocks of this query
   const int tok0 = mt * a.T;
   const int ntok = min(a.T, a.KL - tok0);
@@ -179,6 +357,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ntb = (ncand * a.C + kBN - 1) / kBN;       // blocks over the candidates' own slots
   // valid own slots of the tile's candidates (the own blocks with none are skipped)
   int* n_own = reinterpret_cast<int*>(drain + 1) + 4;
+
   for (int c = threadIdx.x; c < ncand; c += kThreads) {
     int n = a.own_len ? __ldg(&a.own_len[qi * a.K + c_lo + c]) : a.C;
     n_own[c] = n < 0 ? 0 : (n > a.C ? a.C : n);
@@ -221,13 +400,13 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  // own block tb holds a valid slot when some candidate c it overlaps has
-  // c * C + n_c > tb * kBN (each candidate's valid slots are its first n_c)
+  // own block tb holds a valid slot when some candidate c it overlaps has n_c > 0
+  // and c * C + n_c > tb * kBN (each candidate's valid slots are its first n_c)
   auto own_valid = [&](int tb) {
     const int s0 = tb * kBN;
     const int s1 = min(s0 + kBN, ncand * a.C);
     for (int c = s0 / a.C; c * a.C < s1; ++c)
-      if (c * a.C + n_own[c] > s0) return true;
+      if (n_own[c] > 0 && c * a.C + n_own[c] > s0) return true;
     return false;
   };
   auto own_next = [&](int tb) {                      // first valid own block >= tb
@@ -240,9 +419,16 @@ __global__ void __launch_bounds__(kThreads, 1)
   for (int base = 0; base < ntb; base += 32)
     nvt += __popc(__ballot_sync(0xffffffffu, base + lane < ntb && own_valid(base + lane)));
   const int nb = nbp + nvt;
-  const int bps = (nb + a.nsplit - 1) / a.nsplit;
-  const int blk_lo = split * bps;
-  const int nblk = max(0, min(nb, blk_lo + bps) - blk_lo);
+  int blk_lo, nblk;
+  if (a.tile_runs) {              // plan_run counted the same nb for this tile
+    blk_lo = wk.y;
+    nblk = wk.z;
+  } else {
+    const int bps = (nb + a.nsplit - 1) / a.nsplit;
+    blk_lo = split * bps;
+    nblk = max(0, min(nb, blk_lo + bps) - blk_lo);
+  }
+  const bool direct = a.tile_runs ? wk.w != 0 : a.nsplit == 1;   // this CTA writes the output
   // the first own block this run uses: skip the valid own blocks of earlier runs
   int tb_first = ntb;
   {
@@ -547,6 +733,9 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int head = g * a.grp + r % a.grp;
     const size_t rowid = ((size_t)qi * a.KL + tok) * a.hq + head;
     const size_t nrows = (size_t)a.Qn * a.KL * a.hq;
+    // partial slot of this row: [run][row of the tile] (balanced plan) or [split][row]
+    const size_t pidx =
+        a.tile_runs ? (size_t)blockIdx.x * a.slot_rows + r : (size_t)split * nrows + rowid;
     const bool any = l > 0.f;
     const float inv = any ? 1.f / l : 0.f;
     const float lse = any ? kLn2 * (m_ref + __log2f(l)) : -INFINITY;
@@ -562,7 +751,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         for (int c = 0; c < 32; ++c) o[c] = 0u;
       }
       if (rvalid) {
-        if (a.nsplit == 1) {
+        if (direct) {
           uint4* dst = reinterpret_cast<uint4*>(a.out + rowid * D + oc);
 #pragma unroll
           for (int c = 0; c < 32; c += 8)
@@ -572,7 +761,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pack_bf16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
                 pack_bf16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
         } else {
-          float4* dst = reinterpret_cast<float4*>(a.part_o + ((size_t)split * nrows + rowid) * D + oc);
+          float4* dst = reinterpret_cast<float4*>(a.part_o + pidx * D + oc);
 #pragma unroll
           for (int c = 0; c < 32; c += 4)
             dst[c / 4] = make_float4(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv,
@@ -581,10 +770,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       }
     }
     if (rvalid && half == 0) {
-      if (a.nsplit == 1) {
+      if (direct) {
         if (a.lse) a.lse[rowid] = lse;
       } else {
-        a.part_lse[(size_t)split * nrows + rowid] = lse;
+        a.part_lse[pidx] = lse;
       }
     }
   }
@@ -595,21 +784,45 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem_base, kTmemCols);
 }
 
+// Where the partials of a tile live under the balanced plan (null otherwise).
+struct RunTable {
+  const int2* tile_runs;   // [tiles] {first slot, runs}
+  int slot_rows, KL, hq, grp, T, mtiles, hkv;
+};
+
 // One warp per output row: out = sum_s w_s o_s / sum_s w_s with w_s = exp(lse_s - max lse),
 // lse = max + log(sum_s w_s).  Lane s holds split s's weight (and s + 32); all partial
-// loads of a group of 8 splits are issued before any is used.
+// loads of a group of 8 splits are issued before any is used.  Partial s of the row sits
+// at index first + s * stride: [split][row] (static plan), or [slot][row of the tile]
+// with the tile's runs in consecutive slots (balanced plan; a tile with one run was
+// written by its CTA directly).
 template <int D>
 __global__ void merge_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
                              int nsplit, long long nrows, __nv_bfloat16* __restrict__ out,
-                             float* __restrict__ lse_out) {
+                             float* __restrict__ lse_out, const RunTable rt) {
   constexpr int DPL = D / 32;
   griddep_wait();
   griddep_launch_dependents();
   const long long row = (long long)blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
   if (row >= nrows) return;
-  const float l0 = lane < nsplit ? part_lse[(size_t)lane * nrows + row] : -INFINITY;
-  const float l1 = lane + 32 < nsplit ? part_lse[(size_t)(lane + 32) * nrows + row] : -INFINITY;
+  long long first = row, stride = nrows;
+  if (rt.tile_runs) {
+    const int head = (int)(row % rt.hq);
+    const long long tq = row / rt.hq;
+    const int tok = (int)(tq % rt.KL);
+    const int qi = (int)(tq / rt.KL);
+    const int g = head / rt.grp;
+    const int mt = tok / rt.T;
+    const int r = (tok - mt * rt.T) * rt.grp + head % rt.grp;
+    const int2 tr = rt.tile_runs[((long long)qi * rt.hkv + g) * rt.mtiles + mt];
+    if (tr.y <= 1) return;
+    nsplit = tr.y;
+    first = (long long)tr.x * rt.slot_rows + r;
+    stride = rt.slot_rows;
+  }
+  const float l0 = lane < nsplit ? part_lse[first + lane * stride] : -INFINITY;
+  const float l1 = lane + 32 < nsplit ? part_lse[first + (lane + 32) * stride] : -INFINITY;
   const float mx = warp_max(fmaxf(l0, l1));
   const float w0 = l0 == -INFINITY ? 0.f : __expf(l0 - mx);
   const float w1 = l1 == -INFINITY ? 0.f : __expf(l1 - mx);
@@ -617,13 +830,13 @@ __global__ void merge_kernel(const float* __restrict__ part_o, const float* __re
   float res[DPL];
 #pragma unroll
   for (int i = 0; i < DPL; ++i) res[i] = 0.f;
-  const float* base = part_o + (size_t)row * D + lane * DPL;
+  const float* base = part_o + (size_t)first * D + lane * DPL;
   for (int s0 = 0; s0 < nsplit; s0 += 8) {
     float v[8][DPL];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       if (s0 + u < nsplit) {
-        const float* po = base + (size_t)(s0 + u) * nrows * D;
+        const float* po = base + (size_t)(s0 + u) * stride * D;
         if constexpr (DPL == 4) {
           const float4 f = *reinterpret_cast<const float4*>(po);
           v[u][0] = f.x;
@@ -659,6 +872,7 @@ struct Problem {
   int Qn, K, Lq, C, hq, hkv, D, max_prefix, total_prefix;
   float scale;                 // 0 => 1/sqrt(D)
   const int32_t* own_len;      // device [Qn][K] or null (every candidate has C valid slots)
+  bool ragged;                 // the valid own slots n_k are read from the device
 };
 
 struct Plan {
@@ -702,8 +916,42 @@ static Plan make_plan(const Problem& pr, int sms) {
   return p;
 }
 
+// The balanced plan serves problems whose tiles' block lists differ by the n_k on the
+// device (decode): one grid of CTAs, a whole number of waves over the SMs with room for
+// every tile's first run and a quarter more.
+static bool balanced_grid(const Problem& pr, const Plan& p, int sms, int* grid) {
+  if (!pr.ragged) return false;
+  const long long ntiles = (long long)pr.Qn * pr.hkv * p.mtiles;
+  if (ntiles > kMaxPlanTiles || pr.Qn > kMaxPlanQueries || (long long)pr.Qn * pr.K > kMaxPlanOwn)
+    return false;
+  const long long waves = (ntiles + ntiles / 4) / sms + 1;
+  if (waves > 8) return false;
+  *grid = (int)(waves * sms);
+  return true;
+}
+
+// Workspace of the balanced plan: header | tile runs [tiles] | partial O [grid][T * grp][D]
+// | partial lse [grid][T * grp].
+struct BalancedWs {
+  size_t runs, part_o, part_lse, total;
+};
+
+static BalancedWs balanced_ws(const Problem& pr, const Plan& p, int grid) {
+  auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
+  const size_t ntiles = (size_t)pr.Qn * pr.hkv * p.mtiles;
+  const size_t slots = (size_t)grid * p.grp * p.T;
+  BalancedWs w;
+  w.runs = up(kWsHeaderBytes);
+  w.part_o = w.runs + up(ntiles * sizeof(int2));
+  w.part_lse = w.part_o + up(slots * pr.D * 4);
+  w.total = w.part_lse + up(slots * 4);
+  return w;
+}
+
 static size_t ws_bytes(const Problem& pr, int sms) {
   const Plan p = make_plan(pr, sms);
+  int grid = 0;
+  if (balanced_grid(pr, p, sms, &grid)) return balanced_ws(pr, p, grid).total;
   const size_t rows = (size_t)pr.Qn * pr.K * pr.Lq * pr.hq;
   return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)pr.D + 1) * 4 : 0);
 }
@@ -773,13 +1021,22 @@ static fvrag_status run(const Problem& pr, const void* q, const void* k_prefix, 
       maps[2] = maps[4];
     }
   }
+  int bgrid = 0;
+  const bool bal = balanced_grid(pr, p, sms, &bgrid);
+  const BalancedWs bw = bal ? balanced_ws(pr, p, bgrid) : BalancedWs{};
   Args a;
+  a.tile_runs = bal ? reinterpret_cast<int2*>(base + bw.runs) : nullptr;
   a.offs = prefix_offsets;
   a.own_len = pr.own_len;
   a.out = reinterpret_cast<__nv_bfloat16*>(out);
   a.lse = lse;
-  a.part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
-  a.part_lse = a.part_o + (size_t)p.nsplit * nrows * D;
+  if (bal) {
+    a.part_o = reinterpret_cast<float*>(base + bw.part_o);
+    a.part_lse = reinterpret_cast<float*>(base + bw.part_lse);
+  } else {
+    a.part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
+    a.part_lse = a.part_o + (size_t)p.nsplit * nrows * D;
+  }
   a.status = reinterpret_cast<uint32_t*>(base);
   a.limit_ns = wait_limit_ns();
   a.Qn = pr.Qn;
@@ -793,30 +1050,38 @@ static fvrag_status run(const Problem& pr, const void* q, const void* k_prefix, 
   a.T = p.T;
   a.mtiles = p.mtiles;
   a.nsplit = p.nsplit;
+  a.slot_rows = p.grp * p.T;
   a.scale_log2 = scale * kLog2e;
-  const long long grid = (long long)pr.Qn * pr.hkv * p.nsplit * p.mtiles;
+  RunTable rt{nullptr, a.slot_rows, KL, pr.hq, p.grp, p.T, p.mtiles, pr.hkv};
+  long long grid = (long long)pr.Qn * pr.hkv * p.nsplit * p.mtiles;
+  if (bal) {
+    rt.tile_runs = a.tile_runs;
+    grid = bgrid;
+  }
   if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
   fvrag_status st = D == 128 ? launch<128>(maps, a, grid, s) : launch<64>(maps, a, grid, s);
-  if (st != FVRAG_OK || p.nsplit == 1) return st;
+  if (st != FVRAG_OK || (!bal && p.nsplit == 1)) return st;
   const int wpb = 8;
   const long long blocks = (nrows + wpb - 1) / wpb;
   const cudaError_t e =
       D == 128 ? launch_pdl(merge_kernel<128>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
-                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse)
+                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out,
+                            lse, rt)
                : launch_pdl(merge_kernel<64>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
-                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out, lse);
+                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out,
+                            lse, rt);
   if (e != cudaSuccess) return FVRAG_ERR_CUDA;
   return launch_status();
 }
 
 static Problem verify_problem(const fvrag_attn_desc* d) {
   return Problem{d->num_queries, d->num_cand, d->cand_len, d->cand_len, d->hq, d->hkv,
-                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, nullptr};
+                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, nullptr, false};
 }
 
 static Problem decode_problem(const fvrag_decode_desc* d, const int32_t* cache_len) {
   return Problem{d->num_queries, d->num_drafts, 1, d->cache_cap, d->hq, d->hkv,
-                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, cache_len};
+                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, cache_len, true};
 }
 
 }  // namespace attn

@@ -37,6 +37,8 @@ def test_decode_tiny_matches_oracle():
     (3, 4, 8, 1, 64, (100, 900), 300, (1, 1)),           # MQA, D = 64, only the newest token
     (1, 7, 2, 2, 128, (5000, 5000), 2048, (1500, 2048)), # long caches spread over many runs
     (1, 2, 4, 1, 64, (0, 0), 8192, (8000, 8192)),        # no prefix at all, 8K caches
+    (170, 2, 4, 2, 64, (0, 600), 96, (1, 96)),           # 340 row tiles: a grid of 3 waves
+    (1, 1, 1, 1, 64, (300000, 300000), 64, (1, 64)),     # one tile cut into the most runs (64)
 ])
 def test_decode_shapes(Qn, K, hq, hkv, D, pr, C, cr):
     cfg = configs.DEC_TINY.with_(num_queries=Qn, num_drafts=K, hq=hq, hkv=hkv, head_dim=D,

@@ -22,6 +22,28 @@ from .configs import VerifyConfig
 STEP_INPUTS = ("q", "k_prefix", "v_prefix", "prefix_offsets", "k_tail", "v_tail", "hidden",
                "targets", "cand_emb", "frame_emb")
 RESIDENT = ("weight",)   # model parameters: loaded once, not part of a step's inputs
+_ALIGN = 256             # byte alignment of every tensor inside an arena
+
+
+def _arena_layout(tensors: dict):
+    """name -> (byte offset, bytes) for the step inputs present, packed in STEP_INPUTS order."""
+    lay, off = {}, 0
+    for name in STEP_INPUTS:
+        if name in tensors:
+            nb = tensors[name].numel() * tensors[name].element_size()
+            lay[name] = (off, nb)
+            off += (nb + _ALIGN - 1) // _ALIGN * _ALIGN
+    return lay, max(off, _ALIGN)
+
+
+def _view(arena, off, nb, like):
+    return arena[off:off + nb].view(like.dtype).view(like.shape)
+
+
+class HostInputs(dict):
+    """A step's inputs as views into one pinned host buffer (``arena``) laid out like the
+    device buffer of the step, so that one copy moves them all."""
+    arena = None
 
 
 def _to_torch(name, arr):
@@ -52,8 +74,15 @@ class VerifyStep:
         self.argmax = torch.empty((Qn, K), dtype=torch.int32, device=dev)
         self.keep = torch.empty((Qn, K), dtype=torch.uint8, device=dev)
         self.cos = None
-        self.score = torch.empty((Qn, K), dtype=torch.float32, device=dev)
-        self.selected = torch.empty((Qn,), dtype=torch.int32, device=dev)
+        # the step's result (score, selected) shares one buffer so one copy reads it back
+        sb = (Qn * K * 4 + _ALIGN - 1) // _ALIGN * _ALIGN
+        self._result = torch.empty(sb + Qn * 4, dtype=torch.uint8, device=dev)
+        self.score = self._result[:Qn * K * 4].view(torch.float32).view(Qn, K)
+        self.selected = self._result[sb:sb + Qn * 4].view(torch.int32)
+        self._sel_off = sb
+        self._result_h = None
+        self._arena = None
+        self._layout = {}
         lmd = fvrag.LmDesc(M, cfg.hidden, cfg.vocab, cfg.gathers, 0)
         self.lm_ws = torch.zeros(fvrag.lm_workspace_bytes(lmd), dtype=torch.uint8, device=dev)
         self.attn_ws = None
@@ -61,9 +90,20 @@ class VerifyStep:
 
     # ---------------------------------------------------------------- inputs
     def upload(self, inputs: dict) -> None:
-        """Copies numpy inputs (from ``synth.make_inputs``) to the device."""
-        for name, arr in inputs.items():
-            self.t[name] = _to_torch(name, arr).to(self.device)
+        """Copies numpy inputs (from ``synth.make_inputs``) to the device.  The per-step
+        inputs go into one device buffer (the arena), each a 256-byte-aligned view; model
+        parameters get their own allocations."""
+        tens = {name: _to_torch(name, arr) for name, arr in inputs.items()}
+        lay, total = _arena_layout(tens)
+        self._layout = lay
+        self._arena = torch.empty(total, dtype=torch.uint8, device=self.device)
+        for name, x in tens.items():
+            if name in lay:
+                v = _view(self._arena, *lay[name], x)
+                v.copy_(x)
+                self.t[name] = v
+            else:
+                self.t[name] = x.to(self.device)
         if "prefix_offsets" in inputs:
             offs = inputs["prefix_offsets"]
             mp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
@@ -78,14 +118,15 @@ class VerifyStep:
         if self.attn_ws is None or self.attn_ws.numel() < need:
             self.attn_ws = torch.zeros(need, dtype=torch.uint8, device=self.device)
 
-    def host_inputs(self, pin=True) -> dict:
-        """Per-step inputs as (pinned) host tensors, for the end-to-end path."""
-        h = {}
-        for name in STEP_INPUTS:
-            if name in self.t:
-                x = torch.empty(self.t[name].shape, dtype=self.t[name].dtype, pin_memory=pin)
-                x.copy_(self.t[name])
-                h[name] = x
+    def host_inputs(self, pin=True) -> HostInputs:
+        """Per-step inputs as views into one (pinned) host arena laid out like the device
+        arena, for the end-to-end path.  Writing new inputs into the views and passing the
+        result to ``run_from_host`` uploads them with a single copy."""
+        h = HostInputs()
+        h.arena = torch.empty(self._arena.numel(), dtype=torch.uint8, pin_memory=pin)
+        h.arena.copy_(self._arena)
+        for name, (off, nb) in self._layout.items():
+            h[name] = _view(h.arena, off, nb, self.t[name])
         return h
 
     # ---------------------------------------------------------------- the step
@@ -160,19 +201,25 @@ class VerifyStep:
         """End-to-end step: host->device copies of the step's inputs, the four calls, and a
         device->host read of the result (selected index and candidate scores).
         Returns (selected, score) host tensors and the byte counts moved each way."""
-        h2d = 0
-        for name, x in host.items():
-            self.t[name].copy_(x, non_blocking=True)
-            h2d += x.numel() * x.element_size()
+        arena = getattr(host, "arena", None)
+        if (arena is not None and self._arena is not None and arena.numel() == self._arena.numel()
+                and set(host) == set(self._layout)):
+            self._arena.copy_(arena, non_blocking=True)        # all inputs in one copy
+            h2d = arena.numel()
+        else:
+            h2d = 0
+            for name, x in host.items():
+                self.t[name].copy_(x, non_blocking=True)
+                h2d += x.numel() * x.element_size()
         if stream is None:
             self.replay()
         else:
             self.run(stream)
-        if getattr(self, "_sel_h", None) is None:
-            self._sel_h = torch.empty(self.selected.shape, dtype=self.selected.dtype, pin_memory=True)
-            self._sc_h = torch.empty(self.score.shape, dtype=self.score.dtype, pin_memory=True)
-        sel, sc = self._sel_h, self._sc_h
-        sel.copy_(self.selected, non_blocking=True)
-        sc.copy_(self.score, non_blocking=True)
-        d2h = sel.numel() * sel.element_size() + sc.numel() * sc.element_size()
-        return sel, sc, h2d, d2h
+        if self._result_h is None:
+            self._result_h = torch.empty(self._result.numel(), dtype=torch.uint8, pin_memory=True)
+        self._result_h.copy_(self._result, non_blocking=True)   # score and selected in one copy
+        Qn, K = self.score.shape
+        sb = self._sel_off
+        sc = self._result_h[:Qn * K * 4].view(torch.float32).view(Qn, K)
+        sel = self._result_h[sb:sb + Qn * 4].view(torch.int32)
+        return sel, sc, h2d, self._result.numel()

@@ -268,10 +268,20 @@ def test_pipeline_end_to_end_from_host():
     host = step.host_inputs()
     sel, sc, h2d, d2h = step.run_from_host(host)
     torch.cuda.synchronize()
+    ref_sel, ref_sc = step.selected.cpu().numpy().copy(), step.score.cpu().numpy().copy()
+    assert np.array_equal(sel.numpy(), ref_sel) and np.array_equal(sc.numpy(), ref_sc)
+    assert h2d >= sum(v.numel() * v.element_size() for v in host.values())
+    assert d2h >= cfg.num_queries * 4 + cfg.num_queries * cfg.num_cand * 4
+    # new inputs written into the host views travel with the one copy of the arena
+    host["targets"].copy_((host["targets"] + 1) % cfg.vocab)
+    _, sc2, _, _ = step.run_from_host(host)
+    torch.cuda.synchronize()
+    got = sc2.numpy().copy()
+    assert not np.array_equal(got, ref_sc)
+    assert torch.equal(step.t["targets"].cpu(), host["targets"])
     step.run()
     torch.cuda.synchronize()
-    assert h2d > 0 and d2h == cfg.num_queries * 4 + cfg.num_queries * cfg.num_cand * 4
-    assert np.array_equal(sel.numpy(), step.selected.cpu().numpy())
+    assert np.array_equal(step.score.cpu().numpy(), got)
 
 
 # ============================================================ failure detection

@@ -91,8 +91,8 @@ struct Layout {
   static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
   // + row-max exchange [2 slots][2 halves][128 rows] and row-sum exchange [2][128] floats
   static constexpr int kBytes =
-      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4 + 16 +
-      kPlanInts * 4;
+      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4;
+  static_assert(kPlanInts * 4 <= kVStages * kStage, "plan scratch fits the V ring");
   static_assert(kBytes <= 232448, "shared memory per CTA");
 };
 
@@ -301,7 +301,9 @@ __device__ int4 plan_run(const Args& a, int* ps) {
   return make_int4(ctl[2], ctl[3], ctl[4], ctl[5]);
 }
 
-template <int D>
+// BAL: the balanced plan (decode) or the static split (verification); separate
+// instantiations keep the plan's code out of the verification kernel.
+template <int D, bool BAL>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kp,
                 const __grid_constant__ CUtensorMap tm_vp, const __grid_constant__ CUtensorMap tm_kt,
@@ -332,8 +334,10 @@ __global__ void __launch_bounds__(kThreads, 1)
   // ---- work item
   int mt, split = 0, g, qi;
   int4 wk = make_int4(0, 0, 0, 0);
-  if (a.tile_runs) {
-    wk = plan_run<kThreads>(a, reinterpret_cast<int*>(drain + 1) + 4 + ((kMaxCand + 3) & ~3));
+  if constexpr (BAL) {
+    // the plan's scratch is the V ring, whose first writer is the TMA after the prologue
+    wk = plan_run<kThreads>(a, reinterpret_cast<int*>(v_ring));
+    fence_proxy_async_smem();
     if (wk.x < 0) return;         // the plan left this CTA without a run
     mt = wk.x % a.mtiles;
     g = (wk.x / a.mtiles) % a.hkv;
@@ -420,7 +424,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     nvt += __popc(__ballot_sync(0xffffffffu, base + lane < ntb && own_valid(base + lane)));
   const int nb = nbp + nvt;
   int blk_lo, nblk;
-  if (a.tile_runs) {              // plan_run counted the same nb for this tile
+  if constexpr (BAL) {            // plan_run counted the same nb for this tile
     blk_lo = wk.y;
     nblk = wk.z;
   } else {
@@ -428,7 +432,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     blk_lo = split * bps;
     nblk = max(0, min(nb, blk_lo + bps) - blk_lo);
   }
-  const bool direct = a.tile_runs ? wk.w != 0 : a.nsplit == 1;   // this CTA writes the output
+  const bool direct = BAL ? wk.w != 0 : a.nsplit == 1;   // this CTA writes the output
   // the first own block this run uses: skip the valid own blocks of earlier runs
   int tb_first = ntb;
   {
@@ -735,7 +739,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     const size_t nrows = (size_t)a.Qn * a.KL * a.hq;
     // partial slot of this row: [run][row of the tile] (balanced plan) or [split][row]
     const size_t pidx =
-        a.tile_runs ? (size_t)blockIdx.x * a.slot_rows + r : (size_t)split * nrows + rowid;
+        BAL ? (size_t)blockIdx.x * a.slot_rows + r : (size_t)split * nrows + rowid;
     const bool any = l > 0.f;
     const float inv = any ? 1.f / l : 0.f;
     const float lse = any ? kLn2 * (m_ref + __log2f(l)) : -INFINITY;
@@ -961,13 +965,13 @@ static int device_sms() {
   return s > 0 ? s : 148;
 }
 
-template <int D>
+template <int D, bool BAL>
 static fvrag_status launch(const CUtensorMap* maps, const Args& a, long long grid, cudaStream_t s) {
   const int sm = Layout<D>::kBytes;
-  if (cudaFuncSetAttribute(attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) !=
-      cudaSuccess)
+  auto kern = attn_kernel<D, BAL>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) != cudaSuccess)
     return FVRAG_ERR_CUDA;
-  if (launch_pdl(attn_kernel<D>, dim3((unsigned)grid), dim3(kThreads), (size_t)sm, s, maps[0], maps[1],
+  if (launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), (size_t)sm, s, maps[0], maps[1],
                  maps[2], maps[3], maps[4], a) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
@@ -1059,7 +1063,11 @@ static fvrag_status run(const Problem& pr, const void* q, const void* k_prefix, 
     grid = bgrid;
   }
   if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
-  fvrag_status st = D == 128 ? launch<128>(maps, a, grid, s) : launch<64>(maps, a, grid, s);
+  fvrag_status st;
+  if (bal)
+    st = D == 128 ? launch<128, true>(maps, a, grid, s) : launch<64, true>(maps, a, grid, s);
+  else
+    st = D == 128 ? launch<128, false>(maps, a, grid, s) : launch<64, false>(maps, a, grid, s);
   if (st != FVRAG_OK || (!bal && p.nsplit == 1)) return st;
   const int wpb = 8;
   const long long blocks = (nrows + wpb - 1) / wpb;

@@ -344,6 +344,287 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
 }
 
+// ---------------------------------------------------------------------------
+// Pair form for many rows (more than three M-tiles).  A cluster of two CTAs on two SMs
+// runs the GEMM with tcgen05 cta_group::2 MMAs of M = 256: CTA r of the pair holds hidden
+// rows [128 r, 128 r + 128) of every 256-row pair-tile and W rows [v0 + N/2 r, v0 + N/2 (r + 1))
+// of every N-row vocabulary tile, and its tensor memory receives the accumulators of its
+// own 128 rows against all N columns (rank 0's W rows first).  Each SM thus loads half of
+// every W tile, and one pass over W serves PG pair-tiles (PG = 2: 512 rows).  Rank 0
+// issues the MMAs; both CTAs load (their copies complete on rank 0's barriers), and both
+// run the epilogue over their own rows.  The pair owns one contiguous vocabulary range
+// and writes one partial per row.
+template <int PG>
+struct PairCfg {
+  static constexpr int BN = 256;                           // vocabulary rows per tile (MMA N)
+  static constexpr int kABytes = kBM * kBK * 2;            // this CTA's 128 rows of a pair-tile
+  static constexpr int kBBytes = (BN / 2) * kBK * 2;       // this CTA's half of a W tile
+  static constexpr int kStageBytes = PG * kABytes + kBBytes;
+  static constexpr int kSlots = 512 / (PG * BN);
+  static constexpr int kStages = PG == 2 ? 4 : 6;
+  static constexpr int kTmemCols = 512;
+  static constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + 2 * kMaxMTiles * kBM * 4;
+  static_assert(kSlots >= 1 && kSlots * PG * BN <= kTmemCols, "accumulators fit tensor memory");
+  static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+};
+
+template <int PG>
+__global__ void __launch_bounds__(kThreads, 1)
+    lm_head_pair_kernel(const __grid_constant__ CUtensorMap tm_hidden,
+                        const __grid_constant__ CUtensorMap tm_w64,
+                        const __grid_constant__ CUtensorMap tm_w16, const int32_t* __restrict__ targets,
+                        int M, int H, int V, int G, float* __restrict__ part_max,
+                        float* __restrict__ part_sum, float* __restrict__ tgt_logit, uint32_t* status,
+                        uint64_t limit_ns) {
+  using C = PairCfg<PG>;
+  constexpr int BN = C::BN;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* ring = smem;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStages * C::kStageBytes);
+  uint64_t* full = bars;                       // [kStages]  rank 0: both CTAs' copies
+  uint64_t* empty = bars + C::kStages;         // [kStages]  each CTA: its stage is free
+  uint64_t* tfull = bars + 2 * C::kStages;     // [kSlots]   each CTA: accumulators ready
+  uint64_t* tempty = tfull + C::kSlots;        // [kSlots]   rank 0: both epilogues done
+  uint64_t* drain = tempty + C::kSlots;        // [1]        rank 0: every MMA done
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* st_max = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);
+  float* st_sum = st_max + kMaxMTiles * kBM;
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+
+  // ---- this pair's vocabulary range, in units of 16 rows
+  const int nunits = (V + 15) >> 4;
+  const int u_lo = (int)(((long long)pair * nunits) / npairs);
+  const int u_hi = (int)(((long long)(pair + 1) * nunits) / npairs);
+  const int v_lo = u_lo * 16;
+  const int v_hi = min(u_hi * 16, V);
+  const int ntiles = (v_hi - v_lo + BN - 1) / BN;
+  const int ptiles = (M + 2 * kBM - 1) / (2 * kBM);        // 256-row pair-tiles
+  const int ngroups = (ptiles + PG - 1) / PG;
+  const int nitems = ntiles * ngroups;
+  const int kblocks = (H + kBK - 1) / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int s = 0; s < C::kSlots; ++s) {
+      mbar_init(smem_u32(&tfull[s]), 1);
+      mbar_init(smem_u32(&tempty[s]), 8);  // one arrival per epilogue warp of both CTAs
+    }
+    mbar_init(smem_u32(drain), 1);
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_hidden);
+    tma_prefetch_desc(&tm_w64);
+    tma_prefetch_desc(&tm_w16);
+  }
+  for (int i = threadIdx.x; i < ptiles * kBM; i += kThreads) {
+    st_max[i] = -INFINITY;
+    st_sum[i] = 0.f;
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(tmem_holder), C::kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // the peer's barriers are initialised before any remote use
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);      // rank 0's barriers
+  const uint32_t tempty0 = mapa_shared(smem_u32(&tempty[0]), 0);
+  griddep_wait();                 // the prologue above touched no global memory
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer (both CTAs)
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_h = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int t = it / ngroups, grp = it % ngroups;
+        const int v0 = v_lo + t * BN;
+        const int n = min(BN, (v_hi - v0 + 31) & ~31);    // MMA N, a multiple of 32
+        const int half = n >> 1;
+        const int pcount = min(PG, ptiles - grp * PG);
+        const uint32_t bytes = pcount * C::kABytes + half * kBK * 2;   // per CTA
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + (uint32_t)(stage * 8);
+          if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full[stage]), 2 * bytes);
+          uint8_t* st = ring + stage * C::kStageBytes;
+          for (int j = 0; j < pcount; ++j)
+            tma_load_2d_pair(smem_u32(st + j * C::kABytes), &tm_hidden, fb, kb * kBK,
+                             (grp * PG + j) * 2 * kBM + (int)rank * kBM, pol_h);
+          uint8_t* bsm = st + PG * C::kABytes;
+          const int w0 = v0 + (int)rank * half;
+          int r = 0;
+          for (; r + 64 <= half; r += 64)
+            tma_load_2d_pair(smem_u32(bsm + r * 128), &tm_w64, fb, kb * kBK, w0 + r, pol_w);
+          for (; r < half; r += 16)
+            tma_load_2d_pair(smem_u32(bsm + r * 128), &tm_w16, fb, kb * kBK, w0 + r, pol_w);
+          ++issued;
+          if (++stage == C::kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // rank 0 sees both CTAs' copies complete on its barriers: leave none in flight
+      if (rank == 0) {
+        const int pend = issued < C::kStages ? (int)issued : C::kStages;
+        for (int i = 0; i < pend; ++i) {
+          if (--stage < 0) {
+            stage = C::kStages - 1;
+            phase ^= 1;
+          }
+          mbar_wait(smem_u32(&full[stage]), phase, limit_ns);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (rank 0)
+    if (lane == 0 && rank == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int slot = it % C::kSlots;
+        const uint32_t use = it / C::kSlots;
+        const int t = it / ngroups, grp = it % ngroups;
+        const int v0 = v_lo + t * BN;
+        const int n = min(BN, (v_hi - v0 + 31) & ~31);
+        const int pcount = min(PG, ptiles - grp * PG);
+        const uint32_t idesc = idesc_bf16_f32(2 * kBM, n);
+        if (!mbar_wait_cluster(smem_u32(&tempty[slot]), (use & 1) ^ 1, limit_ns)) {
+          record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaTmem);
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&full[stage]), phase, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaFull);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(ring + stage * C::kStageBytes);
+          const uint32_t bsm = st + PG * C::kABytes;
+          for (int j = 0; j < pcount; ++j) {
+            const uint32_t d = tmem_base + (uint32_t)((slot * PG + j) * BN);
+#pragma unroll
+            for (int k16 = 0; k16 < kBK / 16; ++k16)
+              tc_mma_bf16_pair(d, desc_kmajor_sw128(st + j * C::kABytes + k16 * 32),
+                               desc_kmajor_sw128(bsm + k16 * 32), idesc, (kb | k16) != 0);
+          }
+          tc_commit_pair(smem_u32(&empty[stage]), 0x3);
+          if (++stage == C::kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit_pair(smem_u32(&tfull[slot]), 0x3);
+      }
+      // every MMA issued by this thread has finished before tensor memory is freed
+      tc_commit_pair(smem_u32(drain), 0x1);
+      if (!mbar_wait(smem_u32(drain), 0, limit_ns)) record_error(status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (both CTAs)
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;      // this CTA's row inside a pair-tile
+    for (int it = 0; it < nitems; ++it) {
+      const int slot = it % C::kSlots;
+      const uint32_t use = it / C::kSlots;
+      const int t = it / ngroups, grp = it % ngroups;
+      const int v0 = v_lo + t * BN;
+      const int ncols = min(BN, v_hi - v0);
+      const int pcount = min(PG, ptiles - grp * PG);
+      if (!mbar_wait_cluster(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
+        break;
+      }
+      tc_fence_after();
+      for (int j = 0; j < pcount; ++j) {
+        const int pt = grp * PG + j;
+        const int m = pt * 2 * kBM + (int)rank * kBM + row;
+        const bool live = m < M;
+        int tg[kMaxGathers];
+#pragma unroll
+        for (int g = 0; g < kMaxGathers; ++g)
+          tg[g] = (live && g < G) ? __ldg(&targets[(size_t)m * G + g]) - v0 : -1;
+        float rmax = st_max[pt * kBM + row];
+        float rsum = st_sum[pt * kBM + row];
+        const uint32_t tbase =
+            tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * PG + j) * BN);
+        for (int c0 = 0; c0 < ncols; c0 += 32) {
+          uint32_t r[32];
+          tmem_ld_32x32b_x32(tbase + c0, r);
+          tmem_wait_ld();
+          const int nvalid = min(32, ncols - c0);
+          float cmax = -INFINITY;
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nvalid) cmax = fmaxf(cmax, __uint_as_float(r[i]) * kLog2e);
+          const float nmax = fmaxf(rmax, cmax);
+          float sacc = rsum * ex2(rmax - nmax);
+#pragma unroll
+          for (int i = 0; i < 32; ++i)
+            if (i < nvalid) sacc += ex2(fmaf(__uint_as_float(r[i]), kLog2e, -nmax));
+          rsum = sacc;
+          rmax = nmax;
+#pragma unroll
+          for (int g = 0; g < kMaxGathers; ++g) {
+            const int c = tg[g] - c0;
+            if (c >= 0 && c < nvalid) {
+              float val = 0.f;
+#pragma unroll
+              for (int i = 0; i < 32; ++i)
+                if (i == c) val = __uint_as_float(r[i]);
+              tgt_logit[(size_t)m * G + g] = val;
+            }
+          }
+        }
+        st_max[pt * kBM + row] = rmax;
+        st_sum[pt * kBM + row] = rsum;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty0 + (uint32_t)(slot * 8));
+    }
+    // publish this CTA's rows of the pair's partials (log2 domain)
+    for (int pt = 0; pt < ptiles; ++pt) {
+      const int m = pt * 2 * kBM + (int)rank * kBM + row;
+      if (m < M) {
+        part_max[(size_t)pair * M + m] = st_max[pt * kBM + row];
+        part_sum[(size_t)pair * M + m] = st_sum[pt * kBM + row];
+      }
+    }
+  }
+  griddep_launch_dependents();    // the merge kernel may start launching
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // neither CTA frees tensor memory the other may still use
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem_base, C::kTmemCols);
+}
+
 // One warp per row: lse = ln 2 * (M2 + log2 S) with M2 = max_b max_b and
 // S = sum_b sum_b * 2^(max_b - M2) (partials in the log2 domain); logprob = z_target - lse.
 __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float* __restrict__ part_sum,
@@ -387,18 +668,81 @@ __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float*
 }
 
 struct Plan {
-  int ctas;
-  int bn, mg;
+  int ctas;       // CTAs of the 1-CTA forms; pairs of the pair form (the merge's partials)
+  int bn, mg;     // mg = 0: the pair form
 };
+
+// Pairs (2-CTA clusters) of the pair form that can be resident at once, per device.
+static int max_pairs() {
+  static std::mutex mu;
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cached[dev] == 0) {
+    using C = PairCfg<2>;
+    int n = 0;
+    if (cudaFuncSetAttribute(lm_head_pair_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             C::kSmemBytes) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      const int sms = std::max(2, sm_count());
+      cfg.gridDim = dim3(sms / 2 * 2);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = C::kSmemBytes;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 2;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      if (cudaOccupancyMaxActiveClusters(&n, lm_head_pair_kernel<2>, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    cached[dev] = std::max(1, std::min(n, std::min(sm_count() / 2, kMaxCtas)));
+  }
+  return cached[dev];
+}
 
 static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->rows + kBM - 1) / kBM;
   p.bn = mtiles == 3 ? 160 : 256;
-  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : 2;
+  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : mtiles == 2 ? 2 : 0;
   const int nunits = (d->vocab + 15) / 16;
   p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
+  if (p.mg == 0) p.ctas = std::max(1, std::min(max_pairs(), nunits));
   return p;
+}
+
+template <int PG>
+static fvrag_status launch_pair(const Plan& p, const CUtensorMap& th, const CUtensorMap& tw64,
+                                const CUtensorMap& tw16, const int32_t* targets,
+                                const fvrag_lm_desc* d, float* pmax, float* psum, float* ptgt,
+                                uint32_t* status, cudaStream_t s) {
+  using C = PairCfg<PG>;
+  auto kern = lm_head_pair_kernel<PG>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::kSmemBytes) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * p.ctas);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = C::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (cudaLaunchKernelEx(&cfg, kern, th, tw64, tw16, targets, d->rows, d->hidden, d->vocab,
+                         d->gathers, pmax, psum, ptgt, status, wait_limit_ns()) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return launch_status();
 }
 
 static size_t ws_bytes(const fvrag_lm_desc* d) {
@@ -471,7 +815,9 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   fvrag_status st;
-  if (p.mg == 1)
+  if (p.mg == 0)
+    st = launch_pair<2>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
+  else if (p.mg == 1)
     st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else if (p.mg == 3)
     st = launch<160, 3>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);

@@ -112,9 +112,10 @@ LM_CASES = [
     (129, 256, 4103, 1),      # two M-tiles (second with one row)
     (300, 192, 3001, 2),      # three M-tiles: one pass of 160-row vocabulary tiles
     (257, 64, 50021, 1),      # three M-tiles, the third with one row; ~3 vocabulary tiles per CTA
-    (512, 96, 7777, 3),       # four M-tiles: two passes of two
+    (512, 96, 7777, 3),       # four M-tiles: one pass of two CTA-pair tiles (2-SM MMAs)
+    (600, 128, 50021, 2),     # three pair tiles (the last one partly empty), ragged W tiles
     (80, 3584, 9000, 1),      # 7b hidden size, small vocabulary
-    (2048, 64, 1000, 1),      # the most rows supported: 16 M-tiles in 8 groups
+    (2048, 64, 1000, 1),      # the most rows supported: 8 pair tiles in 4 passes
 ]
 
 

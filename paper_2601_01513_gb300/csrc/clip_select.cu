@@ -2,9 +2,13 @@
 // K4: candidate selection (masked mean log-prob; Algorithm 1's two stages,
 // Eq. 12-13 and the final argmax over alignment).
 //
-// Both steps move kilobytes to a few megabytes, so they are latency-bound:
-// K3 uses one CTA per (query, candidate), 16 warps with four frames' 16-byte
-// loads in flight per warp; K4 uses one CTA per query.
+// At the paper's sizes both steps move kilobytes to a few megabytes and are
+// latency-bound.  K3 reads every frame embedding once per group of 16 candidates:
+// a warp scores 16 frames against all of them with mma.sync tensor-core tiles (the
+// contraction is [16 frames x E] x [E x 16 candidates], too small in M for tcgen05
+// tiles), so with many frames it streams at HBM rates; a query's frames are split
+// over a cluster of up to 8 CTAs whose per-candidate bests are merged in distributed
+// shared memory.  K4 uses one CTA per query.
 #include <cuda_fp16.h>
 
 #include "fvrag_common.cuh"
@@ -13,125 +17,239 @@
 namespace fvrag {
 
 constexpr int kClipThreads = 512;
-constexpr int kClipUnroll = 4;   // frames in flight per warp
+constexpr int kClipWarps = kClipThreads / 32;
+constexpr int kClipKG = 16;      // candidates a CTA scores against each frame (two MMA n-tiles)
+constexpr int kClipTile = 16;    // frames per warp tile (MMA m)
+constexpr int kClipUnroll = 4;   // 32-element chunks of E in flight per thread
 constexpr int kClipMaxDim = 4096;
+constexpr int kClipMaxSplit = 8; // CTAs (one cluster) sharing one query's frames
+constexpr int kClipPad = 8;      // fp16 elements of padding per candidate row in shared memory
 
-// One CTA per (query q, candidate k).  The candidate embedding is widened to
-// fp32 in shared memory; warp w handles frames w, w + 16, w + 32, w + 48 together
-// (then the next 64): the 32 lanes split the E dimension in 16-byte (8 x fp16)
-// chunks with the four frames' loads in flight at once, reduce <e, f> and |f|^2
-// with shuffles, and lane 0 keeps the warp's best (cos, frame).  The 16 warp
-// results are then reduced by one warp: larger cos wins, equal cos goes to the
-// lower frame index.
+__device__ __forceinline__ void st_cluster_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void st_cluster_s32(uint32_t addr, int v) {
+  asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+// (v, i) beats (bv, bi): larger cosine, or equal cosine and lower frame index.
+__device__ __forceinline__ bool clip_better(float v, int i, float bv, int bi) {
+  return v > bv || (v == bv && i < bi);
+}
+
+// D = A * B + D for one m16n8k16 tile: A 16 x 16 fp16 (row), B 16 x 8 fp16 (col), fp32 D.
+__device__ __forceinline__ void mma_f16_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                              uint32_t a3, uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Grid: Qn x G x S CTAs, blockIdx.x = (q * G + g) * S + s, in clusters of S along x.
+// CTA (q, g, s) scores frames [s F / S, (s + 1) F / S) of query q against candidates
+// k0 .. k0 + kg - 1 (k0 = 16 g): every frame is read once per group of 16 candidates.
+//
+// The dot products are tensor-core tiles: a warp takes 16 frames as the A operand (rows)
+// and the 16 candidates as B (two n-tiles of 8), accumulating fp32 over E.  The order in
+// which E enters the contraction does not change the sums, so lane (r, t) (r = lane / 4,
+// t = lane % 4) loads elements [32 c + 8 t, 32 c + 8 t + 8) of frames r and r + 8 and of
+// candidates r and r + 8 with 16-byte loads and uses them as its fragment pairs of two
+// consecutive k16 steps; A and B pair up the same elements.  The frames' squared norms
+// come from two more MMAs of the frame tile against itself (B = the tile's own rows), of
+// which the diagonal is kept.  Each lane then holds the cosines of frames r, r + 8 with
+// candidates 2t, 2t + 1, 2t + 8, 2t + 9; the per-candidate best (cos, frame) is reduced over
+// the warp, the CTA and, through rank 0's shared memory, the cluster, which writes max_cos,
+// argmax and keep.
 __global__ void __launch_bounds__(kClipThreads) clip_align_kernel(
     const __half* __restrict__ cand, const __half* __restrict__ frames, int K, int F, int E,
     float tau, float* __restrict__ cos_out, float* __restrict__ max_cos, int32_t* __restrict__ argmax,
-    uint8_t* __restrict__ keep) {
-  __shared__ __align__(16) float e_s[kClipMaxDim];
-  __shared__ float red[kClipThreads / 32];
-  __shared__ float best_v[kClipThreads / 32];
-  __shared__ int best_i[kClipThreads / 32];
+    uint8_t* __restrict__ keep, int G, int S) {
+  extern __shared__ __align__(16) __half c_s[];     // [kClipKG][E + kClipPad], then the
+                                                    // accumulator exchange [warps][32][16] fp32
+  __shared__ float inv_e_s[kClipKG];
+  __shared__ float red_v[kClipWarps][kClipKG];
+  __shared__ int red_i[kClipWarps][kClipKG];
+  __shared__ float part_v[kClipMaxSplit][kClipKG];  // rank 0: one row per CTA of the cluster
+  __shared__ int part_i[kClipMaxSplit][kClipKG];
   griddep_wait();
   griddep_launch_dependents();
-  const int qk = blockIdx.x;
-  const int q = qk / K;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int nchunk = E >> 3;
+  const int s = blockIdx.x % S;
+  const int qg = blockIdx.x / S;
+  const int g = qg % G, q = qg / G;
+  const int k0 = g * kClipKG, kg = min(kClipKG, K - k0);
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int r = lane >> 2, t = lane & 3;
+  const int nchunk = E >> 3;                          // 16-byte chunks per row
+  const int ldc = E + kClipPad;
 
-  const __half* e = cand + (size_t)qk * E;
-  float ee_part = 0.f;
-  for (int c = threadIdx.x; c < nchunk; c += kClipThreads) {
-    const uint4 raw = __ldg(reinterpret_cast<const uint4*>(e) + c);
-    const __half2* h2 = reinterpret_cast<const __half2*>(&raw);
+  // candidates k0 .. k0 + kg - 1 (rows past kg are zero) and their inverse norms
+  for (int idx = tid; idx < kClipKG * nchunk; idx += kClipThreads) {
+    const int k = idx / nchunk, c = idx - k * nchunk;
+    const uint4 raw = k < kg ? __ldg(reinterpret_cast<const uint4*>(cand + ((size_t)q * K + k0 + k) * E) + c)
+                             : make_uint4(0u, 0u, 0u, 0u);
+    *reinterpret_cast<uint4*>(&c_s[(size_t)k * ldc + 8 * c]) = raw;
+  }
+  __syncthreads();
+  for (int k = warp; k < kClipKG; k += kClipWarps) {
+    float ee = 0.f;
+    for (int i = lane; i < E; i += 32) {
+      const float v = __half2float(c_s[(size_t)k * ldc + i]);
+      ee = fmaf(v, v, ee);
+    }
+    ee = warp_sum(ee);
+    if (lane == 0) inv_e_s[k] = ee > 0.f ? rsqrtf(ee) : 0.f;
+  }
+  __syncthreads();
+  const float ie0 = inv_e_s[2 * t], ie1 = inv_e_s[2 * t + 1];
+  const float ie8 = inv_e_s[2 * t + 8], ie9 = inv_e_s[2 * t + 9];
+
+  const int fa = (int)(((long long)s * F) / S), fb = (int)(((long long)(s + 1) * F) / S);
+  const __half* fq = frames + (size_t)q * F * E;
+  const __half* c_lo = c_s + (size_t)r * ldc + 8 * t;          // candidate r
+  const __half* c_hi = c_s + (size_t)(r + 8) * ldc + 8 * t;    // candidate r + 8
+  const int nc32 = (E + 31) >> 5;                              // 32-element chunks
+  // With few frame tiles, ne warps share a tile, each over a slice of E, and add their
+  // accumulators through shared memory before the epilogue (warp part 0).
+  const int ntile = (fb - fa + kClipTile - 1) / kClipTile;
+  int ne = 1;
+  while (ne < 8 && 2 * ne * ntile <= kClipWarps && 2 * ne <= nc32) ne *= 2;
+  const int part = warp % ne, tpi = kClipWarps / ne;
+  const int c_beg = (part * nc32) / ne, c_end = ((part + 1) * nc32) / ne;
+  const int iters = (ntile + tpi - 1) / tpi;
+  float* xch = reinterpret_cast<float*>(c_s + (size_t)kClipKG * ldc);   // [warps][16][32]
+  // running best of candidates 2t, 2t+1, 2t+8, 2t+9 over this warp's frames
+  float bv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+  int bi[4] = {0x7fffffff, 0x7fffffff, 0x7fffffff, 0x7fffffff};
+  for (int it = 0; it < iters; ++it) {
+    const int tile = warp / ne + it * tpi;
+    const int f0 = fa + tile * kClipTile;
+    const int fr0 = f0 + r, fr1 = f0 + r + 8;
+    const bool v0 = tile < ntile && fr0 < fb, v1 = tile < ntile && fr1 < fb;
+    const uint4* p0 = reinterpret_cast<const uint4*>(fq + (size_t)(v0 ? fr0 : fa) * E + 8 * t);
+    const uint4* p1 = reinterpret_cast<const uint4*>(fq + (size_t)(v1 ? fr1 : fa) * E + 8 * t);
+    float acc[16];              // candidates 0-7 | 8-15 | frames x frames 0-7 | 8-15
+#pragma unroll
+    for (int i = 0; i < 16; ++i) acc[i] = 0.f;
+    float(&dc0)[4] = *reinterpret_cast<float(*)[4]>(&acc[0]);
+    float(&dc1)[4] = *reinterpret_cast<float(*)[4]>(&acc[4]);
+    float(&nn0)[4] = *reinterpret_cast<float(*)[4]>(&acc[8]);
+    float(&nn1)[4] = *reinterpret_cast<float(*)[4]>(&acc[12]);
+    for (int cb = c_beg; cb < c_end; cb += kClipUnroll) {
+      uint4 a_lo[kClipUnroll], a_hi[kClipUnroll];
+#pragma unroll
+      for (int u = 0; u < kClipUnroll; ++u) {
+        const int c = cb + u;
+        const bool in = c < c_end && 32 * c + 8 * t < E;
+        a_lo[u] = (in && v0) ? __ldg(p0 + 4 * c) : make_uint4(0u, 0u, 0u, 0u);
+        a_hi[u] = (in && v1) ? __ldg(p1 + 4 * c) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int u = 0; u < kClipUnroll; ++u) {
+        const int c = cb + u;
+        const bool in = c < c_end && 32 * c + 8 * t < E;
+        const uint4 b_lo = in ? *reinterpret_cast<const uint4*>(c_lo + 32 * c) : make_uint4(0u, 0u, 0u, 0u);
+        const uint4 b_hi = in ? *reinterpret_cast<const uint4*>(c_hi + 32 * c) : make_uint4(0u, 0u, 0u, 0u);
+        // k16 step 1: elements 8t .. 8t+3 of the chunk; step 2: 8t+4 .. 8t+7
+        mma_f16_16816(dc0, a_lo[u].x, a_hi[u].x, a_lo[u].y, a_hi[u].y, b_lo.x, b_lo.y);
+        mma_f16_16816(dc0, a_lo[u].z, a_hi[u].z, a_lo[u].w, a_hi[u].w, b_lo.z, b_lo.w);
+        mma_f16_16816(dc1, a_lo[u].x, a_hi[u].x, a_lo[u].y, a_hi[u].y, b_hi.x, b_hi.y);
+        mma_f16_16816(dc1, a_lo[u].z, a_hi[u].z, a_lo[u].w, a_hi[u].w, b_hi.z, b_hi.w);
+        mma_f16_16816(nn0, a_lo[u].x, a_hi[u].x, a_lo[u].y, a_hi[u].y, a_lo[u].x, a_lo[u].y);
+        mma_f16_16816(nn0, a_lo[u].z, a_hi[u].z, a_lo[u].w, a_hi[u].w, a_lo[u].z, a_lo[u].w);
+        mma_f16_16816(nn1, a_lo[u].x, a_hi[u].x, a_lo[u].y, a_hi[u].y, a_hi[u].x, a_hi[u].y);
+        mma_f16_16816(nn1, a_lo[u].z, a_hi[u].z, a_lo[u].w, a_hi[u].w, a_hi[u].z, a_hi[u].w);
+      }
+    }
+    if (ne > 1) {                 // part 0 adds the other parts' accumulators
+#pragma unroll
+      for (int i = 0; i < 16; ++i) xch[((size_t)warp * 16 + i) * 32 + lane] = acc[i];
+      __syncthreads();
+      if (part == 0)
+        for (int pp = 1; pp < ne; ++pp)
+#pragma unroll
+          for (int i = 0; i < 16; ++i) acc[i] += xch[((size_t)(warp + pp) * 16 + i) * 32 + lane];
+      __syncthreads();
+    }
+    if (part != 0 || tile >= ntile) continue;
+    // |f_r|^2 sits in lane (r, r / 2) as nn0[r & 1]; |f_{r+8}|^2 there as nn1[2 + (r & 1)]
+    const float d_lo = (r & 1) ? nn0[1] : nn0[0];
+    const float d_hi = (r & 1) ? nn1[3] : nn1[2];
+    const int src = 4 * r + (r >> 1);
+    const float n_lo = __shfl_sync(0xffffffffu, d_lo, src);
+    const float n_hi = __shfl_sync(0xffffffffu, d_hi, src);
+    const float if0 = n_lo > 0.f ? rsqrtf(n_lo) : 0.f;
+    const float if1 = n_hi > 0.f ? rsqrtf(n_hi) : 0.f;
+    // dc0 = {C[r][2t], C[r][2t+1], C[r+8][2t], C[r+8][2t+1]}, dc1 the same for candidates + 8
+    const float iek[4] = {ie0, ie1, ie8, ie9};
+    const int kk[4] = {2 * t, 2 * t + 1, 2 * t + 8, 2 * t + 9};
+    const float dlo[4] = {dc0[0], dc0[1], dc1[0], dc1[1]};   // frame r
+    const float dhi[4] = {dc0[2], dc0[3], dc1[2], dc1[3]};   // frame r + 8
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      const float2 f = __half22float2(h2[j]);
-      e_s[8 * c + 2 * j] = f.x;
-      e_s[8 * c + 2 * j + 1] = f.y;
-      ee_part = fmaf(f.x, f.x, fmaf(f.y, f.y, ee_part));
+      const bool kv = kk[j] < kg;
+      const float c_a = (if0 > 0.f && iek[j] > 0.f) ? dlo[j] * iek[j] * if0 : 0.f;
+      const float c_b = (if1 > 0.f && iek[j] > 0.f) ? dhi[j] * iek[j] * if1 : 0.f;
+      if (kv && v0) {
+        if (cos_out) cos_out[((size_t)q * K + k0 + kk[j]) * F + fr0] = c_a;
+        if (clip_better(c_a, fr0, bv[j], bi[j])) { bv[j] = c_a; bi[j] = fr0; }
+      }
+      if (kv && v1) {
+        if (cos_out) cos_out[((size_t)q * K + k0 + kk[j]) * F + fr1] = c_b;
+        if (clip_better(c_b, fr1, bv[j], bi[j])) { bv[j] = c_b; bi[j] = fr1; }
+      }
     }
   }
-  ee_part = warp_sum(ee_part);
-  if (lane == 0) red[warp] = ee_part;
-  __syncthreads();
-  float ee = 0.f;
+  // over the 8 lanes that share t (the tile's rows)
 #pragma unroll
-  for (int w = 0; w < kClipThreads / 32; ++w) ee += red[w];
-  const float inv_e = ee > 0.f ? rsqrtf(ee) : 0.f;
-
-  constexpr int NW = kClipThreads / 32;
-  float wbest = -INFINITY;
-  int wbest_i = 0x7fffffff;
-  const __half* fq = frames + (size_t)q * F * E;
-  for (int f0 = warp; f0 < F; f0 += NW * kClipUnroll) {
-    float dot[kClipUnroll], ff[kClipUnroll];
+  for (int j = 0; j < 4; ++j) {
 #pragma unroll
-    for (int u = 0; u < kClipUnroll; ++u) dot[u] = ff[u] = 0.f;
-    for (int c = lane; c < nchunk; c += 32) {
-      const float4 ea = *reinterpret_cast<const float4*>(&e_s[8 * c]);
-      const float4 eb = *reinterpret_cast<const float4*>(&e_s[8 * c + 4]);
-      uint4 raw[kClipUnroll];
-#pragma unroll
-      for (int u = 0; u < kClipUnroll; ++u) {
-        const int f = f0 + u * NW;
-        raw[u] = f < F ? __ldg(reinterpret_cast<const uint4*>(fq + (size_t)f * E) + c)
-                       : make_uint4(0, 0, 0, 0);
-      }
-#pragma unroll
-      for (int u = 0; u < kClipUnroll; ++u) {
-        const __half2* h2 = reinterpret_cast<const __half2*>(&raw[u]);
-        const float2 f0v = __half22float2(h2[0]), f1v = __half22float2(h2[1]);
-        const float2 f2v = __half22float2(h2[2]), f3v = __half22float2(h2[3]);
-        float d = dot[u], n = ff[u];
-        d = fmaf(ea.x, f0v.x, d); d = fmaf(ea.y, f0v.y, d);
-        d = fmaf(ea.z, f1v.x, d); d = fmaf(ea.w, f1v.y, d);
-        d = fmaf(eb.x, f2v.x, d); d = fmaf(eb.y, f2v.y, d);
-        d = fmaf(eb.z, f3v.x, d); d = fmaf(eb.w, f3v.y, d);
-        n = fmaf(f0v.x, f0v.x, n); n = fmaf(f0v.y, f0v.y, n);
-        n = fmaf(f1v.x, f1v.x, n); n = fmaf(f1v.y, f1v.y, n);
-        n = fmaf(f2v.x, f2v.x, n); n = fmaf(f2v.y, f2v.y, n);
-        n = fmaf(f3v.x, f3v.x, n); n = fmaf(f3v.y, f3v.y, n);
-        dot[u] = d;
-        ff[u] = n;
-      }
+    for (int o = 4; o < 32; o <<= 1) {
+      const float ov = __shfl_xor_sync(0xffffffffu, bv[j], o);
+      const int oi = __shfl_xor_sync(0xffffffffu, bi[j], o);
+      if (clip_better(ov, oi, bv[j], bi[j])) { bv[j] = ov; bi[j] = oi; }
     }
+  }
+  if (r == 0) {
+    red_v[warp][2 * t] = bv[0];     red_i[warp][2 * t] = bi[0];
+    red_v[warp][2 * t + 1] = bv[1]; red_i[warp][2 * t + 1] = bi[1];
+    red_v[warp][2 * t + 8] = bv[2]; red_i[warp][2 * t + 8] = bi[2];
+    red_v[warp][2 * t + 9] = bv[3]; red_i[warp][2 * t + 9] = bi[3];
+  }
+  __syncthreads();
+  float v = -INFINITY;
+  int vi = 0x7fffffff;
+  if (tid < kClipKG) {
 #pragma unroll
-    for (int u = 0; u < kClipUnroll; ++u) {
-      const int f = f0 + u * NW;
-      const float dsum = warp_sum(dot[u]);
-      const float nsum = warp_sum(ff[u]);
-      if (f < F && lane == 0) {
-        const float c = (nsum > 0.f && inv_e > 0.f) ? dsum * inv_e * rsqrtf(nsum) : 0.f;
-        if (cos_out) cos_out[(size_t)qk * F + f] = c;
-        if (c > wbest) {  // a warp sees its frames in increasing order: strict > keeps the lowest
-          wbest = c;
-          wbest_i = f;
+    for (int w = 0; w < kClipWarps; ++w)
+      if (clip_better(red_v[w][tid], red_i[w][tid], v, vi)) {
+        v = red_v[w][tid];
+        vi = red_i[w][tid];
+      }
+  }
+  if (S > 1) {
+    if (tid < kClipKG) {
+      st_cluster_f32(mapa_shared(smem_u32(&part_v[s][tid]), 0), v);
+      st_cluster_s32(mapa_shared(smem_u32(&part_i[s][tid]), 0), vi);
+    }
+    cluster_sync();
+    if (s != 0) return;
+    if (tid < kClipKG) {
+      v = part_v[0][tid];
+      vi = part_i[0][tid];
+      for (int rr = 1; rr < S; ++rr)
+        if (clip_better(part_v[rr][tid], part_i[rr][tid], v, vi)) {
+          v = part_v[rr][tid];
+          vi = part_i[rr][tid];
         }
-      }
     }
   }
-  if (lane == 0) {
-    best_v[warp] = wbest;
-    best_i[warp] = wbest_i;
-  }
-  __syncthreads();
-  if (warp == 0) {
-    float v = lane < NW ? best_v[lane] : -INFINITY;
-    int i = lane < NW ? best_i[lane] : 0x7fffffff;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-      const int oi = __shfl_xor_sync(0xffffffffu, i, o);
-      if (ov > v || (ov == v && oi < i)) {
-        v = ov;
-        i = oi;
-      }
-    }
-    if (lane == 0) {
-      max_cos[qk] = v;
-      argmax[qk] = i;
-      keep[qk] = v >= tau ? 1 : 0;
-    }
+  if (tid < kg) {
+    const size_t qk = (size_t)q * K + k0 + tid;
+    max_cos[qk] = v;
+    argmax[qk] = vi;
+    keep[qk] = v >= tau ? 1 : 0;
   }
 }
 
@@ -229,11 +347,34 @@ extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* c
   if (d->dim % 8 != 0 || d->dim > kClipMaxDim) return FVRAG_ERR_UNSUPPORTED;
   if ((int64_t)d->num_queries * d->num_cand > 0x7fffffff) return FVRAG_ERR_UNSUPPORTED;
   if (!aligned16(cand_emb) || !aligned16(frame_emb)) return FVRAG_ERR_MISALIGNED;
-  const int blocks = d->num_queries * d->num_cand;
-  if (launch_pdl(clip_align_kernel, dim3(blocks), dim3(kClipThreads), 0,
-                 reinterpret_cast<cudaStream_t>(stream), reinterpret_cast<const __half*>(cand_emb),
-                 reinterpret_cast<const __half*>(frame_emb), d->num_cand, d->num_frames, d->dim,
-                 d->threshold, cos, max_cos, argmax, keep) != cudaSuccess)
+  // frames split over a cluster of S CTAs (a power of two, at most 8, about 256 frames each)
+  int S = 1;
+  while (S < kClipMaxSplit && (long long)S * 256 < d->num_frames && 2 * S <= d->num_frames) S *= 2;
+  const int G = (d->num_cand + kClipKG - 1) / kClipKG;
+  const long long blocks = (long long)d->num_queries * G * S;
+  if (blocks > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
+  const size_t smem = (size_t)kClipKG * (d->dim + kClipPad) * sizeof(__half) +
+                      (size_t)kClipWarps * 16 * 32 * sizeof(float);
+  if (cudaFuncSetAttribute(clip_align_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           (int)smem) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)blocks);
+  cfg.blockDim = dim3(kClipThreads);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = reinterpret_cast<cudaStream_t>(stream);
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = (unsigned)S;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (cudaLaunchKernelEx(&cfg, clip_align_kernel, reinterpret_cast<const __half*>(cand_emb),
+                         reinterpret_cast<const __half*>(frame_emb), d->num_cand, d->num_frames,
+                         d->dim, d->threshold, cos, max_cos, argmax, keep, G, S) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
 }

@@ -199,6 +199,41 @@ def test_clip_edges():
     assert np.array_equal(mc2, mc) and np.array_equal(am2, am)
 
 
+@pytest.mark.parametrize("Qn,K,F,E", [
+    (2, 13, 300, 64),      # two candidate groups of a CTA; frames over a cluster of 2
+    (3, 8, 4096, 768),     # clusters of 8 CTAs per query
+    (1, 1, 1, 8),          # one frame, the smallest dimension
+    (1, 9, 2, 4096),       # the largest dimension
+    (16, 10, 4096, 768),   # the CLIP bandwidth-sweep size
+])
+def test_clip_shapes(Qn, K, F, E):
+    cand = synth.round_f16(synth.normal_f64((Qn, K, E), 31 + K, 1))
+    frames = synth.round_f16(synth.normal_f64((Qn, F, E), 31 + K, 2))
+    frames[:, F // 2] = cand[:, 0]                     # a planted exact match
+    cos, mc, am, keep = run_clip(cand, frames, 0.2)
+    rcos, rmc, ram, rkeep = oracle.clip_align(cand, frames, 0.2)
+    assert np.max(np.abs(cos - rcos)) <= COS_ATOL
+    assert np.max(np.abs(mc - rmc)) <= COS_ATOL
+    check_argmax_with_margin(am, rcos)
+    check_keep_with_margin(keep, rmc, 0.2)
+    assert np.all(am[:, 0] == F // 2)
+
+
+def test_clip_ties_across_a_cluster():
+    """Equal cosines in frames held by different CTAs of a cluster: the lowest index wins."""
+    E, F = 64, 1024
+    rng = np.random.default_rng(4)
+    x = synth.round_f16(rng.standard_normal(E))
+    y = synth.round_f16(rng.standard_normal(E))
+    cand = np.stack([x, y, 2 * x])[None]
+    frames = np.repeat(x[None, None], F, axis=1)       # every frame equals candidate 0 ...
+    frames[0, 700] = y                                 # ... but two equal to candidate 1,
+    frames[0, 900] = y                                 # held by different CTAs
+    cos, mc, am, keep = run_clip(cand, frames, 0.0, with_cos=False)
+    assert am[0, 0] == 0 and am[0, 2] == 0             # all maxima equal: the first frame
+    assert am[0, 1] == 700
+
+
 # ============================================================ selection
 ALL_MODES = [fvrag.SEL_MASKED_MEAN_LOGPROB, fvrag.SEL_TWO_STAGE, fvrag.SEL_ADDITION, fvrag.SEL_INVERT,
              fvrag.SEL_RELIABILITY_ONLY, fvrag.SEL_ALIGNMENT_ONLY, fvrag.SEL_RANDOM]

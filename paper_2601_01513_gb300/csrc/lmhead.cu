@@ -668,8 +668,8 @@ __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float*
 }
 
 struct Plan {
-  int ctas;       // CTAs of the 1-CTA forms; pairs of the pair form (the merge's partials)
-  int bn, mg;     // mg = 0: the pair form
+  int ctas;       // CTAs of the 1-CTA forms; pairs of the pair forms (the merge's partials)
+  int bn, mg;     // mg = 0 / -1: the pair form with two / one pair-tiles per pass
 };
 
 // Pairs (2-CTA clusters) of the pair form that can be resident at once, per device.
@@ -708,10 +708,13 @@ static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->rows + kBM - 1) / kBM;
   p.bn = mtiles == 3 ? 160 : 256;
-  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : mtiles == 2 ? 2 : 0;
+  // one M-tile: <256, 1>; two: the pair form with one pair-tile and two accumulator sets;
+  // three: <160, 3> (one pass; pairs would pad 384 rows to 512); more: the pair form with
+  // two pair-tiles per pass
+  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : mtiles == 2 ? -1 : 0;
   const int nunits = (d->vocab + 15) / 16;
   p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
-  if (p.mg == 0) p.ctas = std::max(1, std::min(max_pairs(), nunits));
+  if (p.mg <= 0) p.ctas = std::max(1, std::min(max_pairs(), nunits));
   return p;
 }
 
@@ -817,6 +820,8 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   fvrag_status st;
   if (p.mg == 0)
     st = launch_pair<2>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
+  else if (p.mg == -1)
+    st = launch_pair<1>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
   else if (p.mg == 1)
     st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else if (p.mg == 3)

@@ -43,7 +43,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 
 # DRAM traffic of one LM-head launch at the 7B shape, from an ncu capture of the
 # kernel source with this SHA-256 prefix (null once the kernel source changes).
-LM_TRAFFIC = {"sha256_prefix": "973327c92e3674bc", "bytes_per_launch": 1093798144}
+LM_TRAFFIC = {"sha256_prefix": "7afb8471b7320825", "bytes_per_launch": 1093970432}
 
 
 def peaks():
@@ -280,6 +280,20 @@ def _time_calls(fn, stream, steps, dev, between=None):
     return float(ms.mean()), ms
 
 
+def _steps_for_clocks(fn, stream, dev, steps, between=None, min_s=0.6, cap=20000):
+    """At least `steps` calls, and enough for the timed loop to last `min_s` seconds of wall
+    time, so that the clock sampler (one sample per 100 ms) sees the calls running."""
+    import torch
+    t0 = time.perf_counter()
+    for _ in range(5):
+        if between is not None:
+            between()
+        fn()
+    torch.cuda.synchronize(dev)
+    per = (time.perf_counter() - t0) / 5
+    return int(min(cap, max(steps, np.ceil(min_s / max(per, 1e-7)))))
+
+
 def bench_row(args):
     """One JSON line for the retrieval or keyframe step (1 GPU; other ranks replicate)."""
     import torch
@@ -339,6 +353,7 @@ def bench_row(args):
                 call()
                 call_host()
             torch.cuda.synchronize(dev)
+            steps = _steps_for_clocks(call, stream, dev, steps)
             with ClockSampler(dev.index or 0) as clk:
                 clk.wait_first()
                 t_ms, _ = _time_calls(call, stream, steps, dev)
@@ -415,6 +430,7 @@ def bench_row(args):
                 call()
                 call_host()
             torch.cuda.synchronize(dev)
+            steps = _steps_for_clocks(call, stream, dev, steps, between=flush_w.zero_)
             with ClockSampler(dev.index or 0) as clk:
                 clk.wait_first()
                 t_ms, _ = _time_calls(call, stream, steps, dev, between=flush_w.zero_)
@@ -483,6 +499,7 @@ def bench_row(args):
                 call()
                 call_host()
             torch.cuda.synchronize(dev)
+            steps = _steps_for_clocks(call, stream, dev, steps, between=flush_w.zero_)
             with ClockSampler(dev.index or 0) as clk:
                 clk.wait_first()
                 t_ms, _ = _time_calls(call, stream, steps, dev, between=flush_w.zero_)
@@ -557,6 +574,7 @@ def bench_row(args):
                 call()
             call_host()
             torch.cuda.synchronize(dev)
+            steps = _steps_for_clocks(call, stream, dev, steps)
             with ClockSampler(dev.index or 0) as clk:
                 clk.wait_first()
                 t_ms, _ = _time_calls(call, stream, steps, dev)

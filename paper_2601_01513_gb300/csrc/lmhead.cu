@@ -9,7 +9,7 @@
 //
 // Persistent grid, one CTA per SM.  CTA b owns a contiguous vocabulary range
 // (multiples of 16 rows, balanced to within 16 rows) and walks it in tiles of
-// BN = 256 rows.  Per tile it accumulates, for a group of MG M-tiles of 128 hidden rows,
+// BN rows.  Per tile it accumulates, for a group of MG M-tiles of 128 hidden rows,
 // D[128 x BN] = hidden_tile * W_tile^T in tensor memory (fp32), K-loop over H
 // in blocks of 64 (one 128-byte swizzled row per operand row).
 //
@@ -22,11 +22,14 @@
 //   warps 2-5  epilogue: tcgen05.ld of 32 columns at a time (one hidden row per
 //              thread), online max / sum of exp over the CTA's vocabulary slice,
 //              and the gather of target logits that fall in the slice.
-// With one M-tile, two accumulator sets in tensor memory let the epilogue of tile
-// t overlap the MMAs of tile t+1.  With two M-tiles the 512 columns hold a single
-// set: the N = 256 MMAs run at the full tensor rate (N = 128 ones issue at about
-// 80% of it) and each W byte feeds twice the hidden rows, which outweighs the lost
-// overlap while the epilogue is this light.
+// Forms by row count M:
+//   M <= 128        <256, 1>: one M-tile, two accumulator sets, so the epilogue of
+//                   tile t overlaps the MMAs of tile t+1 (HBM-bound: W streams once);
+//   129 .. 256      the pair form with one 256-row pair-tile (two accumulator sets);
+//   257 .. 384      <160, 3>: three M-tiles against 160-row W tiles, one pass over W;
+//   385 .. 2048     the pair form with two pair-tiles (512 rows) per pass over W.
+// The pair form (lm_head_pair_kernel) runs on clusters of two CTAs with tcgen05
+// cta_group::2 MMAs of M = 256, each SM loading half of every W tile.
 //
 // A second small kernel merges the per-CTA (max, sum) partials of every row into
 // lse and writes logprob = z_target - lse (NaN for ids outside [0, V)).
@@ -55,13 +58,11 @@ enum : uint32_t { kSiteProdEmpty = 0x201, kSiteMmaTmem = 0x202, kSiteMmaFull = 0
                   kSiteEpiFull = 0x204, kSiteDrain = 0x205 };
 
 // BN vocabulary rows per tile and MG M-tiles per pass; the accumulators of one item take
-// MG * BN tensor-memory columns, so <256, 1> double-buffers them (two slots) and
-// <256, 2> has a single slot (its epilogue then waits for the MMAs, a small share when H
-// is large).  N = 256 MMAs run at the full tensor rate; two M-tiles per W tile halve the
-// hidden bytes fetched per W byte compared with one.  <160, 3> serves exactly three
-// M-tiles (129-384 rows) in one pass over W (480 of the 512 columns): with <256, 2> the
-// third M-tile would need a second pass, and a CTA's 256-row W tile (2H * 256 bytes, 4 MB
-// at H = 8192) is long gone from L2 by the time the second pass comes back to it.
+// MG * BN tensor-memory columns.  <256, 1> (one M-tile) double-buffers them; <160, 3> serves
+// exactly three M-tiles (257-384 rows) in one pass over W with a single set (480 of the 512
+// columns): pairs of 256-column accumulators would need a second pass for the third M-tile,
+// and a CTA's 256-row W tile (2H * 256 bytes, 4 MB at H = 8192) is long gone from L2 by the
+// time that pass comes back to it.  Two M-tiles and more than three take the pair form below.
 template <int BN, int MG>
 struct Cfg {
   static constexpr int kABytes = kBM * kBK * 2;           // 16 KB per M-tile
@@ -824,10 +825,8 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
     st = launch_pair<1>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
   else if (p.mg == 1)
     st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
-  else if (p.mg == 3)
-    st = launch<160, 3>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else
-    st = launch<256, 2>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
+    st = launch<160, 3>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   if (st != FVRAG_OK) return st;
   const int rows_per_block = 8;
   if (launch_pdl(lm_merge_kernel, dim3((d->rows + rows_per_block - 1) / rows_per_block),

@@ -511,9 +511,12 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         if (moved) {
           t_last = globaltimer_ns();
-        } else if (globaltimer_ns() - t_last > a.limit_ns) {
-          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteProducer);
-          break;
+        } else {
+          __nanosleep(20);
+          if (globaltimer_ns() - t_last > a.limit_ns) {
+            record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteProducer);
+            break;
+          }
         }
       }
       // no copy may still be in flight when the CTA exits
@@ -575,9 +578,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           }
           if (moved) {
             t_last = globaltimer_ns();
-          } else if (globaltimer_ns() - t_last > a.limit_ns) {
-            record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
-            break;
+          } else {
+            __nanosleep(20);
+            if (globaltimer_ns() - t_last > a.limit_ns) {
+              record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
+              break;
+            }
           }
         }
       }

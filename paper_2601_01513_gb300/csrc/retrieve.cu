@@ -5,22 +5,25 @@
 // Shape of the work: sim = frames[Fr x E] * texts[Nt x E]^T with Fr (keyframes of
 // a batch of queries) small (1 .. 2048) and the corpus large (1,048,576 x 768
 // fp16 = 1.6 GB).  It is the LM head's shape with a different epilogue, so the
-// kernel has the same structure: a persistent grid, one CTA per SM, each CTA
-// owning a contiguous range of texts (16-row units) and walking it in tiles of
-// BN texts; per tile a tcgen05 GEMM accumulates D[128 x BN] = frames_tile *
-// texts_tile^T in tensor memory (fp16 inputs, fp32 accumulate), K-loop over E
-// in 64-element blocks (one 128-byte swizzled row per operand row).
+// kernels have the same structure: a persistent grid, each CTA (or CTA pair)
+// owning a contiguous range of texts (16-row units) and walking it in tiles of 256
+// texts; per tile a tcgen05 GEMM accumulates frames_tile * texts_tile^T in tensor
+// memory (fp16 inputs, fp32 accumulate), K-loop over E in 64-element blocks (one
+// 128-byte swizzled row per operand row).
 //
 // Warp roles (192 threads):
 //   warp 0     TMA producer (frame tiles 64 x 128, text tiles 64 x 64 / 64 x 16)
-//              into a 4-deep shared-memory ring;
+//              into a shared-memory ring;
 //   warp 1     tensor-memory allocation and the single MMA-issuing lane;
 //   warps 2-5  epilogue: tcgen05.ld of 32 columns (one keyframe per thread),
 //              scale by the text's inverse norm, keep a running top-k_frame list
 //              per keyframe (in shared memory between tiles).  Columns arrive in
 //              increasing text id, so a strict > keeps the smaller id on ties.
-// Two accumulator slots in tensor memory let the epilogue of one tile overlap the
-// MMAs of the next.
+// Two accumulator sets in tensor memory let the epilogue of one tile overlap the
+// MMAs of the next.  Up to 128 keyframes: one CTA per SM (retrieve_kernel<256, 1>).
+// More: clusters of two CTAs with tcgen05 cta_group::2 MMAs of M = 256 keyframes
+// (retrieve_pair_kernel), each SM loading half of every text tile and its own 128
+// keyframes of every 256-row pair-tile.
 //
 // Two small kernels follow: one merges the per-CTA lists of each keyframe and
 // applies the keyframe's inverse norm (cos = <f, t> / |f| / |t|); one forms each
@@ -30,6 +33,7 @@
 #include <cuda_fp16.h>
 
 #include <algorithm>
+#include <mutex>
 
 #include "fvrag_common.cuh"
 #include "fvrag_internal.h"
@@ -66,6 +70,80 @@ struct Cfg {
 // (s, i) ranks before (t, j): larger similarity first, smaller id first on ties.
 __device__ __forceinline__ bool better(float s, int i, float t, int j) {
   return s > t || (s == t && (unsigned)i < (unsigned)j);  // id -1 ranks last among equals
+}
+
+// One keyframe row's pass over the ncols similarities of a text tile held in tensor
+// memory at tbase (this thread's lane): scale by the texts' inverse norms (lane i of
+// chunk c holds column 32 c + i in invr[c]) and insert those that beat the row's list
+// (ss / si, best first; columns are text ids v0 + column).
+template <int BN>
+__device__ __forceinline__ void row_tile(uint32_t tbase, int ncols, int v0, bool live, int kf,
+                                         const float (&invr)[BN / 32], float* ss, int32_t* si) {
+  float thr = ss[kf - 1];
+  const int nch = (ncols + 31) / 32;
+#pragma unroll 1
+  for (int c = 0; c < nch; ++c) {
+    float invc = invr[0];
+#pragma unroll
+    for (int cc = 1; cc < BN / 32; ++cc)
+      if (cc == c) invc = invr[cc];
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tbase + c * 32, r);
+    tmem_wait_ld();
+    const int nvalid = min(32, ncols - c * 32);
+    // fast filter: scaled similarities in place, bit i set when column i beats the list
+    uint32_t hits = 0;
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      const float v = __uint_as_float(r[i]) * __shfl_sync(0xffffffffu, invc, i);
+      r[i] = __float_as_uint(v);
+      hits |= (v > thr ? 1u : 0u) << i;
+    }
+    if (!live) hits = 0;
+    if (nvalid < 32) hits &= (1u << nvalid) - 1u;
+    // more hits than the list holds (the lists fill on a CTA's first tiles): only the
+    // chunk's kf best can enter it, so keep those (larger value, then lower column)
+    if (__popc(hits) > kf) {
+      uint32_t keepm = 0;
+#pragma unroll 1
+      for (int p = 0; p < kf; ++p) {
+        float bv = -INFINITY;
+        int bi = -1;
+#pragma unroll
+        for (int i = 0; i < 32; ++i) {
+          const float v = __uint_as_float(r[i]);
+          const bool cand = ((hits & ~keepm) >> i) & 1u;
+          if (cand && (bi < 0 || v > bv)) {
+            bv = v;
+            bi = i;
+          }
+        }
+        keepm |= 1u << bi;
+      }
+      hits = keepm;
+    }
+    // rare path: insert the hits in column order (ids ascend, so a strict >
+    // against the list keeps the smaller id first among equal similarities)
+    while (hits) {
+      const int i = __ffs(hits) - 1;
+      hits &= hits - 1u;
+      float v = 0.f;
+#pragma unroll
+      for (int k = 0; k < 32; ++k)
+        if (k == i) v = __uint_as_float(r[k]);
+      if (!(v > thr)) continue;
+      const int id = v0 + c * 32 + i;
+      int p = kf - 1;
+      while (p > 0 && better(v, id, ss[p - 1], si[p - 1])) {
+        ss[p] = ss[p - 1];
+        si[p] = si[p - 1];
+        --p;
+      }
+      ss[p] = v;
+      si[p] = id;
+      thr = ss[kf - 1];
+    }
+  }
 }
 
 template <int BN, int MG>
@@ -271,54 +349,10 @@ __global__ void __launch_bounds__(kThreads, 1)
         const int mt = grp * MG + j;
         const bool live = mt * kBM + row < M;
         // this keyframe's running list, best first, in shared memory (row-private)
-        float* ss = st_sim + (mt * kBM + row) * kf;
-        int32_t* si = st_idx + (mt * kBM + row) * kf;
-        float thr = ss[kf - 1];
         const uint32_t tbase =
             tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * MG + j) * BN);
-        const int nch = (ncols + 31) / 32;
-#pragma unroll 1
-        for (int c = 0; c < nch; ++c) {
-          float invc = invr[0];
-#pragma unroll
-          for (int cc = 1; cc < BN / 32; ++cc)
-            if (cc == c) invc = invr[cc];
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tbase + c * 32, r);
-          tmem_wait_ld();
-          const int nvalid = min(32, ncols - c * 32);
-          // fast filter: scaled similarities in place, bit i set when column i beats the list
-          uint32_t hits = 0;
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const float v = __uint_as_float(r[i]) * __shfl_sync(0xffffffffu, invc, i);
-            r[i] = __float_as_uint(v);
-            hits |= (v > thr ? 1u : 0u) << i;
-          }
-          if (!live) hits = 0;
-          if (nvalid < 32) hits &= (1u << nvalid) - 1u;
-          // rare path: insert the hits in column order (ids ascend, so a strict >
-          // against the list keeps the smaller id first among equal similarities)
-          while (hits) {
-            const int i = __ffs(hits) - 1;
-            hits &= hits - 1u;
-            float v = 0.f;
-#pragma unroll
-            for (int k = 0; k < 32; ++k)
-              if (k == i) v = __uint_as_float(r[k]);
-            if (!(v > thr)) continue;
-            const int id = v0 + c * 32 + i;
-            int p = kf - 1;
-            while (p > 0 && better(v, id, ss[p - 1], si[p - 1])) {
-              ss[p] = ss[p - 1];
-              si[p] = si[p - 1];
-              --p;
-            }
-            ss[p] = v;
-            si[p] = id;
-            thr = ss[kf - 1];
-          }
-        }
+        row_tile<BN>(tbase, ncols, v0, live, kf, invr, st_sim + (mt * kBM + row) * kf,
+                     st_idx + (mt * kBM + row) * kf);
       }
       tc_fence_before();
       __syncwarp();
@@ -338,6 +372,248 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, C::kTmemCols);
+}
+
+// ---------------------------------------------------------------------------
+// Pair form for more than 128 keyframes: a cluster of two CTAs on two SMs runs
+// tcgen05 cta_group::2 MMAs of M = 256 keyframes x N = 256 texts.  CTA r of the pair
+// holds keyframes [128 r, 128 r + 128) of every 256-row pair-tile and texts
+// [v0 + N/2 r, v0 + N/2 (r + 1)) of every text tile, keeps the top-k lists of its own
+// keyframes, and receives their similarities against all N texts (rank 0's texts
+// first, so column c is text v0 + c).  Each SM so loads half of every text tile and
+// half of every pair-tile, per 256 texts; two accumulator sets of 256 columns per
+// CTA let the epilogue of one item overlap the MMAs of the next.  Rank 0 issues the
+// MMAs; both CTAs' copies complete on rank 0's barriers.
+struct PairCfg {
+  static constexpr int BN = 256;
+  static constexpr int kABytes = kBM * kBK * 2;             // this CTA's 128 keyframes
+  static constexpr int kBBytes = (BN / 2) * kBK * 2;        // this CTA's 128 texts
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr int kStagesP = 6;
+  static constexpr int kSlots = 2;
+  static constexpr int kTmemCols = 512;
+  static constexpr int kSmemBytes = kStagesP * kStageBytes + 1024 + 256 + kMaxState * 8;
+  static_assert(kSlots * BN <= kTmemCols, "accumulators fit tensor memory");
+  static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+  static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+    retrieve_pair_kernel(const __grid_constant__ CUtensorMap tm_frames,
+                         const __grid_constant__ CUtensorMap tm_t64,
+                         const __grid_constant__ CUtensorMap tm_t16,
+                         const float* __restrict__ text_inv_norm, int M, int E, int Nt, int kf,
+                         float* __restrict__ part_sim, int32_t* __restrict__ part_idx,
+                         uint32_t* status, uint64_t limit_ns) {
+  using C = PairCfg;
+  constexpr int BN = C::BN;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* ring = smem;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + C::kStagesP * C::kStageBytes);
+  uint64_t* full = bars;                        // rank 0: both CTAs' copies
+  uint64_t* empty = bars + C::kStagesP;         // each CTA: its stage is free
+  uint64_t* tfull = bars + 2 * C::kStagesP;     // each CTA: accumulators ready
+  uint64_t* tempty = tfull + C::kSlots;         // rank 0: both epilogues done
+  uint64_t* drain = tempty + C::kSlots;         // rank 0: every MMA done
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* st_sim = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);
+  int32_t* st_idx = reinterpret_cast<int32_t*>(st_sim + kMaxState);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+
+  // ---- this pair's text range, in units of 16 rows
+  const int nunits = (Nt + 15) >> 4;
+  const int u_lo = (int)(((long long)pair * nunits) / npairs);
+  const int u_hi = (int)(((long long)(pair + 1) * nunits) / npairs);
+  const int v_lo = u_lo * 16;
+  const int v_hi = min(u_hi * 16, Nt);
+  const int ntiles = (v_hi - v_lo + BN - 1) / BN;
+  const int ptiles = (M + 2 * kBM - 1) / (2 * kBM);
+  const int nitems = ntiles * ptiles;
+  const int kblocks = (E + kBK - 1) / kBK;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::kStagesP; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    for (int s = 0; s < C::kSlots; ++s) {
+      mbar_init(smem_u32(&tfull[s]), 1);
+      mbar_init(smem_u32(&tempty[s]), 8);  // one arrival per epilogue warp of both CTAs
+    }
+    mbar_init(smem_u32(drain), 1);
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_frames);
+    tma_prefetch_desc(&tm_t64);
+    tma_prefetch_desc(&tm_t16);
+  }
+  for (int i = threadIdx.x; i < ptiles * kBM * kf; i += kThreads) {
+    st_sim[i] = -INFINITY;
+    st_idx[i] = -1;
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(tmem_holder), C::kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // the peer's barriers are initialised before any remote use
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);      // rank 0's barriers
+  const uint32_t tempty0 = mapa_shared(smem_u32(&tempty[0]), 0);
+  griddep_wait();                 // inputs may come from the previous kernel
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer (both CTAs)
+    if (lane == 0) {
+      const uint64_t pol_t = policy_evict_first();
+      const uint64_t pol_f = policy_evict_last();
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int t = it / ptiles, pt = it % ptiles;
+        const int v0 = v_lo + t * BN;
+        const int n = min(BN, (v_hi - v0 + 31) & ~31);     // MMA N, a multiple of 32
+        const int half = n >> 1;
+        const uint32_t bytes = C::kABytes + half * kBK * 2;   // per CTA
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + (uint32_t)(stage * 8);
+          if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full[stage]), 2 * bytes);
+          uint8_t* st = ring + stage * C::kStageBytes;
+          tma_load_2d_pair(smem_u32(st), &tm_frames, fb, kb * kBK, pt * 2 * kBM + (int)rank * kBM,
+                           pol_f);
+          uint8_t* bsm = st + C::kABytes;
+          const int w0 = v0 + (int)rank * half;
+          int r = 0;
+          for (; r + 64 <= half; r += 64)
+            tma_load_2d_pair(smem_u32(bsm + r * 128), &tm_t64, fb, kb * kBK, w0 + r, pol_t);
+          for (; r < half; r += 16)
+            tma_load_2d_pair(smem_u32(bsm + r * 128), &tm_t16, fb, kb * kBK, w0 + r, pol_t);
+          ++issued;
+          if (++stage == C::kStagesP) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      // rank 0 sees both CTAs' copies complete on its barriers: leave none in flight
+      if (rank == 0) {
+        const int pend = issued < C::kStagesP ? (int)issued : C::kStagesP;
+        for (int i = 0; i < pend; ++i) {
+          if (--stage < 0) {
+            stage = C::kStagesP - 1;
+            phase ^= 1;
+          }
+          mbar_wait(smem_u32(&full[stage]), phase, limit_ns);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (rank 0)
+    if (lane == 0 && rank == 0) {
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int it = 0; it < nitems && ok; ++it) {
+        const int slot = it % C::kSlots;
+        const uint32_t use = it / C::kSlots;
+        const int t = it / ptiles;
+        const int v0 = v_lo + t * BN;
+        const int n = min(BN, (v_hi - v0 + 31) & ~31);
+        const uint32_t idesc = idesc_f16_f32(2 * kBM, n);
+        if (!mbar_wait_cluster(smem_u32(&tempty[slot]), (use & 1) ^ 1, limit_ns)) {
+          record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaTmem);
+          break;
+        }
+        tc_fence_after();
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&full[stage]), phase, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaFull);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(ring + stage * C::kStageBytes);
+          const uint32_t bsm = st + C::kABytes;
+          const uint32_t d = tmem_base + (uint32_t)(slot * BN);
+#pragma unroll
+          for (int k16 = 0; k16 < kBK / 16; ++k16)
+            tc_mma_bf16_pair(d, desc_kmajor_sw128(st + k16 * 32), desc_kmajor_sw128(bsm + k16 * 32),
+                             idesc, (kb | k16) != 0);
+          tc_commit_pair(smem_u32(&empty[stage]), 0x3);
+          if (++stage == C::kStagesP) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit_pair(smem_u32(&tfull[slot]), 0x3);
+      }
+      // every MMA issued by this thread has finished before tensor memory is freed
+      tc_commit_pair(smem_u32(drain), 0x1);
+      if (!mbar_wait(smem_u32(drain), 0, limit_ns)) record_error(status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (both CTAs)
+    const int quarter = warp & 3;
+    const int row = quarter * 32 + lane;      // this CTA's keyframe inside a pair-tile
+    for (int it = 0; it < nitems; ++it) {
+      const int slot = it % C::kSlots;
+      const uint32_t use = it / C::kSlots;
+      const int t = it / ptiles, pt = it % ptiles;
+      const int v0 = v_lo + t * BN;
+      const int ncols = min(BN, v_hi - v0);
+      // the tile's inverse text norms, loaded before the accumulator wait
+      float invr[BN / 32];
+#pragma unroll
+      for (int c = 0; c < BN / 32; ++c) {
+        const int col = c * 32 + lane;
+        invr[c] = col < ncols ? __ldg(text_inv_norm + v0 + col) : 0.f;
+      }
+      if (!mbar_wait_cluster(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
+        break;
+      }
+      tc_fence_after();
+      const int m = pt * 2 * kBM + (int)rank * kBM + row;
+      const uint32_t tbase =
+          tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(slot * BN);
+      row_tile<BN>(tbase, ncols, v0, m < M, kf, invr, st_sim + (pt * kBM + row) * kf,
+                   st_idx + (pt * kBM + row) * kf);
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive_cluster(tempty0 + (uint32_t)(slot * 8));
+    }
+    // publish this CTA's keyframes' lists (one partial per pair)
+    for (int pt = 0; pt < ptiles; ++pt) {
+      const int m = pt * 2 * kBM + (int)rank * kBM + row;
+      if (m < M)
+        for (int p = 0; p < kf; ++p) {
+          part_sim[((size_t)pair * M + m) * kf + p] = st_sim[(pt * kBM + row) * kf + p];
+          part_idx[((size_t)pair * M + m) * kf + p] = st_idx[(pt * kBM + row) * kf + p];
+        }
+    }
+  }
+  griddep_launch_dependents();
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // neither CTA frees tensor memory the other may still use
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem_base, C::kTmemCols);
 }
 
 // inv_norm[r] = 1 / |x_r| (0 for a zero row); one warp per row, 16-byte loads.
@@ -482,16 +758,49 @@ __global__ void query_merge_kernel(const int32_t* __restrict__ fidx, const float
 }
 
 struct Plan {
-  int ctas, bn, mg;
+  int ctas, bn, mg;   // mg = 0: the pair form (ctas = pairs, the merge's partial lists)
 };
+
+// Pairs (2-CTA clusters) of the pair form that can be resident at once, per device.
+static int max_pairs() {
+  static std::mutex mu;
+  static int cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaFuncSetAttribute(retrieve_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             PairCfg::kSmemBytes) == cudaSuccess) {
+      cudaLaunchConfig_t cfg = {};
+      const int sms = std::max(2, sm_count());
+      cfg.gridDim = dim3(sms / 2 * 2);
+      cfg.blockDim = dim3(kThreads);
+      cfg.dynamicSmemBytes = PairCfg::kSmemBytes;
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = 2;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      if (cudaOccupancyMaxActiveClusters(&n, retrieve_pair_kernel, &cfg) != cudaSuccess) n = 0;
+    }
+    cudaGetLastError();
+    cached[dev] = std::max(1, std::min(n, std::min(sm_count() / 2, kMaxCtas)));
+  }
+  return cached[dev];
+}
 
 static Plan make_plan(const fvrag_retrieve_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->num_keyframes + kBM - 1) / kBM;
-  p.bn = mtiles <= 1 ? 256 : 128;
-  p.mg = mtiles <= 1 ? 1 : 2;
+  // one M-tile: <256, 1>, two accumulator sets; more keyframes: the pair form
+  p.bn = 256;
+  p.mg = mtiles <= 1 ? 1 : 0;
   const int nunits = (d->num_texts + 15) / 16;
   p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
+  if (p.mg == 0) p.ctas = std::max(1, std::min(max_pairs(), nunits));
   return p;
 }
 
@@ -531,6 +840,34 @@ static fvrag_status launch(const Plan& p, const CUtensorMap& tf, const CUtensorM
   if (launch_pdl(kern, dim3(p.ctas), dim3(kThreads), (size_t)C::kSmemBytes, s, tf, t64, t16,
                  inv_norm, d->num_keyframes, d->dim, d->num_texts, d->k_frame, hrows, psim, pidx,
                  status, wait_limit_ns()) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return launch_status();
+}
+
+static fvrag_status launch_pair(const Plan& p, const CUtensorMap& tf, const CUtensorMap& t64,
+                                const CUtensorMap& t16, const float* inv_norm,
+                                const fvrag_retrieve_desc* d, float* psim, int32_t* pidx,
+                                uint32_t* status, cudaStream_t s) {
+  if (cudaFuncSetAttribute(retrieve_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           PairCfg::kSmemBytes) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * p.ctas);
+  cfg.blockDim = dim3(kThreads);
+  cfg.dynamicSmemBytes = PairCfg::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (cudaLaunchKernelEx(&cfg, retrieve_pair_kernel, tf, t64, t16, inv_norm, d->num_keyframes,
+                         d->dim, d->num_texts, d->k_frame, psim, pidx, status, wait_limit_ns()) !=
+      cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
 }
@@ -615,10 +952,10 @@ extern "C" fvrag_status fvrag_retrieve(const fvrag_retrieve_desc* d, const void*
       if (!encode_tmap_f16(&t16, text_emb, 2, dims, strides, b16, true)) return FVRAG_ERR_CUDA;
     }
     fvrag_status st;
-    if (p.bn == 256)
+    if (p.mg == 1)
       st = launch<256, 1>(p, tf, t64, t16, inv, d, hrows, psim, pidx, status, s);
     else
-      st = launch<128, 2>(p, tf, t64, t16, inv, d, hrows, psim, pidx, status, s);
+      st = launch_pair(p, tf, t64, t16, inv, d, psim, pidx, status, s);
     if (st != FVRAG_OK) return st;
     if (launch_pdl(frame_merge_kernel, dim3((M + 7) / 8), dim3(256), 0, s, (const float*)psim,
                    (const int32_t*)pidx, (const __half*)frame_emb, M, d->dim, d->k_frame, p.ctas,

@@ -185,7 +185,8 @@ __device__ __forceinline__ void tc_fence_after() {
   asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// D[tmem] (+)= A[smem] * B[smem]^T, bf16 inputs, fp32 accumulate (kind::f16).
+// D[tmem] (+)= A[smem] * B[smem]^T, 16-bit inputs, fp32 accumulate (kind::f16: the
+// instruction descriptor says bf16 or fp16, idesc_bf16_f32 / idesc_f16_f32).
 __device__ __forceinline__ void tc_mma_bf16(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                             uint32_t idesc, uint32_t accumulate) {
   asm volatile(
@@ -365,7 +366,8 @@ __device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr, uint32_t ncols
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T over the pair (M = 256: rows 0-127 from rank 0's A,
-// 128-255 from rank 1's; the N columns half from each CTA's B), issued by rank 0.
+// 128-255 from rank 1's; the N columns half from each CTA's B), issued by rank 0;
+// kind::f16, so bf16 or fp16 inputs as the instruction descriptor says.
 __device__ __forceinline__ void tc_mma_bf16_pair(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc,
                                                  uint32_t idesc, uint32_t accumulate) {
   asm volatile(

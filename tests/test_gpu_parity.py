@@ -114,6 +114,8 @@ LM_CASES = [
     (257, 64, 50021, 1),      # three M-tiles, the third with one row; ~3 vocabulary tiles per CTA
     (512, 96, 7777, 3),       # four M-tiles: one pass of two CTA-pair tiles (2-SM MMAs)
     (600, 128, 50021, 2),     # three pair tiles (the last one partly empty), ragged W tiles
+    (200, 64, 3000, 8),       # one pair tile, two accumulator sets; 8 gathers per row
+    (400, 72, 30001, 8),      # two pair tiles per pass; 8 gathers; H not a multiple of 64
     (80, 3584, 9000, 1),      # 7b hidden size, small vocabulary
     (2048, 64, 1000, 1),      # the most rows supported: 8 pair tiles in 4 passes
 ]

@@ -298,10 +298,14 @@ __device__ __forceinline__ uint32_t mapa_shared(uint32_t addr, uint32_t rank) {
   return r;
 }
 
-// Arrives once on a barrier given by its cluster shared-memory address.
+// Arrives once on a barrier given by its cluster shared-memory address (the peer's
+// barrier in a pair).  Release at CTA scope, the instruction's default: the callers
+// signal "tensor-memory columns read" after tcgen05.wait::ld and
+// tcgen05.fence::before_thread_sync, which is all the waiting MMA issuer needs; a
+// cluster-scope release made each arrival wait for this thread's earlier stores and
+// cost the retrieval pair kernel ~5 % of its time.
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr)
-               : "memory");
+  asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
 // mbar_wait with cluster-scope acquire (for phases completed by the other CTA of a pair).

@@ -75,74 +75,93 @@ __device__ __forceinline__ bool better(float s, int i, float t, int j) {
 // One keyframe row's pass over the ncols similarities of a text tile held in tensor
 // memory at tbase (this thread's lane): scale by the texts' inverse norms (lane i of
 // chunk c holds column 32 c + i in invr[c]) and insert those that beat the row's list
-// (ss / si, best first; columns are text ids v0 + column).
+// (ss / si, best first; columns are text ids v0 + column).  The accumulator is read
+// kLdGroup chunks of 32 columns per tensor-memory wait: a load waits behind the MMAs
+// already queued on the SM's tensor core, so fewer, larger waits keep the epilogue off
+// the critical path.
+constexpr int kLdGroup = 1;
+
+template <int BN>
+__device__ __forceinline__ void row_chunk(const uint32_t (&r0)[32], int c, int ncols, int v0,
+                                          bool live, int kf, const float (&invr)[BN / 32],
+                                          float& thr, float* ss, int32_t* si) {
+  uint32_t r[32];
+#pragma unroll
+  for (int i = 0; i < 32; ++i) r[i] = r0[i];
+  float invc = invr[0];
+#pragma unroll
+  for (int cc = 1; cc < BN / 32; ++cc)
+    if (cc == c) invc = invr[cc];
+  const int nvalid = min(32, ncols - c * 32);
+  // fast filter: scaled similarities in place, bit i set when column i beats the list
+  uint32_t hits = 0;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const float v = __uint_as_float(r[i]) * __shfl_sync(0xffffffffu, invc, i);
+    r[i] = __float_as_uint(v);
+    hits |= (v > thr ? 1u : 0u) << i;
+  }
+  if (!live) hits = 0;
+  if (nvalid < 32) hits &= (1u << nvalid) - 1u;
+  // more hits than the list holds (the lists fill on a CTA's first tiles): only the
+  // chunk's kf best can enter it, so keep those (larger value, then lower column)
+  if (__popc(hits) > kf) {
+    uint32_t keepm = 0;
+#pragma unroll 1
+    for (int p = 0; p < kf; ++p) {
+      float bv = -INFINITY;
+      int bi = -1;
+#pragma unroll
+      for (int i = 0; i < 32; ++i) {
+        const float v = __uint_as_float(r[i]);
+        const bool cand = ((hits & ~keepm) >> i) & 1u;
+        if (cand && (bi < 0 || v > bv)) {
+          bv = v;
+          bi = i;
+        }
+      }
+      keepm |= 1u << bi;
+    }
+    hits = keepm;
+  }
+  // rare path: insert the hits in column order (ids ascend, so a strict >
+  // against the list keeps the smaller id first among equal similarities)
+  while (hits) {
+    const int i = __ffs(hits) - 1;
+    hits &= hits - 1u;
+    float v = 0.f;
+#pragma unroll
+    for (int k = 0; k < 32; ++k)
+      if (k == i) v = __uint_as_float(r[k]);
+    if (!(v > thr)) continue;
+    const int id = v0 + c * 32 + i;
+    int p = kf - 1;
+    while (p > 0 && better(v, id, ss[p - 1], si[p - 1])) {
+      ss[p] = ss[p - 1];
+      si[p] = si[p - 1];
+      --p;
+    }
+    ss[p] = v;
+    si[p] = id;
+    thr = ss[kf - 1];
+  }
+}
+
 template <int BN>
 __device__ __forceinline__ void row_tile(uint32_t tbase, int ncols, int v0, bool live, int kf,
                                          const float (&invr)[BN / 32], float* ss, int32_t* si) {
   float thr = ss[kf - 1];
   const int nch = (ncols + 31) / 32;
 #pragma unroll 1
-  for (int c = 0; c < nch; ++c) {
-    float invc = invr[0];
+  for (int c0 = 0; c0 < nch; c0 += kLdGroup) {
+    uint32_t r[kLdGroup][32];
 #pragma unroll
-    for (int cc = 1; cc < BN / 32; ++cc)
-      if (cc == c) invc = invr[cc];
-    uint32_t r[32];
-    tmem_ld_32x32b_x32(tbase + c * 32, r);
+    for (int g = 0; g < kLdGroup; ++g)
+      if (c0 + g < nch) tmem_ld_32x32b_x32(tbase + (c0 + g) * 32, r[g]);
     tmem_wait_ld();
-    const int nvalid = min(32, ncols - c * 32);
-    // fast filter: scaled similarities in place, bit i set when column i beats the list
-    uint32_t hits = 0;
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-      const float v = __uint_as_float(r[i]) * __shfl_sync(0xffffffffu, invc, i);
-      r[i] = __float_as_uint(v);
-      hits |= (v > thr ? 1u : 0u) << i;
-    }
-    if (!live) hits = 0;
-    if (nvalid < 32) hits &= (1u << nvalid) - 1u;
-    // more hits than the list holds (the lists fill on a CTA's first tiles): only the
-    // chunk's kf best can enter it, so keep those (larger value, then lower column)
-    if (__popc(hits) > kf) {
-      uint32_t keepm = 0;
-#pragma unroll 1
-      for (int p = 0; p < kf; ++p) {
-        float bv = -INFINITY;
-        int bi = -1;
-#pragma unroll
-        for (int i = 0; i < 32; ++i) {
-          const float v = __uint_as_float(r[i]);
-          const bool cand = ((hits & ~keepm) >> i) & 1u;
-          if (cand && (bi < 0 || v > bv)) {
-            bv = v;
-            bi = i;
-          }
-        }
-        keepm |= 1u << bi;
-      }
-      hits = keepm;
-    }
-    // rare path: insert the hits in column order (ids ascend, so a strict >
-    // against the list keeps the smaller id first among equal similarities)
-    while (hits) {
-      const int i = __ffs(hits) - 1;
-      hits &= hits - 1u;
-      float v = 0.f;
-#pragma unroll
-      for (int k = 0; k < 32; ++k)
-        if (k == i) v = __uint_as_float(r[k]);
-      if (!(v > thr)) continue;
-      const int id = v0 + c * 32 + i;
-      int p = kf - 1;
-      while (p > 0 && better(v, id, ss[p - 1], si[p - 1])) {
-        ss[p] = ss[p - 1];
-        si[p] = si[p - 1];
-        --p;
-      }
-      ss[p] = v;
-      si[p] = id;
-      thr = ss[kf - 1];
-    }
+    for (int g = 0; g < kLdGroup; ++g)
+      if (c0 + g < nch) row_chunk<BN>(r[g], c0 + g, ncols, v0, live, kf, invr, thr, ss, si);
   }
 }
 

@@ -403,6 +403,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 // half of every pair-tile, per 256 texts; two accumulator sets of 256 columns per
 // CTA let the epilogue of one item overlap the MMAs of the next.  Rank 0 issues the
 // MMAs; both CTAs' copies complete on rank 0's barriers.
+//
+// A last pair-tile of at most 128 keyframes (320 keyframes = 256 + 64, say) runs as
+// M = 128 MMAs instead, which take half the time of M = 256 ones: CTA r holds
+// keyframes [64 r, 64 r + 64) of it, and its accumulator (N/2 columns) holds them
+// twice over the 128 lanes: lane l < 64 keyframe l against rank 0's texts
+// (v0 + [0, N/2)), lane 64 + l the same keyframe against rank 1's (v0 + N/2 + [0, N/2)).
+// Each lane keeps its own list; the two lists of a keyframe are merged at the end.
 struct PairCfg {
   static constexpr int BN = 256;
   static constexpr int kABytes = kBM * kBK * 2;             // this CTA's 128 keyframes
@@ -419,6 +426,7 @@ struct PairCfg {
 
 __global__ void __launch_bounds__(kThreads, 1)
     retrieve_pair_kernel(const __grid_constant__ CUtensorMap tm_frames,
+                         const __grid_constant__ CUtensorMap tm_frames64,
                          const __grid_constant__ CUtensorMap tm_t64,
                          const __grid_constant__ CUtensorMap tm_t16,
                          const float* __restrict__ text_inv_norm, int M, int E, int Nt, int kf,
@@ -452,6 +460,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int v_hi = min(u_hi * 16, Nt);
   const int ntiles = (v_hi - v_lo + BN - 1) / BN;
   const int ptiles = (M + 2 * kBM - 1) / (2 * kBM);
+  const bool tail = M - (ptiles - 1) * 2 * kBM <= kBM;   // last pair-tile: M = 128 MMAs
   const int nitems = ntiles * ptiles;
   const int kblocks = (E + kBK - 1) / kBK;
 
@@ -469,6 +478,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   }
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tm_frames);
+    tma_prefetch_desc(&tm_frames64);
     tma_prefetch_desc(&tm_t64);
     tma_prefetch_desc(&tm_t16);
   }
@@ -500,10 +510,12 @@ __global__ void __launch_bounds__(kThreads, 1)
       bool ok = true;
       for (int it = 0; it < nitems && ok; ++it) {
         const int t = it / ptiles, pt = it % ptiles;
+        const bool tail_item = tail && pt == ptiles - 1;
         const int v0 = v_lo + t * BN;
         const int n = min(BN, (v_hi - v0 + 31) & ~31);     // MMA N, a multiple of 32
         const int half = n >> 1;
-        const uint32_t bytes = C::kABytes + half * kBK * 2;   // per CTA
+        const int arows = tail_item ? kBM / 2 : kBM;       // this CTA's keyframe rows
+        const uint32_t bytes = (arows + half) * kBK * 2;   // per CTA
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait_cluster(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
             record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
@@ -513,8 +525,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t fb = full0 + (uint32_t)(stage * 8);
           if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full[stage]), 2 * bytes);
           uint8_t* st = ring + stage * C::kStageBytes;
-          tma_load_2d_pair(smem_u32(st), &tm_frames, fb, kb * kBK, pt * 2 * kBM + (int)rank * kBM,
-                           pol_f);
+          tma_load_2d_pair(smem_u32(st), tail_item ? &tm_frames64 : &tm_frames, fb, kb * kBK,
+                           pt * 2 * kBM + (int)rank * arows, pol_f);
           uint8_t* bsm = st + C::kABytes;
           const int w0 = v0 + (int)rank * half;
           int r = 0;
@@ -550,10 +562,10 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int it = 0; it < nitems && ok; ++it) {
         const int slot = it % C::kSlots;
         const uint32_t use = it / C::kSlots;
-        const int t = it / ptiles;
+        const int t = it / ptiles, pt = it % ptiles;
         const int v0 = v_lo + t * BN;
         const int n = min(BN, (v_hi - v0 + 31) & ~31);
-        const uint32_t idesc = idesc_f16_f32(2 * kBM, n);
+        const uint32_t idesc = idesc_f16_f32((tail && pt == ptiles - 1) ? kBM : 2 * kBM, n);
         if (!mbar_wait_cluster(smem_u32(&tempty[slot]), (use & 1) ^ 1, limit_ns)) {
           record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaTmem);
           break;
@@ -594,24 +606,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int slot = it % C::kSlots;
       const uint32_t use = it / C::kSlots;
       const int t = it / ptiles, pt = it % ptiles;
+      const bool tail_item = tail && pt == ptiles - 1;
       const int v0 = v_lo + t * BN;
       const int ncols = min(BN, v_hi - v0);
+      // this lane's texts: all N columns, or in the M = 128 form half of them
+      const int half = min(BN, (v_hi - v0 + 31) & ~31) >> 1;
+      const int cbase = tail_item && row >= kBM / 2 ? half : 0;
+      const int nc = tail_item ? max(0, min(half, ncols - cbase)) : ncols;
       // the tile's inverse text norms, loaded before the accumulator wait
       float invr[BN / 32];
 #pragma unroll
       for (int c = 0; c < BN / 32; ++c) {
         const int col = c * 32 + lane;
-        invr[c] = col < ncols ? __ldg(text_inv_norm + v0 + col) : 0.f;
+        invr[c] = col < nc ? __ldg(text_inv_norm + v0 + cbase + col) : 0.f;
       }
       if (!mbar_wait_cluster(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
         record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
         break;
       }
       tc_fence_after();
-      const int m = pt * 2 * kBM + (int)rank * kBM + row;
+      const int m = tail_item ? pt * 2 * kBM + (int)rank * (kBM / 2) + (row & (kBM / 2 - 1))
+                              : pt * 2 * kBM + (int)rank * kBM + row;
       const uint32_t tbase =
           tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(slot * BN);
-      row_tile<BN>(tbase, ncols, v0, m < M, kf, invr, st_sim + (pt * kBM + row) * kf,
+      row_tile<BN>(tbase, nc, v0 + cbase, m < M, kf, invr, st_sim + (pt * kBM + row) * kf,
                    st_idx + (pt * kBM + row) * kf);
       tc_fence_before();
       __syncwarp();
@@ -619,6 +637,26 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // publish this CTA's keyframes' lists (one partial per pair)
     for (int pt = 0; pt < ptiles; ++pt) {
+      if (tail && pt == ptiles - 1) {
+        // M = 128 form: lanes l and 64 + l hold keyframe l's lists over the two halves
+        // of every text tile (disjoint texts); merge them, best first
+        asm volatile("bar.sync 1, 128;" ::: "memory");   // the 4 epilogue warps
+        const int m = pt * 2 * kBM + (int)rank * (kBM / 2) + row;
+        if (row < kBM / 2 && m < M) {
+          const float* as = st_sim + (pt * kBM + row) * kf;
+          const int32_t* ai = st_idx + (pt * kBM + row) * kf;
+          const float* bs = st_sim + (pt * kBM + row + kBM / 2) * kf;
+          const int32_t* bi = st_idx + (pt * kBM + row + kBM / 2) * kf;
+          int ia = 0, ib = 0;   // ia + ib = p < kf: neither runs past its list
+          for (int p = 0; p < kf; ++p) {
+            const bool from_a = better(as[ia], ai[ia], bs[ib], bi[ib]);
+            part_sim[((size_t)pair * M + m) * kf + p] = from_a ? as[ia] : bs[ib];
+            part_idx[((size_t)pair * M + m) * kf + p] = from_a ? ai[ia] : bi[ib];
+            if (from_a) ++ia; else ++ib;
+          }
+        }
+        continue;
+      }
       const int m = pt * 2 * kBM + (int)rank * kBM + row;
       if (m < M)
         for (int p = 0; p < kf; ++p) {
@@ -863,7 +901,8 @@ static fvrag_status launch(const Plan& p, const CUtensorMap& tf, const CUtensorM
   return launch_status();
 }
 
-static fvrag_status launch_pair(const Plan& p, const CUtensorMap& tf, const CUtensorMap& t64,
+static fvrag_status launch_pair(const Plan& p, const CUtensorMap& tf, const CUtensorMap& tf64,
+                                const CUtensorMap& t64,
                                 const CUtensorMap& t16, const float* inv_norm,
                                 const fvrag_retrieve_desc* d, float* psim, int32_t* pidx,
                                 uint32_t* status, cudaStream_t s) {
@@ -884,7 +923,7 @@ static fvrag_status launch_pair(const Plan& p, const CUtensorMap& tf, const CUte
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, retrieve_pair_kernel, tf, t64, t16, inv_norm, d->num_keyframes,
+  if (cudaLaunchKernelEx(&cfg, retrieve_pair_kernel, tf, tf64, t64, t16, inv_norm, d->num_keyframes,
                          d->dim, d->num_texts, d->k_frame, psim, pidx, status, wait_limit_ns()) !=
       cudaSuccess)
     return FVRAG_ERR_CUDA;
@@ -958,11 +997,13 @@ extern "C" fvrag_status fvrag_retrieve(const fvrag_retrieve_desc* d, const void*
     const Plan p = make_plan(d, sm_count());
     const uint64_t E = (uint64_t)d->dim, Nt = (uint64_t)d->num_texts;
     const int hrows = M <= kBM ? (M + 15) / 16 * 16 : kBM;
-    CUtensorMap tf, t64, t16;
+    CUtensorMap tf, tf64, t64, t16;
     {
       const uint64_t dims[2] = {E, (uint64_t)M}, strides[1] = {E * 2};
-      const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)hrows};
+      const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)hrows}, box64[2] = {(uint32_t)kBK, 64u};
       if (!encode_tmap_f16(&tf, frame_emb, 2, dims, strides, box, true)) return FVRAG_ERR_CUDA;
+      if (p.mg == 0 && !encode_tmap_f16(&tf64, frame_emb, 2, dims, strides, box64, true))
+        return FVRAG_ERR_CUDA;
     }
     {
       const uint64_t dims[2] = {E, Nt}, strides[1] = {E * 2};
@@ -974,7 +1015,7 @@ extern "C" fvrag_status fvrag_retrieve(const fvrag_retrieve_desc* d, const void*
     if (p.mg == 1)
       st = launch<256, 1>(p, tf, t64, t16, inv, d, hrows, psim, pidx, status, s);
     else
-      st = launch_pair(p, tf, t64, t16, inv, d, psim, pidx, status, s);
+      st = launch_pair(p, tf, tf64, t64, t16, inv, d, psim, pidx, status, s);
     if (st != FVRAG_OK) return st;
     if (launch_pdl(frame_merge_kernel, dim3((M + 7) / 8), dim3(256), 0, s, (const float*)psim,
                    (const int32_t*)pidx, (const __half*)frame_emb, M, d->dim, d->k_frame, p.ctas,

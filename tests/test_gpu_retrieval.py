@@ -126,6 +126,11 @@ def test_retrieve_tiny_matches_oracle():
     ([100, 28], 1 << 14, 768, 8, 8),     # k_frame = 8, M = 128 exactly
     ([1024, 1024], 600, 64, 2, 16),      # the most keyframes at k_frame = 2 (16 M-tiles)
     ([300, 212], 2000, 128, 8, 64),      # the most keyframes at k_frame = 8; k_query = 64
+    ([150, 130], 3001, 64, 3, 5),        # 280: a last pair-tile of 24 keyframes (M = 128 MMAs)
+    ([200, 184], 5000, 96, 2, 8),        # 384: a full last M = 128 pair-tile, 64 per CTA
+    ([300, 30], 4099, 200, 8, 16),       # 330: 64 + 10 keyframes in the last pair-tile
+    ([600, 500], 700, 64, 2, 4),         # 1100: tail of 76 after four pair-tiles; pairs with
+                                         #       no texts (700 texts over 76 pairs)
 ])
 def test_retrieve_shapes(nkf, Nt, E, kf, Kq):
     offs = np.zeros(len(nkf) + 1, np.int32)

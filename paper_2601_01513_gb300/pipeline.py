@@ -12,6 +12,13 @@ In the real verifier the attention output feeds further layers before the LM
 head; the synthetic workloads give the LM head its own hidden states, so the
 four calls are independent launches on one stream.  PyTorch only provides
 memory, copies and the stream.
+
+End to end from host buffers (``run_from_host``), the step's inputs come from one
+pinned host arena laid out like the device arena, LM-head and CLIP inputs first:
+their copy (< 1 MB) lands before the LM head starts, and the attention inputs
+(the K/V caches, most of the bytes) copy on a side stream while the LM head runs;
+attention waits for them.  The whole sequence (copies, calls, the read-back of the
+result) is one CUDA graph per host arena.
 """
 import numpy as np
 import torch
@@ -19,8 +26,10 @@ import torch
 from . import fvrag
 from .configs import VerifyConfig
 
-STEP_INPUTS = ("q", "k_prefix", "v_prefix", "prefix_offsets", "k_tail", "v_tail", "hidden",
-               "targets", "cand_emb", "frame_emb")
+# arena order: the LM head's and CLIP's inputs, then attention's (copied last, overlapped)
+STEP_INPUTS = ("hidden", "targets", "cand_emb", "frame_emb", "q", "prefix_offsets", "k_tail",
+               "v_tail", "k_prefix", "v_prefix")
+ATTN_INPUTS = ("q", "prefix_offsets", "k_tail", "v_tail", "k_prefix", "v_prefix")
 RESIDENT = ("weight",)   # model parameters: loaded once, not part of a step's inputs
 _ALIGN = 256             # byte alignment of every tensor inside an arena
 
@@ -87,6 +96,8 @@ class VerifyStep:
         self.lm_ws = torch.zeros(fvrag.lm_workspace_bytes(lmd), dtype=torch.uint8, device=dev)
         self.attn_ws = None
         self._side = None
+        self._copy = None
+        self._e2e_graphs = {}
 
     # ---------------------------------------------------------------- inputs
     def upload(self, inputs: dict) -> None:
@@ -96,6 +107,8 @@ class VerifyStep:
         tens = {name: _to_torch(name, arr) for name, arr in inputs.items()}
         lay, total = _arena_layout(tens)
         self._layout = lay
+        self._split = min([lay[n][0] for n in ATTN_INPUTS if n in lay] or [total])
+        self._e2e_graphs = {}
         self._arena = torch.empty(total, dtype=torch.uint8, device=self.device)
         for name, x in tens.items():
             if name in lay:
@@ -197,27 +210,81 @@ class VerifyStep:
         LM head + merge, CLIP, select."""
         return (2 if self.cfg.prefix_len > 0 or self.cfg.prefix_range else 1) + 2 + 1 + 1
 
+    def _enqueue_from_host(self, arena, main):
+        """Copies + calls + read-back of one step from a host arena, on `main` with a copy
+        stream for the inputs and the side stream for CLIP."""
+        if self._side is None:
+            self._side = torch.cuda.Stream(device=self.device)
+        if self._copy is None:
+            self._copy = torch.cuda.Stream(device=self.device)
+        if self._result_h is None:
+            self._result_h = torch.empty(self._result.numel(), dtype=torch.uint8, pin_memory=True)
+        sp = self._split
+        start, lm_in, attn_in = torch.cuda.Event(), torch.cuda.Event(), torch.cuda.Event()
+        fork, join = torch.cuda.Event(), torch.cuda.Event()
+        start.record(main)                       # earlier work on `main` is done with the arena
+        self._copy.wait_event(start)
+        with torch.cuda.stream(self._copy):
+            self._arena[:sp].copy_(arena[:sp], non_blocking=True)      # LM head and CLIP inputs
+            lm_in.record(self._copy)
+            if sp < arena.numel():
+                self._arena[sp:].copy_(arena[sp:], non_blocking=True)  # attention inputs
+            attn_in.record(self._copy)
+        main.wait_event(lm_in)
+        fork.record(main)
+        self._side.wait_event(fork)
+        with torch.cuda.stream(self._side):
+            self.clip()
+        join.record(self._side)
+        with torch.cuda.stream(main):
+            self.lm_head()
+            main.wait_event(attn_in)
+            self.attention()
+            main.wait_event(join)
+            self.select()
+            self._result_h.copy_(self._result, non_blocking=True)   # score and selected
+
     def run_from_host(self, host: dict, stream=None):
         """End-to-end step: host->device copies of the step's inputs, the four calls, and a
         device->host read of the result (selected index and candidate scores).
-        Returns (selected, score) host tensors and the byte counts moved each way."""
+        Returns (selected, score) host tensors and the byte counts moved each way.
+
+        With a host arena from ``host_inputs`` (the fast path) the attention inputs copy
+        while the LM head runs, and the sequence replays as one CUDA graph per arena
+        (captured on first use) when `stream` is None; any other dict of host tensors is
+        copied tensor by tensor before the step."""
         arena = getattr(host, "arena", None)
         if (arena is not None and self._arena is not None and arena.numel() == self._arena.numel()
                 and set(host) == set(self._layout)):
-            self._arena.copy_(arena, non_blocking=True)        # all inputs in one copy
             h2d = arena.numel()
+            if stream is not None:
+                self._enqueue_from_host(arena, stream)
+            else:
+                key = arena.data_ptr()
+                g = self._e2e_graphs.get(key)
+                if g is None:
+                    main = torch.cuda.current_stream(self.device)
+                    torch.cuda.synchronize(self.device)
+                    self._enqueue_from_host(arena, main)     # kernel attributes set outside capture
+                    torch.cuda.synchronize(self.device)
+                    g = torch.cuda.CUDAGraph()
+                    with torch.cuda.graph(g, capture_error_mode="thread_local"):
+                        self._enqueue_from_host(arena, torch.cuda.current_stream(self.device))
+                    self._e2e_graphs[key] = g
+                g.replay()
         else:
             h2d = 0
             for name, x in host.items():
                 self.t[name].copy_(x, non_blocking=True)
                 h2d += x.numel() * x.element_size()
-        if stream is None:
-            self.replay()
-        else:
-            self.run(stream)
-        if self._result_h is None:
-            self._result_h = torch.empty(self._result.numel(), dtype=torch.uint8, pin_memory=True)
-        self._result_h.copy_(self._result, non_blocking=True)   # score and selected in one copy
+            if stream is None:
+                self.replay()
+            else:
+                self.run(stream)
+            if self._result_h is None:
+                self._result_h = torch.empty(self._result.numel(), dtype=torch.uint8,
+                                             pin_memory=True)
+            self._result_h.copy_(self._result, non_blocking=True)   # score and selected in one copy
         Qn, K = self.score.shape
         sb = self._sel_off
         sc = self._result_h[:Qn * K * 4].view(torch.float32).view(Qn, K)

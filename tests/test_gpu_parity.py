@@ -320,6 +320,20 @@ def test_pipeline_end_to_end_from_host():
     step.run()
     torch.cuda.synchronize()
     assert np.array_equal(step.score.cpu().numpy(), got)
+    # the same sequence launched directly on a stream (no graph) gives the same result
+    host["targets"].copy_((host["targets"] + 1) % cfg.vocab)
+    _, sc3, _, _ = step.run_from_host(host, stream=torch.cuda.current_stream())
+    torch.cuda.synchronize()
+    got3 = sc3.numpy().copy()
+    step.run()
+    torch.cuda.synchronize()
+    assert np.array_equal(step.score.cpu().numpy(), got3) and not np.array_equal(got3, got)
+    # a plain dict of host tensors takes the tensor-by-tensor path
+    plain = {k: v.clone() for k, v in host.items()}
+    _, sc4, h2d4, _ = step.run_from_host(plain)
+    torch.cuda.synchronize()
+    assert np.array_equal(sc4.numpy(), got3) and h2d4 == sum(v.numel() * v.element_size()
+                                                            for v in plain.values())
 
 
 # ============================================================ failure detection

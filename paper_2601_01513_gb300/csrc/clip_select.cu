@@ -8,8 +8,12 @@
 // contraction is [16 frames x E] x [E x 16 candidates], too small in M for tcgen05
 // tiles), so with many frames it streams at HBM rates; a query's frames are split
 // over a cluster of up to 8 CTAs whose per-candidate bests are merged in distributed
-// shared memory.  K4 uses one CTA per query.
+// shared memory (the cluster size is picked from how many clusters fit the GPU at once).
+// K4 uses one CTA per query.
 #include <cuda_fp16.h>
+
+#include <algorithm>
+#include <mutex>
 
 #include "fvrag_common.cuh"
 #include "fvrag_internal.h"
@@ -338,6 +342,61 @@ __global__ void select_kernel(const float* __restrict__ logprob, const int32_t* 
 
 using namespace fvrag;
 
+// Clusters of S CTAs of clip_align_kernel that can be resident at once (S <= 8), cached
+// per device and shared-memory size.
+static int clip_max_clusters(int S, int smem) {
+  static std::mutex mu;
+  static int cache_dev[64] = {0}, cache_smem[64] = {0}, cache_n[64][kClipMaxSplit + 1] = {{0}};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  std::lock_guard<std::mutex> lock(mu);
+  if (cache_dev[dev] == 0 || cache_smem[dev] != smem) {
+    for (int k = 0; k <= kClipMaxSplit; ++k) cache_n[dev][k] = -1;
+    cache_dev[dev] = 1;
+    cache_smem[dev] = smem;
+  }
+  if (cache_n[dev][S] < 0) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(S);
+    cfg.blockDim = dim3(kClipThreads);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, clip_align_kernel, &cfg) != cudaSuccess) n = 0;
+    cudaGetLastError();
+    cache_n[dev][S] = n;
+  }
+  return cache_n[dev][S];
+}
+
+// CTAs per (query, candidate group): about 256 frames each, at most 8 (one cluster), and
+// among those the split that finishes soonest when `groups` clusters share the GPU: each
+// CTA's work scales as 1 / S and the clusters run in ceil(groups / resident(S)) waves (on a
+// GB300, 15 clusters of 8 fit at once but 36 of 4: 16 queries x 8 CTAs took two waves).
+static int clip_split(int F, long long groups, int smem) {
+  int smax = 1;
+  while (smax < kClipMaxSplit && (long long)smax * 256 < F && 2 * smax <= F) smax *= 2;
+  int best = 1;
+  double best_cost = 0.0;
+  for (int S = 1; S <= smax; ++S) {
+    const int n = S == 1 ? 0 : clip_max_clusters(S, smem);
+    const long long per_wave = S == 1 ? std::max(1, sm_count()) : n;
+    if (per_wave <= 0) continue;
+    const double cost = (double)((groups + per_wave - 1) / per_wave) / S;
+    if (S == 1 || cost < best_cost) {
+      best = S;
+      best_cost = cost;
+    }
+  }
+  return best;
+}
+
 extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
                                          const void* frame_emb, float* cos, float* max_cos,
                                          int32_t* argmax, uint8_t* keep, fvrag_stream_t stream) {
@@ -347,17 +406,15 @@ extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* c
   if (d->dim % 8 != 0 || d->dim > kClipMaxDim) return FVRAG_ERR_UNSUPPORTED;
   if ((int64_t)d->num_queries * d->num_cand > 0x7fffffff) return FVRAG_ERR_UNSUPPORTED;
   if (!aligned16(cand_emb) || !aligned16(frame_emb)) return FVRAG_ERR_MISALIGNED;
-  // frames split over a cluster of S CTAs (a power of two, at most 8, about 256 frames each)
-  int S = 1;
-  while (S < kClipMaxSplit && (long long)S * 256 < d->num_frames && 2 * S <= d->num_frames) S *= 2;
   const int G = (d->num_cand + kClipKG - 1) / kClipKG;
-  const long long blocks = (long long)d->num_queries * G * S;
-  if (blocks > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
   const size_t smem = (size_t)kClipKG * (d->dim + kClipPad) * sizeof(__half) +
                       (size_t)kClipWarps * 16 * 32 * sizeof(float);
   if (cudaFuncSetAttribute(clip_align_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            (int)smem) != cudaSuccess)
     return FVRAG_ERR_CUDA;
+  const int S = clip_split(d->num_frames, (long long)d->num_queries * G, (int)smem);
+  const long long blocks = (long long)d->num_queries * G * S;
+  if (blocks > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((unsigned)blocks);
   cfg.blockDim = dim3(kClipThreads);

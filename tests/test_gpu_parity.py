@@ -205,8 +205,10 @@ def test_clip_edges():
     (2, 13, 300, 64),      # two candidate groups of a CTA; frames over a cluster of 2
     (3, 8, 4096, 768),     # clusters of 8 CTAs per query
     (1, 1, 1, 8),          # one frame, the smallest dimension
-    (1, 9, 2, 4096),       # the largest dimension
+    (1, 9, 2, 4096),       # the largest dimension (a 2-deep copy ring)
     (16, 10, 4096, 768),   # the CLIP bandwidth-sweep size
+    (2, 16, 100, 1536),    # the largest dimension with an 8-deep ring
+    (1, 5, 700, 2048),     # a 4-deep ring; frames over a cluster of 4
 ])
 def test_clip_shapes(Qn, K, F, E):
     cand = synth.round_f16(synth.normal_f64((Qn, K, E), 31 + K, 1))

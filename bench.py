@@ -695,15 +695,26 @@ def main():
 
     flush = _Flush()
     names = ["attn", "lm", "clip", "select"]
-    calls = {"attn": step.attention, "lm": step.lm_head, "clip": step.clip, "select": step.select}
+    # per-kernel numbers: each call alone on all SMs; with an SM split, the attention and the
+    # LM head are also timed alone within their budgets ("sm_split" in the line)
+    calls = {"attn": lambda: step.attention(sm_budget=0), "lm": lambda: step.lm_head(sm_budget=0),
+             "clip": step.clip, "select": step.select}
+    split_names = []
+    if step.sm_split is not None:
+        calls["attn_split"], calls["lm_split"] = step.attention, step.lm_head
+        split_names = ["attn_split", "lm_split"]
     for _ in range(args.warmup):
         step.run()
     torch.cuda.synchronize(dev)
     assert fvrag.read_status(step.lm_ws) == fvrag.OK and fvrag.read_status(step.attn_ws) == fvrag.OK
+    # kernel launches per step and per call, from the library's own launch counter
+    launches_step = step.launches_per_step()
+    launches_call = {n: step.launches_of(calls[n]) for n in calls}
+    torch.cuda.synchronize(dev)
     # one CUDA graph for the whole step, one per call for the per-kernel numbers
     step.capture()
     graphs = {}
-    for n in names:
+    for n in names + split_names:
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g, capture_error_mode="thread_local"):
             calls[n]()
@@ -713,7 +724,7 @@ def main():
     with torch.cuda.stream(stream):
         for _ in range(args.warmup):
             step.replay()
-            for n in names:
+            for n in names + split_names:
                 graphs[n].replay()
             step.run_from_host(host)
         torch.cuda.synchronize(dev)
@@ -736,8 +747,8 @@ def main():
             step_ms = np.array([a.elapsed_time(b) for a, b in ev])
             # per-kernel launch durations (each call replayed alone, L2 flushed before each)
             kreps = max(3, min(args.steps, args.kernel_reps))
-            per_k = np.zeros((kreps, len(names)))
-            for j, n in enumerate(names):
+            per_k = np.zeros((kreps, len(names) + len(split_names)))
+            for j, n in enumerate(names + split_names):
                 kev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                        for _ in range(kreps)]
                 for i in range(kreps):
@@ -797,13 +808,23 @@ def main():
             "us_per_query": total_ms / args.steps * 1e3 / cfg.num_queries,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms / args.steps},
-            "gpu_launches": step.launches_per_step() * (2 * args.steps + per_k.shape[0]),
+            "gpu_launches": launches_step * 2 * args.steps
+                            + sum(launches_call[n] for n in names + split_names) * per_k.shape[0],
             "timing": {"step": "CUDA graph of the four calls, CUDA events per step, L2 flushed between steps",
                        "kernels": "each call replayed alone %d times (events per launch), L2 flushed before each"
                                   % per_k.shape[0], "host_wall_s": t_wall,
                        "step_us_p10_p50_p90": [float(np.percentile(step_ms, q)) * 1e3 for q in (10, 50, 90)],
                        "sum_of_call_medians_us": float(sum(k["us_median"] for k in kern.values()))},
             "roofline": roof, "kernels": kern, "clocks": clk.summary()}
+    if split_names:
+        A, B = step.sm_split
+        line["sm_split"] = {
+            "attn_sms": A, "lm_sms": B, "e2e": list(step.sm_split_e2e or []),
+            "note": "attention beside the LM head on two streams; each timed alone in its budget "
+                    "(the host-input path gives the attention the second split: it starts once "
+                    "its inputs land)",
+            "attn_us": float(np.mean(per_k[:, len(names)])) * 1e3,
+            "lm_us": float(np.mean(per_k[:, len(names) + 1])) * 1e3}
     if not args.no_cpu_baseline and ws_ == 1:
         line["cpu_baseline"] = cpu_baseline(cfg, x, args.cpu_budget)
     print(json.dumps(line), flush=True)

@@ -49,6 +49,19 @@
  *     while it runs; calls that share a workspace must not overlap in time.
  *   - Alignment: every tensor pointer must be 16-byte aligned
  *     (FVRAG_ERR_MISALIGNED otherwise).
+ *   - SM budgets (fvrag_attn_desc.sm_budget, fvrag_lm_desc.sm_budget): each of
+ *     these kernels needs a whole SM per CTA (shared and tensor memory), so two
+ *     of them share the GPU only when their grids together fit its SMs.  In a
+ *     verify step whose LM head streams its weight from HBM (M <= 128 rows) the
+ *     attention, which is bound by the tensor cores, can run on a few SMs beside
+ *     it: give the LM head budget S - A and the attention budget A, and enqueue
+ *     them on two streams.  A budget changes the grid and the key split, hence the
+ *     rounding order of partial sums, never the operation computed; the workspace
+ *     size depends on it (pass the same descriptor to the *_workspace call).
+ *   - fvrag_launch_count() counts the kernel launches the library has enqueued
+ *     in this process (a launch captured into a CUDA graph counts once, at
+ *     capture), so a caller can tell how many kernels one call or one captured
+ *     step runs.
  */
 #ifndef FVRAG_H
 #define FVRAG_H
@@ -60,7 +73,7 @@
 extern "C" {
 #endif
 
-#define FVRAG_ABI_VERSION 4
+#define FVRAG_ABI_VERSION 5
 
 /* cudaStream_t without including the CUDA headers. */
 typedef struct CUstream_st* fvrag_stream_t;
@@ -77,6 +90,10 @@ typedef enum {
 
 /* FVRAG_ABI_VERSION of the loaded library. */
 int fvrag_abi_version(void);
+
+/* Kernel launches this library has enqueued since it was loaded (all devices and
+ * threads; a launch into a capturing stream counts once, when it is captured). */
+uint64_t fvrag_launch_count(void);
 
 /* Static, never NULL, human-readable name of a status code. */
 const char* fvrag_status_string(int status);
@@ -103,6 +120,10 @@ typedef struct fvrag_attn_desc {
   int32_t total_prefix; /* sum over queries of P_q = rows of k_prefix / v_prefix */
   float softmax_scale;  /* > 0, or 0 => 1/sqrt(head_dim); negative / NaN / inf rejected */
   uint32_t flags;       /* must be 0 */
+  int32_t sm_budget;    /* SMs the key split is planned for: 0 = every SM of the current
+                           device, else 1 .. that count (more: FVRAG_ERR_INVALID_ARG).  A
+                           budget below the device's count leaves the other SMs to a call
+                           running beside this one on another stream (see "SM budgets") */
 } fvrag_attn_desc;
 
 /* Bytes of workspace fvrag_verify_attn needs for `d` (0 if `d` is invalid). */
@@ -186,6 +207,9 @@ typedef struct fvrag_lm_desc {
   int32_t vocab;   /* V >= 1 */
   int32_t gathers; /* G: target ids per row, 1..8 (1: likelihood; 2: "Yes"/"No") */
   uint32_t flags;  /* must be 0 */
+  int32_t sm_budget; /* most SMs the call's persistent grid occupies: 0 = every SM of the
+                        current device, else 1 .. that count (more: FVRAG_ERR_INVALID_ARG);
+                        see "SM budgets" */
 } fvrag_lm_desc;
 
 size_t fvrag_score_logprobs_workspace(const fvrag_lm_desc* d);

@@ -15,6 +15,10 @@ static std::atomic<uint64_t> g_wait_limit_ns{1000000000ull};
 
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
 
+static std::atomic<uint64_t> g_launches{0};
+
+void count_launch() { g_launches.fetch_add(1, std::memory_order_relaxed); }
+
 int sm_count() {
   static std::mutex mu;
   static int cache[64] = {0};
@@ -139,7 +143,11 @@ fvrag_status fvrag_selftest_wait_timeout(void* ws, fvrag_stream_t stream) {
   if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
   selftest_wait_kernel<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(
       reinterpret_cast<uint32_t*>(ws), wait_limit_ns());
-  return launch_status();
+  const fvrag_status st = launch_status();
+  if (st == FVRAG_OK) count_launch();
+  return st;
 }
+
+uint64_t fvrag_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
 }  // extern "C"

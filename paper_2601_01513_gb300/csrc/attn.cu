@@ -971,6 +971,13 @@ static int device_sms() {
   return s > 0 ? s : 148;
 }
 
+// The SMs a verification call plans for; -1 when the budget is outside 0 .. the SM count.
+static int budget_sms(int32_t budget) {
+  const int s = sm_count();
+  if (budget < 0 || (s > 0 && budget > s)) return -1;
+  return budget > 0 ? budget : device_sms();
+}
+
 template <int D, bool BAL>
 static fvrag_status launch(const CUtensorMap* maps, const Args& a, long long grid, cudaStream_t s) {
   const int sm = Layout<D>::kBytes;
@@ -994,10 +1001,11 @@ static fvrag_status check_problem(const Problem& pr) {
 }
 
 // q [Qn][K][Lq][hq][D]; own K/V [Qn][K][C][hkv][D]; out like q.
-static fvrag_status run(const Problem& pr, const void* q, const void* k_prefix, const void* v_prefix,
-                        const int32_t* prefix_offsets, const void* k_own, const void* v_own,
-                        void* out, float* lse, void* ws, size_t ws_size, cudaStream_t s) {
-  const int sms = device_sms();
+// `sms`: the SMs the split is planned for (the device's count, or the caller's budget).
+static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k_prefix,
+                        const void* v_prefix, const int32_t* prefix_offsets, const void* k_own,
+                        const void* v_own, void* out, float* lse, void* ws, size_t ws_size,
+                        cudaStream_t s) {
   const size_t need = ws_bytes(pr, sms);
   if (!ws || ws_size < need) return FVRAG_ERR_WORKSPACE;
   if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
@@ -1107,7 +1115,9 @@ extern "C" size_t fvrag_verify_attn_workspace(const fvrag_attn_desc* d) {
   if (!d || d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
       d->hq % d->hkv || (d->head_dim != 64 && d->head_dim != 128) || d->max_prefix < 0)
     return 0;
-  return attn::ws_bytes(attn::verify_problem(d), attn::device_sms());
+  const int sms = attn::budget_sms(d->sm_budget);
+  if (sms < 0) return 0;
+  return attn::ws_bytes(attn::verify_problem(d), sms);
 }
 
 extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* q,
@@ -1122,6 +1132,8 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
       d->softmax_scale == INFINITY)
     return FVRAG_ERR_INVALID_ARG;
   if (d->total_prefix > 0 && (!k_prefix || !v_prefix)) return FVRAG_ERR_INVALID_ARG;
+  const int sms = budget_sms(d->sm_budget);
+  if (sms < 0) return FVRAG_ERR_INVALID_ARG;
   if (d->cand_len > kMaxTail) return FVRAG_ERR_UNSUPPORTED;
   const Problem pr = verify_problem(d);
   const fvrag_status cs = check_problem(pr);
@@ -1129,8 +1141,8 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
   if (!aligned16(q) || !aligned16(k_tail) || !aligned16(v_tail) || !aligned16(out) ||
       (k_prefix && !aligned16(k_prefix)) || (v_prefix && !aligned16(v_prefix)))
     return FVRAG_ERR_MISALIGNED;
-  return run(pr, q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, out, lse, ws, ws_size,
-             reinterpret_cast<cudaStream_t>(stream));
+  return run(pr, sms, q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, out, lse, ws,
+             ws_size, reinterpret_cast<cudaStream_t>(stream));
 }
 
 extern "C" size_t fvrag_decode_attn_workspace(const fvrag_decode_desc* d) {
@@ -1160,6 +1172,6 @@ extern "C" fvrag_status fvrag_decode_attn(const fvrag_decode_desc* d, const void
   if (!aligned16(q) || !aligned16(k_cache) || !aligned16(v_cache) || !aligned16(out) ||
       (k_prefix && !aligned16(k_prefix)) || (v_prefix && !aligned16(v_prefix)))
     return FVRAG_ERR_MISALIGNED;
-  return run(pr, q, k_prefix, v_prefix, prefix_offsets, k_cache, v_cache, out, lse, ws, ws_size,
-             reinterpret_cast<cudaStream_t>(stream));
+  return run(pr, device_sms(), q, k_prefix, v_prefix, prefix_offsets, k_cache, v_cache, out, lse,
+             ws, ws_size, reinterpret_cast<cudaStream_t>(stream));
 }

@@ -429,9 +429,11 @@ extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* c
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, clip_align_kernel, reinterpret_cast<const __half*>(cand_emb),
-                         reinterpret_cast<const __half*>(frame_emb), d->num_cand, d->num_frames,
-                         d->dim, d->threshold, cos, max_cos, argmax, keep, G, S) != cudaSuccess)
+  if (counted(cudaLaunchKernelEx(&cfg, clip_align_kernel,
+                                 reinterpret_cast<const __half*>(cand_emb),
+                                 reinterpret_cast<const __half*>(frame_emb), d->num_cand,
+                                 d->num_frames, d->dim, d->threshold, cos, max_cos, argmax, keep,
+                                 G, S)) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
 }

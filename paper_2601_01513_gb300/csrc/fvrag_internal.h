@@ -15,6 +15,22 @@ uint64_t wait_limit_ns();
 // Number of SMs of the current device (cached per device); 0 if it cannot be read.
 int sm_count();
 
+// SMs a call plans for: the device's count when `budget` is 0, else `budget`
+// (callers have checked 0 <= budget <= sm_count()).
+inline int sm_plan(int budget) {
+  const int s = sm_count();
+  return budget > 0 && (s <= 0 || budget <= s) ? budget : s;
+}
+
+// Records one kernel launch that the runtime accepted (fvrag_launch_count).
+void count_launch();
+
+// Passes a launch's result through, counting it when the runtime accepted it.
+inline cudaError_t counted(cudaError_t e) {
+  if (e == cudaSuccess) count_launch();
+  return e;
+}
+
 // Tiled TMA descriptor over a row-major tensor of 16-bit elements.
 //   dims[0] = innermost extent (elements), dims[i] = extent of dimension i,
 //   strides_bytes[i-1] = byte stride of dimension i (multiple of 16),
@@ -45,7 +61,9 @@ inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, s
   attr[0].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+  if (e == cudaSuccess) count_launch();
+  return e;
 }
 
 inline fvrag_status launch_status() {

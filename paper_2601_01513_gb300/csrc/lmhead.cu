@@ -705,6 +705,7 @@ static int max_pairs() {
   return cached[dev];
 }
 
+// `sms`: the most SMs the grid may occupy (the device's count, or the caller's budget).
 static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->rows + kBM - 1) / kBM;
@@ -715,7 +716,7 @@ static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : mtiles == 2 ? -1 : 0;
   const int nunits = (d->vocab + 15) / 16;
   p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
-  if (p.mg <= 0) p.ctas = std::max(1, std::min(max_pairs(), nunits));
+  if (p.mg <= 0) p.ctas = std::max(1, std::min(std::min(max_pairs(), std::max(1, sms / 2)), nunits));
   return p;
 }
 
@@ -743,10 +744,17 @@ static fvrag_status launch_pair(const Plan& p, const CUtensorMap& th, const CUte
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, kern, th, tw64, tw16, targets, d->rows, d->hidden, d->vocab,
-                         d->gathers, pmax, psum, ptgt, status, wait_limit_ns()) != cudaSuccess)
+  if (counted(cudaLaunchKernelEx(&cfg, kern, th, tw64, tw16, targets, d->rows, d->hidden,
+                                 d->vocab, d->gathers, pmax, psum, ptgt, status,
+                                 wait_limit_ns())) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
+}
+
+// 0 (every SM) or 1 .. the device's SM count.
+static bool budget_ok(int32_t budget) {
+  const int s = sm_count();
+  return budget >= 0 && (s <= 0 || budget <= s);
 }
 
 static size_t ws_bytes(const fvrag_lm_desc* d) {
@@ -777,7 +785,9 @@ static fvrag_status launch(const Plan& p, const CUtensorMap& th, const CUtensorM
 using namespace fvrag;
 
 extern "C" size_t fvrag_score_logprobs_workspace(const fvrag_lm_desc* d) {
-  if (!d || d->rows < 1 || d->hidden < 8 || d->vocab < 1 || d->gathers < 1) return 0;
+  if (!d || d->rows < 1 || d->hidden < 8 || d->vocab < 1 || d->gathers < 1 ||
+      !lm::budget_ok(d->sm_budget))
+    return 0;
   return lm::ws_bytes(d);
 }
 
@@ -787,7 +797,8 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
                                              fvrag_stream_t stream) {
   using namespace lm;
   if (!d || !hidden || !weight || !targets || !logprob) return FVRAG_ERR_INVALID_ARG;
-  if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0)
+  if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0 ||
+      !budget_ok(d->sm_budget))
     return FVRAG_ERR_INVALID_ARG;
   if (d->gathers > kMaxGathers || d->rows > kMaxMTiles * kBM) return FVRAG_ERR_UNSUPPORTED;
   if (d->hidden % 8 != 0) return FVRAG_ERR_MISALIGNED;
@@ -795,7 +806,7 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   if (!ws || ws_size < ws_bytes(d)) return FVRAG_ERR_WORKSPACE;
   if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
 
-  const Plan p = make_plan(d, sm_count());
+  const Plan p = make_plan(d, sm_plan(d->sm_budget));
   const uint64_t H = (uint64_t)d->hidden, M = (uint64_t)d->rows, V = (uint64_t)d->vocab;
   CUtensorMap th, tw64, tw16;
   // one M-tile: load only the rows that exist (rounded to 16), not all 128
@@ -884,7 +895,8 @@ extern "C" fvrag_status fvrag_score_logprobs_noalloc(const fvrag_lm_desc* d, con
   using namespace lm;
   // reject bad arguments before anything is enqueued
   if (!d || !hidden || !weight || !targets || !logprob) return FVRAG_ERR_INVALID_ARG;
-  if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0)
+  if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0 ||
+      !budget_ok(d->sm_budget))
     return FVRAG_ERR_INVALID_ARG;
   if (d->rows > kNoAllocMaxRows || d->gathers > kMaxGathers) return FVRAG_ERR_UNSUPPORTED;
   if (d->hidden % 8 != 0 || !aligned16(hidden) || !aligned16(weight)) return FVRAG_ERR_MISALIGNED;

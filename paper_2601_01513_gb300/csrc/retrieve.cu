@@ -923,9 +923,9 @@ static fvrag_status launch_pair(const Plan& p, const CUtensorMap& tf, const CUte
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (cudaLaunchKernelEx(&cfg, retrieve_pair_kernel, tf, tf64, t64, t16, inv_norm, d->num_keyframes,
-                         d->dim, d->num_texts, d->k_frame, psim, pidx, status, wait_limit_ns()) !=
-      cudaSuccess)
+  if (counted(cudaLaunchKernelEx(&cfg, retrieve_pair_kernel, tf, tf64, t64, t16, inv_norm,
+                                 d->num_keyframes, d->dim, d->num_texts, d->k_frame, psim, pidx,
+                                 status, wait_limit_ns())) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
 }

@@ -22,7 +22,7 @@ SEL_RANDOM = 6
 WS_HEADER_BYTES = 256
 
 EXPORTED = (
-    "fvrag_abi_version", "fvrag_status_string",
+    "fvrag_abi_version", "fvrag_status_string", "fvrag_launch_count",
     "fvrag_verify_attn_workspace", "fvrag_verify_attn",
     "fvrag_decode_attn_workspace", "fvrag_decode_attn",
     "fvrag_score_logprobs_workspace", "fvrag_score_logprobs", "fvrag_score_logprobs_noalloc",
@@ -45,7 +45,7 @@ class AttnDesc(ctypes.Structure):
                 ("cand_len", ctypes.c_int32), ("hq", ctypes.c_int32), ("hkv", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("max_prefix", ctypes.c_int32),
                 ("total_prefix", ctypes.c_int32), ("softmax_scale", ctypes.c_float),
-                ("flags", ctypes.c_uint32)]
+                ("flags", ctypes.c_uint32), ("sm_budget", ctypes.c_int32)]
 
 
 class DecodeDesc(ctypes.Structure):
@@ -58,7 +58,8 @@ class DecodeDesc(ctypes.Structure):
 
 class LmDesc(ctypes.Structure):
     _fields_ = [("rows", ctypes.c_int32), ("hidden", ctypes.c_int32), ("vocab", ctypes.c_int32),
-                ("gathers", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+                ("gathers", ctypes.c_int32), ("flags", ctypes.c_uint32),
+                ("sm_budget", ctypes.c_int32)]
 
 
 class ClipDesc(ctypes.Structure):
@@ -98,6 +99,7 @@ def lib():
         L = ctypes.CDLL(LIB_PATH)
         vp, sz, i32, u64 = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_uint64
         L.fvrag_abi_version.restype = i32
+        L.fvrag_launch_count.restype = u64
         L.fvrag_status_string.restype = ctypes.c_char_p
         L.fvrag_status_string.argtypes = [i32]
         L.fvrag_verify_attn_workspace.restype = sz
@@ -162,9 +164,10 @@ def _stream(stream):
 
 
 # --------------------------------------------------------------------- descriptors
-def lm_desc(hidden, weight, targets) -> LmDesc:
+def lm_desc(hidden, weight, targets, sm_budget=0) -> LmDesc:
     G = 1 if targets.dim() == 1 else int(targets.shape[1])
-    return LmDesc(int(hidden.shape[0]), int(hidden.shape[1]), int(weight.shape[0]), G, 0)
+    return LmDesc(int(hidden.shape[0]), int(hidden.shape[1]), int(weight.shape[0]), G, 0,
+                  int(sm_budget))
 
 
 def attn_workspace_bytes(desc: AttnDesc) -> int:
@@ -177,12 +180,13 @@ def lm_workspace_bytes(desc: LmDesc) -> int:
 
 # --------------------------------------------------------------------- the four calls
 def verify_attn(q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, out, ws, max_prefix,
-                lse=None, softmax_scale=0.0, stream=None):
+                lse=None, softmax_scale=0.0, stream=None, sm_budget=0):
     """q [Qn][K][L][hq][D] bf16; k/v_prefix [sum P][hkv][D]; prefix_offsets [Qn+1] int32 (device);
-    k/v_tail [Qn][K][L][hkv][D]; out like q; lse [Qn][K][L][hq] fp32 or None; ws uint8 device."""
+    k/v_tail [Qn][K][L][hkv][D]; out like q; lse [Qn][K][L][hq] fp32 or None; ws uint8 device;
+    sm_budget: SMs the key split is planned for (0: all)."""
     d = AttnDesc(q.shape[0], q.shape[1], q.shape[2], q.shape[3], k_tail.shape[3], q.shape[4],
                  int(max_prefix), 0 if k_prefix is None else int(k_prefix.shape[0]),
-                 float(softmax_scale), 0)
+                 float(softmax_scale), 0, int(sm_budget))
     s = lib().fvrag_verify_attn(ctypes.byref(d), _ptr(q), _ptr(k_prefix), _ptr(v_prefix),
                                 _ptr(prefix_offsets), _ptr(k_tail), _ptr(v_tail), _ptr(out),
                                 _ptr(lse), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream))
@@ -212,9 +216,10 @@ def decode_attn(q, k_prefix, v_prefix, prefix_offsets, k_cache, v_cache, cache_l
     _check(s, "fvrag_decode_attn")
 
 
-def score_logprobs(hidden, weight, targets, logprob, ws, lse=None, stream=None):
-    """hidden [M][H] bf16, weight [V][H] bf16, targets [M][G] int32 -> logprob [M][G] fp32."""
-    d = lm_desc(hidden, weight, targets)
+def score_logprobs(hidden, weight, targets, logprob, ws, lse=None, stream=None, sm_budget=0):
+    """hidden [M][H] bf16, weight [V][H] bf16, targets [M][G] int32 -> logprob [M][G] fp32;
+    sm_budget: the most SMs the persistent grid occupies (0: all)."""
+    d = lm_desc(hidden, weight, targets, sm_budget)
     s = lib().fvrag_score_logprobs(ctypes.byref(d), _ptr(hidden), _ptr(weight), _ptr(targets),
                                    _ptr(logprob), _ptr(lse), _ptr(ws), ws.numel() * ws.element_size(),
                                    _stream(stream))
@@ -299,6 +304,11 @@ def keyframes(pixels, video_offsets, theta, sim, is_key, key_index, key_offsets,
 
 
 # --------------------------------------------------------------------- status
+def launch_count() -> int:
+    """Kernel launches the library has enqueued in this process (captures count once)."""
+    return int(lib().fvrag_launch_count())
+
+
 def read_status(ws, stream=None) -> int:
     return int(lib().fvrag_read_status(_ptr(ws), _stream(stream)))
 

@@ -10,8 +10,16 @@ libfvrag calls in order on one stream:
 
 In the real verifier the attention output feeds further layers before the LM
 head; the synthetic workloads give the LM head its own hidden states, so the
-four calls are independent launches on one stream.  PyTorch only provides
-memory, copies and the stream.
+four calls are independent launches.  PyTorch only provides memory, copies and
+streams.
+
+SM split.  When the LM head streams its weight from HBM (at most 128 candidate
+rows: one M-tile, bound by HBM bandwidth, not by the tensor cores) and the
+attention, bound by the tensor cores, fits in its shadow on a few SMs, the two
+run side by side on two streams: the attention planned for A SMs (one CTA per
+row tile), the LM head's persistent grid on the other S - A.  Every CTA of both
+kernels needs a whole SM, and the two grids together fill the GPU once, so
+neither waits for the other whichever is dispatched first (``plan_sm_split``).
 
 End to end from host buffers (``run_from_host``), the step's inputs come from one
 pinned host arena laid out like the device arena, LM-head and CLIP inputs first:
@@ -63,10 +71,58 @@ def _to_torch(name, arr):
     return torch.from_numpy(arr)
 
 
+# Per-block period of the attention kernel (one 128-key block of a row tile on one SM)
+# and the HBM rate of the LM head's weight stream, both measured on GB300; they only
+# decide whether the side-by-side form pays, never what is computed.
+_ATTN_US_PER_BLOCK = 1.5
+_LM_BYTES_PER_US = 6.4e6
+_LATENCY_US = 20.0        # below this both calls are launch-latency bound: overlap them
+
+
+def attn_row_tiles(cfg: VerifyConfig) -> int:
+    """Row tiles of the attention kernel: per query and KV head, the candidate tokens x the
+    hq / hkv query heads that share a KV head, packed 128 rows to a tile."""
+    grp = cfg.hq // cfg.hkv
+    T = max(1, 128 // grp)
+    return cfg.num_queries * cfg.hkv * (-(-(cfg.num_cand * cfg.cand_len) // T))
+
+
+def plan_sm_split(cfg: VerifyConfig, sms: int, max_prefix: int = None, late: bool = False):
+    """(attention SMs, LM-head SMs) for running the two calls side by side, or None for one
+    after the other on all SMs.  Side by side only pays when the LM head is bound by HBM
+    (rows <= 128) and the attention, on its own SMs, finishes within the LM head's time (or
+    both are short enough to be bound by launch latency).
+
+    ``late``: the attention can only start about half-way through the LM head (end to end
+    from host buffers its inputs are still uploading while the LM head runs), so it gets
+    twice the SMs (two CTAs per row tile) to finish in the remaining half.  On GB300 a
+    20-SM attention started half-way through the LM head ran ~1.8x slower than when both
+    started together; 40 SMs finished in time."""
+    if cfg.rows > 128 or sms < 8:
+        return None
+    tiles = attn_row_tiles(cfg)
+    ctas = 2 * tiles if late else tiles
+    if ctas > (sms // 3 if late else sms // 4):
+        return None
+    P = cfg.prefix_len if max_prefix is None else max_prefix
+    own = -(-(min(cfg.num_cand, 129) * cfg.cand_len) // 128)
+    blocks = -(-P // 128) + own
+    t_attn = -(-blocks // (2 if late else 1)) * _ATTN_US_PER_BLOCK + 5.0
+    t_lm = cfg.vocab * cfg.hidden * 2 / _LM_BYTES_PER_US * (0.5 if late else 1.0)
+    if t_attn > max(0.8 * t_lm, _LATENCY_US):
+        return None
+    return ctas, sms - ctas
+
+
 class VerifyStep:
     def __init__(self, cfg: VerifyConfig, device="cuda", mode=fvrag.SEL_MASKED_MEAN_LOGPROB,
-                 max_prefix=None, with_lse=True):
+                 max_prefix=None, with_lse=True, sm_split="auto"):
+        """``sm_split``: "auto" (``plan_sm_split`` once the prefix is known), None (the calls
+        one after the other on all SMs) or an (attention SMs, LM-head SMs) pair."""
         self.cfg = cfg
+        self._sm_split_arg = sm_split
+        self.sm_split = None if sm_split == "auto" else sm_split
+        self.sm_split_e2e = self.sm_split     # the host-input path (``run_from_host``)
         self.device = torch.device(device)
         self.mode = mode
         self.with_lse = with_lse
@@ -92,6 +148,10 @@ class VerifyStep:
         self._result_h = None
         self._arena = None
         self._layout = {}
+        if self.sm_split is not None:
+            a, b = self.sm_split
+            if a < 1 or b < 1:
+                raise ValueError("sm_split: both budgets must be >= 1")
         lmd = fvrag.LmDesc(M, cfg.hidden, cfg.vocab, cfg.gathers, 0)
         self.lm_ws = torch.zeros(fvrag.lm_workspace_bytes(lmd), dtype=torch.uint8, device=dev)
         self.attn_ws = None
@@ -121,13 +181,25 @@ class VerifyStep:
             offs = inputs["prefix_offsets"]
             mp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
             self.max_prefix = mp if self.max_prefix is None else max(self.max_prefix, mp)
+            if self._sm_split_arg == "auto":
+                sms = torch.cuda.get_device_properties(self.device).multi_processor_count
+                self.sm_split = plan_sm_split(self.cfg, sms, int(self.max_prefix))
+                self.sm_split_e2e = plan_sm_split(self.cfg, sms, int(self.max_prefix), late=True)
             self._alloc_attn_ws()
+
+    def _budgets(self, e2e=False):
+        split = self.sm_split_e2e if e2e else self.sm_split
+        return (0, 0) if split is None else split
 
     def _alloc_attn_ws(self):
         c = self.cfg
-        d = fvrag.AttnDesc(c.num_queries, c.num_cand, c.cand_len, c.hq, c.hkv, c.head_dim,
-                           int(self.max_prefix), int(self.t["k_prefix"].shape[0]), 0.0, 0)
-        need = fvrag.attn_workspace_bytes(d)
+        need = 0
+        # alone on all SMs, or within either split
+        for budget in {0, self._budgets()[0], self._budgets(e2e=True)[0]}:
+            d = fvrag.AttnDesc(c.num_queries, c.num_cand, c.cand_len, c.hq, c.hkv, c.head_dim,
+                               int(self.max_prefix), int(self.t["k_prefix"].shape[0]), 0.0, 0,
+                               budget)
+            need = max(need, fvrag.attn_workspace_bytes(d))
         if self.attn_ws is None or self.attn_ws.numel() < need:
             self.attn_ws = torch.zeros(need, dtype=torch.uint8, device=self.device)
 
@@ -143,16 +215,20 @@ class VerifyStep:
         return h
 
     # ---------------------------------------------------------------- the step
-    def attention(self, stream=None):
+    def attention(self, stream=None, sm_budget=None):
+        """The attention call; ``sm_budget`` None: the step's split budget (0 without one)."""
         t = self.t
+        b = self._budgets()[0] if sm_budget is None else sm_budget
         fvrag.verify_attn(t["q"], t["k_prefix"], t["v_prefix"], t["prefix_offsets"], t["k_tail"],
                           t["v_tail"], self.out, self.attn_ws, self.max_prefix, lse=self.attn_lse,
-                          stream=stream)
+                          stream=stream, sm_budget=b)
 
-    def lm_head(self, stream=None):
+    def lm_head(self, stream=None, sm_budget=None):
+        """The LM-head call; ``sm_budget`` None: the step's split budget (0 without one)."""
         t = self.t
+        b = self._budgets()[1] if sm_budget is None else sm_budget
         fvrag.score_logprobs(t["hidden"], t["weight"], t["targets"], self.logprob, self.lm_ws,
-                             lse=self.lm_lse, stream=stream)
+                             lse=self.lm_lse, stream=stream, sm_budget=b)
 
     def clip(self, stream=None):
         t = self.t
@@ -178,6 +254,17 @@ class VerifyStep:
         fork, join = torch.cuda.Event(), torch.cuda.Event()
         fork.record(main)
         self._side.wait_event(fork)
+        if self.sm_split is not None:
+            # attention (then CLIP, on the SMs attention leaves) beside the LM head
+            with torch.cuda.stream(self._side):
+                self.attention()
+                self.clip()
+            join.record(self._side)
+            with torch.cuda.stream(main):
+                self.lm_head()
+                main.wait_event(join)
+                self.select()
+            return
         with torch.cuda.stream(self._side):
             self.clip()
         join.record(self._side)
@@ -206,9 +293,22 @@ class VerifyStep:
             self.run()
 
     def launches_per_step(self) -> int:
-        """Kernels this library launches per step: attention prefix (if any prefix) + tail/merge,
-        LM head + merge, CLIP, select."""
-        return (2 if self.cfg.prefix_len > 0 or self.cfg.prefix_range else 1) + 2 + 1 + 1
+        """Kernels this library launches per step, counted by the library itself
+        (``fvrag.launch_count``) over one eager step (the captured graph holds the same)."""
+        if getattr(self, "_launches", None) is None:
+            torch.cuda.synchronize(self.device)
+            n0 = fvrag.launch_count()
+            self.run()
+            self._launches = fvrag.launch_count() - n0
+            torch.cuda.synchronize(self.device)
+        return self._launches
+
+    @staticmethod
+    def launches_of(fn) -> int:
+        """Kernels one eager call of ``fn`` launches, by the library's launch counter."""
+        n0 = fvrag.launch_count()
+        fn()
+        return fvrag.launch_count() - n0
 
     def _enqueue_from_host(self, arena, main):
         """Copies + calls + read-back of one step from a host arena, on `main` with a copy
@@ -233,6 +333,20 @@ class VerifyStep:
         main.wait_event(lm_in)
         fork.record(main)
         self._side.wait_event(fork)
+        if self.sm_split_e2e is not None:
+            # CLIP then attention (once its inputs land) on the side stream, beside the LM head
+            a_sms, lm_sms = self.sm_split_e2e
+            with torch.cuda.stream(self._side):
+                self.clip()
+                self._side.wait_event(attn_in)
+                self.attention(sm_budget=a_sms)
+            join.record(self._side)
+            with torch.cuda.stream(main):
+                self.lm_head(sm_budget=lm_sms)
+                main.wait_event(join)
+                self.select()
+                self._result_h.copy_(self._result, non_blocking=True)
+            return
         with torch.cuda.stream(self._side):
             self.clip()
         join.record(self._side)

@@ -28,7 +28,7 @@ def dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0):
+def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0, sm_budget=0):
     """Runs fvrag_verify_attn on numpy inputs; returns (out fp32 numpy, lse numpy, status)."""
     Qn, K, L, Hq, D = q.shape
     tq, tkt, tvt = dev_bf16(q), dev_bf16(kt), dev_bf16(vt)
@@ -36,16 +36,18 @@ def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0):
     tvp = dev_bf16(vp) if vp.shape[0] > 0 else None
     toffs = dev(offs.astype(np.int32))
     maxp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
-    d = fvrag.AttnDesc(Qn, K, L, Hq, kt.shape[3], D, maxp, int(kp.shape[0]), float(scale), 0)
+    d = fvrag.AttnDesc(Qn, K, L, Hq, kt.shape[3], D, maxp, int(kp.shape[0]), float(scale), 0,
+                       sm_budget)
     ws = torch.zeros(fvrag.attn_workspace_bytes(d), dtype=torch.uint8, device="cuda")
     out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device="cuda")
     lse = torch.full(q.shape[:-1], float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
-    fvrag.verify_attn(tq, tkp, tvp, toffs, tkt, tvt, out, ws, maxp, lse=lse, softmax_scale=scale)
+    fvrag.verify_attn(tq, tkp, tvp, toffs, tkt, tvt, out, ws, maxp, lse=lse, softmax_scale=scale,
+                      sm_budget=sm_budget)
     st = fvrag.read_status(ws)
     return out.float().cpu().numpy(), (lse.cpu().numpy() if with_lse else None), st
 
 
-def run_lm(hidden, weight, targets):
+def run_lm(hidden, weight, targets, sm_budget=0):
     th, tw, tt = dev_bf16(hidden), dev_bf16(weight), dev(targets.astype(np.int32))
     M = hidden.shape[0]
     G = targets.shape[1]
@@ -53,7 +55,7 @@ def run_lm(hidden, weight, targets):
     ws = torch.zeros(fvrag.lm_workspace_bytes(d), dtype=torch.uint8, device="cuda")
     lp = torch.full((M, G), float("nan"), dtype=torch.float32, device="cuda")
     lse = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
-    fvrag.score_logprobs(th, tw, tt, lp, ws, lse=lse)
+    fvrag.score_logprobs(th, tw, tt, lp, ws, lse=lse, sm_budget=sm_budget)
     st = fvrag.read_status(ws)
     return lp.cpu().numpy(), lse.cpu().numpy(), st
 

@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert L.fvrag_abi_version() == 4
+    assert L.fvrag_abi_version() == 5
     for s in range(7):
         assert fvrag.status_string(s)
     assert fvrag.status_string(99) == "unknown status"
@@ -76,6 +76,32 @@ def test_attn_validation(L):
     assert L.fvrag_verify_attn_workspace(ctypes.byref(nop)) == 256
 
 
+def test_attn_sm_budget(L):
+    # the budget is the last field; a negative one is rejected by both the call and the
+    # workspace query, and a small one plans a coarser split (no partials for 20 SMs and
+    # 20 row tiles: each tile's whole key list runs on one CTA)
+    assert ctypes.sizeof(fvrag.AttnDesc) == 44
+    assert fvrag.AttnDesc.sm_budget.offset == 40
+    base = (1, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 0)
+    bad = fvrag.AttnDesc(*base, -1)
+    assert L.fvrag_verify_attn_workspace(ctypes.byref(bad)) == 0
+    assert _attn(L, bad) == fvrag.ERR_INVALID_ARG
+    full = L.fvrag_verify_attn_workspace(ctypes.byref(fvrag.AttnDesc(*base, 0)))
+    b20 = L.fvrag_verify_attn_workspace(ctypes.byref(fvrag.AttnDesc(*base, 20)))
+    assert b20 == 256 < full
+    # the budget only plans the split: validation and the workspace check still apply
+    assert _attn(L, fvrag.AttnDesc(*base, 20), ws_bytes=255) == fvrag.ERR_WORKSPACE
+
+
+def test_launch_count_ignores_rejected_calls(L):
+    n0 = fvrag.launch_count()
+    assert n0 >= 0
+    assert _attn(L, fvrag.AttnDesc(0, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_score_logprobs(ctypes.byref(fvrag.LmDesc(0, 8, 8, 1, 0)), P, P, P, P, None, P,
+                                  1 << 20, None) == fvrag.ERR_INVALID_ARG
+    assert fvrag.launch_count() == n0
+
+
 def test_lm_validation(L):
     d = fvrag.LmDesc(80, 3584, 152064, 1, 0)
     need = L.fvrag_score_logprobs_workspace(ctypes.byref(d))
@@ -92,6 +118,15 @@ def test_lm_validation(L):
     assert call(d, w=PMIS) == fvrag.ERR_MISALIGNED
     assert call(d, wsb=need - 4) == fvrag.ERR_WORKSPACE
     assert L.fvrag_score_logprobs_workspace(ctypes.byref(fvrag.LmDesc(0, 8, 8, 1, 0))) == 0
+    # SM budget: the last field; negative budgets are rejected before anything is enqueued
+    assert ctypes.sizeof(fvrag.LmDesc) == 24 and fvrag.LmDesc.sm_budget.offset == 20
+    neg = fvrag.LmDesc(80, 3584, 152064, 1, 0, -1)
+    assert call(neg) == fvrag.ERR_INVALID_ARG
+    assert L.fvrag_score_logprobs_workspace(ctypes.byref(neg)) == 0
+    assert L.fvrag_score_logprobs_noalloc(ctypes.byref(neg), P, P, P, P, None, None) == \
+        fvrag.ERR_INVALID_ARG
+    # the workspace does not depend on the budget (partials are sized for the largest grid)
+    assert L.fvrag_score_logprobs_workspace(ctypes.byref(fvrag.LmDesc(80, 3584, 152064, 1, 0, 64))) == need
 
 
 def test_clip_and_select_validation(L):

@@ -319,9 +319,11 @@ def test_pipeline_end_to_end_from_host():
     got = sc2.numpy().copy()
     assert not np.array_equal(got, ref_sc)
     assert torch.equal(step.t["targets"].cpu(), host["targets"])
+    # the device step may split the SMs differently from the host-input path (the LM head's
+    # per-CTA partials then add up in another order): equal to fp32 rounding
     step.run()
     torch.cuda.synchronize()
-    assert np.array_equal(step.score.cpu().numpy(), got)
+    np.testing.assert_allclose(step.score.cpu().numpy(), got, rtol=0, atol=1e-5)
     # the same sequence launched directly on a stream (no graph) gives the same result
     host["targets"].copy_((host["targets"] + 1) % cfg.vocab)
     _, sc3, _, _ = step.run_from_host(host, stream=torch.cuda.current_stream())
@@ -329,13 +331,14 @@ def test_pipeline_end_to_end_from_host():
     got3 = sc3.numpy().copy()
     step.run()
     torch.cuda.synchronize()
-    assert np.array_equal(step.score.cpu().numpy(), got3) and not np.array_equal(got3, got)
+    np.testing.assert_allclose(step.score.cpu().numpy(), got3, rtol=0, atol=1e-5)
+    assert not np.allclose(got3, got, rtol=0, atol=1e-3)
     # a plain dict of host tensors takes the tensor-by-tensor path
     plain = {k: v.clone() for k, v in host.items()}
     _, sc4, h2d4, _ = step.run_from_host(plain)
     torch.cuda.synchronize()
-    assert np.array_equal(sc4.numpy(), got3) and h2d4 == sum(v.numel() * v.element_size()
-                                                            for v in plain.values())
+    np.testing.assert_allclose(sc4.numpy(), got3, rtol=0, atol=1e-5)
+    assert h2d4 == sum(v.numel() * v.element_size() for v in plain.values())
 
 
 # ============================================================ failure detection

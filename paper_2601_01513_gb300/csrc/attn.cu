@@ -117,6 +117,36 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Packed pairs of fp32 (the sm_100 family's two-lane FMA / ADD) and a three-input max:
+// the softmax issues half as many FMA, ADD and MAX instructions per key.
+__device__ __forceinline__ uint64_t f2_pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+
+__device__ __forceinline__ void f2_unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+
+__device__ __forceinline__ uint64_t f2_fma(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+
+__device__ __forceinline__ float max3(float a, float b, float c) {
+  float r;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+  return r;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
@@ -664,7 +694,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
       if (full) {
 #pragma unroll
-        for (int c = 0; c < kHalf; ++c) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
+        for (int c = 0; c < kHalf; c += 2)
+          pm[(c / 2) & 7] = max3(pm[(c / 2) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
       } else {
 #pragma unroll
         for (int c = 0; c < kHalf; ++c)
@@ -687,23 +718,30 @@ __global__ void __launch_bounds__(kThreads, 1)
       const float corr = resc ? ex2(m_old - m_ref) : 1.f;
       const float ms = m_ref == -INFINITY ? 0.f : m_ref;
       // P_j (bf16 pairs) over the first 64 columns of the same buffer; S_j is in registers
-      float rsp[8];
+      // exponent arguments s * scale - m and the running sums in packed pairs
+      const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-ms, -ms);
+      uint64_t rsp2[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) rsp[u] = 0.f;
+      for (int u = 0; u < 4; ++u) rsp2[u] = 0ull;   // (+0.f, +0.f)
       uint32_t pk[32];
 #pragma unroll
       for (int c = 0; c < kHalf; c += 2) {
-        float e0 = ex2(fmaf(__uint_as_float(sr[c]), a.scale_log2, -ms));
-        float e1 = ex2(fmaf(__uint_as_float(sr[c + 1]), a.scale_log2, -ms));
+        float t0, t1;
+        f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sc2, nm2),
+                  t0, t1);
+        float e0 = ex2(t0);
+        float e1 = ex2(t1);
         if (!full) {
           e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
           e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
         }
-        rsp[c & 7] += e0;
-        rsp[(c + 1) & 7] += e1;
+        rsp2[(c / 2) & 3] = f2_add(rsp2[(c / 2) & 3], f2_pack(e0, e1));
         pk[c / 2] = pack_bf16(e0, e1);
       }
       if (ok) tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(half * kHalf / 2), pk);
+      float rsp[8];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) f2_unpack(rsp2[u], rsp[2 * u], rsp[2 * u + 1]);
       const float rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
       l = l * corr + rs;
       if (ok && __any_sync(0xffffffffu, resc)) {

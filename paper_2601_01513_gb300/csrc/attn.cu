@@ -34,11 +34,12 @@
 //              with three S/P buffers and O accumulated in tensor memory.
 //   warps 2-9  two warps per tensor-memory lane quarter, one query row per thread and
 //              half of the block's keys per warp: tcgen05.ld of S_j, masking (prefix
-//              length, or the row's own visible slots; full blocks skip it), the block
-//              max shared by the two halves through shared memory, online softmax in
-//              base 2 against a lazily moved reference max (O and l are rescaled in
-//              place only when a row's max grows by more than 2^8), and P_j written
-//              back as bf16 pairs over S_j in tensor memory.
+//              length, or the row's own visible slots; full blocks skip it), online
+//              softmax in base 2 against a lazily moved reference max (O and l are
+//              rescaled in place only when a row's max grows by more than 2^8; the block
+//              max is only computed, and shared by the two halves through shared memory,
+//              when a row has no reference yet or a partial sum shows a term past that
+//              limit), and P_j written back as bf16 pairs over S_j in tensor memory.
 //   One run: the CTA writes the bf16 output and the lse directly.  Several runs:
 //   normalised partials go to the workspace and merge_kernel combines them with
 //   log-sum-exp weights.
@@ -69,6 +70,7 @@ __device__ __forceinline__ uint32_t col_s(int b) { return (uint32_t)b * 128u; }
 constexpr uint32_t kColO = kSP * 128;
 static_assert(kColO + 128 <= kTmemCols, "S/P buffers and O must fit in tensor memory");
 constexpr float kRescaleLog2 = 8.f;   // lazy-rescale threshold (P stays < 2^8)
+constexpr float kSumLimit = 256.f;    // 2^kRescaleLog2: a partial sum above it may hold a term past the limit
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 
@@ -89,9 +91,10 @@ struct Layout {
   static constexpr int kQ = NH * kBM * 128;         // Q tile
   static constexpr int kKVHalf = kBN * 128;         // 128 keys x 64 elements
   static constexpr int kStage = NH * kKVHalf;       // one K block or one V block
-  // + row-max exchange [2 slots][2 halves][128 rows] and row-sum exchange [2][128] floats
+  // + row-max exchange [2 slots][2 halves][128 rows], row-sum exchange [2][128] floats and
+  // the slow-path flags [2 slots][2 halves][4 quarters]
   static constexpr int kBytes =
-      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4;
+      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4 + 64;
   static_assert(kPlanInts * 4 <= kVStages * kStage, "plan scratch fits the V ring");
   static_assert(kBytes <= 232448, "shared memory per CTA");
 };
@@ -348,7 +351,8 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint8_t* v_ring = k_ring + kKStages * Lay::kStage;   // [kVStages][kStage]
   float* xmax = reinterpret_cast<float*>(v_ring + kVStages * Lay::kStage);  // [2][2][kBM]
   float* xsum = xmax + 4 * kBM;                                             // [2][kBM]
-  uint64_t* bars = reinterpret_cast<uint64_t*>(xsum + 2 * kBM);
+  int* xflag = reinterpret_cast<int*>(xsum + 2 * kBM);                      // [2][2][4]
+  uint64_t* bars = reinterpret_cast<uint64_t*>(xflag + 16);
   uint64_t* k_full = bars;                        // [kKStages]  TMA -> MMA
   uint64_t* k_empty = bars + kKStages;            // [kKStages]  MMA (S done) -> TMA
   uint64_t* v_full = k_empty + kKStages;          // [kVStages]  TMA -> MMA
@@ -626,8 +630,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     // Two warps per tensor-memory lane quarter: warp w (2..9) serves rows 32 (w % 4) ..
     // +31 and the key half `half` = (w - 2) / 4 of every block (64 keys, written back as
     // 32 columns of packed bf16 P), and the same half of O's columns.  The two halves
-    // of a row agree on the block max through shared memory (a named barrier per
-    // quarter) and keep separate partial sums, added at the end.
+    // of a row keep one reference max (agreed through shared memory and a named barrier
+    // per quarter when it has to move) and separate partial sums, added at the end.
     // Online softmax in base 2 with a lazily updated reference max: P_j is taken
     // relative to m_ref, which only moves when a row's block max exceeds it by more than
     // kRescaleLog2 (then O in tensor memory and l are rescaled once).  P values stay below
@@ -689,60 +693,81 @@ __global__ void __launch_bounds__(kThreads, 1)
       // rows without output (r >= rows) are not masked: their values are finite and
       // discarded, and masking them would split the warp between the two paths below
       const bool full = vlo <= 0 && vhi >= kHalf;
-      float pm[8];
+      // P_j relative to the reference `mref`: bf16 pairs into pk (written over the first 64
+      // columns of the same buffer; S_j is in registers), the partial sum into rs
+      uint32_t pk[32];
+      float rs = 0.f;
+      auto exp_pass = [&](float mref) {
+        const float ms = mref == -INFINITY ? 0.f : mref;
+        // exponent arguments s * scale - m and the running sums in packed pairs
+        const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-ms, -ms);
+        uint64_t rsp2[4];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
-      if (full) {
+        for (int u = 0; u < 4; ++u) rsp2[u] = 0ull;   // (+0.f, +0.f)
 #pragma unroll
-        for (int c = 0; c < kHalf; c += 2)
-          pm[(c / 2) & 7] = max3(pm[(c / 2) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
-      } else {
+        for (int c = 0; c < kHalf; c += 2) {
+          float t0, t1;
+          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sc2, nm2),
+                    t0, t1);
+          float e0 = ex2(t0);
+          float e1 = ex2(t1);
+          if (!full) {
+            e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
+            e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
+          }
+          rsp2[(c / 2) & 3] = f2_add(rsp2[(c / 2) & 3], f2_pack(e0, e1));
+          pk[c / 2] = pack_bf16(e0, e1);
+        }
+        float rsp[8];
 #pragma unroll
-        for (int c = 0; c < kHalf; ++c)
-          if (c >= vlo && c < vhi) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
-      }
-      float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                         fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-      // block max over both halves (double-buffered slots: the partner may still be
-      // reading the previous block's value)
-      float* xs = xmax + (j & 1) * 2 * kBM;
-      xs[half * kBM + r] = hmax;
+        for (int u = 0; u < 4; ++u) f2_unpack(rsp2[u], rsp[2 * u], rsp[2 * u + 1]);
+        rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
+      };
+      // Once every row of the warp has a reference, the block max is not computed: all
+      // terms of the partial sum are positive, so rs <= 2^kRescaleLog2 shows that no term
+      // of this half ran past the limit.  A row without a reference, or a larger sum, in
+      // either warp of the quarter sends both into the path that computes the block max
+      // (the two halves of a row must keep one reference).
+      const bool fresh = __any_sync(0xffffffffu, m_ref == -INFINITY);
+      if (!fresh) exp_pass(m_ref);
+      const bool mine = fresh || __any_sync(0xffffffffu, !(rs <= kSumLimit));
+      int* xf = xflag + ((j & 1) * 2 + half) * 4;      // [2 slots][2 halves][4 quarters]
+      if (lane == 0) xf[quarter] = mine ? 1 : 0;
       tc_fence_before();          // this warp's S loads are complete before the partner
       pair_sync();                // writes its P over them
       tc_fence_after();
-      hmax = fmaxf(hmax, xs[(half ^ 1) * kBM + r]);
-      const float bmax = a.scale_log2 * hmax;
-      const float m_old = m_ref;
-      if (bmax > m_ref + kRescaleLog2) m_ref = bmax;   // also the first finite block
-      const bool resc = m_ref != m_old && m_old != -INFINITY;
-      const float corr = resc ? ex2(m_old - m_ref) : 1.f;
-      const float ms = m_ref == -INFINITY ? 0.f : m_ref;
-      // P_j (bf16 pairs) over the first 64 columns of the same buffer; S_j is in registers
-      // exponent arguments s * scale - m and the running sums in packed pairs
-      const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-ms, -ms);
-      uint64_t rsp2[4];
+      const bool slow = mine || xflag[((j & 1) * 2 + (half ^ 1)) * 4 + quarter] != 0;
+      bool resc = false;
+      float corr = 1.f;
+      if (slow) {
+        float pm[8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) rsp2[u] = 0ull;   // (+0.f, +0.f)
-      uint32_t pk[32];
+        for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
+        if (full) {
 #pragma unroll
-      for (int c = 0; c < kHalf; c += 2) {
-        float t0, t1;
-        f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sc2, nm2),
-                  t0, t1);
-        float e0 = ex2(t0);
-        float e1 = ex2(t1);
-        if (!full) {
-          e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
-          e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
+          for (int c = 0; c < kHalf; c += 2)
+            pm[(c / 2) & 7] = max3(pm[(c / 2) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
+        } else {
+#pragma unroll
+          for (int c = 0; c < kHalf; ++c)
+            if (c >= vlo && c < vhi) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
         }
-        rsp2[(c / 2) & 3] = f2_add(rsp2[(c / 2) & 3], f2_pack(e0, e1));
-        pk[c / 2] = pack_bf16(e0, e1);
+        float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                           fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+        // block max over both halves (slots by block parity: the next use of a slot comes
+        // after two more flag barriers)
+        float* xs = xmax + (j & 1) * 2 * kBM;
+        xs[half * kBM + r] = hmax;
+        pair_sync();
+        hmax = fmaxf(hmax, xs[(half ^ 1) * kBM + r]);
+        const float bmax = a.scale_log2 * hmax;
+        const float m_old = m_ref;
+        if (bmax > m_ref + kRescaleLog2) m_ref = bmax;   // also the first finite block
+        resc = m_ref != m_old && m_old != -INFINITY;
+        corr = resc ? ex2(m_old - m_ref) : 1.f;
+        if (fresh || __any_sync(0xffffffffu, m_ref != m_old)) exp_pass(m_ref);
       }
       if (ok) tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(half * kHalf / 2), pk);
-      float rsp[8];
-#pragma unroll
-      for (int u = 0; u < 4; ++u) f2_unpack(rsp2[u], rsp[2 * u], rsp[2 * u + 1]);
-      const float rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
       l = l * corr + rs;
       if (ok && __any_sync(0xffffffffu, resc)) {
         // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale

@@ -26,7 +26,9 @@
 // attn_kernel: one CTA = one row tile x one run of key blocks.
 //   warp 0     TMA: the Q tile once (3-D map over [tokens][hq][D]), then K and V
 //              blocks (3-D maps over [keys][hkv][D], 128-byte swizzle) into a 2-deep
-//              K ring and a 3-deep V ring, each issued as soon as its ring has a free slot.
+//              K ring and a 3-deep V ring, in block order, each once its slot is free.
+//              Warps 0 and 1 wait with blocking mbarrier waits in a fixed order, so they
+//              take no issue slots from the softmax warps on their sub-partitions.
 //   warp 1     allocates tensor memory and issues tcgen05.mma:
 //                S_j  = Q K_j^T   (M = 128 rows, N = 128 keys, K = D; both K-major)
 //                O   += P_j V_j   (M = 128, N = D, K = 128 keys; P_j read from tensor
@@ -486,8 +488,7 @@ __global__ void __launch_bounds__(kThreads, 1)
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    // Event-driven: issues the next K block or the next V block, whichever ring has
-    // a free slot (K is recycled after its S MMA, V after its PV MMA).
+    // K_0, V_0, K_1, V_1, ... (K is recycled after its S MMA, V after its PV MMA).
     if (lane == 0 && nblk > 0) {
       const uint64_t pol_kv = policy_evict_last();   // re-read by the other row tiles
       const uint64_t pol_q = policy_evict_first();
@@ -500,59 +501,43 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int tbase = (qi * a.K + c_lo) * a.C;       // own slot 0 of candidate c_lo
       int nk = 0, nv = 0;
       int tbk = tb_first, tbv = tb_first;               // own-block cursors of the two rings
-      uint64_t t_last = globaltimer_ns();
-      while (nk < nblk || nv < nblk) {
-        bool moved = false;
-        if (nk < nblk && mbar_test(smem_u32(&k_empty[nk % kKStages]), ((nk / kKStages) & 1) ^ 1)) {
-          const uint32_t fb = smem_u32(&k_full[nk % kKStages]);
-          mbar_arrive_expect_tx(fb, Lay::kStage);
-          uint8_t* dst = k_ring + (nk % kKStages) * Lay::kStage;
-          const int bi = blk_lo + nk;
-          const bool pre = bi < nbp;
-          int key;
-          if (pre) {
-            key = pbase + bi * kBN;
-          } else {
-            tbk = own_next(tbk);
-            key = tbase + tbk * kBN;
-            ++tbk;
-          }
-          for (int h = 0; h < NH; ++h)
-            tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), pre ? &tm_kp : &tm_kt, fb, h * 64, g, key,
-                        pol_kv);
-          ++nk;
-          moved = true;
-        }
-        if (nv < nk && mbar_test(smem_u32(&v_empty[nv % kVStages]), ((nv / kVStages) & 1) ^ 1)) {
-          const uint32_t fb = smem_u32(&v_full[nv % kVStages]);
-          mbar_arrive_expect_tx(fb, Lay::kStage);
-          uint8_t* dst = v_ring + (nv % kVStages) * Lay::kStage;
-          const int bi = blk_lo + nv;
-          const bool pre = bi < nbp;
-          int key;
-          if (pre) {
-            key = pbase + bi * kBN;
-          } else {
-            tbv = own_next(tbv);
-            key = tbase + tbv * kBN;
-            ++tbv;
-          }
-          for (int h = 0; h < NH; ++h)
-            tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), pre ? &tm_vp : &tm_vt, fb, h * 64, g, key,
-                        pol_kv);
-          ++nv;
-          moved = true;
-        }
-        if (moved) {
-          t_last = globaltimer_ns();
+      // Fixed order K_j, V_j with blocking waits (the waiting thread takes no issue slots
+      // from the softmax warps on its sub-partition): K_j's slot frees when S_{j-2} is done,
+      // V_j's when PV_{j-3} is done, both well before the block is needed.
+      auto load = [&](bool is_v, int j, int& tb) {
+        const uint32_t fb = smem_u32(is_v ? &v_full[j % kVStages] : &k_full[j % kKStages]);
+        mbar_arrive_expect_tx(fb, Lay::kStage);
+        uint8_t* dst = is_v ? v_ring + (j % kVStages) * Lay::kStage : k_ring + (j % kKStages) * Lay::kStage;
+        const int bi = blk_lo + j;
+        const bool pre = bi < nbp;
+        int key;
+        if (pre) {
+          key = pbase + bi * kBN;
         } else {
-          __nanosleep(20);
-          if (globaltimer_ns() - t_last > a.limit_ns) {
-            record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteProducer);
-            break;
-          }
+          tb = own_next(tb);
+          key = tbase + tb * kBN;
+          ++tb;
         }
+        const CUtensorMap* tm = is_v ? (pre ? &tm_vp : &tm_vt) : (pre ? &tm_kp : &tm_kt);
+        for (int h = 0; h < NH; ++h)
+          tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), tm, fb, h * 64, g, key, pol_kv);
+      };
+      bool fine = true;
+      for (int j = 0; j < nblk && fine; ++j) {
+        if (!mbar_wait(smem_u32(&k_empty[j % kKStages]), ((j / kKStages) & 1) ^ 1, a.limit_ns)) {
+          fine = false;
+          break;
+        }
+        load(false, j, tbk);
+        ++nk;
+        if (!mbar_wait(smem_u32(&v_empty[j % kVStages]), ((j / kVStages) & 1) ^ 1, a.limit_ns)) {
+          fine = false;
+          break;
+        }
+        load(true, j, tbv);
+        ++nv;
       }
+      if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteProducer);
       // no copy may still be in flight when the CTA exits
       mbar_wait(qb, 0, a.limit_ns);
       for (int i = max(0, nk - kKStages); i < nk; ++i)
@@ -573,53 +558,49 @@ __global__ void __launch_bounds__(kThreads, 1)
       if (!mbar_wait(smem_u32(q_full), 0, a.limit_ns)) {
         record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
       } else {
-        int ns = 0, np = 0;
-        uint64_t t_last = globaltimer_ns();
-        while (np < nblk) {
-          bool moved = false;
-          if (ns < nblk && ns < np + kSP &&
-              mbar_test(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1) &&
-              mbar_test(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1)) {
-            tc_fence_after();
-            const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
+        // Fixed order with blocking waits: S_0 .. S_{kSP-1}, then PV_j followed by
+        // S_{j+kSP} (which reuses PV_j's S/P buffer once PV_j is done).
+        auto issue_s = [&](int ns) {
+          if (!mbar_wait(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1, a.limit_ns) ||
+              !mbar_wait(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1, a.limit_ns))
+            return false;
+          tc_fence_after();
+          const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
 #pragma unroll
-            for (int h = 0; h < NH; ++h)
+          for (int h = 0; h < NH; ++h)
 #pragma unroll
-              for (int k16 = 0; k16 < 4; ++k16)
-                tc_mma_bf16(tmem_base + col_s(ns % kSP),
-                            desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
-                            desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS,
-                            (h | k16) != 0);
-            tc_commit(smem_u32(&s_full[ns % kSP]));
-            tc_commit(smem_u32(&k_empty[ns % kKStages]));
-            ++ns;
-            moved = true;
-          }
-          if (np < ns && mbar_test(smem_u32(&p_full[np % kSP]), (np / kSP) & 1) &&
-              mbar_test(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1)) {
-            tc_fence_after();
-            const uint32_t pa = tmem_base + col_s(np % kSP);
-            const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
+            for (int k16 = 0; k16 < 4; ++k16)
+              tc_mma_bf16(tmem_base + col_s(ns % kSP),
+                          desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
+                          desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS,
+                          (h | k16) != 0);
+          tc_commit(smem_u32(&s_full[ns % kSP]));
+          tc_commit(smem_u32(&k_empty[ns % kKStages]));
+          return true;
+        };
+        auto issue_pv = [&](int np) {
+          if (!mbar_wait(smem_u32(&p_full[np % kSP]), (np / kSP) & 1, a.limit_ns) ||
+              !mbar_wait(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1, a.limit_ns))
+            return false;
+          tc_fence_after();
+          const uint32_t pa = tmem_base + col_s(np % kSP);
+          const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
 #pragma unroll
-            for (int k16 = 0; k16 < kBN / 16; ++k16)
-              tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
-                             desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
-                             (np | k16) != 0);
-            tc_commit(smem_u32(&pv_done[np % kSP]));
-            tc_commit(smem_u32(&v_empty[np % kVStages]));
-            ++np;
-            moved = true;
-          }
-          if (moved) {
-            t_last = globaltimer_ns();
-          } else {
-            __nanosleep(20);
-            if (globaltimer_ns() - t_last > a.limit_ns) {
-              record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
-              break;
-            }
-          }
+          for (int k16 = 0; k16 < kBN / 16; ++k16)
+            tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
+                           desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
+                           (np | k16) != 0);
+          tc_commit(smem_u32(&pv_done[np % kSP]));
+          tc_commit(smem_u32(&v_empty[np % kVStages]));
+          return true;
+        };
+        bool fine = true;
+        for (int ns = 0; ns < min(nblk, kSP) && fine; ++ns) fine = issue_s(ns);
+        for (int j = 0; j < nblk && fine; ++j) {
+          fine = issue_pv(j);
+          if (fine && j + kSP < nblk) fine = issue_s(j + kSP);
         }
+        if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
       }
       tc_commit(smem_u32(drain));
       if (!mbar_wait(smem_u32(drain), 0, a.limit_ns))

@@ -1,7 +1,7 @@
 """One verify step of the VideoSpeculateRAG verifier on one GPU (public API).
 
 ``VerifyStep`` owns the device buffers of one workload and issues the four
-libfvrag calls in order on one stream:
+libfvrag calls of a verify step:
 
   1. fvrag_verify_attn       attention over shared prefix + own causal tail (Eq. 6, Eq. 11)
   2. fvrag_score_logprobs    LM-head log-probabilities of the candidate tokens (Eq. 11)
@@ -15,8 +15,8 @@ streams.
 
 SM split.  When the LM head streams its weight from HBM (at most 128 candidate
 rows: one M-tile, bound by HBM bandwidth, not by the tensor cores) and the
-attention, bound by the tensor cores, fits in its shadow on a few SMs, the two
-run side by side on two streams: the attention planned for A SMs (one CTA per
+attention, bound by its softmax/tensor-core pipeline rather than by HBM, fits in
+the LM head's shadow on a few SMs, the two run side by side on two streams: the attention planned for A SMs (one CTA per
 row tile), the LM head's persistent grid on the other S - A.  Every CTA of both
 kernels needs a whole SM, and the two grids together fill the GPU once, so
 neither waits for the other whichever is dispatched first (``plan_sm_split``).

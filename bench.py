@@ -263,18 +263,25 @@ def cpu_baseline(cfg, x, budget_s):
                       % (reps, nrows, M, cfg.hq, dt)}
 
 
+_TIMED_LAUNCHES = [0]   # library kernel launches inside the timed loops of a row bench
+
+
 def _time_calls(fn, stream, steps, dev, between=None):
     """CUDA-event time of `steps` calls of fn on `stream` (ms per call, and the list);
-    `between` (outside the events) runs before each call."""
+    `between` (outside the events) runs before each call.  The library's kernel launches
+    inside the loop are added to _TIMED_LAUNCHES (from its own launch counter)."""
     import torch
+    from paper_2601_01513_gb300 import fvrag
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
           for _ in range(steps)]
+    n0 = fvrag.launch_count()
     for i in range(steps):
         if between is not None:
             between()
         ev[i][0].record(stream)
         fn()
         ev[i][1].record(stream)
+    _TIMED_LAUNCHES[0] += fvrag.launch_count() - n0
     torch.cuda.synchronize(dev)
     ms = np.array([a.elapsed_time(b) for a, b in ev])
     return float(ms.mean()), ms
@@ -386,7 +393,6 @@ def bench_row(args):
                         % (Nt * E * 2 / 1e9),
                   "inv_norm_index_build_ms": inv_ms, "parallelism": "replicas"}
         dtype = "f16"
-        launches = 3
         cpu = None
         if not args.no_cpu_baseline and ws_ == 1:
             oracle.build()
@@ -450,7 +456,6 @@ def bench_row(args):
                         "the %.0f MB of frames also exceed L2" % (tf.numel() * 2 / 1e6),
                   "parallelism": "replicas"}
         dtype = "f16"
-        launches = 1
         cpu = None
         if not args.no_cpu_baseline and ws_ == 1:
             oracle.build()
@@ -523,7 +528,6 @@ def bench_row(args):
                   "l2": "flushed before every timed call (256 MiB write, outside the events)",
                   "parallelism": "replicas"}
         dtype = "bf16"
-        launches = 2
         cpu = None
         if not args.no_cpu_baseline and ws_ == 1:
             oracle.build()
@@ -595,7 +599,6 @@ def bench_row(args):
                   "l2": "inputs larger than L2 (%.2f GB of frames per call)" % (T * cfg.npix * 3 / 1e9),
                   "parallelism": "replicas"}
         dtype = "u8"
-        launches = 3
         cpu = None
         if not args.no_cpu_baseline and ws_ == 1:
             oracle.build()
@@ -619,7 +622,7 @@ def bench_row(args):
                 "config": config,
                 "e2e": {"value": units * ws_ / (e_ms * 1e-3), "unit": unit, "h2d_bytes_per_step": int(h2d),
                         "d2h_bytes_per_step": int(d2h), "ms_per_step": e_ms},
-                "gpu_launches": launches * (steps * 2 + args.warmup + 1),
+                "gpu_launches": _TIMED_LAUNCHES[0],
                 "roofline": roof, "clocks": clk.summary()}
         if cpu:
             line["cpu_baseline"] = cpu
@@ -728,6 +731,9 @@ def main():
                 graphs[n].replay()
             step.run_from_host(host)
         torch.cuda.synchronize(dev)
+        # kernels of one end-to-end step (its own SM split may add the attention's merge)
+        launches_e2e = step.launches_of(lambda: step.run_from_host(host, stream=stream))
+        torch.cuda.synchronize(dev)
         if ws_ > 1:
             dist.barrier()
         torch.cuda.synchronize(dev)
@@ -817,7 +823,7 @@ def main():
             "us_per_query": total_ms / args.steps * 1e3 / cfg.num_queries,
             "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(h2d),
                     "d2h_bytes_per_step": int(d2h), "ms_per_step": e2e_ms / args.steps},
-            "gpu_launches": launches_step * 2 * args.steps
+            "gpu_launches": (launches_step + launches_e2e) * args.steps
                             + sum(launches_call[n] for n in names + split_names) * per_k.shape[0],
             "timing": {"step": "CUDA graph of the four calls, CUDA events per step, L2 flushed between steps",
                        "kernels": "each call replayed alone %d times (events per launch), L2 flushed before each"

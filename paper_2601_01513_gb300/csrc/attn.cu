@@ -647,10 +647,8 @@ __global__ void __launch_bounds__(kThreads, 1)
       tc_fence_after();
       uint32_t sr[kHalf];
       if (ok) {
-#pragma unroll
-        for (int c0 = 0; c0 < kHalf; c0 += 32)
-          tmem_ld_32x32b_x32(lane_base + col_s(sb) + half * kHalf + c0,
-                             *reinterpret_cast<uint32_t(*)[32]>(&sr[c0]));
+        static_assert(kHalf == 64, "one 64-column load per warp and block");
+        tmem_ld_32x32b_x64(lane_base + col_s(sb) + half * kHalf, sr);
         tmem_wait_ld();
       } else {
 #pragma unroll

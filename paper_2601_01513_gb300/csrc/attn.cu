@@ -49,6 +49,7 @@
 
 #include <algorithm>
 #include <cmath>
+#include <type_traits>
 
 #include "fvrag_common.cuh"
 #include "fvrag_internal.h"
@@ -676,7 +677,9 @@ __global__ void __launch_bounds__(kThreads, 1)
       // columns of the same buffer; S_j is in registers), the partial sum into rs
       uint32_t pk[32];
       float rs = 0.f;
-      auto exp_pass = [&](float mref) {
+      // kMask: 0 = no masking, 1 = mask every element, 2 = mask when the block is not full
+      auto exp_pass_t = [&](float mref, auto mask_mode) {
+        constexpr int kMask = decltype(mask_mode)::value;
         const float ms = mref == -INFINITY ? 0.f : mref;
         // exponent arguments s * scale - m and the running sums in packed pairs
         const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-ms, -ms);
@@ -690,7 +693,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                     t0, t1);
           float e0 = ex2(t0);
           float e1 = ex2(t1);
-          if (!full) {
+          if (kMask == 1 || (kMask == 2 && !full)) {
             e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
             e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
           }
@@ -701,6 +704,21 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
         for (int u = 0; u < 4; ++u) f2_unpack(rsp2[u], rsp[2 * u], rsp[2 * u + 1]);
         rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
+      };
+      // Verification: full blocks (almost all of them) run a copy of the loop without the
+      // masking selects, which the compiler otherwise keeps in the loop as predicated
+      // instructions (long 145.9 -> 133.6 us per call).  Decode (the balanced plan), whose own
+      // blocks are mostly partial, keeps the one loop with the test inside (74.2 us
+      // unswitched against 71.7).
+      auto exp_pass = [&](float mref) {
+        if constexpr (BAL) {
+          exp_pass_t(mref, std::integral_constant<int, 2>{});
+        } else {
+          if (full)
+            exp_pass_t(mref, std::integral_constant<int, 0>{});
+          else
+            exp_pass_t(mref, std::integral_constant<int, 1>{});
+        }
       };
       // Once every row of the warp has a reference, the block max is not computed: all
       // terms of the partial sum are positive, so rs <= 2^kRescaleLog2 shows that no term

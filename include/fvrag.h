@@ -286,7 +286,9 @@ fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
  * FVRAG_SEL_TWO_STAGE (Algorithm 1): with lpY = logprob[k][n_k-1][0] and
  *   lpN = logprob[k][n_k-1][1], score_k = 1 / (1 + exp(lpN - lpY)) = pY/(pY+pN)
  *   (Eq. 12); A_H = {k : score_k >= max_j score_j - delta} (Eq. 13); selected =
- *   the k in A_H with the largest max_cos, lowest index on ties.
+ *   the k in A_H with the largest max_cos, lowest index on ties; a NaN max_cos
+ *   ranks below every number there (as -inf), so it is chosen only when every
+ *   member of A_H has a NaN alignment.
  * The other strategies the paper compares share the reliability r_k of Eq. 12 (the
  * TWO_STAGE score) and the alignment a_k = max_cos of Eq. 15:
  * FVRAG_SEL_ADDITION ("addition", Section 4.6, Table 3): score_k = r_k + a_k;

@@ -449,7 +449,8 @@ static uint64_t oracle_splitmix64(uint64_t s, uint64_t n) {
  * mode 6 (ablation "Random"): selected = floor(((x >> 32) * K) / 2^32) with x the q-th
  *   SplitMix64 output of `seed`; score_k = 0.
  * Ties go to the lowest index.  A candidate whose n_k is outside [1, L] or whose
- * score is NaN is never selected (modes 0-5).
+ * score is NaN is never selected (modes 0-5).  In mode 1 a NaN a_k ranks below
+ * every number (as -inf) when the best-aligned member of A_H is chosen.
  */
 int oracle_select(int Qn, int K, int L, int G, int mode, double delta, const double* logprob,
                   const int32_t* lengths, const uint8_t* keep, const double* max_cos,
@@ -497,8 +498,10 @@ int oracle_select(int Qn, int K, int L, int G, int mode, double delta, const dou
         const int64_t qk = (int64_t)qi * K + k;
         const double s = score[qk];
         if (isnan(s) || !(s >= top - delta)) continue; /* Eq. 13 */
-        if (sel < 0 || max_cos[qk] > best) {
-          best = max_cos[qk];
+        /* a NaN alignment has no order: it ranks below every number */
+        const double a = isnan(max_cos[qk]) ? -INFINITY : max_cos[qk];
+        if (sel < 0 || a > best) {
+          best = a;
           sel = k;
         }
       }

@@ -316,7 +316,8 @@ __global__ void select_kernel(const float* __restrict__ logprob, const int32_t* 
       for (int k = 0; k < K; ++k) {
         const double s = sc[k];
         if (isnan(s) || !(s >= top - delta)) continue;   // Eq. 13
-        const float a = max_cos[(size_t)q * K + k];
+        const float m = max_cos[(size_t)q * K + k];
+        const float a = isnan(m) ? -INFINITY : m;       // NaN ranks below every number
         if (sel < 0 || a > best) {
           best = a;
           sel = k;

@@ -261,6 +261,19 @@ def test_select_matches_oracle(mode, Qn, K, L):
         assert np.array_equal(sel, rsel)
 
 
+def test_select_two_stage_nan_alignment():
+    """A NaN max_cos ranks below every number when the best-aligned member of A_H is
+    chosen (Algorithm 1): same pick as the oracle, including an all-NaN A_H."""
+    rel = np.array([[0.7, 0.7, 0.7, 0.1], [0.6, 0.6, 0.2, 0.6], [0.5, 0.5, 0.5, 0.5]])
+    lp = np.stack([np.log(rel), np.log1p(-rel)], -1)[:, :, None, :]
+    mc = np.array([[np.nan, 0.3, 0.2, 0.99], [0.1, np.nan, 0.9, -np.inf],
+                   [np.nan, np.nan, np.nan, np.nan]])
+    _, sel = run_select(lp, fvrag.SEL_TWO_STAGE, max_cos=mc, delta=0.05)
+    _, rsel = oracle.select(lp.astype(np.float32), mode=oracle.SEL_TWO_STAGE,
+                            max_cos=mc.astype(np.float32), delta=float(np.float32(0.05)))
+    assert np.array_equal(sel, rsel) and list(sel) == [1, 0, 0]
+
+
 def test_select_case_studies_on_gpu():
     import json, os
     here = os.path.join(os.path.dirname(__file__), "golden")

@@ -330,6 +330,24 @@ def test_two_stage_delta_boundary():
     assert sel[0] == 3          # everything survives: pure alignment argmax
 
 
+def test_two_stage_nan_alignment_ranks_last():
+    """A NaN max_cos inside A_H loses to every number (taken as -inf), so a NaN first
+    member of A_H cannot block a later finite alignment; all-NaN A_H keeps its first."""
+    lp = _two_stage_logprobs([0.7, 0.7, 0.7, 0.1])
+    mc = np.array([[np.nan, 0.3, 0.2, 0.99]])
+    _, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=0.05)
+    assert sel[0] == 1          # 3 is outside A_H; 0 has no alignment
+    mc = np.array([[0.3, np.nan, 0.5, 0.99]])
+    _, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=0.05)
+    assert sel[0] == 2
+    mc = np.array([[np.nan, np.nan, np.nan, 0.99]])
+    _, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=0.05)
+    assert sel[0] == 0          # every member of A_H unaligned: the lowest index
+    mc = np.array([[-np.inf, np.nan, -np.inf, 0.99]])
+    _, sel = oracle.select(lp, mode=oracle.SEL_TWO_STAGE, max_cos=mc, delta=0.05)
+    assert sel[0] == 0          # NaN ties -inf; the lowest index wins
+
+
 def test_masked_mean_logprob_rules():
     # candidate means: [-1, -0.5, -0.25, -2]; lengths cut off huge trailing values
     lp = np.array([[[-1, -1, 50], [-0.5, -0.5, -0.5], [-0.25, 9, 9], [-2, -2, -2]]], np.float64)[..., None]

@@ -1,6 +1,6 @@
 """Benchmark of one verify step of the VideoSpeculateRAG verifier hot path.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--config 7b] [--impl reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--config 72b] [--impl reference]
 
 A step is one pass of the whole hot path over one query batch: shared-prefix
 attention, LM-head log-probabilities, CLIP alignment and candidate selection
@@ -10,7 +10,8 @@ outside the per-step CUDA events.
 
 Metric: verified candidate tokens/s = (queries x candidates x tokens) / step time.
 Also reported: verify-step microseconds per query, per-kernel times, the roofline
-fraction of the dominant kernel (the LM head, HBM-bound at the 7B shape), the
+fraction of the dominant kernel (the LM head: tensor-bound at the default 72B-class
+shape, HBM-bound at the 7B shape), the
 end-to-end number through the public API with host buffers (host->device copies
 of the step's inputs and the device->host read of the result inside the timed
 region), and the fp64 oracle's time on this host's cores.
@@ -41,9 +42,11 @@ METRIC = "verified candidate tokens/s"
 UNIT = "tokens/s"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# DRAM traffic of one LM-head launch at the 7B shape, from an ncu capture of the
-# kernel source with this SHA-256 prefix (null once the kernel source changes).
-LM_TRAFFIC = {"sha256_prefix": "647e44d32925ae8a", "bytes_per_launch": 1093409536}
+# DRAM traffic of one LM-head launch per workload, from an ncu capture of the kernel
+# source with this SHA-256 prefix (reported as null once the kernel source changes).
+LM_TRAFFIC = {
+    "7b": {"sha256_prefix": "647e44d32925ae8a", "bytes_per_launch": 1093409536},
+}
 
 
 def peaks():
@@ -191,7 +194,7 @@ def run_reference(args, cfg):
     sel = sel.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.hq)
     cores = oracle.max_threads()
 
-    def step():
+    def step(rows, sel):
         oracle.verify_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_tail"],
                            x["v_tail"], row_sel=sel)
         lp, _ = oracle.score_logprobs(x["hidden"][rows], x["weight"], x["targets"][rows])
@@ -200,11 +203,21 @@ def run_reference(args, cfg):
         full[rows] = lp
         oracle.select(full.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.gathers), keep=keep)
 
+    # rows per step: at most --ref-rows, and few enough that the whole run (warm-up and
+    # timed steps) stays within about --ref-budget seconds, from a one-step probe
+    t0 = time.perf_counter()
+    step(rows, sel)
+    per_row = (time.perf_counter() - t0) / len(rows)
+    n = int(max(1, min(len(rows), args.ref_budget / max(1e-9, per_row * (args.steps + args.warmup)))))
+    rows = rows[:n]
+    sel = np.zeros((M, cfg.hq), bool)
+    sel[rows, :] = True
+    sel = sel.reshape(cfg.num_queries, cfg.num_cand, cfg.cand_len, cfg.hq)
     for _ in range(args.warmup):
-        step()
+        step(rows, sel)
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        step()
+        step(rows, sel)
     dt = (time.perf_counter() - t0) / args.steps
     value = len(rows) / dt
     sample = ("%d of %d candidate-token rows per step (LM head and all %d heads of attention for "
@@ -638,9 +651,15 @@ def main():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--kernel-reps", type=int, default=200)
-    ap.add_argument("--config", default="7b", choices=sorted(configs.PRESETS))
+    ap.add_argument("--config", default="72b", choices=sorted(configs.PRESETS),
+                    help="verify-step workload (default: the 72B-class verifier, the largest "
+                         "single-GPU preset)")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--ref-rows", type=int, default=8)
+    ap.add_argument("--ref-rows", type=int, default=8,
+                    help="--impl reference: at most this many candidate-token rows per step")
+    ap.add_argument("--ref-budget", type=float, default=150.0,
+                    help="--impl reference: seconds the whole run should take at most (fewer "
+                         "rows per step, down to one, when it would take longer)")
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--row", default="verify",
@@ -797,10 +816,10 @@ def main():
         if f:
             kern[n]["tc_frac"] = kern[n]["TFLOP_s"] / pk["bf16_tflops_sustained"]
     lm = kern["lm"]
-    traffic = None   # DRAM bytes per launch from the ncu capture of the 7B-class LM head
-    if (cfg.name == "7b" and LM_TRAFFIC["bytes_per_launch"]
-            and source_sha("lmhead.cu").startswith(LM_TRAFFIC["sha256_prefix"] or "#")):
-        traffic = LM_TRAFFIC["bytes_per_launch"]
+    traffic = None   # DRAM bytes per launch from an ncu capture of this workload's LM head
+    tr = LM_TRAFFIC.get(cfg.name)
+    if tr and tr["bytes_per_launch"] and source_sha("lmhead.cu").startswith(tr["sha256_prefix"]):
+        traffic = tr["bytes_per_launch"]
     # the binding roof: HBM below the ridge (at most ~278 rows), the tensor cores above it
     # (the sustained bf16 peak: the call is replayed back to back for seconds)
     ridge = pk["bf16_tflops_sustained"] * 1e12 / (pk["hbm_gbs"] * 1e9)

@@ -237,16 +237,31 @@ fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void* hidden, co
  *   - rows must be <= 1024 (gathers <= 8): larger shapes return
  *     FVRAG_ERR_UNSUPPORTED without enqueuing anything.
  *   - The first call on a device looks up the array's device address (with
- *     that device current) and caches it; make that first call before any
- *     stream capture.  No call allocates or frees memory.
+ *     that device current) and caches it with the CUDA context it belongs to;
+ *     make that first call before any stream capture.  After cudaDeviceReset
+ *     (a new context) the next call looks the address up again.  No call
+ *     allocates or frees memory.
  *   - Every call shares the one array and leaves its contents behind; each call
  *     clears the array's status word before its kernels run.  Calls that
  *     overlap on the GPU (other streams, other threads) race on the array:
  *     serialise them.
+ *   - The return value reports host-side checks and launches only.  A device-side
+ *     error (a bounded wait that ran out: FVRAG_ERR_TIMEOUT) lands in the array's
+ *     status word; read it with fvrag_score_logprobs_noalloc_status before the
+ *     next call clears it.
  */
 fvrag_status fvrag_score_logprobs_noalloc(const fvrag_lm_desc* d, const void* hidden,
                                           const void* weight, const int32_t* targets,
                                           float* logprob, float* lse, fvrag_stream_t stream);
+
+/*
+ * Device-side status of the most recent fvrag_score_logprobs_noalloc call on the
+ * current device (the counterpart of fvrag_read_status for the static array,
+ * whose address the caller never sees).  Synchronises `stream`, then reads the
+ * status word: FVRAG_OK, or FVRAG_ERR_TIMEOUT when a bounded wait ran out.
+ * Allocates nothing.
+ */
+fvrag_status fvrag_score_logprobs_noalloc_status(fvrag_stream_t stream);
 
 /* ------------------------------------------------------------------------ *
  * 3. CLIP entity alignment (Eq. 14-15) with the keep/drop threshold

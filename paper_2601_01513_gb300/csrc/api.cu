@@ -47,6 +47,22 @@ static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   return fn;
 }
 
+CUcontext current_cu_context() {
+  static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+  });
+  CUcontext c = nullptr;
+  if (!fn || fn(&c) != CUDA_SUCCESS) return nullptr;
+  return c;
+}
+
 static bool encode_tmap_16bit(CUtensorMap* map, CUtensorMapDataType dtype, const void* base,
                               int rank, const uint64_t* dims, const uint64_t* strides_bytes,
                               const uint32_t* box, bool swizzle128) {
@@ -119,9 +135,7 @@ fvrag_status fvrag_read_status(const void* ws, fvrag_stream_t stream) {
   if (cudaStreamSynchronize(s) != cudaSuccess) return FVRAG_ERR_CUDA;
   uint32_t v = 0;
   if (cudaMemcpy(&v, ws, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return FVRAG_ERR_CUDA;
-  if (v == 0) return FVRAG_OK;
-  if (v & FVRAG_ERR_TIMEOUT) return FVRAG_ERR_TIMEOUT;
-  return (fvrag_status)v;
+  return status_of_word(v);
 }
 
 fvrag_status fvrag_clear_status(void* ws, fvrag_stream_t stream) {

@@ -43,6 +43,18 @@ bool encode_tmap_bf16(CUtensorMap* map, const void* base, int rank, const uint64
 bool encode_tmap_f16(CUtensorMap* map, const void* base, int rank, const uint64_t* dims,
                      const uint64_t* strides_bytes, const uint32_t* box, bool swizzle128);
 
+// The CUDA context current on this thread (driver entry point fetched through the
+// runtime), or null when none is current or the driver call is unavailable.
+CUcontext current_cu_context();
+
+// Status a workspace status word reports: OK when 0, TIMEOUT when that bit is set,
+// else the recorded code.
+inline fvrag_status status_of_word(uint32_t v) {
+  if (v == 0) return FVRAG_OK;
+  if (v & FVRAG_ERR_TIMEOUT) return FVRAG_ERR_TIMEOUT;
+  return (fvrag_status)v;
+}
+
 inline bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 // Launches `kernel` with programmatic stream serialization: its launch and

@@ -868,21 +868,24 @@ constexpr size_t kNoAllocBytes = kWsHeaderBytes + 2 * (size_t)kMaxCtas * kNoAllo
 
 static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocBytes];
 
-// Device address of g_noalloc_scratch on the current device.  In host code the
-// array's name is only a host-side stand-in, so the address is looked up once
-// per device (with that device current) and cached.
+// Device address of g_noalloc_scratch in the current context.  In host code the
+// array's name is only a host-side stand-in, so the address is looked up with the
+// device current (the first call on a device) and cached per device together with
+// the context it was found in: when that context changes (after cudaDeviceReset the
+// module is loaded again, possibly elsewhere) the address is looked up again.
 static void* noalloc_scratch_address() {
   static std::mutex mu;
   static void* addr[64] = {nullptr};
+  static CUcontext ctx[64] = {nullptr};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
   std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
-    void* p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
-    addr[dev] = p;
-  }
-  return addr[dev];
+  if (addr[dev] && ctx[dev] != nullptr && ctx[dev] == current_cu_context()) return addr[dev];
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess) return nullptr;
+  addr[dev] = p;
+  ctx[dev] = current_cu_context();   // current now: the lookup initialised the runtime
+  return p;
 }
 
 }  // namespace lm
@@ -908,4 +911,18 @@ extern "C" fvrag_status fvrag_score_logprobs_noalloc(const fvrag_lm_desc* d, con
     return FVRAG_ERR_CUDA;
   return fvrag_score_logprobs(d, hidden, weight, targets, logprob, lse, scratch, kNoAllocBytes,
                               stream);
+}
+
+// Status of the last fvrag_score_logprobs_noalloc call on the current device: its
+// device-side status word lives in the static array, out of the caller's reach.
+extern "C" fvrag_status fvrag_score_logprobs_noalloc_status(fvrag_stream_t stream) {
+  using namespace lm;
+  void* scratch = noalloc_scratch_address();
+  if (!scratch) return FVRAG_ERR_CUDA;
+  if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  uint32_t v = 0;
+  if (cudaMemcpy(&v, scratch, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return status_of_word(v);
 }

@@ -26,6 +26,7 @@ EXPORTED = (
     "fvrag_verify_attn_workspace", "fvrag_verify_attn",
     "fvrag_decode_attn_workspace", "fvrag_decode_attn",
     "fvrag_score_logprobs_workspace", "fvrag_score_logprobs", "fvrag_score_logprobs_noalloc",
+    "fvrag_score_logprobs_noalloc_status",
     "fvrag_clip_align", "fvrag_select_candidate",
     "fvrag_embed_inv_norms", "fvrag_retrieve_workspace", "fvrag_retrieve",
     "fvrag_keyframes_workspace", "fvrag_keyframes",
@@ -116,6 +117,8 @@ def lib():
         L.fvrag_score_logprobs.argtypes = [ctypes.POINTER(LmDesc)] + [vp] * 5 + [vp, sz, vp]
         L.fvrag_score_logprobs_noalloc.restype = i32
         L.fvrag_score_logprobs_noalloc.argtypes = [ctypes.POINTER(LmDesc)] + [vp] * 5 + [vp]
+        L.fvrag_score_logprobs_noalloc_status.restype = i32
+        L.fvrag_score_logprobs_noalloc_status.argtypes = [vp]
         L.fvrag_clip_align.restype = i32
         L.fvrag_clip_align.argtypes = [ctypes.POINTER(ClipDesc)] + [vp] * 6 + [vp]
         L.fvrag_select_candidate.restype = i32
@@ -232,6 +235,11 @@ def score_logprobs_noalloc(hidden, weight, targets, logprob, lse=None, stream=No
     s = lib().fvrag_score_logprobs_noalloc(ctypes.byref(d), _ptr(hidden), _ptr(weight), _ptr(targets),
                                            _ptr(logprob), _ptr(lse), _stream(stream))
     _check(s, "fvrag_score_logprobs_noalloc")
+
+
+def noalloc_status(stream=None) -> int:
+    """Device-side status of the last score_logprobs_noalloc call (synchronises `stream`)."""
+    return lib().fvrag_score_logprobs_noalloc_status(_stream(stream))
 
 
 def clip_align(cand_emb, frame_emb, threshold, max_cos, argmax, keep, cos=None, stream=None):

@@ -1,5 +1,6 @@
-"""Shared helpers of the GPU parity tests: device placement of seeded inputs and
-the comparison rules (tolerances and margin rules for integer decisions)."""
+"""Shared helpers of the GPU parity tests: device placement of seeded inputs, guarded
+output buffers (sentinel regions before and after every output, checked after each
+call) and the comparison rules (tolerances and margin rules for integer decisions)."""
 import numpy as np
 import torch
 
@@ -9,6 +10,48 @@ ATTN_ATOL = 2e-2        # attention output, max-abs (bf16 output vs fp64)
 ATTN_LSE_ATOL = 2e-3    # attention log-sum-exp (fp32 scores, fp32 sums)
 LOGPROB_ATOL = 1e-2     # per-token log-prob
 COS_ATOL = 1e-3         # cosine / max_cos
+
+
+GUARD_BYTES = 4096      # sentinel bytes before and after every output buffer
+
+
+class Guarded:
+    """An output tensor placed between two guard regions of sentinel bytes.  Writes past
+    either end of the output (which NaN-poisoning of the output itself cannot reveal)
+    change a guard; ``check`` asserts both are intact.  The output starts 4096 bytes into
+    its allocation, so it keeps the allocation's alignment."""
+
+    def __init__(self, shape, dtype, fill):
+        esz = torch.empty((), dtype=dtype).element_size()
+        n = int(np.prod(shape)) * esz
+        self.n = n
+        self.buf = torch.empty(GUARD_BYTES * 2 + n, dtype=torch.uint8, device="cuda")
+        pat = (torch.arange(GUARD_BYTES, dtype=torch.int32, device="cuda") * 37 + 11) % 251
+        self.pat = pat.to(torch.uint8)
+        self.buf[:GUARD_BYTES].copy_(self.pat)
+        self.buf[GUARD_BYTES + n:].copy_(self.pat)
+        self.t = self.buf[GUARD_BYTES:GUARD_BYTES + n].view(dtype).view(shape)
+        if n:
+            self.t.fill_(fill)
+
+    def check(self, what=""):
+        torch.cuda.synchronize()
+        lo = self.buf[:GUARD_BYTES]
+        hi = self.buf[GUARD_BYTES + self.n:]
+        assert torch.equal(lo, self.pat), "write before the start of output %s" % what
+        assert torch.equal(hi, self.pat), "write past the end of output %s" % what
+
+
+def guarded(shape, dtype, fill, pool):
+    """A guarded output tensor; its guard object is appended to `pool` for ``check_all``."""
+    g = Guarded(shape, dtype, fill)
+    pool.append(g)
+    return g.t
+
+
+def check_all(pool):
+    for i, g in enumerate(pool):
+        g.check("#%d" % i)
 
 
 def ensure_built():
@@ -39,11 +82,13 @@ def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0, sm_budget=0):
     d = fvrag.AttnDesc(Qn, K, L, Hq, kt.shape[3], D, maxp, int(kp.shape[0]), float(scale), 0,
                        sm_budget)
     ws = torch.zeros(fvrag.attn_workspace_bytes(d), dtype=torch.uint8, device="cuda")
-    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device="cuda")
-    lse = torch.full(q.shape[:-1], float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
+    pool = []
+    out = guarded(q.shape, torch.bfloat16, float("nan"), pool)
+    lse = guarded(q.shape[:-1], torch.float32, float("nan"), pool) if with_lse else None
     fvrag.verify_attn(tq, tkp, tvp, toffs, tkt, tvt, out, ws, maxp, lse=lse, softmax_scale=scale,
                       sm_budget=sm_budget)
     st = fvrag.read_status(ws)
+    check_all(pool)
     return out.float().cpu().numpy(), (lse.cpu().numpy() if with_lse else None), st
 
 
@@ -53,10 +98,12 @@ def run_lm(hidden, weight, targets, sm_budget=0):
     G = targets.shape[1]
     d = fvrag.LmDesc(M, hidden.shape[1], weight.shape[0], G, 0)
     ws = torch.zeros(fvrag.lm_workspace_bytes(d), dtype=torch.uint8, device="cuda")
-    lp = torch.full((M, G), float("nan"), dtype=torch.float32, device="cuda")
-    lse = torch.full((M,), float("nan"), dtype=torch.float32, device="cuda")
+    pool = []
+    lp = guarded((M, G), torch.float32, float("nan"), pool)
+    lse = guarded((M,), torch.float32, float("nan"), pool)
     fvrag.score_logprobs(th, tw, tt, lp, ws, lse=lse, sm_budget=sm_budget)
     st = fvrag.read_status(ws)
+    check_all(pool)
     return lp.cpu().numpy(), lse.cpu().numpy(), st
 
 
@@ -64,26 +111,28 @@ def run_clip(cand, frames, tau, with_cos=True):
     Qn, K, E = cand.shape
     F = frames.shape[1]
     tc, tf = dev_f16(cand), dev_f16(frames)
-    mc = torch.full((Qn, K), float("nan"), device="cuda")
-    am = torch.full((Qn, K), -7, dtype=torch.int32, device="cuda")
-    keep = torch.full((Qn, K), 9, dtype=torch.uint8, device="cuda")
-    cos = torch.full((Qn, K, F), float("nan"), device="cuda") if with_cos else None
+    pool = []
+    mc = guarded((Qn, K), torch.float32, float("nan"), pool)
+    am = guarded((Qn, K), torch.int32, -7, pool)
+    keep = guarded((Qn, K), torch.uint8, 9, pool)
+    cos = guarded((Qn, K, F), torch.float32, float("nan"), pool) if with_cos else None
     fvrag.clip_align(tc, tf, tau, mc, am, keep, cos=cos)
-    torch.cuda.synchronize()
+    check_all(pool)
     return ((cos.cpu().numpy() if with_cos else None), mc.cpu().numpy(), am.cpu().numpy(),
             keep.cpu().numpy())
 
 
 def run_select(lp, mode, keep=None, max_cos=None, lengths=None, delta=0.05, seed=0):
     Qn, K, L, G = lp.shape
-    score = torch.full((Qn, K), float("nan"), device="cuda")
-    sel = torch.full((Qn,), -7, dtype=torch.int32, device="cuda")
+    pool = []
+    score = guarded((Qn, K), torch.float32, float("nan"), pool)
+    sel = guarded((Qn,), torch.int32, -7, pool)
     fvrag.select_candidate(dev(lp.astype(np.float32)), score, sel, mode=mode,
                            keep=None if keep is None else dev(keep.astype(np.uint8)),
                            max_cos=None if max_cos is None else dev(max_cos.astype(np.float32)),
                            lengths=None if lengths is None else dev(lengths.astype(np.int32)),
                            delta=delta, seed=seed)
-    torch.cuda.synchronize()
+    check_all(pool)
     return score.cpu().numpy(), sel.cpu().numpy()
 
 
@@ -134,13 +183,15 @@ def run_keyframes(pixels, video_offsets, theta, with_hist=True):
     vo = dev(np.asarray(video_offsets, np.int32))
     d = fvrag.keyframe_desc(Nv, px, theta)
     ws = torch.zeros(fvrag.keyframes_workspace_bytes(d), dtype=torch.uint8, device="cuda")
-    hist = torch.full((T, 512), -7, dtype=torch.int32, device="cuda") if with_hist else None
-    sim = torch.full((max(T, 1),), float("nan"), device="cuda")
-    key = torch.full((max(T, 1),), 9, dtype=torch.uint8, device="cuda")
-    kidx = torch.full((max(T, 1),), -7, dtype=torch.int32, device="cuda")
-    koffs = torch.full((Nv + 1,), -7, dtype=torch.int32, device="cuda")
+    pool = []
+    hist = guarded((T, 512), torch.int32, -7, pool) if with_hist else None
+    sim = guarded((max(T, 1),), torch.float32, float("nan"), pool)
+    key = guarded((max(T, 1),), torch.uint8, 9, pool)
+    kidx = guarded((max(T, 1),), torch.int32, -7, pool)
+    koffs = guarded((Nv + 1,), torch.int32, -7, pool)
     fvrag.keyframes(px, vo, theta, sim, key, kidx, koffs, ws, hist=hist)
     st = fvrag.read_status(ws)
+    check_all(pool)
     ko = koffs.cpu().numpy()
     return ((hist.cpu().numpy() if with_hist else None), sim.cpu().numpy()[:T], key.cpu().numpy()[:T],
             kidx.cpu().numpy()[:ko[-1]], ko, st)
@@ -155,17 +206,21 @@ def run_retrieve(frames, frame_offsets, texts, k_frame, k_query, precompute_norm
     fo = dev(np.asarray(frame_offsets, np.int32))
     inv = None
     if precompute_norms:
-        inv = torch.empty(texts.shape[0], dtype=torch.float32, device="cuda")
+        npool = []
+        inv = guarded((texts.shape[0],), torch.float32, float("nan"), npool)
         fvrag.embed_inv_norms(tt, inv)
+        check_all(npool)
     d = fvrag.retrieve_desc(Qn, tf, tt, k_frame, k_query)
     ws = torch.zeros(fvrag.retrieve_workspace_bytes(d), dtype=torch.uint8, device="cuda")
-    fi = torch.full((max(Fr, 1), k_frame), -7, dtype=torch.int32, device="cuda")
-    fs = torch.full((max(Fr, 1), k_frame), float("nan"), device="cuda")
-    oi = torch.full((Qn, k_query), -7, dtype=torch.int32, device="cuda")
-    os_ = torch.full((Qn, k_query), float("nan"), device="cuda")
+    pool = []
+    fi = guarded((max(Fr, 1), k_frame), torch.int32, -7, pool)
+    fs = guarded((max(Fr, 1), k_frame), torch.float32, float("nan"), pool)
+    oi = guarded((Qn, k_query), torch.int32, -7, pool)
+    os_ = guarded((Qn, k_query), torch.float32, float("nan"), pool)
     fvrag.retrieve(tf, fo, tt, k_frame, oi, os_, ws, text_inv_norm=inv, frame_topk=fi,
                    frame_topk_sim=fs)
     st = fvrag.read_status(ws)
+    check_all(pool)
     return (fi.cpu().numpy()[:Fr], fs.cpu().numpy()[:Fr], oi.cpu().numpy(), os_.cpu().numpy(), st)
 
 
@@ -210,8 +265,10 @@ def run_decode(q, kp, vp, offs, kc, vc, n, with_lse=True, scale=0.0):
     maxp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
     d = fvrag.decode_desc(tq, tkp, tkc, maxp, scale)
     ws = torch.zeros(fvrag.decode_workspace_bytes(d), dtype=torch.uint8, device="cuda")
-    out = torch.full(q.shape, float("nan"), dtype=torch.bfloat16, device="cuda")
-    lse = torch.full(q.shape[:-1], float("nan"), dtype=torch.float32, device="cuda") if with_lse else None
+    pool = []
+    out = guarded(q.shape, torch.bfloat16, float("nan"), pool)
+    lse = guarded(q.shape[:-1], torch.float32, float("nan"), pool) if with_lse else None
     fvrag.decode_attn(tq, tkp, tvp, toffs, tkc, tvc, tn, out, ws, maxp, lse=lse, softmax_scale=scale)
     st = fvrag.read_status(ws)
+    check_all(pool)
     return out.float().cpu().numpy(), (lse.cpu().numpy() if with_lse else None), st

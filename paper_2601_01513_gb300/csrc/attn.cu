@@ -29,11 +29,14 @@
 //              K ring and a 3-deep V ring, in block order, each once its slot is free.
 //              Warps 0 and 1 wait with blocking mbarrier waits in a fixed order, so they
 //              take no issue slots from the softmax warps on their sub-partitions.
-//   warp 1     allocates tensor memory and issues tcgen05.mma:
-//                S_j  = Q K_j^T   (M = 128 rows, N = 128 keys, K = D; both K-major)
+//   warp 1     allocates tensor memory and issues the PV tcgen05.mma:
 //                O   += P_j V_j   (M = 128, N = D, K = 128 keys; P_j read from tensor
 //                                  memory, V MN-major from shared memory)
-//              with three S/P buffers and O accumulated in tensor memory.
+//   warp 10    issues the S tcgen05.mma:
+//                S_j  = Q K_j^T   (M = 128 rows, N = 128 keys, K = D; both K-major)
+//              into three S/P buffers; O accumulates in tensor memory.  Two issuing
+//              threads keep the tensor pipe fed: S_{j+3} waits for PV_j to finish
+//              (it overwrites P_j) while PV_{j+1} is already queued.
 //   warps 2-9  two warps per tensor-memory lane quarter, one query row per thread and
 //              half of the block's keys per warp: tcgen05.ld of S_j, masking (prefix
 //              length, or the row's own visible slots; full blocks skip it), online
@@ -57,7 +60,8 @@
 namespace fvrag {
 namespace attn {
 
-constexpr int kThreads = 320;      // producer, MMA issuer, 8 softmax warps
+constexpr int kThreads = 352;      // producer, PV issuer, 8 softmax warps, S issuer
+constexpr int kWarpS = 10;         // the warp whose lane 0 issues the S MMAs
 constexpr int kBM = 128;          // query rows per tile (MMA M)
 constexpr int kBN = 128;          // keys per block (MMA N of S, K of PV)
 constexpr int kKStages = 2;       // depth of the K ring (K_j is consumed early, by S_j)
@@ -364,8 +368,9 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* p_full = s_full + kSP;                // [kSP]  P_j in tensor memory (4 warps)
   uint64_t* pv_done = s_full + 2 * kSP;           // [kSP]  PV_j done: S/P buffer free
   uint64_t* q_full = s_full + 3 * kSP;
-  uint64_t* drain = q_full + 1;
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  uint64_t* drain = q_full + 1;                   // every PV MMA done
+  uint64_t* drain_s = drain + 1;                  // every S MMA done
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain_s + 1);
 
   griddep_wait();                 // inputs may come from the previous kernel
   // ---- work item
@@ -397,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 1)
   const int ncand = (tok0 + ntok - 1) / a.Lq - c_lo + 1;
   const int ntb = (ncand * a.C + kBN - 1) / kBN;       // blocks over the candidates' own slots
   // valid own slots of the tile's candidates (the own blocks with none are skipped)
-  int* n_own = reinterpret_cast<int*>(drain + 1) + 4;
+  int* n_own = reinterpret_cast<int*>(drain_s + 1) + 4;
 
   for (int c = threadIdx.x; c < ncand; c += kThreads) {
     int n = a.own_len ? __ldg(&a.own_len[qi * a.K + c_lo + c]) : a.C;
@@ -420,6 +425,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     mbar_init(smem_u32(q_full), 1);
     mbar_init(smem_u32(drain), 1);
+    mbar_init(smem_u32(drain_s), 1);
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -547,64 +553,67 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_wait(smem_u32(&v_full[i % kVStages]), (i / kVStages) & 1, a.limit_ns);
     }
   } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    //   S_ns  = Q K_ns^T         into S/P buffer ns % kSP, once K_ns is in and PV_{ns-kSP}
-    //                            (the previous user of that buffer) is done;
-    //   O    += P_np V_np        with P_np read from tensor memory, once the softmax
-    //                            warps published P_np and V_np is in.
+    // ------------------------------------------------------------ PV issuer
+    //   O += P_j V_j   with P_j read from tensor memory, once the softmax warps published
+    //                  P_j and V_j is in; its commit frees V_j's stage and S/P buffer j.
+    // The S MMAs come from another thread (warp kWarpS), so neither kind of MMA waits
+    // behind the other's inputs: the S issuer waits for PV_j to finish before it reuses
+    // P_j's buffer while this thread already has PV_{j+1} queued, and the tensor pipe is
+    // never drained between blocks.
     if (lane == 0 && nblk > 0) {
-      const uint32_t idS = idesc_bf16_f32(kBM, kBN);
       const uint32_t idPV = idesc_bf16_f32(kBM, D) | (1u << 16);   // B (= V) MN-major
-      const uint32_t qa = smem_u32(q_s);
-      if (!mbar_wait(smem_u32(q_full), 0, a.limit_ns)) {
-        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
-      } else {
-        // Fixed order with blocking waits: S_0 .. S_{kSP-1}, then PV_j followed by
-        // S_{j+kSP} (which reuses PV_j's S/P buffer once PV_j is done).
-        auto issue_s = [&](int ns) {
-          if (!mbar_wait(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1, a.limit_ns) ||
-              !mbar_wait(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1, a.limit_ns))
-            return false;
-          tc_fence_after();
-          const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
-#pragma unroll
-          for (int h = 0; h < NH; ++h)
-#pragma unroll
-            for (int k16 = 0; k16 < 4; ++k16)
-              tc_mma_bf16(tmem_base + col_s(ns % kSP),
-                          desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
-                          desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS,
-                          (h | k16) != 0);
-          tc_commit(smem_u32(&s_full[ns % kSP]));
-          tc_commit(smem_u32(&k_empty[ns % kKStages]));
-          return true;
-        };
-        auto issue_pv = [&](int np) {
-          if (!mbar_wait(smem_u32(&p_full[np % kSP]), (np / kSP) & 1, a.limit_ns) ||
-              !mbar_wait(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1, a.limit_ns))
-            return false;
-          tc_fence_after();
-          const uint32_t pa = tmem_base + col_s(np % kSP);
-          const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
-#pragma unroll
-          for (int k16 = 0; k16 < kBN / 16; ++k16)
-            tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
-                           desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
-                           (np | k16) != 0);
-          tc_commit(smem_u32(&pv_done[np % kSP]));
-          tc_commit(smem_u32(&v_empty[np % kVStages]));
-          return true;
-        };
-        bool fine = true;
-        for (int ns = 0; ns < min(nblk, kSP) && fine; ++ns) fine = issue_s(ns);
-        for (int j = 0; j < nblk && fine; ++j) {
-          fine = issue_pv(j);
-          if (fine && j + kSP < nblk) fine = issue_s(j + kSP);
+      bool fine = true;
+      for (int np = 0; np < nblk && fine; ++np) {
+        if (!mbar_wait(smem_u32(&p_full[np % kSP]), (np / kSP) & 1, a.limit_ns) ||
+            !mbar_wait(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1, a.limit_ns)) {
+          fine = false;
+          break;
         }
-        if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
+        tc_fence_after();
+        const uint32_t pa = tmem_base + col_s(np % kSP);
+        const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
+#pragma unroll
+        for (int k16 = 0; k16 < kBN / 16; ++k16)
+          tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
+                         desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
+                         (np | k16) != 0);
+        tc_commit(smem_u32(&pv_done[np % kSP]));
+        tc_commit(smem_u32(&v_empty[np % kVStages]));
       }
+      if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
       tc_commit(smem_u32(drain));
       if (!mbar_wait(smem_u32(drain), 0, a.limit_ns))
+        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else if (warp == kWarpS) {
+    // ------------------------------------------------------------ S issuer
+    //   S_j = Q K_j^T  into S/P buffer j % kSP, once K_j is in and PV_{j-kSP} (the previous
+    //                  user of that buffer) is done; its commit frees K_j's stage.
+    if (lane == 0 && nblk > 0) {
+      const uint32_t idS = idesc_bf16_f32(kBM, kBN);
+      const uint32_t qa = smem_u32(q_s);
+      bool fine = mbar_wait(smem_u32(q_full), 0, a.limit_ns);
+      if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
+      for (int ns = 0; ns < nblk && fine; ++ns) {
+        if (!mbar_wait(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1, a.limit_ns) ||
+            !mbar_wait(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1, a.limit_ns)) {
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
+          fine = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
+#pragma unroll
+        for (int h = 0; h < NH; ++h)
+#pragma unroll
+          for (int k16 = 0; k16 < 4; ++k16)
+            tc_mma_bf16(tmem_base + col_s(ns % kSP), desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
+                        desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS, (h | k16) != 0);
+        tc_commit(smem_u32(&s_full[ns % kSP]));
+        tc_commit(smem_u32(&k_empty[ns % kKStages]));
+      }
+      tc_commit(smem_u32(drain_s));
+      if (!mbar_wait(smem_u32(drain_s), 0, a.limit_ns))
         record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteDrain);
     }
   } else {

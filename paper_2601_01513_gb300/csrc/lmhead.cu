@@ -85,6 +85,63 @@ __device__ __forceinline__ float ex2(float x) {
   return y;
 }
 
+// Online (max, sum of exp2) update of one row's state with a 32-column chunk of logits
+// (natural units in r).  FULL: all 32 columns are valid (no per-element tests).  The max
+// is a tree and the sum four interleaved partial sums, so neither is one long dependency
+// chain.
+template <bool FULL>
+__device__ __forceinline__ void lse_chunk(const uint32_t (&r)[32], int nvalid, float& rmax,
+                                          float& rsum) {
+  float mx[8];
+#pragma unroll
+  for (int u = 0; u < 8; ++u) mx[u] = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    if (FULL || i < nvalid) mx[i & 7] = fmaxf(mx[i & 7], __uint_as_float(r[i]));
+  const float cmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
+                           fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7]))) * kLog2e;
+  const float nmax = fmaxf(rmax, cmax);
+  float sp[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+  for (int i = 0; i < 32; ++i)
+    if (FULL || i < nvalid) sp[i & 3] += ex2(fmaf(__uint_as_float(r[i]), kLog2e, -nmax));
+  rsum = rsum * ex2(rmax - nmax) + ((sp[0] + sp[1]) + (sp[2] + sp[3]));
+  rmax = nmax;
+}
+
+// The epilogue of one row over `ncols` accumulator columns at tensor-memory address tbase
+// (this warp's lane quarter), whose column c is vocabulary id v0 + c: folds them into the
+// row's (rmax, rsum) and writes the logits of the row's targets found among them.
+__device__ __forceinline__ void lse_row(uint32_t tbase, int ncols, int v0, bool live, int m,
+                                        int G, const int32_t* __restrict__ targets,
+                                        float* __restrict__ tgt_logit, float& rmax, float& rsum) {
+  int tg[kMaxGathers];
+#pragma unroll
+  for (int g = 0; g < kMaxGathers; ++g)
+    tg[g] = (live && g < G) ? __ldg(&targets[(size_t)m * G + g]) - v0 : -1;
+  for (int c0 = 0; c0 < ncols; c0 += 32) {
+    uint32_t r[32];
+    tmem_ld_32x32b_x32(tbase + c0, r);
+    tmem_wait_ld();
+    const int nvalid = min(32, ncols - c0);
+    if (nvalid == 32)
+      lse_chunk<true>(r, 32, rmax, rsum);
+    else
+      lse_chunk<false>(r, nvalid, rmax, rsum);
+#pragma unroll
+    for (int g = 0; g < kMaxGathers; ++g) {
+      const int c = tg[g] - c0;
+      if (c >= 0 && c < nvalid) {
+        float val = 0.f;
+#pragma unroll
+        for (int i = 0; i < 32; ++i)
+          if (i == c) val = __uint_as_float(r[i]);
+        tgt_logit[(size_t)m * G + g] = val;
+      }
+    }
+  }
+}
+
 template <int BN, int MG>
 __global__ void __launch_bounds__(kThreads, 1)
     lm_head_kernel(const __grid_constant__ CUtensorMap tm_hidden,
@@ -275,7 +332,6 @@ __global__ void __launch_bounds__(kThreads, 1)
       const int t = it / ngroups, grp = it % ngroups;
       const int v0 = v_lo + t * BN;
       const int ncols = min(BN, v_hi - v0);
-      const int rows16 = (ncols + 15) & ~15;
       const int mcount = min(MG, mtiles - grp * MG);
       if (!mbar_wait(smem_u32(&tfull[slot]), use & 1, limit_ns)) {
         record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
@@ -285,43 +341,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < mcount; ++j) {
         const int mt = grp * MG + j;
         const int m = mt * kBM + row;
-        const bool live = m < M;
-        int tg[kMaxGathers];
-#pragma unroll
-        for (int g = 0; g < kMaxGathers; ++g)
-          tg[g] = (live && g < G) ? __ldg(&targets[(size_t)m * G + g]) - v0 : -1;
         float rmax = st_max[mt * kBM + row];  // running max of z * log2(e)
         float rsum = st_sum[mt * kBM + row];
         const uint32_t tbase =
             tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * MG + j) * BN);
-        for (int c0 = 0; c0 < rows16; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tbase + c0, r);
-          tmem_wait_ld();
-          const int nvalid = min(32, ncols - c0);
-          float cmax = -INFINITY;
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < nvalid) cmax = fmaxf(cmax, __uint_as_float(r[i]) * kLog2e);
-          const float nmax = fmaxf(rmax, cmax);
-          float s = rsum * ex2(rmax - nmax);
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < nvalid) s += ex2(fmaf(__uint_as_float(r[i]), kLog2e, -nmax));
-          rsum = s;
-          rmax = nmax;
-#pragma unroll
-          for (int g = 0; g < kMaxGathers; ++g) {
-            const int c = tg[g] - c0;
-            if (c >= 0 && c < nvalid) {
-              float val = 0.f;
-#pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (i == c) val = __uint_as_float(r[i]);
-              tgt_logit[(size_t)m * G + g] = val;
-            }
-          }
-        }
+        lse_row(tbase, ncols, v0, m < M, m, G, targets, tgt_logit, rmax, rsum);
         st_max[mt * kBM + row] = rmax;
         st_sum[mt * kBM + row] = rsum;
       }
@@ -565,43 +589,11 @@ __global__ void __launch_bounds__(kThreads, 1)
       for (int j = 0; j < pcount; ++j) {
         const int pt = grp * PG + j;
         const int m = pt * 2 * kBM + (int)rank * kBM + row;
-        const bool live = m < M;
-        int tg[kMaxGathers];
-#pragma unroll
-        for (int g = 0; g < kMaxGathers; ++g)
-          tg[g] = (live && g < G) ? __ldg(&targets[(size_t)m * G + g]) - v0 : -1;
         float rmax = st_max[pt * kBM + row];
         float rsum = st_sum[pt * kBM + row];
         const uint32_t tbase =
             tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)((slot * PG + j) * BN);
-        for (int c0 = 0; c0 < ncols; c0 += 32) {
-          uint32_t r[32];
-          tmem_ld_32x32b_x32(tbase + c0, r);
-          tmem_wait_ld();
-          const int nvalid = min(32, ncols - c0);
-          float cmax = -INFINITY;
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < nvalid) cmax = fmaxf(cmax, __uint_as_float(r[i]) * kLog2e);
-          const float nmax = fmaxf(rmax, cmax);
-          float sacc = rsum * ex2(rmax - nmax);
-#pragma unroll
-          for (int i = 0; i < 32; ++i)
-            if (i < nvalid) sacc += ex2(fmaf(__uint_as_float(r[i]), kLog2e, -nmax));
-          rsum = sacc;
-          rmax = nmax;
-#pragma unroll
-          for (int g = 0; g < kMaxGathers; ++g) {
-            const int c = tg[g] - c0;
-            if (c >= 0 && c < nvalid) {
-              float val = 0.f;
-#pragma unroll
-              for (int i = 0; i < 32; ++i)
-                if (i == c) val = __uint_as_float(r[i]);
-              tgt_logit[(size_t)m * G + g] = val;
-            }
-          }
-        }
+        lse_row(tbase, ncols, v0, m < M, m, G, targets, tgt_logit, rmax, rsum);
         st_max[pt * kBM + row] = rmax;
         st_sum[pt * kBM + row] = rsum;
       }

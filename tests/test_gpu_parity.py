@@ -54,6 +54,12 @@ ATTN_CASES = [
     (2, 3, 9, 16, 2, 128, [700, 2049]),    # 8 heads per KV head, several key splits
     (1, 2, 64, 8, 8, 64, [300]),           # longest supported tail
     (1, 2, 3, 128, 1, 64, [200]),          # hq / hkv = 128: one token per row tile
+    # pairs of row tiles on CTA pairs (cta_group::2 MMAs), D = 128
+    (1, 3, 16, 16, 2, 128, [500]),         # 3 tiles: the second pair's rank-1 tile is empty
+    (2, 4, 16, 16, 2, 128, [300, 1111]),   # 4 tiles, ragged prefixes, several key splits
+    (1, 2, 40, 8, 1, 128, [129]),          # 5 tiles, tiles spanning two candidates
+    (1, 8, 8, 28, 4, 128, [0]),            # no prefix: own blocks only
+    (3, 5, 16, 28, 4, 128, [4000, 100, 2500]),   # 7b-style GQA over three ragged queries
 ]
 
 
@@ -134,6 +140,8 @@ LM_CASES = [
     (129, 256, 4103, 1),      # two M-tiles (second with one row)
     (300, 192, 3001, 2),      # three M-tiles: one pass of 160-row vocabulary tiles
     (257, 64, 50021, 1),      # three M-tiles, the third with one row; ~3 vocabulary tiles per CTA
+    (384, 96, 10007, 8),      # three full M-tiles; 8 gathers
+    (320, 8192, 5000, 1),     # the 72b shape's rows and hidden size, small vocabulary
     (512, 96, 7777, 3),       # four M-tiles: one pass of two CTA-pair tiles (2-SM MMAs)
     (600, 128, 50021, 2),     # three pair tiles (the last one partly empty), ragged W tiles
     (200, 64, 3000, 8),       # one pair tile, two accumulator sets; 8 gathers per row

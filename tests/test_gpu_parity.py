@@ -54,8 +54,8 @@ ATTN_CASES = [
     (2, 3, 9, 16, 2, 128, [700, 2049]),    # 8 heads per KV head, several key splits
     (1, 2, 64, 8, 8, 64, [300]),           # longest supported tail
     (1, 2, 3, 128, 1, 64, [200]),          # hq / hkv = 128: one token per row tile
-    # pairs of row tiles on CTA pairs (cta_group::2 MMAs), D = 128
-    (1, 3, 16, 16, 2, 128, [500]),         # 3 tiles: the second pair's rank-1 tile is empty
+    # several row tiles per KV head, D = 128
+    (1, 3, 16, 16, 2, 128, [500]),         # 3 tiles of 16 tokens x 8 heads
     (2, 4, 16, 16, 2, 128, [300, 1111]),   # 4 tiles, ragged prefixes, several key splits
     (1, 2, 40, 8, 1, 128, [129]),          # 5 tiles, tiles spanning two candidates
     (1, 8, 8, 28, 4, 128, [0]),            # no prefix: own blocks only

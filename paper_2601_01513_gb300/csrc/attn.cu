@@ -46,9 +46,12 @@
 //              when a row has no reference yet or a partial sum shows a term past that
 //              limit), and P_j written back as bf16 pairs over S_j in tensor memory.
 //   One run: the CTA writes the bf16 output and the lse directly.  Several runs:
-//   normalised partials go to the workspace and merge_kernel combines them with
+//   normalised partials go to the workspace (fp16: the outputs are convex combinations
+//   of V rows, so 11 mantissa bits keep them well inside the bf16 output's rounding) and
+//   merge_kernel combines them with
 //   log-sum-exp weights.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include <algorithm>
 #include <cmath>
@@ -112,7 +115,7 @@ struct Args {
   const int32_t* own_len;  // [Qn][K] valid own slots n_k, or null (n_k = C)
   __nv_bfloat16* out;     // final output (one split)
   float* lse;             // final lse (one split), may be null
-  float* part_o;          // [nsplit][rows][D]  (several splits)
+  __half* part_o;         // [nsplit][rows][D] fp16 (several splits)
   float* part_lse;        // [nsplit][rows]
   uint32_t* status;
   uint64_t limit_ns;
@@ -159,6 +162,11 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
   __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ uint32_t pack_f16(float lo, float hi) {
+  __half2 v = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
@@ -840,11 +848,14 @@ __global__ void __launch_bounds__(kThreads, 1)
                 pack_bf16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
                 pack_bf16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
         } else {
-          float4* dst = reinterpret_cast<float4*>(a.part_o + pidx * D + oc);
+          uint4* dst = reinterpret_cast<uint4*>(a.part_o + pidx * D + oc);
 #pragma unroll
-          for (int c = 0; c < 32; c += 4)
-            dst[c / 4] = make_float4(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv,
-                                     __uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv);
+          for (int c = 0; c < 32; c += 8)
+            dst[c / 8] = make_uint4(
+                pack_f16(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
+                pack_f16(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
+                pack_f16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
+                pack_f16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
         }
       }
     }
@@ -876,7 +887,7 @@ struct RunTable {
 // with the tile's runs in consecutive slots (balanced plan; a tile with one run was
 // written by its CTA directly).
 template <int D>
-__global__ void merge_kernel(const float* __restrict__ part_o, const float* __restrict__ part_lse,
+__global__ void merge_kernel(const __half* __restrict__ part_o, const float* __restrict__ part_lse,
                              int nsplit, long long nrows, __nv_bfloat16* __restrict__ out,
                              float* __restrict__ lse_out, const RunTable rt) {
   constexpr int DPL = D / 32;
@@ -909,22 +920,28 @@ __global__ void merge_kernel(const float* __restrict__ part_o, const float* __re
   float res[DPL];
 #pragma unroll
   for (int i = 0; i < DPL; ++i) res[i] = 0.f;
-  const float* base = part_o + (size_t)first * D + lane * DPL;
+  const __half* base = part_o + (size_t)first * D + lane * DPL;
   for (int s0 = 0; s0 < nsplit; s0 += 8) {
     float v[8][DPL];
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       if (s0 + u < nsplit) {
-        const float* po = base + (size_t)(s0 + u) * stride * D;
+        const __half2* po = reinterpret_cast<const __half2*>(base + (size_t)(s0 + u) * stride * D);
         if constexpr (DPL == 4) {
-          const float4 f = *reinterpret_cast<const float4*>(po);
-          v[u][0] = f.x;
-          v[u][1] = f.y;
-          v[u][2] = f.z;
-          v[u][3] = f.w;
+          const uint2 raw = *reinterpret_cast<const uint2*>(po);
+          const float2 f0 = __half22float2(*reinterpret_cast<const __half2*>(&raw.x));
+          const float2 f1 = __half22float2(*reinterpret_cast<const __half2*>(&raw.y));
+          v[u][0] = f0.x;
+          v[u][1] = f0.y;
+          v[u][2] = f1.x;
+          v[u][3] = f1.y;
         } else {
 #pragma unroll
-          for (int i = 0; i < DPL; ++i) v[u][i] = po[i];
+          for (int i = 0; i < DPL; i += 2) {
+            const float2 f = __half22float2(po[i / 2]);
+            v[u][i] = f.x;
+            v[u][i + 1] = f.y;
+          }
         }
       }
     }
@@ -962,8 +979,13 @@ struct Plan {
 // own blocks of its candidates) is cut on the device into nsplit equal runs, one
 // CTA each, so a short ragged prefix gives short CTAs that the block scheduler
 // backfills.  Pick nsplit to minimise an estimate of the time: the larger of the
-// mean work per SM (waves x mean run) and the longest run, plus the cost of
-// writing and merging the partials (a 128-key block is ~0.6 us).
+// mean work per SM (waves x mean run, three blocks added per run for its prologue and
+// epilogue) and the longest run, plus the cost of writing and merging the fp16
+// partials.  The constants (~0.8 us per 128-key block; per split count, a fixed 20 us
+// and the partials written and read at ~3 TB/s) were fitted on GB300 to per-call times
+// measured at every split
+// count from 1 to 12 on the 72B-class, long-context and batch-16 workloads, where they
+// pick the fastest measured split (5, 5 and 1).
 static Plan make_plan(const Problem& pr, int sms) {
   Plan p;
   p.grp = pr.hq / pr.hkv;
@@ -985,8 +1007,8 @@ static Plan make_plan(const Problem& pr, int sms) {
     const double waves = (double)((ctas + sms - 1) / sms);
     const double t_mean = waves * (std::ceil(nb_mean / ns) + 3);
     const double t_max = std::ceil((double)nb / ns) + 3;
-    double t = std::max(t_mean, t_max) * 0.6;
-    if (ns > 1) t += 3.0 + ns * rows * (pr.D + 1) * 8.0 / 8.0e6;
+    double t = std::max(t_mean, t_max) * 0.8;
+    if (ns > 1) t += 20.0 + ns * rows * (pr.D * 2 + 4) * 2.0 / 3.0e6;
     if (t < best - 1e-9) {
       best = t;
       p.nsplit = ns;
@@ -1022,7 +1044,7 @@ static BalancedWs balanced_ws(const Problem& pr, const Plan& p, int grid) {
   BalancedWs w;
   w.runs = up(kWsHeaderBytes);
   w.part_o = w.runs + up(ntiles * sizeof(int2));
-  w.part_lse = w.part_o + up(slots * pr.D * 4);
+  w.part_lse = w.part_o + up(slots * pr.D * 2);
   w.total = w.part_lse + up(slots * 4);
   return w;
 }
@@ -1032,7 +1054,8 @@ static size_t ws_bytes(const Problem& pr, int sms) {
   int grid = 0;
   if (balanced_grid(pr, p, sms, &grid)) return balanced_ws(pr, p, grid).total;
   const size_t rows = (size_t)pr.Qn * pr.K * pr.Lq * pr.hq;
-  return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)pr.D + 1) * 4 : 0);
+  // partial outputs fp16 [nsplit][rows][D], then their lse fp32 [nsplit][rows]
+  return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)pr.D * 2 + 4) : 0);
 }
 
 static int device_sms() {
@@ -1118,11 +1141,11 @@ static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k
   a.out = reinterpret_cast<__nv_bfloat16*>(out);
   a.lse = lse;
   if (bal) {
-    a.part_o = reinterpret_cast<float*>(base + bw.part_o);
+    a.part_o = reinterpret_cast<__half*>(base + bw.part_o);
     a.part_lse = reinterpret_cast<float*>(base + bw.part_lse);
   } else {
-    a.part_o = reinterpret_cast<float*>(base + kWsHeaderBytes);
-    a.part_lse = a.part_o + (size_t)p.nsplit * nrows * D;
+    a.part_o = reinterpret_cast<__half*>(base + kWsHeaderBytes);
+    a.part_lse = reinterpret_cast<float*>(a.part_o + (size_t)p.nsplit * nrows * D);
   }
   a.status = reinterpret_cast<uint32_t*>(base);
   a.limit_ns = wait_limit_ns();
@@ -1156,10 +1179,10 @@ static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k
   const long long blocks = (nrows + wpb - 1) / wpb;
   const cudaError_t e =
       D == 128 ? launch_pdl(merge_kernel<128>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
-                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out,
+                            (const __half*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out,
                             lse, rt)
                : launch_pdl(merge_kernel<64>, dim3((unsigned)blocks), dim3(32 * wpb), 0, s,
-                            (const float*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out,
+                            (const __half*)a.part_o, (const float*)a.part_lse, p.nsplit, nrows, a.out,
                             lse, rt);
   if (e != cudaSuccess) return FVRAG_ERR_CUDA;
   return launch_status();

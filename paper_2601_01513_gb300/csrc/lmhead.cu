@@ -26,7 +26,8 @@
 //   M <= 128        <256, 1>: one M-tile, two accumulator sets, so the epilogue of
 //                   tile t overlaps the MMAs of tile t+1 (HBM-bound: W streams once);
 //   129 .. 256      the pair form with one 256-row pair-tile (two accumulator sets);
-//   257 .. 384      <160, 3>: three M-tiles against 160-row W tiles, one pass over W;
+//   257 .. 384      the vocabulary-major pair form: W rows along the MMA's M axis, the
+//                   hidden rows along N (no padding of 320 rows to 384);
 //   385 .. 2048     the pair form with two pair-tiles (512 rows) per pass over W.
 // The pair form (lm_head_pair_kernel) runs on clusters of two CTAs with tcgen05
 // cta_group::2 MMAs of M = 256, each SM loading half of every W tile.
@@ -58,11 +59,8 @@ enum : uint32_t { kSiteProdEmpty = 0x201, kSiteMmaTmem = 0x202, kSiteMmaFull = 0
                   kSiteEpiFull = 0x204, kSiteDrain = 0x205 };
 
 // BN vocabulary rows per tile and MG M-tiles per pass; the accumulators of one item take
-// MG * BN tensor-memory columns.  <256, 1> (one M-tile) double-buffers them; <160, 3> serves
-// exactly three M-tiles (257-384 rows) in one pass over W with a single set (480 of the 512
-// columns): pairs of 256-column accumulators would need a second pass for the third M-tile,
-// and a CTA's 256-row W tile (2H * 256 bytes, 4 MB at H = 8192) is long gone from L2 by the
-// time that pass comes back to it.  Two M-tiles and more than three take the pair form below.
+// MG * BN tensor-memory columns.  The one form built, <256, 1> (one M-tile), double-buffers
+// them; more rows take the pair forms below.
 template <int BN, int MG>
 struct Cfg {
   static constexpr int kABytes = kBM * kBK * 2;           // 16 KB per M-tile
@@ -618,6 +616,355 @@ __global__ void __launch_bounds__(kThreads, 1)
   if (warp == 1) tmem_dealloc_pair(tmem_base, C::kTmemCols);
 }
 
+// ---------------------------------------------------------------------------
+// Vocabulary-major pair form for 257 .. 384 rows.  An MMA's M axis comes in 128 rows per
+// SM, so 257-384 hidden rows as the A operand cost 384 rows of tensor work (320 rows: a
+// ceiling of 83 %).  Here the operands swap: W is A (M = 256 vocabulary rows per pair MMA,
+// 128 per CTA) and the hidden rows lie along N, which comes in steps of 16: Mp = rows
+// rounded up to 32, issued as two MMAs of N = Mp / 2 per K step.  Each CTA of the pair loads
+// its 128 W rows of a tile and a quarter Mp / 4 of the hidden rows of each of the two MMAs.
+//
+// Tensor memory then holds z with vocabulary ids in lanes and hidden rows in columns, so
+// the log-sum-exp over the vocabulary runs across the lanes of a warp.  Per 32-column chunk
+// a transposed butterfly of 31 shuffles leaves lane c with the sum over the warp's 32 ids of
+// column c.  Every (lane quarter, column) keeps a reference max R in the log2 domain, raised
+// only when a value passes it by more than 2^8 (one warp vote per chunk), so an ordinary
+// chunk takes no max reduction at all.  Consecutive tiles alternate their accumulators
+// between columns [0, Mp) and [512 - Mp, 512); the next tile's MMAs wait only until the
+// epilogue has read the columns the two ranges share, which it reads first.  Eight epilogue
+// warps (two per lane quarter) split the chunks.  The target logits are direct dot products
+// of the hidden row with the target's W row (the definition of z_target), taken by the
+// epilogue warps while the first tile's MMAs run.
+namespace vt {
+constexpr int kThreads = 320;                   // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
+constexpr int kEpiWarps = 8;
+constexpr int kMaxRows = 384;
+constexpr int kStages = 5;
+constexpr int kTile = 256;                      // vocabulary rows per pair MMA (128 per CTA)
+constexpr int kABytes = kBM * kBK * 2;          // this CTA's 128 W rows x 64 K: 16 KB
+constexpr int kStageBytes = kABytes + kMaxRows / 2 * kBK * 2;   // + up to 192 hidden rows
+constexpr int kSmemBytes = kStages * kStageBytes + 1024 + 256 + 2 * 4 * kMaxRows * 4;
+constexpr float kLazy = 8.f;                    // R is raised once a value exceeds it by 2^8
+static_assert(kStageBytes % 1024 == 0, "stages must keep 1024-byte alignment");
+static_assert(kSmemBytes <= 232448, "shared memory per CTA");
+}  // namespace vt
+
+// On entry v[i] is this lane's value of column i of a 32 x 32 block (lanes x columns); on
+// exit v[0] holds the reduction over the 32 lanes of column `lane`.  Each step halves the
+// columns a lane keeps and combines them with the partner's across the step's lane bit.
+template <bool MAX>
+__device__ __forceinline__ float warp_transpose_reduce(float (&v)[32], int lane) {
+#pragma unroll
+  for (int w = 16; w >= 1; w >>= 1) {
+    const bool hi = (lane & w) != 0;
+#pragma unroll
+    for (int i = 0; i < w; ++i) {
+      const float send = hi ? v[i] : v[i + w];
+      const float keep = hi ? v[i + w] : v[i];
+      const float got = __shfl_xor_sync(0xffffffffu, send, w);
+      v[i] = MAX ? fmaxf(keep, got) : keep + got;
+    }
+  }
+  return v[0];
+}
+
+// One 32-column chunk of a vocabulary-major accumulator: lanes are vocabulary ids, columns
+// hidden rows.  nR / S: this lane quarter's -R and running sums of the chunk's 32 columns
+// (lane c owns column c).  MASKED: lanes with `valid` false lie past the pair's range.
+template <bool MASKED>
+__device__ __forceinline__ void vt_chunk(uint32_t taddr, bool valid, float* nR, float* S, int lane) {
+  uint32_t r[32];
+  tmem_ld_32x32b_x32(taddr, r);
+  tmem_wait_ld();
+  float nr[32], e[32];
+  const float4* nr4 = reinterpret_cast<const float4*>(nR);
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    const float4 x = nr4[q];
+    nr[4 * q] = x.x;
+    nr[4 * q + 1] = x.y;
+    nr[4 * q + 2] = x.z;
+    nr[4 * q + 3] = x.w;
+  }
+  float dmax = -INFINITY;
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    float d = fmaf(__uint_as_float(r[i]), kLog2e, nr[i]);
+    if (MASKED && !valid) d = -INFINITY;
+    dmax = fmaxf(dmax, d);
+    e[i] = ex2(d);
+  }
+  if (__any_sync(0xffffffffu, dmax > vt::kLazy)) {
+    // rare: some value passed its column's R by more than 2^8 (always on the first tile,
+    // where R = -inf): raise R to the column max and redo the chunk
+#pragma unroll
+    for (int i = 0; i < 32; ++i)
+      e[i] = (MASKED && !valid) ? -INFINITY : __uint_as_float(r[i]) * kLog2e;
+    const float cmax = warp_transpose_reduce<true>(e, lane);
+    const float rold = -nR[lane];
+    const float rnew = fmaxf(rold, cmax);
+    if (rnew > rold) {
+      S[lane] *= ex2(rold - rnew);
+      nR[lane] = -rnew;
+    }
+    __syncwarp();
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 x = nr4[q];
+      nr[4 * q] = x.x;
+      nr[4 * q + 1] = x.y;
+      nr[4 * q + 2] = x.z;
+      nr[4 * q + 3] = x.w;
+    }
+#pragma unroll
+    for (int i = 0; i < 32; ++i) {
+      float d = fmaf(__uint_as_float(r[i]), kLog2e, nr[i]);
+      if (MASKED && !valid) d = -INFINITY;
+      e[i] = ex2(d);
+    }
+  }
+  const float csum = warp_transpose_reduce<false>(e, lane);
+  S[lane] += csum;
+}
+
+// Sum of the products of eight bf16 pairs packed in two 16-byte vectors, in fp32.
+__device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b) {
+  const uint32_t av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+  float s = 0.f;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    s = fmaf(__uint_as_float(av[i] << 16), __uint_as_float(bv[i] << 16), s);
+    s = fmaf(__uint_as_float(av[i] & 0xffff0000u), __uint_as_float(bv[i] & 0xffff0000u), s);
+  }
+  return s;
+}
+
+__global__ void __launch_bounds__(vt::kThreads, 1)
+    lm_head_vt_kernel(const __grid_constant__ CUtensorMap tm_hb,
+                      const __grid_constant__ CUtensorMap tm_w64, const uint16_t* __restrict__ hidden,
+                      const uint16_t* __restrict__ weight, const int32_t* __restrict__ targets, int M,
+                      int Mp, int H, int V, int G, float* __restrict__ part_max,
+                      float* __restrict__ part_sum, float* __restrict__ tgt_logit, uint32_t* status,
+                      uint64_t limit_ns) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~uintptr_t(1023));
+  uint8_t* ring = smem;
+  uint64_t* bars = reinterpret_cast<uint64_t*>(ring + vt::kStages * vt::kStageBytes);
+  uint64_t* full = bars;                       // [vt::kStages]  rank 0: both CTAs' copies
+  uint64_t* empty = bars + vt::kStages;            // [vt::kStages]  each CTA: its stage is free
+  uint64_t* tfull = bars + 2 * vt::kStages;        // each CTA: the tile's accumulators are ready
+  uint64_t* ovl = tfull + 1;                   // rank 0: both epilogues read the shared columns
+  uint64_t* drain = ovl + 1;                   // rank 0: every MMA done
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain + 1);
+  float* negR = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(bars) + 256);  // [4][vt::kMaxRows]
+  float* Ssum = negR + 4 * vt::kMaxRows;                                                // [4][vt::kMaxRows]
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const int pair = blockIdx.x >> 1, npairs = gridDim.x >> 1;
+
+  // ---- this pair's vocabulary range, in units of 16 rows
+  const int nunits = (V + 15) >> 4;
+  const int u_lo = (int)(((long long)pair * nunits) / npairs);
+  const int u_hi = (int)(((long long)(pair + 1) * nunits) / npairs);
+  const int v_lo = u_lo * 16;
+  const int v_hi = min(u_hi * 16, V);
+  const int ntiles = (v_hi - v_lo + vt::kTile - 1) / vt::kTile;
+  const int kblocks = (H + kBK - 1) / kBK;
+  const int N = Mp >> 1, nb = Mp >> 2, nch = Mp >> 5;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < vt::kStages; ++s) {
+      mbar_init(smem_u32(&full[s]), 1);
+      mbar_init(smem_u32(&empty[s]), 1);
+    }
+    mbar_init(smem_u32(tfull), 1);
+    mbar_init(smem_u32(ovl), 2 * vt::kEpiWarps);   // every epilogue warp of both CTAs
+    mbar_init(smem_u32(drain), 1);
+    fence_barrier_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tm_hb);
+    tma_prefetch_desc(&tm_w64);
+  }
+  for (int i = threadIdx.x; i < 4 * vt::kMaxRows; i += vt::kThreads) {
+    negR[i] = INFINITY;     // R = -inf
+    Ssum[i] = 0.f;
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(smem_u32(tmem_holder), 512);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // the peer's barriers are initialised before any remote use
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_holder;
+  const uint32_t full0 = mapa_shared(smem_u32(&full[0]), 0);
+  const uint32_t ovl0 = mapa_shared(smem_u32(ovl), 0);
+  griddep_wait();                 // the prologue above touched no global memory
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer (both CTAs)
+    if (lane == 0) {
+      const uint64_t pol_w = policy_evict_first();
+      const uint64_t pol_h = policy_evict_last();
+      const uint32_t bytes = vt::kABytes + (uint32_t)Mp * kBK;   // per CTA: 128 W rows + Mp/2 hidden rows
+      int stage = 0;
+      uint32_t phase = 0;
+      long long issued = 0;
+      bool ok = true;
+      for (int t = 0; t < ntiles && ok; ++t) {
+        const int w0 = v_lo + t * vt::kTile + (int)rank * kBM;
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
+            ok = false;
+            break;
+          }
+          const uint32_t fb = full0 + (uint32_t)(stage * 8);
+          if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full[stage]), 2 * bytes);
+          const uint32_t st = smem_u32(ring + stage * vt::kStageBytes);
+          tma_load_2d_pair(st, &tm_w64, fb, kb * kBK, w0, pol_w);
+          tma_load_2d_pair(st + 64 * 128, &tm_w64, fb, kb * kBK, w0 + 64, pol_w);
+          tma_load_2d_pair(st + vt::kABytes, &tm_hb, fb, kb * kBK, (int)rank * nb, pol_h);
+          tma_load_2d_pair(st + vt::kABytes + nb * 128, &tm_hb, fb, kb * kBK, N + (int)rank * nb, pol_h);
+          ++issued;
+          if (++stage == vt::kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+      }
+      if (rank == 0) {
+        const int pend = issued < vt::kStages ? (int)issued : vt::kStages;
+        for (int i = 0; i < pend; ++i) {
+          if (--stage < 0) {
+            stage = vt::kStages - 1;
+            phase ^= 1;
+          }
+          mbar_wait(smem_u32(&full[stage]), phase, limit_ns);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------ MMA issuer (rank 0)
+    if (lane == 0 && rank == 0) {
+      const uint32_t idesc = idesc_bf16_f32(2 * kBM, (uint32_t)N);
+      int stage = 0;
+      uint32_t phase = 0;
+      bool ok = true;
+      for (int t = 0; t < ntiles && ok; ++t) {
+        // the previous tile's epilogue has read the columns this tile shares with it (and,
+        // before that, all of the tile before it, whose columns this one reuses)
+        if (t > 0 && !mbar_wait_cluster(smem_u32(ovl), (uint32_t)((t - 1) & 1), limit_ns)) {
+          record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaTmem);
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d0 = tmem_base + (uint32_t)((t & 1) ? 512 - Mp : 0);
+        for (int kb = 0; kb < kblocks; ++kb) {
+          if (!mbar_wait_cluster(smem_u32(&full[stage]), phase, limit_ns)) {
+            record_error(status, FVRAG_ERR_TIMEOUT, kSiteMmaFull);
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t st = smem_u32(ring + stage * vt::kStageBytes);
+#pragma unroll
+          for (int k16 = 0; k16 < kBK / 16; ++k16) {
+            const uint64_t a = desc_kmajor_sw128(st + k16 * 32);
+            tc_mma_bf16_pair(d0, a, desc_kmajor_sw128(st + vt::kABytes + k16 * 32), idesc,
+                             (kb | k16) != 0);
+            tc_mma_bf16_pair(d0 + (uint32_t)N, a,
+                             desc_kmajor_sw128(st + vt::kABytes + nb * 128 + k16 * 32), idesc,
+                             (kb | k16) != 0);
+          }
+          tc_commit_pair(smem_u32(&empty[stage]), 0x3);
+          if (++stage == vt::kStages) {
+            stage = 0;
+            phase ^= 1;
+          }
+        }
+        if (!ok) break;
+        tc_commit_pair(smem_u32(tfull), 0x3);
+      }
+      tc_commit_pair(smem_u32(drain), 0x1);
+      if (!mbar_wait(smem_u32(drain), 0, limit_ns)) record_error(status, FVRAG_ERR_TIMEOUT, kSiteDrain);
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue (both CTAs)
+    const int ew = warp - 2, quarter = warp & 3, grp = ew >> 2;
+    // target logits z[m, t] = <hidden[m], W[t]>, split over every epilogue warp of the grid
+    for (int i = (int)blockIdx.x * vt::kEpiWarps + ew; i < M * G; i += (int)gridDim.x * vt::kEpiWarps) {
+      const int tg = __ldg(&targets[i]);
+      if (tg < 0 || tg >= V) continue;          // the merge writes NaN for these
+      const uint4* hp = reinterpret_cast<const uint4*>(hidden + (size_t)(i / G) * H);
+      const uint4* wp = reinterpret_cast<const uint4*>(weight + (size_t)tg * H);
+      float acc = 0.f;
+      for (int c = lane; c < (H >> 3); c += 32) acc += dot8_bf16(__ldg(hp + c), __ldg(wp + c));
+      acc = warp_sum(acc);
+      if (lane == 0) tgt_logit[i] = acc;
+    }
+    float* nRq = negR + quarter * vt::kMaxRows;
+    float* Sq = Ssum + quarter * vt::kMaxRows;
+    const int vl = (int)rank * kBM + quarter * 32 + lane;   // this thread's row inside a tile
+    const uint32_t lane_addr = tmem_base + ((uint32_t)(quarter * 32) << 16);
+    for (int t = 0; t < ntiles; ++t) {
+      if (!mbar_wait_cluster(smem_u32(tfull), (uint32_t)(t & 1), limit_ns)) {
+        record_error(status, FVRAG_ERR_TIMEOUT, kSiteEpiFull);
+        break;
+      }
+      tc_fence_after();
+      const int v0 = v_lo + t * vt::kTile;
+      const bool masked = v0 + vt::kTile > v_hi;
+      const bool valid = v0 + vl < v_hi;
+      const uint32_t tb = lane_addr + (uint32_t)((t & 1) ? 512 - Mp : 0);
+      // chunks whose columns the next tile's accumulators share: [16 - nch, nch) of an even
+      // tile, [0, 2 nch - 16) of an odd one
+      const int lo = (t & 1) ? 0 : 16 - nch, hi = (t & 1) ? 2 * nch - 16 : nch;
+      for (int pass = 0; pass < 2; ++pass) {
+        for (int k = grp; k < nch; k += 2) {
+          if ((k >= lo && k < hi) != (pass == 0)) continue;
+          if (masked)
+            vt_chunk<true>(tb + (uint32_t)(32 * k), valid, nRq + 32 * k, Sq + 32 * k, lane);
+          else
+            vt_chunk<false>(tb + (uint32_t)(32 * k), valid, nRq + 32 * k, Sq + 32 * k, lane);
+        }
+        if (pass == 0) {
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive_cluster(ovl0);
+        }
+      }
+    }
+    // fold the four lane quarters of every column into this CTA's partial (log2 domain)
+    asm volatile("bar.sync 1, %0;" ::"n"(vt::kEpiWarps * 32) : "memory");
+    for (int m = ew * 32 + lane; m < M; m += vt::kEpiWarps * 32) {
+      float mx = -INFINITY;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) mx = fmaxf(mx, -negR[q * vt::kMaxRows + m]);
+      float s = 0.f;
+      if (mx != -INFINITY) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float rq = -negR[q * vt::kMaxRows + m];
+          if (rq != -INFINITY) s += Ssum[q * vt::kMaxRows + m] * ex2(rq - mx);
+        }
+      }
+      part_max[(size_t)blockIdx.x * M + m] = mx;
+      part_sum[(size_t)blockIdx.x * M + m] = s;
+    }
+  }
+  griddep_launch_dependents();    // the merge kernel may start launching
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();                 // neither CTA frees tensor memory the other may still use
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem_base, 512);
+}
+
 // One warp per row: lse = ln 2 * (M2 + log2 S) with M2 = max_b max_b and
 // S = sum_b sum_b * 2^(max_b - M2) (partials in the log2 domain); logprob = z_target - lse.
 __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float* __restrict__ part_sum,
@@ -661,27 +1008,27 @@ __global__ void lm_merge_kernel(const float* __restrict__ part_max, const float*
 }
 
 struct Plan {
-  int ctas;       // CTAs of the 1-CTA forms; pairs of the pair forms (the merge's partials)
-  int bn, mg;     // mg = 0 / -1: the pair form with two / one pair-tiles per pass
+  int ctas;       // CTAs of the 1-CTA forms; pairs of the pair forms
+  int parts;      // per-row partials the merge folds: one per CTA, or per pair
+  int bn, mg;     // mg = 0 / -1: the pair form with two / one pair-tiles per pass;
+                  // mg = 2: the vocabulary-major pair form
 };
 
-// Pairs (2-CTA clusters) of the pair form that can be resident at once, per device.
-static int max_pairs() {
-  static std::mutex mu;
-  static int cached[64] = {0};
+// Pairs (2-CTA clusters) of a pair-form kernel that can be resident at once on the current
+// device; `cache` holds one entry per device.
+static int resident_pairs(const void* kern, int threads, int smem, int* cache, std::mutex& mu) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
   std::lock_guard<std::mutex> lock(mu);
-  if (cached[dev] == 0) {
-    using C = PairCfg<2>;
+  if (cache[dev] == 0) {
     int n = 0;
-    if (cudaFuncSetAttribute(lm_head_pair_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             C::kSmemBytes) == cudaSuccess) {
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) ==
+        cudaSuccess) {
       cudaLaunchConfig_t cfg = {};
       const int sms = std::max(2, sm_count());
       cfg.gridDim = dim3(sms / 2 * 2);
-      cfg.blockDim = dim3(kThreads);
-      cfg.dynamicSmemBytes = C::kSmemBytes;
+      cfg.blockDim = dim3(threads);
+      cfg.dynamicSmemBytes = smem;
       cudaLaunchAttribute attr[1];
       attr[0].id = cudaLaunchAttributeClusterDimension;
       attr[0].val.clusterDim.x = 2;
@@ -689,26 +1036,47 @@ static int max_pairs() {
       attr[0].val.clusterDim.z = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      if (cudaOccupancyMaxActiveClusters(&n, lm_head_pair_kernel<2>, &cfg) != cudaSuccess) n = 0;
+      if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess) n = 0;
     }
     cudaGetLastError();
-    cached[dev] = std::max(1, std::min(n, std::min(sm_count() / 2, kMaxCtas)));
+    cache[dev] = std::max(1, std::min(n, std::min(sm_count() / 2, kMaxCtas / 2)));
   }
-  return cached[dev];
+  return cache[dev];
+}
+
+static int max_pairs() {
+  static std::mutex mu;
+  static int cache[64] = {0};
+  return resident_pairs(reinterpret_cast<const void*>(lm_head_pair_kernel<2>), kThreads,
+                        PairCfg<2>::kSmemBytes, cache, mu);
+}
+
+static int max_pairs_vt() {
+  static std::mutex mu;
+  static int cache[64] = {0};
+  return resident_pairs(reinterpret_cast<const void*>(lm_head_vt_kernel), vt::kThreads,
+                        vt::kSmemBytes, cache, mu);
 }
 
 // `sms`: the most SMs the grid may occupy (the device's count, or the caller's budget).
 static Plan make_plan(const fvrag_lm_desc* d, int sms) {
   Plan p;
   const int mtiles = (d->rows + kBM - 1) / kBM;
-  p.bn = mtiles == 3 ? 160 : 256;
+  p.bn = 256;
   // one M-tile: <256, 1>; two: the pair form with one pair-tile and two accumulator sets;
-  // three: <160, 3> (one pass; pairs would pad 384 rows to 512); more: the pair form with
-  // two pair-tiles per pass
-  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 3 : mtiles == 2 ? -1 : 0;
+  // three: the vocabulary-major pair form (hidden rows along N, no padding to 384); more:
+  // the pair form with two pair-tiles per pass
+  p.mg = mtiles == 1 ? 1 : mtiles == 3 ? 2 : mtiles == 2 ? -1 : 0;
   const int nunits = (d->vocab + 15) / 16;
-  p.ctas = std::max(1, std::min(std::min(sms > 0 ? sms : 148, kMaxCtas), nunits));
-  if (p.mg <= 0) p.ctas = std::max(1, std::min(std::min(max_pairs(), std::max(1, sms / 2)), nunits));
+  const int budget = sms > 0 ? sms : 148;
+  if (p.mg == 1) {
+    p.ctas = std::max(1, std::min(std::min(budget, kMaxCtas), nunits));
+    p.parts = p.ctas;
+  } else {
+    const int pairs = p.mg == 2 ? max_pairs_vt() : max_pairs();
+    p.ctas = std::max(1, std::min(std::min(pairs, std::max(1, budget / 2)), nunits));
+    p.parts = p.mg == 2 ? 2 * p.ctas : p.ctas;
+  }
   return p;
 }
 
@@ -738,6 +1106,36 @@ static fvrag_status launch_pair(const Plan& p, const CUtensorMap& th, const CUte
   cfg.numAttrs = 2;
   if (counted(cudaLaunchKernelEx(&cfg, kern, th, tw64, tw16, targets, d->rows, d->hidden,
                                  d->vocab, d->gathers, pmax, psum, ptgt, status,
+                                 wait_limit_ns())) != cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  return launch_status();
+}
+
+static fvrag_status launch_vt(const Plan& p, const CUtensorMap& thb, const CUtensorMap& tw64,
+                              const void* hidden, const void* weight, const int32_t* targets,
+                              const fvrag_lm_desc* d, int Mp, float* pmax, float* psum,
+                              float* ptgt, uint32_t* status, cudaStream_t s) {
+  auto kern = lm_head_vt_kernel;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, vt::kSmemBytes) !=
+      cudaSuccess)
+    return FVRAG_ERR_CUDA;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(2 * p.ctas);
+  cfg.blockDim = dim3(vt::kThreads);
+  cfg.dynamicSmemBytes = vt::kSmemBytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 2;
+  if (counted(cudaLaunchKernelEx(&cfg, kern, thb, tw64, static_cast<const uint16_t*>(hidden),
+                                 static_cast<const uint16_t*>(weight), targets, d->rows, Mp,
+                                 d->hidden, d->vocab, d->gathers, pmax, psum, ptgt, status,
                                  wait_limit_ns())) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();
@@ -822,19 +1220,25 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
 
   fvrag_status st;
-  if (p.mg == 0)
+  if (p.mg == 2) {
+    // vocabulary-major form: hidden rows in boxes of Mp / 4 (a quarter of the padded rows)
+    const int Mp = (int)((M + 31) / 32 * 32);
+    CUtensorMap thb;
+    const uint64_t dims[2] = {H, M}, strides[1] = {H * 2};
+    const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)(Mp / 4)};
+    if (!encode_tmap_bf16(&thb, hidden, 2, dims, strides, box, true)) return FVRAG_ERR_CUDA;
+    st = launch_vt(p, thb, tw64, hidden, weight, targets, d, Mp, pmax, psum, ptgt, status, s);
+  } else if (p.mg == 0)
     st = launch_pair<2>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
   else if (p.mg == -1)
     st = launch_pair<1>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
-  else if (p.mg == 1)
-    st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   else
-    st = launch<160, 3>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
+    st = launch<256, 1>(p, th, tw64, tw16, targets, d, hrows, pmax, psum, ptgt, status, s);
   if (st != FVRAG_OK) return st;
   const int rows_per_block = 8;
   if (launch_pdl(lm_merge_kernel, dim3((d->rows + rows_per_block - 1) / rows_per_block),
                  dim3(32 * rows_per_block), 0, s, (const float*)pmax, (const float*)psum,
-                 (const float*)ptgt, targets, d->rows, d->vocab, d->gathers, p.ctas, logprob,
+                 (const float*)ptgt, targets, d->rows, d->vocab, d->gathers, p.parts, logprob,
                  lse) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   return launch_status();

@@ -138,10 +138,13 @@ LM_CASES = [
     (33, 72, 1007, 2),        # H not a multiple of 64; V not a multiple of 16
     (128, 128, 5000, 8),      # one full M-tile, 8 gathers
     (129, 256, 4103, 1),      # two M-tiles (second with one row)
-    (300, 192, 3001, 2),      # three M-tiles: one pass of 160-row vocabulary tiles
-    (257, 64, 50021, 1),      # three M-tiles, the third with one row; ~3 vocabulary tiles per CTA
-    (384, 96, 10007, 8),      # three full M-tiles; 8 gathers
+    (300, 192, 3001, 2),      # 257-384 rows: the vocabulary-major pair form (Mp = 320)
+    (257, 64, 50021, 1),      # vocabulary-major, Mp = 288 (boxes of 72 rows); ~1.3 tiles per pair
+    (384, 96, 10007, 8),      # vocabulary-major, Mp = 384 (two accumulator ranges sharing 256 columns)
     (320, 8192, 5000, 1),     # the 72b shape's rows and hidden size, small vocabulary
+    (352, 136, 40000, 3),     # vocabulary-major, Mp = 352; H not a multiple of 64
+    (290, 64, 40, 2),         # vocabulary-major with 3 pairs of 16 rows: most lanes past the range
+    (320, 64, 152064, 1),     # vocabulary-major over the full vocabulary: 8 tiles per pair
     (512, 96, 7777, 3),       # four M-tiles: one pass of two CTA-pair tiles (2-SM MMAs)
     (600, 128, 50021, 2),     # three pair tiles (the last one partly empty), ragged W tiles
     (200, 64, 3000, 8),       # one pair tile, two accumulator sets; 8 gathers per row
@@ -170,15 +173,33 @@ def test_lm_matches_oracle(case):
     assert np.max(np.abs(lse - ref_lse)) <= LOGPROB_ATOL
 
 
-def test_lm_all_targets_sum_to_one():
+@pytest.mark.parametrize("M", [3, 300])
+def test_lm_all_targets_sum_to_one(M):
     """Gathering every vocabulary id of a row: sum of probabilities is 1 (any size)."""
-    M, H, V = 3, 128, 8
+    H, V = 128, 8
     hid = synth.normal_bf16((M, H), 5, 1)
     W = synth.normal_bf16((V, H), 5, 2, 0.0, 0.3)
     tgt = np.tile(np.arange(V, dtype=np.int32), (M, 1))
     lp, _, st = run_lm(hid, W, tgt)
     assert st == fvrag.OK
     np.testing.assert_allclose(np.exp(lp.astype(np.float64)).sum(1), 1.0, atol=1e-4)
+
+
+@pytest.mark.parametrize("M", [40, 300])
+def test_lm_growing_logits_match_oracle(M):
+    """Logits whose scale grows along the vocabulary (W row v scaled by 1 + 6 v / V), so
+    later vocabulary tiles keep passing the running maxima of earlier ones: the online
+    log-sum-exp rescales (and the vocabulary-major form raises its reference max) often."""
+    H, V, G = 128, 30011, 2
+    hid = synth.normal_bf16((M, H), 77 + M, 1)
+    W = synth.bf16_bits_to_f32(synth.normal_bf16((V, H), 77 + M, 2, 0.0, 0.3)).astype(np.float64)
+    W = synth.round_bf16(W * (1.0 + 6.0 * np.arange(V, dtype=np.float64) / V)[:, None])
+    tgt = synth.uniform_i32((M, G), 77 + M, 3, 0, V)
+    lp, lse, st = run_lm(hid, W, tgt)
+    assert st == fvrag.OK
+    ref, ref_lse = oracle.score_logprobs(hid, W, tgt)
+    assert np.max(np.abs(lp - ref)) <= LOGPROB_ATOL
+    assert np.max(np.abs(lse - ref_lse)) <= LOGPROB_ATOL
 
 
 @pytest.mark.parametrize("name", ["7b", "long", "72b", "batch16"])

@@ -27,7 +27,7 @@ pytestmark = pytest.mark.gpu
 # rows, hidden, vocabulary, gathers: the kernel form each selects
 CASES = [
     (1024, 256, 9001, 8),    # eight M-tiles: 2-SM pair form, two pair tiles per pass; the array's limit
-    (300, 512, 20011, 2),    # three M-tiles: <160, 3>
+    (300, 512, 20011, 2),    # three M-tiles: the vocabulary-major 2-SM pair form
     (200, 128, 7001, 3),     # two M-tiles: 2-SM pair form, one pair tile
     (37, 256, 4099, 1),      # one M-tile: <256, 1>
 ]

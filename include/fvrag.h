@@ -73,7 +73,7 @@
 extern "C" {
 #endif
 
-#define FVRAG_ABI_VERSION 5
+#define FVRAG_ABI_VERSION 6
 
 /* cudaStream_t without including the CUDA headers. */
 typedef struct CUstream_st* fvrag_stream_t;
@@ -119,12 +119,23 @@ typedef struct fvrag_attn_desc {
   int32_t max_prefix;   /* upper bound on every P_q (plans the key split); >= 0 */
   int32_t total_prefix; /* sum over queries of P_q = rows of k_prefix / v_prefix */
   float softmax_scale;  /* > 0, or 0 => 1/sqrt(head_dim); negative / NaN / inf rejected */
-  uint32_t flags;       /* must be 0 */
+  uint32_t flags;       /* 0 (the library picks the key split), or one FVRAG_ATTN_SPLIT_* */
   int32_t sm_budget;    /* SMs the key split is planned for: 0 = every SM of the current
                            device, else 1 .. that count (more: FVRAG_ERR_INVALID_ARG).  A
                            budget below the device's count leaves the other SMs to a call
                            running beside this one on another stream (see "SM budgets") */
 } fvrag_attn_desc;
+
+/* fvrag_attn_desc.flags: how the keys of every row tile (a group of candidate tokens x the
+ * query heads of one KV head) are split over CTAs.  Every split gives the same result up to
+ * the order of floating-point additions; with flags = 0 the library picks one by its cost
+ * model.  Any other value: FVRAG_ERR_INVALID_ARG. */
+#define FVRAG_ATTN_SPLIT_STATIC 1u  /* each tile's key list cut into equal runs, one CTA per run */
+#define FVRAG_ATTN_SPLIT_STREAM 2u  /* one CTA per SM (of the budget), each an equal share of all
+                                       tiles' key lists in tile order; needs num_queries <= 64,
+                                       at most 64 tiles per KV head and query, and every P_q <=
+                                       max_prefix, else FVRAG_ERR_UNSUPPORTED (and a workspace
+                                       size of 0) */
 
 /* Bytes of workspace fvrag_verify_attn needs for `d` (0 if `d` is invalid). */
 size_t fvrag_verify_attn_workspace(const fvrag_attn_desc* d);

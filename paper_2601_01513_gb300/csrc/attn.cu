@@ -90,10 +90,13 @@ constexpr int kMaxPlanQueries = 1024; // queries whose offsets it stages
 constexpr int kMaxPlanOwn = 2048;     // Qn * K own lengths it stages
 constexpr int kMaxRuns = 64;          // runs of one tile that merge_kernel combines
 constexpr int kPlanScratch = 256;     // reduction and control words
+constexpr int kMaxStreamQueries = 64; // streamed plan: queries and row tiles per KV head
+constexpr int kMaxStreamMtiles = 64;  // whose prefix sums it keeps in shared memory
+constexpr int kStreamPlanBytes = 1024;
 constexpr int kPlanInts = kPlanScratch + kMaxPlanTiles + kMaxPlanQueries + 4 + kMaxPlanOwn;
 
 enum : uint32_t { kSiteQ = 0x101, kSiteMma = 0x102, kSiteProducer = 0x103, kSiteSFull = 0x107,
-                  kSitePvDone = 0x109, kSiteDrain = 0x10A };
+                  kSitePvDone = 0x109, kSiteDrain = 0x10A, kSitePlan = 0x10B };
 
 template <int D>
 struct Layout {
@@ -104,7 +107,8 @@ struct Layout {
   // + row-max exchange [2 slots][2 halves][128 rows], row-sum exchange [2][128] floats and
   // the slow-path flags [2 slots][2 halves][4 quarters]
   static constexpr int kBytes =
-      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4 + 64;
+      kQ + (kKStages + kVStages) * kStage + 1024 + 256 + kMaxCand * 4 + 6 * kBM * 4 + 64 +
+      kStreamPlanBytes;
   static_assert(kPlanInts * 4 <= kVStages * kStage, "plan scratch fits the V ring");
   static_assert(kBytes <= 232448, "shared memory per CTA");
 };
@@ -120,7 +124,8 @@ struct Args {
   uint32_t* status;
   uint64_t limit_ns;
   int Qn, K, Lq, C, KL, hq, hkv, grp, T, mtiles, nsplit;
-  int slot_rows;           // balanced plan: rows per partial slot (T * grp)
+  int slot_rows;           // balanced and streamed plans: rows per partial slot (T * grp)
+  int maxparts;            // streamed plan: partial slots per tile
   float scale_log2;
 };
 
@@ -349,13 +354,73 @@ __device__ int4 plan_run(const Args& a, int* ps) {
   return make_int4(ctl[2], ctl[3], ctl[4], ctl[5]);
 }
 
-// BAL: the balanced plan (decode) or the static split (verification); separate
-// instantiations keep the plan's code out of the verification kernel.
-template <int D, bool BAL>
+// ---------------------------------------------------------------------------
+// Streamed plan (verification, own lengths all C).  The block lists of all tiles, in tile
+// order (query, KV head, row tile), form one sequence of W blocks; CTA c takes the blocks
+// [c W / grid, (c + 1) W / grid): the tail of one tile, whole tiles and the head of another,
+// run as consecutive segments in one pass of its pipelines.  Every SM then does the same
+// number of blocks (to within one) in a single wave, whatever the number of tiles, and pays
+// the pipeline fill once.  A tile cut between CTAs leaves one normalised partial per CTA in
+// slots [t * maxparts, t * maxparts + parts) of the balanced plan's layout, merged by
+// merge_kernel; a tile that lies inside one CTA's range is written directly.
+//
+// The sequence position of tile t (query qi, KV head g, row tile mt) is closed-form:
+// tile t has npb(qi) prefix blocks and ntb(mt) own blocks, so with the prefix sums qcum over
+// queries and tcum over row tiles (NTB = tcum[mtiles]),
+//   G0(t) = hkv (mtiles qcum[qi] + qi NTB) + g (mtiles npb(qi) + NTB) + mt npb(qi) + tcum[mt].
+struct StreamPlan {
+  long long W;                         // blocks in all
+  int t0;                              // first tile of this CTA's range
+  int qcum[kMaxStreamQueries + 1];
+  int npb[kMaxStreamQueries];
+  int tcum[kMaxStreamMtiles + 1];
+};
+static_assert(sizeof(StreamPlan) + 16 <= kStreamPlanBytes, "the streamed plan fits its space");
+
+// Own blocks of row tile mt: the 128-key blocks over its candidates' C slots each.
+__device__ __forceinline__ int tile_own_blocks(const Args& a, int mt) {
+  const int tok0 = mt * a.T;
+  const int ntok = min(a.T, a.KL - tok0);
+  const int c_lo = tok0 / a.Lq;
+  const int ncand = (tok0 + ntok - 1) / a.Lq - c_lo + 1;
+  return (ncand * a.C + kBN - 1) / kBN;
+}
+
+__device__ __forceinline__ long long stream_g0(const Args& a, const StreamPlan& sp, int t) {
+  if (t >= a.Qn * a.hkv * a.mtiles) return sp.W;
+  const int mt = t % a.mtiles;
+  const int g = (t / a.mtiles) % a.hkv;
+  const int qi = t / a.mtiles / a.hkv;
+  const long long ntb_all = sp.tcum[a.mtiles];
+  return (long long)a.hkv * ((long long)a.mtiles * sp.qcum[qi] + (long long)qi * ntb_all) +
+         (long long)g * ((long long)a.mtiles * sp.npb[qi] + ntb_all) +
+         (long long)mt * sp.npb[qi] + sp.tcum[mt];
+}
+
+// The CTA whose range holds sequence position x: the largest c with c W / grid <= x.
+__device__ __forceinline__ int stream_cta(long long x, long long W, int grid) {
+  return (int)(((x + 1) * grid + W - 1) / W) - 1;
+}
+
+// One contiguous run of a tile's block list that a CTA processes.
+struct Seg {
+  int t;            // tile
+  int blk_lo;       // first block of the tile's list
+  int nblk;         // blocks
+  bool direct;      // the run is the whole list: the CTA writes the output itself
+  int pslot;        // partial slot (runs that are not direct), or the static plan's split
+};
+
+// MODE 0: static split (verification: tile x nsplit runs, one per CTA); 1: balanced plan
+// (decode: runs fitted on the device into one grid); 2: streamed plan (verification: a
+// share of the concatenated block lists per CTA).  Separate instantiations keep each plan's
+// code out of the other kernels.
+template <int D, int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_kernel(const __grid_constant__ CUtensorMap tm_q, const __grid_constant__ CUtensorMap tm_kp,
                 const __grid_constant__ CUtensorMap tm_vp, const __grid_constant__ CUtensorMap tm_kt,
                 const __grid_constant__ CUtensorMap tm_vt, const Args a) {
+  constexpr bool BAL = MODE == 1, STREAM = MODE == 2;
   using Lay = Layout<D>;
   constexpr int NH = Lay::NH;
   extern __shared__ uint8_t smem_raw[];
@@ -375,48 +440,124 @@ __global__ void __launch_bounds__(kThreads, 1)
   uint64_t* s_full = v_empty + kVStages;          // [kSP]  S_j in tensor memory
   uint64_t* p_full = s_full + kSP;                // [kSP]  P_j in tensor memory (4 warps)
   uint64_t* pv_done = s_full + 2 * kSP;           // [kSP]  PV_j done: S/P buffer free
-  uint64_t* q_full = s_full + 3 * kSP;
+  uint64_t* q_full = s_full + 3 * kSP;            // the segment's Q tile is in
   uint64_t* drain = q_full + 1;                   // every PV MMA done
   uint64_t* drain_s = drain + 1;                  // every S MMA done
-  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(drain_s + 1);
+  uint64_t* q_empty = drain_s + 1;                // the segment's S MMAs are done: Q may be reloaded
+  uint64_t* o_free = q_empty + 1;                 // the softmax warps have read the segment's O
+  uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(o_free + 1);
+  // valid own slots of the tile's candidates (single-segment plans; the own blocks with
+  // none are skipped)
+  int* n_own = reinterpret_cast<int*>(o_free + 1) + 4;
+  StreamPlan* sp = reinterpret_cast<StreamPlan*>(
+      (reinterpret_cast<uintptr_t>(n_own + kMaxCand) + 15) & ~uintptr_t(15));
 
   griddep_wait();                 // inputs may come from the previous kernel
-  // ---- work item
-  int mt, split = 0, g, qi;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // ---- work: one run (static, balanced plans) or this CTA's share of the sequence
+  Seg seg0 = {0, 0, 0, false, 0};
   int4 wk = make_int4(0, 0, 0, 0);
   if constexpr (BAL) {
     // the plan's scratch is the V ring, whose first writer is the TMA after the prologue
     wk = plan_run<kThreads>(a, reinterpret_cast<int*>(v_ring));
     fence_proxy_async_smem();
     if (wk.x < 0) return;         // the plan left this CTA without a run
-    mt = wk.x % a.mtiles;
-    g = (wk.x / a.mtiles) % a.hkv;
-    qi = wk.x / a.mtiles / a.hkv;
-  } else {
+    seg0.t = wk.x;
+  } else if constexpr (!STREAM) {
     int b = blockIdx.x;
-    mt = b % a.mtiles;
+    const int mt = b % a.mtiles;
     b /= a.mtiles;
-    split = b % a.nsplit;
+    seg0.pslot = b % a.nsplit;    // the split
     b /= a.nsplit;
-    g = b % a.hkv;
-    qi = b / a.hkv;
+    seg0.t = b * a.mtiles + mt;   // (qi, g) then mt
+  } else {
+    const int ntiles = a.Qn * a.hkv * a.mtiles;
+    for (int i = threadIdx.x; i < a.Qn; i += kThreads)
+      sp->npb[i] = (max(0, __ldg(&a.offs[i + 1]) - __ldg(&a.offs[i])) + kBN - 1) / kBN;
+    for (int i = threadIdx.x; i < a.mtiles; i += kThreads) sp->tcum[i + 1] = tile_own_blocks(a, i);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      sp->qcum[0] = 0;
+      for (int i = 0; i < a.Qn; ++i) sp->qcum[i + 1] = sp->qcum[i] + sp->npb[i];
+      sp->tcum[0] = 0;
+      for (int i = 0; i < a.mtiles; ++i) sp->tcum[i + 1] += sp->tcum[i];
+      sp->W = (long long)a.hkv *
+              ((long long)a.mtiles * sp->qcum[a.Qn] + (long long)a.Qn * sp->tcum[a.mtiles]);
+      const long long W = sp->W, grid = gridDim.x;
+      const long long x0 = (long long)blockIdx.x * W / grid, x1 = ((long long)blockIdx.x + 1) * W / grid;
+      // first tile whose list reaches past x0
+      int lo = 0, hi = ntiles;            // G0(lo) <= x0 < G0(hi)
+      while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (stream_g0(a, *sp, mid) <= x0) lo = mid; else hi = mid;
+      }
+      sp->t0 = lo;
+      // record {first slot, runs} of every tile whose first block lies in this range
+      for (int t = lo; t < ntiles; ++t) {
+        const long long g0 = stream_g0(a, *sp, t);
+        if (g0 >= x1) break;
+        if (g0 < x0) continue;
+        const long long g1 = stream_g0(a, *sp, t + 1);
+        const int parts = g1 > g0 ? stream_cta(g1 - 1, W, (int)grid) - stream_cta(g0, W, (int)grid) + 1 : 1;
+        a.tile_runs[t] = make_int2(t * a.maxparts, parts);
+      }
+    }
   }
-  const int P = max(0, __ldg(&a.offs[qi + 1]) - __ldg(&a.offs[qi]));
-  const int nbp = (P + kBN - 1) / kBN;                 // prefix blocks of this query
-  const int tok0 = mt * a.T;
-  const int ntok = min(a.T, a.KL - tok0);
-  const int rows = ntok * a.grp;
-  const int c_lo = tok0 / a.Lq;
-  const int ncand = (tok0 + ntok - 1) / a.Lq - c_lo + 1;
-  const int ntb = (ncand * a.C + kBN - 1) / kBN;       // blocks over the candidates' own slots
-  // valid own slots of the tile's candidates (the own blocks with none are skipped)
-  int* n_own = reinterpret_cast<int*>(drain_s + 1) + 4;
+  // segment s of this CTA (s = 0 only for the static and balanced plans); false past the last
+  auto segment = [&](int s, Seg& sg) -> bool {
+    if constexpr (!STREAM) {
+      if (s > 0) return false;
+      sg = seg0;
+      return true;
+    } else {
+      const int ntiles = a.Qn * a.hkv * a.mtiles;
+      const long long W = sp->W, grid = gridDim.x;
+      const long long x0 = (long long)blockIdx.x * W / grid, x1 = ((long long)blockIdx.x + 1) * W / grid;
+      const int t = sp->t0 + s;
+      if (t >= ntiles) return false;
+      const long long g0 = stream_g0(a, *sp, t);
+      if (g0 >= x1) return false;
+      const long long g1 = stream_g0(a, *sp, t + 1);
+      const long long lo = max(x0, g0), hi = min(x1, g1);
+      if (hi <= lo) return false;   // an empty range (more CTAs than blocks)
+      sg.t = t;
+      sg.blk_lo = (int)(lo - g0);
+      sg.nblk = (int)max(0LL, hi - lo);
+      const int cf = stream_cta(g0, W, (int)grid);
+      const int parts = g1 > g0 ? stream_cta(g1 - 1, W, (int)grid) - cf + 1 : 1;
+      sg.direct = parts == 1;
+      const int part = (int)blockIdx.x - cf;
+      sg.pslot = part < a.maxparts ? t * a.maxparts + part : -1;   // -1: no room (bad plan)
+      return true;
+    }
+  };
+  // the tile a segment covers
+  struct TileInfo {
+    int mt, g, qi, P, nbp, tok0, ntok, rows, c_lo, ncand, ntb;
+  };
+  auto tile_info = [&](int t) {
+    TileInfo ti;
+    ti.mt = t % a.mtiles;
+    ti.g = (t / a.mtiles) % a.hkv;
+    ti.qi = t / a.mtiles / a.hkv;
+    ti.P = max(0, __ldg(&a.offs[ti.qi + 1]) - __ldg(&a.offs[ti.qi]));
+    ti.nbp = (ti.P + kBN - 1) / kBN;               // prefix blocks of this query
+    ti.tok0 = ti.mt * a.T;
+    ti.ntok = min(a.T, a.KL - ti.tok0);
+    ti.rows = ti.ntok * a.grp;
+    ti.c_lo = ti.tok0 / a.Lq;
+    ti.ncand = (ti.tok0 + ti.ntok - 1) / a.Lq - ti.c_lo + 1;
+    ti.ntb = (ti.ncand * a.C + kBN - 1) / kBN;     // blocks over the candidates' own slots
+    return ti;
+  };
 
-  for (int c = threadIdx.x; c < ncand; c += kThreads) {
-    int n = a.own_len ? __ldg(&a.own_len[qi * a.K + c_lo + c]) : a.C;
-    n_own[c] = n < 0 ? 0 : (n > a.C ? a.C : n);
+  if constexpr (!STREAM) {
+    const TileInfo ti = tile_info(seg0.t);
+    for (int c = threadIdx.x; c < ti.ncand; c += kThreads) {
+      int n = a.own_len ? __ldg(&a.own_len[ti.qi * a.K + ti.c_lo + c]) : a.C;
+      n_own[c] = n < 0 ? 0 : (n > a.C ? a.C : n);
+    }
   }
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kKStages; ++s) {
       mbar_init(smem_u32(&k_full[s]), 1);
@@ -434,6 +575,8 @@ __global__ void __launch_bounds__(kThreads, 1)
     mbar_init(smem_u32(q_full), 1);
     mbar_init(smem_u32(drain), 1);
     mbar_init(smem_u32(drain_s), 1);
+    mbar_init(smem_u32(q_empty), 1);
+    mbar_init(smem_u32(o_free), 8);         // one arrival per softmax warp
     fence_barrier_init();
   }
   if (warp == 1) {
@@ -455,106 +598,132 @@ __global__ void __launch_bounds__(kThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_holder;
-  // own block tb holds a valid slot when some candidate c it overlaps has n_c > 0
-  // and c * C + n_c > tb * kBN (each candidate's valid slots are its first n_c)
-  auto own_valid = [&](int tb) {
-    const int s0 = tb * kBN;
-    const int s1 = min(s0 + kBN, ncand * a.C);
-    for (int c = s0 / a.C; c * a.C < s1; ++c)
-      if (n_own[c] > 0 && c * a.C + n_own[c] > s0) return true;
-    return false;
+  // own block tb of a tile holds a valid slot when some candidate c it overlaps has n_c > 0
+  // and c * C + n_c > tb * kBN (each candidate's valid slots are its first n_c); under the
+  // streamed plan every candidate has C valid slots, so every own block does
+  auto own_valid = [&](const TileInfo& ti, int tb) {
+    if constexpr (STREAM) {
+      return tb < ti.ntb;
+    } else {
+      const int s0 = tb * kBN;
+      const int s1 = min(s0 + kBN, ti.ncand * a.C);
+      for (int c = s0 / a.C; c * a.C < s1; ++c)
+        if (n_own[c] > 0 && c * a.C + n_own[c] > s0) return true;
+      return false;
+    }
   };
-  auto own_next = [&](int tb) {                      // first valid own block >= tb
-    while (tb < ntb && !own_valid(tb)) ++tb;
+  auto own_next = [&](const TileInfo& ti, int tb) {   // first valid own block >= tb
+    while (tb < ti.ntb && !own_valid(ti, tb)) ++tb;
     return tb;
   };
-  // count the valid own blocks, 32 per step of the warp (every warp computes the
-  // same values); this tile's list of nb blocks is cut into nsplit equal runs
-  int nvt = 0;
-  for (int base = 0; base < ntb; base += 32)
-    nvt += __popc(__ballot_sync(0xffffffffu, base + lane < ntb && own_valid(base + lane)));
-  const int nb = nbp + nvt;
-  int blk_lo, nblk;
-  if constexpr (BAL) {            // plan_run counted the same nb for this tile
-    blk_lo = wk.y;
-    nblk = wk.z;
-  } else {
-    const int bps = (nb + a.nsplit - 1) / a.nsplit;
-    blk_lo = split * bps;
-    nblk = max(0, min(nb, blk_lo + bps) - blk_lo);
-  }
-  const bool direct = BAL ? wk.w != 0 : a.nsplit == 1;   // this CTA writes the output
-  // the first own block this run uses: skip the valid own blocks of earlier runs
-  int tb_first = ntb;
-  {
-    int skip = max(0, blk_lo - nbp);
-    for (int base = 0; base < ntb; base += 32) {
-      const uint32_t m = __ballot_sync(0xffffffffu, base + lane < ntb && own_valid(base + lane));
+  // Single-run plans: every warp computes the run and its first own block (the valid own
+  // blocks of earlier runs of the tile are skipped) with the same warp votes.  The static
+  // split cuts the tile's list of nb blocks into nsplit equal runs here; the balanced plan
+  // fixed the run already.  The streamed plan's segments carry their runs, and every own
+  // block is valid there.
+  int tb_first0 = 0;
+  if constexpr (!STREAM) {
+    const TileInfo ti = tile_info(seg0.t);
+    int nvt = 0;
+    for (int base = 0; base < ti.ntb; base += 32)
+      nvt += __popc(__ballot_sync(0xffffffffu, base + lane < ti.ntb && own_valid(ti, base + lane)));
+    const int nb = ti.nbp + nvt;
+    if constexpr (BAL) {            // plan_run counted the same nb for this tile
+      seg0.blk_lo = wk.y;
+      seg0.nblk = wk.z;
+      seg0.direct = wk.w != 0;
+      seg0.pslot = blockIdx.x;
+    } else {
+      const int bps = (nb + a.nsplit - 1) / a.nsplit;
+      seg0.blk_lo = seg0.pslot * bps;
+      seg0.nblk = max(0, min(nb, seg0.blk_lo + bps) - seg0.blk_lo);
+      seg0.direct = a.nsplit == 1;
+    }
+    tb_first0 = ti.ntb;
+    int skip = max(0, seg0.blk_lo - ti.nbp);
+    for (int base = 0; base < ti.ntb; base += 32) {
+      const uint32_t m = __ballot_sync(0xffffffffu, base + lane < ti.ntb && own_valid(ti, base + lane));
       const int cnt = __popc(m);
       if (skip < cnt) {
         uint32_t mm = m;
         for (int i = 0; i < skip; ++i) mm &= mm - 1u;
-        tb_first = base + __ffs(mm) - 1;
+        tb_first0 = base + __ffs(mm) - 1;
         break;
       }
       skip -= cnt;
     }
   }
+  auto first_own = [&](const TileInfo& ti, const Seg& sg) {
+    return STREAM ? max(0, sg.blk_lo - ti.nbp) : tb_first0;
+  };
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
-    // K_0, V_0, K_1, V_1, ... (K is recycled after its S MMA, V after its PV MMA).
-    if (lane == 0 && nblk > 0) {
+    // Per segment: its Q tile (once the previous segment's S MMAs are done with the last
+    // one), then K_0, V_0, K_1, V_1, ... (K is recycled after its S MMA, V after its PV MMA).
+    // The rings and their phases run on over the CTA's whole sequence of blocks.
+    Seg sg;
+    int nk = 0, nv = 0, nq = 0;
+    bool fine = true;
+    for (int s = 0; fine && segment(s, sg); ++s) {
+      if (lane != 0 || sg.nblk == 0) continue;
+      const TileInfo ti = tile_info(sg.t);
+      const int tb_first = first_own(ti, sg);
       const uint64_t pol_kv = policy_evict_last();   // re-read by the other row tiles
       const uint64_t pol_q = policy_evict_first();
       const uint32_t qb = smem_u32(q_full);
+      if (nq > 0 && !mbar_wait(smem_u32(q_empty), (nq - 1) & 1, a.limit_ns)) {
+        fine = false;
+        break;
+      }
       mbar_arrive_expect_tx(qb, NH * a.grp * a.T * 128);
       for (int h = 0; h < NH; ++h)
-        tma_load_3d(smem_u32(q_s + h * kBM * 128), &tm_q, qb, h * 64, g * a.grp,
-                    qi * a.KL + tok0, pol_q);
-      const int pbase = __ldg(&a.offs[qi]);
-      const int tbase = (qi * a.K + c_lo) * a.C;       // own slot 0 of candidate c_lo
-      int nk = 0, nv = 0;
+        tma_load_3d(smem_u32(q_s + h * kBM * 128), &tm_q, qb, h * 64, ti.g * a.grp,
+                    ti.qi * a.KL + ti.tok0, pol_q);
+      ++nq;
+      const int pbase = __ldg(&a.offs[ti.qi]);
+      const int tbase = (ti.qi * a.K + ti.c_lo) * a.C;   // own slot 0 of candidate c_lo
       int tbk = tb_first, tbv = tb_first;               // own-block cursors of the two rings
       // Fixed order K_j, V_j with blocking waits (the waiting thread takes no issue slots
       // from the softmax warps on its sub-partition): K_j's slot frees when S_{j-2} is done,
       // V_j's when PV_{j-3} is done, both well before the block is needed.
-      auto load = [&](bool is_v, int j, int& tb) {
-        const uint32_t fb = smem_u32(is_v ? &v_full[j % kVStages] : &k_full[j % kKStages]);
+      auto load = [&](bool is_v, int jj, int j, int& tb) {
+        const uint32_t fb = smem_u32(is_v ? &v_full[jj % kVStages] : &k_full[jj % kKStages]);
         mbar_arrive_expect_tx(fb, Lay::kStage);
-        uint8_t* dst = is_v ? v_ring + (j % kVStages) * Lay::kStage : k_ring + (j % kKStages) * Lay::kStage;
-        const int bi = blk_lo + j;
-        const bool pre = bi < nbp;
+        uint8_t* dst = is_v ? v_ring + (jj % kVStages) * Lay::kStage : k_ring + (jj % kKStages) * Lay::kStage;
+        const int bi = sg.blk_lo + j;
+        const bool pre = bi < ti.nbp;
         int key;
         if (pre) {
           key = pbase + bi * kBN;
         } else {
-          tb = own_next(tb);
+          tb = own_next(ti, tb);
           key = tbase + tb * kBN;
           ++tb;
         }
         const CUtensorMap* tm = is_v ? (pre ? &tm_vp : &tm_vt) : (pre ? &tm_kp : &tm_kt);
         for (int h = 0; h < NH; ++h)
-          tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), tm, fb, h * 64, g, key, pol_kv);
+          tma_load_3d(smem_u32(dst + h * Lay::kKVHalf), tm, fb, h * 64, ti.g, key, pol_kv);
       };
-      bool fine = true;
-      for (int j = 0; j < nblk && fine; ++j) {
-        if (!mbar_wait(smem_u32(&k_empty[j % kKStages]), ((j / kKStages) & 1) ^ 1, a.limit_ns)) {
+      for (int j = 0; j < sg.nblk; ++j) {
+        if (!mbar_wait(smem_u32(&k_empty[nk % kKStages]), ((nk / kKStages) & 1) ^ 1, a.limit_ns)) {
           fine = false;
           break;
         }
-        load(false, j, tbk);
+        load(false, nk, j, tbk);
         ++nk;
-        if (!mbar_wait(smem_u32(&v_empty[j % kVStages]), ((j / kVStages) & 1) ^ 1, a.limit_ns)) {
+        if (!mbar_wait(smem_u32(&v_empty[nv % kVStages]), ((nv / kVStages) & 1) ^ 1, a.limit_ns)) {
           fine = false;
           break;
         }
-        load(true, j, tbv);
+        load(true, nv, j, tbv);
         ++nv;
       }
+    }
+    if (lane == 0) {
       if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteProducer);
       // no copy may still be in flight when the CTA exits
-      mbar_wait(qb, 0, a.limit_ns);
+      if (nq > 0) mbar_wait(smem_u32(q_full), (nq - 1) & 1, a.limit_ns);
       for (int i = max(0, nk - kKStages); i < nk; ++i)
         mbar_wait(smem_u32(&k_full[i % kKStages]), (i / kKStages) & 1, a.limit_ns);
       for (int i = max(0, nv - kVStages); i < nv; ++i)
@@ -567,26 +736,37 @@ __global__ void __launch_bounds__(kThreads, 1)
     // The S MMAs come from another thread (warp kWarpS), so neither kind of MMA waits
     // behind the other's inputs: the S issuer waits for PV_j to finish before it reuses
     // P_j's buffer while this thread already has PV_{j+1} queued, and the tensor pipe is
-    // never drained between blocks.
-    if (lane == 0 && nblk > 0) {
+    // never drained between blocks.  A segment's first PV starts O afresh, once the
+    // softmax warps have read the previous segment's O.
+    if (lane == 0) {
       const uint32_t idPV = idesc_bf16_f32(kBM, D) | (1u << 16);   // B (= V) MN-major
       bool fine = true;
-      for (int np = 0; np < nblk && fine; ++np) {
-        if (!mbar_wait(smem_u32(&p_full[np % kSP]), (np / kSP) & 1, a.limit_ns) ||
-            !mbar_wait(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1, a.limit_ns)) {
+      Seg sg;
+      int np = 0, nseg = 0;
+      for (int s = 0; fine && segment(s, sg); ++s) {
+        if (sg.nblk == 0) continue;
+        if (nseg > 0 && !mbar_wait(smem_u32(o_free), (nseg - 1) & 1, a.limit_ns)) {
           fine = false;
           break;
         }
-        tc_fence_after();
-        const uint32_t pa = tmem_base + col_s(np % kSP);
-        const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
+        ++nseg;
+        for (int j = 0; j < sg.nblk; ++j, ++np) {
+          if (!mbar_wait(smem_u32(&p_full[np % kSP]), (np / kSP) & 1, a.limit_ns) ||
+              !mbar_wait(smem_u32(&v_full[np % kVStages]), (np / kVStages) & 1, a.limit_ns)) {
+            fine = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t pa = tmem_base + col_s(np % kSP);
+          const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
 #pragma unroll
-        for (int k16 = 0; k16 < kBN / 16; ++k16)
-          tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
-                         desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
-                         (np | k16) != 0);
-        tc_commit(smem_u32(&pv_done[np % kSP]));
-        tc_commit(smem_u32(&v_empty[np % kVStages]));
+          for (int k16 = 0; k16 < kBN / 16; ++k16)
+            tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
+                           desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
+                           (j | k16) != 0);
+          tc_commit(smem_u32(&pv_done[np % kSP]));
+          tc_commit(smem_u32(&v_empty[np % kVStages]));
+        }
       }
       if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
       tc_commit(smem_u32(drain));
@@ -596,29 +776,41 @@ __global__ void __launch_bounds__(kThreads, 1)
   } else if (warp == kWarpS) {
     // ------------------------------------------------------------ S issuer
     //   S_j = Q K_j^T  into S/P buffer j % kSP, once K_j is in and PV_{j-kSP} (the previous
-    //                  user of that buffer) is done; its commit frees K_j's stage.
-    if (lane == 0 && nblk > 0) {
+    //                  user of that buffer) is done; its commit frees K_j's stage.  After a
+    //                  segment's last S its Q tile is released for the next segment's.
+    if (lane == 0) {
       const uint32_t idS = idesc_bf16_f32(kBM, kBN);
       const uint32_t qa = smem_u32(q_s);
-      bool fine = mbar_wait(smem_u32(q_full), 0, a.limit_ns);
-      if (!fine) record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
-      for (int ns = 0; ns < nblk && fine; ++ns) {
-        if (!mbar_wait(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1, a.limit_ns) ||
-            !mbar_wait(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1, a.limit_ns)) {
-          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
+      bool fine = true;
+      Seg sg;
+      int ns = 0, nq = 0;
+      for (int s = 0; fine && segment(s, sg); ++s) {
+        if (sg.nblk == 0) continue;
+        if (!mbar_wait(smem_u32(q_full), nq & 1, a.limit_ns)) {
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteQ);
           fine = false;
           break;
         }
-        tc_fence_after();
-        const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
+        ++nq;
+        for (int j = 0; j < sg.nblk; ++j, ++ns) {
+          if (!mbar_wait(smem_u32(&k_full[ns % kKStages]), (ns / kKStages) & 1, a.limit_ns) ||
+              !mbar_wait(smem_u32(&pv_done[ns % kSP]), ((ns / kSP) & 1) ^ 1, a.limit_ns)) {
+            record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteMma);
+            fine = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t ks = smem_u32(k_ring + (ns % kKStages) * Lay::kStage);
 #pragma unroll
-        for (int h = 0; h < NH; ++h)
+          for (int h = 0; h < NH; ++h)
 #pragma unroll
-          for (int k16 = 0; k16 < 4; ++k16)
-            tc_mma_bf16(tmem_base + col_s(ns % kSP), desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
-                        desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS, (h | k16) != 0);
-        tc_commit(smem_u32(&s_full[ns % kSP]));
-        tc_commit(smem_u32(&k_empty[ns % kKStages]));
+            for (int k16 = 0; k16 < 4; ++k16)
+              tc_mma_bf16(tmem_base + col_s(ns % kSP), desc_kmajor_sw128(qa + h * kBM * 128 + k16 * 32),
+                          desc_kmajor_sw128(ks + h * Lay::kKVHalf + k16 * 32), idS, (h | k16) != 0);
+          tc_commit(smem_u32(&s_full[ns % kSP]));
+          tc_commit(smem_u32(&k_empty[ns % kKStages]));
+        }
+        tc_commit(smem_u32(q_empty));
       }
       tc_commit(smem_u32(drain_s));
       if (!mbar_wait(smem_u32(drain_s), 0, a.limit_ns))
@@ -641,230 +833,246 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int half = (warp - 2) >> 2;
     const int r = quarter * 32 + lane;                 // tile row = tensor-memory lane
     const uint32_t lane_base = tmem_base + ((uint32_t)(quarter * 32) << 16);
-    const bool rvalid = r < rows;
-    const int tok = tok0 + r / a.grp;
-    const int crow = min(tok / a.Lq - c_lo, ncand - 1);  // rows past the tile: any candidate
-    const int lrow = tok % a.Lq;
-    // visible own slots of this row, in the tile's concatenated own-slot space
-    const int tlo = crow * a.C;
-    const int thi = tlo + max(0, n_own[crow] - a.Lq + lrow + 1);
-    int tbs = tb_first;                                // own-block cursor
-    float m_ref = -INFINITY, l = 0.f;
-    bool ok = true;
     auto pair_sync = [&]() {                           // the two warps of this quarter
       asm volatile("bar.sync %0, 64;" ::"r"(1 + quarter) : "memory");
     };
-    for (int j = 0; j < nblk; ++j) {
-      const int sb = j % kSP;
-      // `ok` stays warp-uniform (the warp votes on every bounded wait), so a timed-out
-      // warp still meets its partner at every barrier below and the kernel drains
-      if (ok && !__all_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[sb]), (j / kSP) & 1, a.limit_ns))) {
-        record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteSFull);
-        ok = false;
-      }
-      tc_fence_after();
-      uint32_t sr[kHalf];
-      if (ok) {
-        static_assert(kHalf == 64, "one 64-column load per warp and block");
-        tmem_ld_32x32b_x64(lane_base + col_s(sb) + half * kHalf, sr);
-        tmem_wait_ld();
-      } else {
-#pragma unroll
-        for (int c = 0; c < kHalf; ++c) sr[c] = 0u;
-      }
-      int vlo, vhi;   // valid columns of this block for this row
-      if (blk_lo + j < nbp) {
-        vlo = 0;
-        vhi = min(kBN, P - (blk_lo + j) * kBN);
-      } else {
-        tbs = own_next(tbs);
-        const int base = tbs * kBN;
-        ++tbs;
-        vlo = max(0, tlo - base);
-        vhi = min(kBN, thi - base);
-      }
-      // this warp's columns are [c_off, c_off + kHalf) of the block
-      const int c_off = half * kHalf;
-      vlo -= c_off;
-      vhi -= c_off;
-      // rows without output (r >= rows) are not masked: their values are finite and
-      // discarded, and masking them would split the warp between the two paths below
-      const bool full = vlo <= 0 && vhi >= kHalf;
-      // P_j relative to the reference `mref`: bf16 pairs into pk (written over the first 64
-      // columns of the same buffer; S_j is in registers), the partial sum into rs
-      uint32_t pk[32];
-      float rs = 0.f;
-      // kMask: 0 = no masking, 1 = mask every element, 2 = mask when the block is not full
-      auto exp_pass_t = [&](float mref, auto mask_mode) {
-        constexpr int kMask = decltype(mask_mode)::value;
-        const float ms = mref == -INFINITY ? 0.f : mref;
-        // exponent arguments s * scale - m and the running sums in packed pairs
-        const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-ms, -ms);
-        uint64_t rsp2[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) rsp2[u] = 0ull;   // (+0.f, +0.f)
-#pragma unroll
-        for (int c = 0; c < kHalf; c += 2) {
-          float t0, t1;
-          f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sc2, nm2),
-                    t0, t1);
-          float e0 = ex2(t0);
-          float e1 = ex2(t1);
-          if (kMask == 1 || (kMask == 2 && !full)) {
-            e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
-            e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
-          }
-          rsp2[(c / 2) & 3] = f2_add(rsp2[(c / 2) & 3], f2_pack(e0, e1));
-          pk[c / 2] = pack_bf16(e0, e1);
-        }
-        float rsp[8];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) f2_unpack(rsp2[u], rsp[2 * u], rsp[2 * u + 1]);
-        rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
-      };
-      // Verification: full blocks (almost all of them) run a copy of the loop without the
-      // masking selects, which the compiler otherwise keeps in the loop as predicated
-      // instructions (long 145.9 -> 133.6 us per call).  Decode (the balanced plan), whose own
-      // blocks are mostly partial, keeps the one loop with the test inside (74.2 us
-      // unswitched against 71.7).
-      auto exp_pass = [&](float mref) {
-        if constexpr (BAL) {
-          exp_pass_t(mref, std::integral_constant<int, 2>{});
-        } else {
-          if (full)
-            exp_pass_t(mref, std::integral_constant<int, 0>{});
-          else
-            exp_pass_t(mref, std::integral_constant<int, 1>{});
-        }
-      };
-      // Once every row of the warp has a reference, the block max is not computed: all
-      // terms of the partial sum are positive, so rs <= 2^kRescaleLog2 shows that no term
-      // of this half ran past the limit.  A row without a reference, or a larger sum, in
-      // either warp of the quarter sends both into the path that computes the block max
-      // (the two halves of a row must keep one reference).
-      const bool fresh = __any_sync(0xffffffffu, m_ref == -INFINITY);
-      if (!fresh) exp_pass(m_ref);
-      const bool mine = fresh || __any_sync(0xffffffffu, !(rs <= kSumLimit));
-      int* xf = xflag + ((j & 1) * 2 + half) * 4;      // [2 slots][2 halves][4 quarters]
-      if (lane == 0) xf[quarter] = mine ? 1 : 0;
-      tc_fence_before();          // this warp's S loads are complete before the partner
-      pair_sync();                // writes its P over them
-      tc_fence_after();
-      const bool slow = mine || xflag[((j & 1) * 2 + (half ^ 1)) * 4 + quarter] != 0;
-      bool resc = false;
-      float corr = 1.f;
-      if (slow) {
-        float pm[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
-        if (full) {
-#pragma unroll
-          for (int c = 0; c < kHalf; c += 2)
-            pm[(c / 2) & 7] = max3(pm[(c / 2) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
-        } else {
-#pragma unroll
-          for (int c = 0; c < kHalf; ++c)
-            if (c >= vlo && c < vhi) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
-        }
-        float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
-                           fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
-        // block max over both halves (slots by block parity: the next use of a slot comes
-        // after two more flag barriers)
-        float* xs = xmax + (j & 1) * 2 * kBM;
-        xs[half * kBM + r] = hmax;
-        pair_sync();
-        hmax = fmaxf(hmax, xs[(half ^ 1) * kBM + r]);
-        const float bmax = a.scale_log2 * hmax;
-        const float m_old = m_ref;
-        if (bmax > m_ref + kRescaleLog2) m_ref = bmax;   // also the first finite block
-        resc = m_ref != m_old && m_old != -INFINITY;
-        corr = resc ? ex2(m_old - m_ref) : 1.f;
-        if (fresh || __any_sync(0xffffffffu, m_ref != m_old)) exp_pass(m_ref);
-      }
-      if (ok) tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(half * kHalf / 2), pk);
-      l = l * corr + rs;
-      if (ok && __any_sync(0xffffffffu, resc)) {
-        // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale
-        const int i = j - 1;
-        if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))) {
-          record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
+    bool ok = true;
+    Seg sg;
+    int J = 0;                                         // blocks of earlier segments
+    for (int s = 0; segment(s, sg); ++s) {
+      const TileInfo ti = tile_info(sg.t);
+      const int tb_first = first_own(ti, sg);
+      const bool rvalid = r < ti.rows;
+      const int tok = ti.tok0 + r / a.grp;
+      const int crow = min(tok / a.Lq - ti.c_lo, ti.ncand - 1);  // rows past the tile: any candidate
+      const int lrow = tok % a.Lq;
+      // visible own slots of this row, in the tile's concatenated own-slot space
+      const int tlo = crow * a.C;
+      const int thi = tlo + max(0, (STREAM ? a.C : n_own[crow]) - a.Lq + lrow + 1);
+      int tbs = tb_first;                                // own-block cursor
+      float m_ref = -INFINITY, l = 0.f;
+      for (int j = 0; j < sg.nblk; ++j) {
+        const int jj = J + j;                            // position in the CTA's sequence
+        const int sb = jj % kSP;
+        // `ok` stays warp-uniform (the warp votes on every bounded wait), so a timed-out
+        // warp still meets its partner at every barrier below and the kernel drains
+        if (ok && !__all_sync(0xffffffffu, mbar_wait(smem_u32(&s_full[sb]), (jj / kSP) & 1, a.limit_ns))) {
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSiteSFull);
           ok = false;
+        }
+        tc_fence_after();
+        uint32_t sr[kHalf];
+        if (ok) {
+          static_assert(kHalf == 64, "one 64-column load per warp and block");
+          tmem_ld_32x32b_x64(lane_base + col_s(sb) + half * kHalf, sr);
+          tmem_wait_ld();
         } else {
-          tc_fence_after();
 #pragma unroll
-          for (int c0 = 0; c0 < kOHalf; c0 += 32) {
-            uint32_t o[32];
-            tmem_ld_32x32b_x32(lane_base + kColO + half * kOHalf + c0, o);
-            tmem_wait_ld();
+          for (int c = 0; c < kHalf; ++c) sr[c] = 0u;
+        }
+        int vlo, vhi;   // valid columns of this block for this row
+        if (sg.blk_lo + j < ti.nbp) {
+          vlo = 0;
+          vhi = min(kBN, ti.P - (sg.blk_lo + j) * kBN);
+        } else {
+          tbs = own_next(ti, tbs);
+          const int base = tbs * kBN;
+          ++tbs;
+          vlo = max(0, tlo - base);
+          vhi = min(kBN, thi - base);
+        }
+        // this warp's columns are [c_off, c_off + kHalf) of the block
+        const int c_off = half * kHalf;
+        vlo -= c_off;
+        vhi -= c_off;
+        // rows without output (r >= rows) are not masked: their values are finite and
+        // discarded, and masking them would split the warp between the two paths below
+        const bool full = vlo <= 0 && vhi >= kHalf;
+        // P_j relative to the reference `mref`: bf16 pairs into pk (written over the first 64
+        // columns of the same buffer; S_j is in registers), the partial sum into rs
+        uint32_t pk[32];
+        float rs = 0.f;
+        // kMask: 0 = no masking, 1 = mask every element, 2 = mask when the block is not full
+        auto exp_pass_t = [&](float mref, auto mask_mode) {
+          constexpr int kMask = decltype(mask_mode)::value;
+          const float ms = mref == -INFINITY ? 0.f : mref;
+          // exponent arguments s * scale - m and the running sums in packed pairs
+          const uint64_t sc2 = f2_pack(a.scale_log2, a.scale_log2), nm2 = f2_pack(-ms, -ms);
+          uint64_t rsp2[4];
 #pragma unroll
-            for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
-            tmem_st_32x32b_x32(lane_base + kColO + half * kOHalf + c0, o);
+          for (int u = 0; u < 4; ++u) rsp2[u] = 0ull;   // (+0.f, +0.f)
+#pragma unroll
+          for (int c = 0; c < kHalf; c += 2) {
+            float t0, t1;
+            f2_unpack(f2_fma(f2_pack(__uint_as_float(sr[c]), __uint_as_float(sr[c + 1])), sc2, nm2),
+                      t0, t1);
+            float e0 = ex2(t0);
+            float e1 = ex2(t1);
+            if (kMask == 1 || (kMask == 2 && !full)) {
+              e0 = (c >= vlo && c < vhi) ? e0 : 0.f;
+              e1 = (c + 1 >= vlo && c + 1 < vhi) ? e1 : 0.f;
+            }
+            rsp2[(c / 2) & 3] = f2_add(rsp2[(c / 2) & 3], f2_pack(e0, e1));
+            pk[c / 2] = pack_bf16(e0, e1);
+          }
+          float rsp[8];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) f2_unpack(rsp2[u], rsp[2 * u], rsp[2 * u + 1]);
+          rs = ((rsp[0] + rsp[1]) + (rsp[2] + rsp[3])) + ((rsp[4] + rsp[5]) + (rsp[6] + rsp[7]));
+        };
+        // Verification: full blocks (almost all of them) run a copy of the loop without the
+        // masking selects, which the compiler otherwise keeps in the loop as predicated
+        // instructions (long 145.9 -> 133.6 us per call).  Decode (the balanced plan), whose own
+        // blocks are mostly partial, keeps the one loop with the test inside (74.2 us
+        // unswitched against 71.7).
+        auto exp_pass = [&](float mref) {
+          if constexpr (BAL) {
+            exp_pass_t(mref, std::integral_constant<int, 2>{});
+          } else {
+            if (full)
+              exp_pass_t(mref, std::integral_constant<int, 0>{});
+            else
+              exp_pass_t(mref, std::integral_constant<int, 1>{});
+          }
+        };
+        // Once every row of the warp has a reference, the block max is not computed: all
+        // terms of the partial sum are positive, so rs <= 2^kRescaleLog2 shows that no term
+        // of this half ran past the limit.  A row without a reference, or a larger sum, in
+        // either warp of the quarter sends both into the path that computes the block max
+        // (the two halves of a row must keep one reference).
+        const bool fresh = __any_sync(0xffffffffu, m_ref == -INFINITY);
+        if (!fresh) exp_pass(m_ref);
+        const bool mine = fresh || __any_sync(0xffffffffu, !(rs <= kSumLimit));
+        int* xf = xflag + ((jj & 1) * 2 + half) * 4;     // [2 slots][2 halves][4 quarters]
+        if (lane == 0) xf[quarter] = mine ? 1 : 0;
+        tc_fence_before();          // this warp's S loads are complete before the partner
+        pair_sync();                // writes its P over them
+        tc_fence_after();
+        const bool slow = mine || xflag[((jj & 1) * 2 + (half ^ 1)) * 4 + quarter] != 0;
+        bool resc = false;
+        float corr = 1.f;
+        if (slow) {
+          float pm[8];
+#pragma unroll
+          for (int u = 0; u < 8; ++u) pm[u] = -INFINITY;
+          if (full) {
+#pragma unroll
+            for (int c = 0; c < kHalf; c += 2)
+              pm[(c / 2) & 7] = max3(pm[(c / 2) & 7], __uint_as_float(sr[c]), __uint_as_float(sr[c + 1]));
+          } else {
+#pragma unroll
+            for (int c = 0; c < kHalf; ++c)
+              if (c >= vlo && c < vhi) pm[c & 7] = fmaxf(pm[c & 7], __uint_as_float(sr[c]));
+          }
+          float hmax = fmaxf(fmaxf(fmaxf(pm[0], pm[1]), fmaxf(pm[2], pm[3])),
+                             fmaxf(fmaxf(pm[4], pm[5]), fmaxf(pm[6], pm[7])));
+          // block max over both halves (slots by block parity: the next use of a slot comes
+          // after two more flag barriers)
+          float* xs = xmax + (jj & 1) * 2 * kBM;
+          xs[half * kBM + r] = hmax;
+          pair_sync();
+          hmax = fmaxf(hmax, xs[(half ^ 1) * kBM + r]);
+          const float bmax = a.scale_log2 * hmax;
+          const float m_old = m_ref;
+          if (bmax > m_ref + kRescaleLog2) m_ref = bmax;   // also the first finite block
+          resc = m_ref != m_old && m_old != -INFINITY;
+          corr = resc ? ex2(m_old - m_ref) : 1.f;
+          if (fresh || __any_sync(0xffffffffu, m_ref != m_old)) exp_pass(m_ref);
+        }
+        if (ok) tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(half * kHalf / 2), pk);
+        l = l * corr + rs;
+        if (ok && __any_sync(0xffffffffu, resc)) {
+          // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale
+          const int i = jj - 1;
+          if (!__all_sync(0xffffffffu, mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))) {
+            record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
+            ok = false;
+          } else {
+            tc_fence_after();
+#pragma unroll
+            for (int c0 = 0; c0 < kOHalf; c0 += 32) {
+              uint32_t o[32];
+              tmem_ld_32x32b_x32(lane_base + kColO + half * kOHalf + c0, o);
+              tmem_wait_ld();
+#pragma unroll
+              for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * corr);
+              tmem_st_32x32b_x32(lane_base + kColO + half * kOHalf + c0, o);
+            }
+          }
+        }
+        tmem_wait_st();
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(smem_u32(&p_full[sb]));
+      }
+      // ---- epilogue: wait for the last PV, add the two halves' sums, normalise O by l
+      if (ok && sg.nblk > 0) {
+        const int i = J + sg.nblk - 1;
+        if (!mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))
+          record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
+        tc_fence_after();
+      }
+      xsum[half * kBM + r] = l;
+      pair_sync();
+      l += xsum[(half ^ 1) * kBM + r];
+      const int head = ti.g * a.grp + r % a.grp;
+      const size_t rowid = ((size_t)ti.qi * a.KL + tok) * a.hq + head;
+      const size_t nrows = (size_t)a.Qn * a.KL * a.hq;
+      // partial slot of this row: [slot][row of the tile] (balanced and streamed plans) or
+      // [split][row] (static split)
+      const bool store = sg.direct || MODE == 0 || sg.pslot >= 0;
+      const size_t pidx = MODE == 0 ? (size_t)sg.pslot * nrows + rowid
+                                    : (size_t)max(sg.pslot, 0) * a.slot_rows + r;
+      const bool any = l > 0.f;
+      const float inv = any ? 1.f / l : 0.f;
+      const float lse = any ? kLn2 * (m_ref + __log2f(l)) : -INFINITY;
+#pragma unroll
+      for (int c0 = 0; c0 < kOHalf; c0 += 32) {
+        const int oc = half * kOHalf + c0;               // O column of this chunk
+        uint32_t o[32];
+        if (sg.nblk > 0) {
+          tmem_ld_32x32b_x32(lane_base + kColO + oc, o);
+          tmem_wait_ld();
+        } else {
+#pragma unroll
+          for (int c = 0; c < 32; ++c) o[c] = 0u;
+        }
+        if (rvalid && store) {
+          if (sg.direct) {
+            uint4* dst = reinterpret_cast<uint4*>(a.out + rowid * D + oc);
+#pragma unroll
+            for (int c = 0; c < 32; c += 8)
+              dst[c / 8] = make_uint4(
+                  pack_bf16(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
+                  pack_bf16(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
+                  pack_bf16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
+                  pack_bf16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
+          } else {
+            uint4* dst = reinterpret_cast<uint4*>(a.part_o + pidx * D + oc);
+#pragma unroll
+            for (int c = 0; c < 32; c += 8)
+              dst[c / 8] = make_uint4(
+                  pack_f16(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
+                  pack_f16(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
+                  pack_f16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
+                  pack_f16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
           }
         }
       }
-      tmem_wait_st();
+      if (rvalid && half == 0 && store) {
+        if (sg.direct) {
+          if (a.lse) a.lse[rowid] = lse;
+        } else {
+          a.part_lse[pidx] = lse;
+        }
+      }
+      if (!store && lane == 0 && half == 0 && quarter == 0)
+        record_error(a.status, FVRAG_ERR_UNSUPPORTED, kSitePlan);
+      // O has been read: the next segment's first PV may overwrite it
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(smem_u32(&p_full[sb]));
-    }
-    // ---- epilogue: wait for the last PV, add the two halves' sums, normalise O by l
-    if (ok && nblk > 0) {
-      const int i = nblk - 1;
-      if (!mbar_wait(smem_u32(&pv_done[i % kSP]), (i / kSP) & 1, a.limit_ns))
-        record_error(a.status, FVRAG_ERR_TIMEOUT, kSitePvDone);
-      tc_fence_after();
-    }
-    xsum[half * kBM + r] = l;
-    pair_sync();
-    l += xsum[(half ^ 1) * kBM + r];
-    const int head = g * a.grp + r % a.grp;
-    const size_t rowid = ((size_t)qi * a.KL + tok) * a.hq + head;
-    const size_t nrows = (size_t)a.Qn * a.KL * a.hq;
-    // partial slot of this row: [run][row of the tile] (balanced plan) or [split][row]
-    const size_t pidx =
-        BAL ? (size_t)blockIdx.x * a.slot_rows + r : (size_t)split * nrows + rowid;
-    const bool any = l > 0.f;
-    const float inv = any ? 1.f / l : 0.f;
-    const float lse = any ? kLn2 * (m_ref + __log2f(l)) : -INFINITY;
-#pragma unroll
-    for (int c0 = 0; c0 < kOHalf; c0 += 32) {
-      const int oc = half * kOHalf + c0;               // O column of this chunk
-      uint32_t o[32];
-      if (nblk > 0) {
-        tmem_ld_32x32b_x32(lane_base + kColO + oc, o);
-        tmem_wait_ld();
-      } else {
-#pragma unroll
-        for (int c = 0; c < 32; ++c) o[c] = 0u;
-      }
-      if (rvalid) {
-        if (direct) {
-          uint4* dst = reinterpret_cast<uint4*>(a.out + rowid * D + oc);
-#pragma unroll
-          for (int c = 0; c < 32; c += 8)
-            dst[c / 8] = make_uint4(
-                pack_bf16(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
-                pack_bf16(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
-                pack_bf16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
-                pack_bf16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
-        } else {
-          uint4* dst = reinterpret_cast<uint4*>(a.part_o + pidx * D + oc);
-#pragma unroll
-          for (int c = 0; c < 32; c += 8)
-            dst[c / 8] = make_uint4(
-                pack_f16(__uint_as_float(o[c]) * inv, __uint_as_float(o[c + 1]) * inv),
-                pack_f16(__uint_as_float(o[c + 2]) * inv, __uint_as_float(o[c + 3]) * inv),
-                pack_f16(__uint_as_float(o[c + 4]) * inv, __uint_as_float(o[c + 5]) * inv),
-                pack_f16(__uint_as_float(o[c + 6]) * inv, __uint_as_float(o[c + 7]) * inv));
-        }
-      }
-    }
-    if (rvalid && half == 0) {
-      if (direct) {
-        if (a.lse) a.lse[rowid] = lse;
-      } else {
-        a.part_lse[pidx] = lse;
-      }
+      if (lane == 0) mbar_arrive(smem_u32(o_free));
+      J += sg.nblk;
     }
   }
   griddep_launch_dependents();
@@ -969,38 +1177,72 @@ struct Problem {
   float scale;                 // 0 => 1/sqrt(D)
   const int32_t* own_len;      // device [Qn][K] or null (every candidate has C valid slots)
   bool ragged;                 // the valid own slots n_k are read from the device
+  uint32_t split;              // FVRAG_ATTN_SPLIT_* request (verification), 0 = by the cost model
 };
 
 struct Plan {
   int grp, T, mtiles, nsplit;
+  bool stream;             // the streamed plan (grid CTAs, maxparts partial slots per tile)
+  int grid, maxparts;
+  bool unsupported;        // the streamed plan was requested but cannot serve the problem
 };
 
-// Key-split plan: every row tile's block list (its query's prefix blocks plus the
-// own blocks of its candidates) is cut on the device into nsplit equal runs, one
-// CTA each, so a short ragged prefix gives short CTAs that the block scheduler
-// backfills.  Pick nsplit to minimise an estimate of the time: the larger of the
-// mean work per SM (waves x mean run, three blocks added per run for its prologue and
-// epilogue) and the longest run, plus the cost of writing and merging the fp16
-// partials.  The constants (~0.8 us per 128-key block; per split count, a fixed 20 us
-// and the partials written and read at ~3 TB/s) were fitted on GB300 to per-call times
-// measured at every split
-// count from 1 to 12 on the 72B-class, long-context and batch-16 workloads, where they
-// pick the fastest measured split (5, 5 and 1).
+// L2 capacity of the current device (cached per device; 126.5 MB if it cannot be read).
+static double l2_bytes() {
+  static double cached[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 126.5e6;
+  if (cached[dev] == 0) {
+    int v = 0;
+    cached[dev] = cudaDeviceGetAttribute(&v, cudaDevAttrL2CacheSize, dev) == cudaSuccess && v > 0
+                      ? (double)v : 126.5e6;
+  }
+  return cached[dev];
+}
+
+// Own blocks of row tile mt (every candidate with all C slots valid).
+static int own_blocks(const Problem& pr, const Plan& p, int mt) {
+  const int KL = pr.K * pr.Lq;
+  const int tok0 = mt * p.T;
+  const int ntok = std::min(p.T, KL - tok0);
+  const int c_lo = tok0 / pr.Lq;
+  const int ncand = (tok0 + ntok - 1) / pr.Lq - c_lo + 1;
+  return (ncand * pr.C + kBN - 1) / kBN;
+}
+
+// Key-split plan.  Static split: every row tile's block list (its query's prefix blocks
+// plus the own blocks of its candidates) is cut on the device into nsplit equal runs, one
+// CTA each, so a short ragged prefix gives short CTAs that the block scheduler backfills.
+// Streamed plan (verification only): each of `grid` CTAs takes an equal share of all tiles'
+// blocks in one wave.  Pick the plan with the smaller estimate of the time: for the static
+// split the larger of the mean work per SM (waves x mean run, three blocks added per run for
+// its prologue and epilogue) and the longest run, for the streamed plan its share; plus the
+// cost of writing and merging the fp16 partials.  The constants (~0.8 us per 128-key block;
+// per split count, a fixed 20 us and the partials written and read at ~3 TB/s) were fitted
+// on GB300 to per-call times of the static split measured at every split count from 1 to 12
+// on the 72B-class, long-context and batch-16 workloads; the streamed plan's terms to its
+// times on the same workloads (72B-class: 158 us against the static split's 181 us; long
+// context: 117 against 111 us; batch-16, whose K/V does not fit L2: 233 against 177 us).
 static Plan make_plan(const Problem& pr, int sms) {
   Plan p;
   p.grp = pr.hq / pr.hkv;
   p.T = std::max(1, kBM / p.grp);
   const int KL = pr.K * pr.Lq;
   p.mtiles = (KL + p.T - 1) / p.T;
+  p.stream = false;
+  p.grid = 0;
+  p.maxparts = 1;
+  p.unsupported = false;
   const long long base = (long long)pr.Qn * pr.hkv * p.mtiles;
   const int ncand = std::min(pr.K, (p.T + pr.Lq - 1) / pr.Lq + 1);
   const int nb_own = (int)(((long long)ncand * pr.C + kBN - 1) / kBN);
   const int nb = (std::max(pr.max_prefix, 0) + kBN - 1) / kBN + nb_own;
   const double nb_mean = std::ceil((double)std::max(pr.total_prefix, 0) / pr.Qn / kBN) + nb_own;
   p.nsplit = 1;
-  if (nb <= 1) return p;
   if (sms <= 0) sms = 148;
+  if (nb <= 1 && pr.split != FVRAG_ATTN_SPLIT_STREAM) return p;
   const double rows = (double)pr.Qn * KL * pr.hq;
+  auto merge_us = [&](double ns) { return 20.0 + ns * rows * (pr.D * 2 + 4) * 2.0 / 3.0e6; };
   double best = 1e30;
   for (int ns = 1; ns <= std::min(nb, 64); ++ns) {
     const long long ctas = base * ns;
@@ -1008,12 +1250,53 @@ static Plan make_plan(const Problem& pr, int sms) {
     const double t_mean = waves * (std::ceil(nb_mean / ns) + 3);
     const double t_max = std::ceil((double)nb / ns) + 3;
     double t = std::max(t_mean, t_max) * 0.8;
-    if (ns > 1) t += 20.0 + ns * rows * (pr.D * 2 + 4) * 2.0 / 3.0e6;
+    if (ns > 1) t += merge_us(ns);
     if (t < best - 1e-9) {
       best = t;
       p.nsplit = ns;
     }
   }
+  // the streamed plan's CTAs read different K/V blocks of a KV head at the same time, so it
+  // needs every query's prefix K/V resident in L2 (3/4 of it) to keep one HBM read per block
+  const double kv_bytes = 4.0 * pr.hkv * pr.D * (double)std::max(pr.total_prefix, 0);
+  const bool want_stream = pr.split == FVRAG_ATTN_SPLIT_STREAM;
+  if (want_stream) best = 1e30;            // requested: no comparison with the static split
+  if (pr.split == FVRAG_ATTN_SPLIT_STATIC) {
+    // requested: the static split as chosen above
+  } else if (!pr.ragged && pr.Qn <= kMaxStreamQueries && p.mtiles <= kMaxStreamMtiles &&
+             (want_stream || kv_bytes <= 0.75 * l2_bytes())) {
+    long long ntb_all = 0;
+    int ntb_max = 0;
+    for (int mt = 0; mt < p.mtiles; ++mt) {
+      const int b = own_blocks(pr, p, mt);
+      ntb_all += b;
+      ntb_max = std::max(ntb_max, b);
+    }
+    // sum over queries of ceil(P_q / 128) lies between these two (P_q sum to total_prefix)
+    const long long tp = std::max(pr.total_prefix, 0);
+    const long long pre_lb = (tp + kBN - 1) / kBN;
+    const long long pre_ub = (tp + (long long)pr.Qn * (kBN - 1)) / kBN;
+    const long long w_lb = (long long)pr.hkv * (p.mtiles * pre_lb + (long long)pr.Qn * ntb_all);
+    const long long w_ub = (long long)pr.hkv * (p.mtiles * pre_ub + (long long)pr.Qn * ntb_all);
+    const int grid = (int)std::max(1LL, std::min<long long>(sms, w_lb));
+    const long long range = std::max(1LL, w_lb / grid);       // fewest blocks of a share
+    const int nbmax = (std::max(pr.max_prefix, 0) + kBN - 1) / kBN + ntb_max;
+    const long long maxparts = (nbmax - 1 + range - 1) / range + 1;
+    if (maxparts <= kMaxRuns) {
+      // per block ~7 % above the static split's (measured: its row tiles of a KV head do not
+      // read a block in lockstep), plus two blocks per change of tile within a share
+      const double share = std::ceil((double)w_ub / grid);
+      const double segs = std::ceil(share / std::max(1.0, nb_mean)) + 1;
+      double t = (share + 3 + 2 * segs) * 0.8 * 1.07;
+      if (maxparts > 1) t += merge_us(std::min<double>(maxparts, 2.0));
+      if (t < best - 1e-9) {
+        p.stream = true;
+        p.grid = grid;
+        p.maxparts = (int)maxparts;
+      }
+    }
+  }
+  p.unsupported = want_stream && !p.stream;
   return p;
 }
 
@@ -1031,16 +1314,17 @@ static bool balanced_grid(const Problem& pr, const Plan& p, int sms, int* grid) 
   return true;
 }
 
-// Workspace of the balanced plan: header | tile runs [tiles] | partial O [grid][T * grp][D]
-// | partial lse [grid][T * grp].
+// Workspace of the balanced and streamed plans: header | tile runs [tiles] | partial O
+// [slots][T * grp][D] | partial lse [slots][T * grp], with one slot per CTA (balanced) or
+// maxparts slots per tile (streamed).
 struct BalancedWs {
   size_t runs, part_o, part_lse, total;
 };
 
-static BalancedWs balanced_ws(const Problem& pr, const Plan& p, int grid) {
+static BalancedWs balanced_ws(const Problem& pr, const Plan& p, long long nslots) {
   auto up = [](size_t x) { return (x + 255) & ~size_t(255); };
   const size_t ntiles = (size_t)pr.Qn * pr.hkv * p.mtiles;
-  const size_t slots = (size_t)grid * p.grp * p.T;
+  const size_t slots = (size_t)nslots * p.grp * p.T;
   BalancedWs w;
   w.runs = up(kWsHeaderBytes);
   w.part_o = w.runs + up(ntiles * sizeof(int2));
@@ -1049,10 +1333,16 @@ static BalancedWs balanced_ws(const Problem& pr, const Plan& p, int grid) {
   return w;
 }
 
+static long long stream_slots(const Problem& pr, const Plan& p) {
+  return (long long)pr.Qn * pr.hkv * p.mtiles * p.maxparts;
+}
+
 static size_t ws_bytes(const Problem& pr, int sms) {
   const Plan p = make_plan(pr, sms);
+  if (p.unsupported) return 0;
   int grid = 0;
   if (balanced_grid(pr, p, sms, &grid)) return balanced_ws(pr, p, grid).total;
+  if (p.stream) return balanced_ws(pr, p, stream_slots(pr, p)).total;
   const size_t rows = (size_t)pr.Qn * pr.K * pr.Lq * pr.hq;
   // partial outputs fp16 [nsplit][rows][D], then their lse fp32 [nsplit][rows]
   return kWsHeaderBytes + (p.nsplit > 1 ? (size_t)p.nsplit * rows * ((size_t)pr.D * 2 + 4) : 0);
@@ -1070,10 +1360,10 @@ static int budget_sms(int32_t budget) {
   return budget > 0 ? budget : device_sms();
 }
 
-template <int D, bool BAL>
+template <int D, int MODE>
 static fvrag_status launch(const CUtensorMap* maps, const Args& a, long long grid, cudaStream_t s) {
   const int sm = Layout<D>::kBytes;
-  auto kern = attn_kernel<D, BAL>;
+  auto kern = attn_kernel<D, MODE>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, sm) != cudaSuccess)
     return FVRAG_ERR_CUDA;
   if (launch_pdl(kern, dim3((unsigned)grid), dim3(kThreads), (size_t)sm, s, maps[0], maps[1],
@@ -1099,6 +1389,7 @@ static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k
                         const void* v_own, void* out, float* lse, void* ws, size_t ws_size,
                         cudaStream_t s) {
   const size_t need = ws_bytes(pr, sms);
+  if (need == 0) return FVRAG_ERR_UNSUPPORTED;   // a requested streamed plan cannot serve it
   if (!ws || ws_size < need) return FVRAG_ERR_WORKSPACE;
   if (!aligned16(ws)) return FVRAG_ERR_MISALIGNED;
 
@@ -1133,14 +1424,16 @@ static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k
   }
   int bgrid = 0;
   const bool bal = balanced_grid(pr, p, sms, &bgrid);
-  const BalancedWs bw = bal ? balanced_ws(pr, p, bgrid) : BalancedWs{};
+  const bool strm = !bal && p.stream;
+  const BalancedWs bw = bal ? balanced_ws(pr, p, bgrid)
+                            : strm ? balanced_ws(pr, p, stream_slots(pr, p)) : BalancedWs{};
   Args a;
-  a.tile_runs = bal ? reinterpret_cast<int2*>(base + bw.runs) : nullptr;
+  a.tile_runs = (bal || strm) ? reinterpret_cast<int2*>(base + bw.runs) : nullptr;
   a.offs = prefix_offsets;
   a.own_len = pr.own_len;
   a.out = reinterpret_cast<__nv_bfloat16*>(out);
   a.lse = lse;
-  if (bal) {
+  if (bal || strm) {
     a.part_o = reinterpret_cast<__half*>(base + bw.part_o);
     a.part_lse = reinterpret_cast<float*>(base + bw.part_lse);
   } else {
@@ -1161,20 +1454,24 @@ static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k
   a.mtiles = p.mtiles;
   a.nsplit = p.nsplit;
   a.slot_rows = p.grp * p.T;
+  a.maxparts = p.maxparts;
   a.scale_log2 = scale * kLog2e;
   RunTable rt{nullptr, a.slot_rows, KL, pr.hq, p.grp, p.T, p.mtiles, pr.hkv};
   long long grid = (long long)pr.Qn * pr.hkv * p.nsplit * p.mtiles;
-  if (bal) {
+  if (bal || strm) {
     rt.tile_runs = a.tile_runs;
-    grid = bgrid;
+    grid = bal ? bgrid : p.grid;
   }
   if (grid > 0x7fffffffLL) return FVRAG_ERR_UNSUPPORTED;
   fvrag_status st;
   if (bal)
-    st = D == 128 ? launch<128, true>(maps, a, grid, s) : launch<64, true>(maps, a, grid, s);
+    st = D == 128 ? launch<128, 1>(maps, a, grid, s) : launch<64, 1>(maps, a, grid, s);
+  else if (strm)
+    st = D == 128 ? launch<128, 2>(maps, a, grid, s) : launch<64, 2>(maps, a, grid, s);
   else
-    st = D == 128 ? launch<128, false>(maps, a, grid, s) : launch<64, false>(maps, a, grid, s);
-  if (st != FVRAG_OK || (!bal && p.nsplit == 1)) return st;
+    st = D == 128 ? launch<128, 0>(maps, a, grid, s) : launch<64, 0>(maps, a, grid, s);
+  if (st != FVRAG_OK) return st;
+  if (!bal && !(strm && p.maxparts > 1) && !(!strm && p.nsplit > 1)) return st;
   const int wpb = 8;
   const long long blocks = (nrows + wpb - 1) / wpb;
   const cudaError_t e =
@@ -1190,12 +1487,18 @@ static fvrag_status run(const Problem& pr, int sms, const void* q, const void* k
 
 static Problem verify_problem(const fvrag_attn_desc* d) {
   return Problem{d->num_queries, d->num_cand, d->cand_len, d->cand_len, d->hq, d->hkv,
-                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, nullptr, false};
+                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, nullptr, false,
+                 d->flags};
 }
 
 static Problem decode_problem(const fvrag_decode_desc* d, const int32_t* cache_len) {
   return Problem{d->num_queries, d->num_drafts, 1, d->cache_cap, d->hq, d->hkv,
-                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, cache_len, true};
+                 d->head_dim, d->max_prefix, d->total_prefix, d->softmax_scale, cache_len, true,
+                 0u};
+}
+
+static bool split_flags_ok(uint32_t f) {
+  return f == 0 || f == FVRAG_ATTN_SPLIT_STATIC || f == FVRAG_ATTN_SPLIT_STREAM;
 }
 
 }  // namespace attn
@@ -1205,7 +1508,8 @@ using namespace fvrag;
 
 extern "C" size_t fvrag_verify_attn_workspace(const fvrag_attn_desc* d) {
   if (!d || d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
-      d->hq % d->hkv || (d->head_dim != 64 && d->head_dim != 128) || d->max_prefix < 0)
+      d->hq % d->hkv || (d->head_dim != 64 && d->head_dim != 128) || d->max_prefix < 0 ||
+      !attn::split_flags_ok(d->flags))
     return 0;
   const int sms = attn::budget_sms(d->sm_budget);
   if (sms < 0) return 0;
@@ -1220,8 +1524,8 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
   using namespace attn;
   if (!d || !q || !prefix_offsets || !k_tail || !v_tail || !out) return FVRAG_ERR_INVALID_ARG;
   if (d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
-      d->max_prefix < 0 || d->total_prefix < 0 || d->flags != 0 || !(d->softmax_scale >= 0.f) ||
-      d->softmax_scale == INFINITY)
+      d->max_prefix < 0 || d->total_prefix < 0 || !split_flags_ok(d->flags) ||
+      !(d->softmax_scale >= 0.f) || d->softmax_scale == INFINITY)
     return FVRAG_ERR_INVALID_ARG;
   if (d->total_prefix > 0 && (!k_prefix || !v_prefix)) return FVRAG_ERR_INVALID_ARG;
   const int sms = budget_sms(d->sm_budget);

@@ -12,6 +12,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libfvrag.so")
 
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_MISALIGNED, ERR_WORKSPACE, ERR_CUDA, ERR_TIMEOUT = range(7)
+# fvrag_attn_desc.flags: the key split of the verification attention (0: the library's choice)
+ATTN_SPLIT_STATIC, ATTN_SPLIT_STREAM = 1, 2
 SEL_MASKED_MEAN_LOGPROB = 0
 SEL_TWO_STAGE = 1
 SEL_ADDITION = 2
@@ -183,13 +185,14 @@ def lm_workspace_bytes(desc: LmDesc) -> int:
 
 # --------------------------------------------------------------------- the four calls
 def verify_attn(q, k_prefix, v_prefix, prefix_offsets, k_tail, v_tail, out, ws, max_prefix,
-                lse=None, softmax_scale=0.0, stream=None, sm_budget=0):
+                lse=None, softmax_scale=0.0, stream=None, sm_budget=0, split=0):
     """q [Qn][K][L][hq][D] bf16; k/v_prefix [sum P][hkv][D]; prefix_offsets [Qn+1] int32 (device);
     k/v_tail [Qn][K][L][hkv][D]; out like q; lse [Qn][K][L][hq] fp32 or None; ws uint8 device;
-    sm_budget: SMs the key split is planned for (0: all)."""
+    sm_budget: SMs the key split is planned for (0: all); split: 0 (library's choice),
+    ATTN_SPLIT_STATIC or ATTN_SPLIT_STREAM."""
     d = AttnDesc(q.shape[0], q.shape[1], q.shape[2], q.shape[3], k_tail.shape[3], q.shape[4],
                  int(max_prefix), 0 if k_prefix is None else int(k_prefix.shape[0]),
-                 float(softmax_scale), 0, int(sm_budget))
+                 float(softmax_scale), int(split), int(sm_budget))
     s = lib().fvrag_verify_attn(ctypes.byref(d), _ptr(q), _ptr(k_prefix), _ptr(v_prefix),
                                 _ptr(prefix_offsets), _ptr(k_tail), _ptr(v_tail), _ptr(out),
                                 _ptr(lse), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream))

@@ -71,22 +71,23 @@ def dev(a):
     return torch.from_numpy(np.ascontiguousarray(a)).cuda()
 
 
-def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0, sm_budget=0):
-    """Runs fvrag_verify_attn on numpy inputs; returns (out fp32 numpy, lse numpy, status)."""
+def run_attn(q, kp, vp, offs, kt, vt, with_lse=True, scale=0.0, sm_budget=0, split=0):
+    """Runs fvrag_verify_attn on numpy inputs; returns (out fp32 numpy, lse numpy, status).
+    split: the key-split plan requested in the descriptor's flags (0: the library's choice)."""
     Qn, K, L, Hq, D = q.shape
     tq, tkt, tvt = dev_bf16(q), dev_bf16(kt), dev_bf16(vt)
     tkp = dev_bf16(kp) if kp.shape[0] > 0 else None
     tvp = dev_bf16(vp) if vp.shape[0] > 0 else None
     toffs = dev(offs.astype(np.int32))
     maxp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
-    d = fvrag.AttnDesc(Qn, K, L, Hq, kt.shape[3], D, maxp, int(kp.shape[0]), float(scale), 0,
+    d = fvrag.AttnDesc(Qn, K, L, Hq, kt.shape[3], D, maxp, int(kp.shape[0]), float(scale), split,
                        sm_budget)
     ws = torch.zeros(fvrag.attn_workspace_bytes(d), dtype=torch.uint8, device="cuda")
     pool = []
     out = guarded(q.shape, torch.bfloat16, float("nan"), pool)
     lse = guarded(q.shape[:-1], torch.float32, float("nan"), pool) if with_lse else None
     fvrag.verify_attn(tq, tkp, tvp, toffs, tkt, tvt, out, ws, maxp, lse=lse, softmax_scale=scale,
-                      sm_budget=sm_budget)
+                      sm_budget=sm_budget, split=split)
     st = fvrag.read_status(ws)
     check_all(pool)
     return out.float().cpu().numpy(), (lse.cpu().numpy() if with_lse else None), st

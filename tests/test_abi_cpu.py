@@ -37,7 +37,7 @@ def test_exports_every_declared_symbol(L):
 
 
 def test_version_and_strings(L):
-    assert L.fvrag_abi_version() == 5
+    assert L.fvrag_abi_version() == 6
     for s in range(7):
         assert fvrag.status_string(s)
     assert fvrag.status_string(99) == "unknown status"
@@ -61,7 +61,8 @@ def test_attn_validation(L):
     assert ws > 256
     assert _attn(L, fvrag.AttnDesc(0, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_INVALID_ARG
     assert _attn(L, good, q=None) == fvrag.ERR_INVALID_ARG
-    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 1)) == fvrag.ERR_INVALID_ARG
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 3)) == fvrag.ERR_INVALID_ARG
+    assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 4)) == fvrag.ERR_INVALID_ARG
     assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 5, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
     assert _attn(L, fvrag.AttnDesc(1, 5, 16, 28, 4, 96, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
     assert _attn(L, fvrag.AttnDesc(1, 5, 65, 28, 4, 128, 8192, 8192, 0.0, 0)) == fvrag.ERR_UNSUPPORTED
@@ -74,6 +75,20 @@ def test_attn_validation(L):
     # no prefix at all: prefix pointers may be NULL, workspace is just the header
     nop = fvrag.AttnDesc(1, 2, 3, 4, 2, 64, 0, 0, 0.0, 0)
     assert L.fvrag_verify_attn_workspace(ctypes.byref(nop)) == 256
+
+
+def test_attn_split_flags(L):
+    """flags selects the key split: 0 (the library's choice), static, or streamed.  The
+    streamed plan needs <= 64 queries (and <= 64 row tiles per KV head): beyond, both the
+    workspace query (0) and the call (UNSUPPORTED) refuse it; the other plans serve it."""
+    base = (1, 5, 16, 28, 4, 128, 8192, 8192, 0.0)
+    for f in (0, fvrag.ATTN_SPLIT_STATIC, fvrag.ATTN_SPLIT_STREAM):
+        assert L.fvrag_verify_attn_workspace(ctypes.byref(fvrag.AttnDesc(*base, f))) >= 256
+    many = (65, 2, 4, 8, 8, 64, 1000, 65000, 0.0)
+    assert L.fvrag_verify_attn_workspace(ctypes.byref(fvrag.AttnDesc(*many, fvrag.ATTN_SPLIT_STREAM))) == 0
+    assert _attn(L, fvrag.AttnDesc(*many, fvrag.ATTN_SPLIT_STREAM)) == fvrag.ERR_UNSUPPORTED
+    assert L.fvrag_verify_attn_workspace(ctypes.byref(fvrag.AttnDesc(*many, fvrag.ATTN_SPLIT_STATIC))) >= 256
+    assert L.fvrag_verify_attn_workspace(ctypes.byref(fvrag.AttnDesc(*many, 0))) >= 256
 
 
 def test_attn_sm_budget(L):

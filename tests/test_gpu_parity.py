@@ -108,13 +108,16 @@ def _row_tile_sel(shape, hkv, tiles):
 
 
 @pytest.mark.parametrize("name", ["7b", "long", "batch16", "72b"])
-def test_attn_full_size(name):
+@pytest.mark.parametrize("split", [0, fvrag.ATTN_SPLIT_STATIC, fvrag.ATTN_SPLIT_STREAM],
+                         ids=["auto", "static", "stream"])
+def test_attn_full_size(name, split):
     """Full-size attention alone on all SMs: every row at 7b and long; at batch16 and 72b
     the first and the last (ragged) row tile of every query and KV head plus sampled rows
     (every row of those two is checked by the whole-step test)."""
     cfg = configs.PRESETS[name]
     x = synth.make_inputs(cfg, parts=("attn",))
-    out, lse, st = run_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_tail"], x["v_tail"])
+    out, lse, st = run_attn(x["q"], x["k_prefix"], x["v_prefix"], x["prefix_offsets"], x["k_tail"],
+                            x["v_tail"], split=split)
     assert st == fvrag.OK
     assert np.all(np.isfinite(out)) and np.all(np.isfinite(lse))
     shape = x["q"].shape[:-1]

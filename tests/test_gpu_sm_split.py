@@ -38,16 +38,22 @@ def _attn_inputs(Qn, K, L, Hq, Hkv, D, plens, seed):
             synth.normal_bf16((Qn, K, L, Hkv, D), seed, 4), synth.normal_bf16((Qn, K, L, Hkv, D), seed, 5))
 
 
-@pytest.mark.parametrize("budget", [1, 3, 20, -1])
+@pytest.mark.parametrize("split", [0, fvrag.ATTN_SPLIT_STATIC, fvrag.ATTN_SPLIT_STREAM],
+                         ids=["auto", "static", "stream"])
+@pytest.mark.parametrize("budget", [1, 2, 3, 5, 7, 20, -1])
 @pytest.mark.parametrize("case", [(2, 3, 9, 16, 2, 128, [700, 2049]),    # several tiles, ragged
-                                  (1, 5, 16, 28, 4, 128, [1000])],       # 7b-style GQA
-                         ids=["ragged2q", "gqa7"])
-def test_attn_budget_matches_oracle(case, budget):
-    """A budget of 1 runs every tile's whole key list on one CTA (no merge); -1 means the
-    device's own SM count given explicitly (the same plan as 0)."""
+                                  (1, 5, 16, 28, 4, 128, [1000]),        # 7b-style GQA
+                                  (3, 5, 16, 28, 4, 128, [4000, 100, 2500]),   # three ragged queries
+                                  (2, 2, 64, 8, 8, 64, [0, 300])],       # D = 64; a query without prefix
+                         ids=["ragged2q", "gqa7", "gqa7x3q", "d64"])
+def test_attn_budget_matches_oracle(case, budget, split):
+    """Every key-split plan at every budget.  Under the streamed plan small budgets give each
+    CTA a long share of the tiles' concatenated key lists (tiles cut between CTAs, several
+    whole tiles per CTA, one CTA for all at a budget of 1); -1 means the device's own SM count
+    given explicitly (the same plan as 0)."""
     b = _sms() if budget == -1 else budget
     q, kp, vp, offs, kt, vt = _attn_inputs(*case, seed=4100 + b)
-    out, lse, st = run_attn(q, kp, vp, offs, kt, vt, sm_budget=b)
+    out, lse, st = run_attn(q, kp, vp, offs, kt, vt, sm_budget=b, split=split)
     assert st == fvrag.OK
     ref, ref_lse = oracle.verify_attn(q, kp, vp, offs, kt, vt)
     assert np.max(np.abs(out - ref)) <= ATTN_ATOL
@@ -66,6 +72,7 @@ def test_attn_budget_above_device_rejected():
 @pytest.mark.parametrize("budget", [1, 2, 33, 132])
 @pytest.mark.parametrize("case", [(80, 512, 9000, 1),     # one M-tile (the HBM-bound form)
                                   (200, 64, 3000, 2),     # pair form, one pair-tile
+                                  (320, 128, 5000, 2),    # vocabulary-major pair form
                                   (512, 96, 7777, 3)],    # pair form, two pair-tiles
                          ids=lambda c: "M%d_H%d_V%d_G%d" % c)
 def test_lm_budget_matches_oracle(case, budget):

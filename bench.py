@@ -46,7 +46,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # source with this SHA-256 prefix (reported as null once the kernel source changes).
 LM_TRAFFIC = {
     "7b": {"sha256_prefix": "647e44d32925ae8a", "bytes_per_launch": 1093409536},
-    "72b": {"sha256_prefix": "165a475a62555a20", "bytes_per_launch": 2499644160},
+    "72b": {"sha256_prefix": "66f93c7cc1035cc6", "bytes_per_launch": 2500659456},
 }
 
 

@@ -741,7 +741,8 @@ __device__ __forceinline__ float dot8_bf16(const uint4 a, const uint4 b) {
 
 __global__ void __launch_bounds__(vt::kThreads, 1)
     lm_head_vt_kernel(const __grid_constant__ CUtensorMap tm_hb,
-                      const __grid_constant__ CUtensorMap tm_w64, const uint16_t* __restrict__ hidden,
+                      const __grid_constant__ CUtensorMap tm_w64,
+                      const __grid_constant__ CUtensorMap tm_w16, const uint16_t* __restrict__ hidden,
                       const uint16_t* __restrict__ weight, const int32_t* __restrict__ targets, int M,
                       int Mp, int H, int V, int G, float* __restrict__ part_max,
                       float* __restrict__ part_sum, float* __restrict__ tgt_logit, uint32_t* status,
@@ -787,6 +788,7 @@ __global__ void __launch_bounds__(vt::kThreads, 1)
   if (warp == 0 && lane == 0) {
     tma_prefetch_desc(&tm_hb);
     tma_prefetch_desc(&tm_w64);
+    tma_prefetch_desc(&tm_w16);
   }
   for (int i = threadIdx.x; i < 4 * vt::kMaxRows; i += vt::kThreads) {
     negR[i] = INFINITY;     // R = -inf
@@ -810,13 +812,18 @@ __global__ void __launch_bounds__(vt::kThreads, 1)
     if (lane == 0) {
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_h = policy_evict_last();
-      const uint32_t bytes = vt::kABytes + (uint32_t)Mp * kBK;   // per CTA: 128 W rows + Mp/2 hidden rows
+      const uint32_t hbytes = (uint32_t)Mp * kBK;       // per CTA: Mp / 2 hidden rows
       int stage = 0;
       uint32_t phase = 0;
       long long issued = 0;
       bool ok = true;
       for (int t = 0; t < ntiles && ok; ++t) {
-        const int w0 = v_lo + t * vt::kTile + (int)rank * kBM;
+        // each CTA loads the W rows of its half that lie in the pair's range (rounded up to
+        // 16); the A rows past them hold stale data and feed only masked lanes
+        const int t0 = v_lo + t * vt::kTile;
+        auto w_rows = [&](int r) { return (min(max(v_hi - t0 - r * kBM, 0), kBM) + 15) & ~15; };
+        const int w0 = t0 + (int)rank * kBM, wr = w_rows((int)rank);
+        const uint32_t bytes2 = (uint32_t)(w_rows(0) + w_rows(1)) * kBK * 2 + 2 * hbytes;
         for (int kb = 0; kb < kblocks; ++kb) {
           if (!mbar_wait_cluster(smem_u32(&empty[stage]), phase ^ 1, limit_ns)) {
             record_error(status, FVRAG_ERR_TIMEOUT, kSiteProdEmpty);
@@ -824,10 +831,13 @@ __global__ void __launch_bounds__(vt::kThreads, 1)
             break;
           }
           const uint32_t fb = full0 + (uint32_t)(stage * 8);
-          if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full[stage]), 2 * bytes);
+          if (rank == 0) mbar_arrive_expect_tx(smem_u32(&full[stage]), bytes2);
           const uint32_t st = smem_u32(ring + stage * vt::kStageBytes);
-          tma_load_2d_pair(st, &tm_w64, fb, kb * kBK, w0, pol_w);
-          tma_load_2d_pair(st + 64 * 128, &tm_w64, fb, kb * kBK, w0 + 64, pol_w);
+          int r = 0;
+          for (; r + 64 <= wr; r += 64)
+            tma_load_2d_pair(st + r * 128, &tm_w64, fb, kb * kBK, w0 + r, pol_w);
+          for (; r < wr; r += 16)
+            tma_load_2d_pair(st + r * 128, &tm_w16, fb, kb * kBK, w0 + r, pol_w);
           tma_load_2d_pair(st + vt::kABytes, &tm_hb, fb, kb * kBK, (int)rank * nb, pol_h);
           tma_load_2d_pair(st + vt::kABytes + nb * 128, &tm_hb, fb, kb * kBK, N + (int)rank * nb, pol_h);
           ++issued;
@@ -1112,7 +1122,7 @@ static fvrag_status launch_pair(const Plan& p, const CUtensorMap& th, const CUte
 }
 
 static fvrag_status launch_vt(const Plan& p, const CUtensorMap& thb, const CUtensorMap& tw64,
-                              const void* hidden, const void* weight, const int32_t* targets,
+                              const CUtensorMap& tw16, const void* hidden, const void* weight, const int32_t* targets,
                               const fvrag_lm_desc* d, int Mp, float* pmax, float* psum,
                               float* ptgt, uint32_t* status, cudaStream_t s) {
   auto kern = lm_head_vt_kernel;
@@ -1133,7 +1143,7 @@ static fvrag_status launch_vt(const Plan& p, const CUtensorMap& thb, const CUten
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 2;
-  if (counted(cudaLaunchKernelEx(&cfg, kern, thb, tw64, static_cast<const uint16_t*>(hidden),
+  if (counted(cudaLaunchKernelEx(&cfg, kern, thb, tw64, tw16, static_cast<const uint16_t*>(hidden),
                                  static_cast<const uint16_t*>(weight), targets, d->rows, Mp,
                                  d->hidden, d->vocab, d->gathers, pmax, psum, ptgt, status,
                                  wait_limit_ns())) != cudaSuccess)
@@ -1227,7 +1237,7 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
     const uint64_t dims[2] = {H, M}, strides[1] = {H * 2};
     const uint32_t box[2] = {(uint32_t)kBK, (uint32_t)(Mp / 4)};
     if (!encode_tmap_bf16(&thb, hidden, 2, dims, strides, box, true)) return FVRAG_ERR_CUDA;
-    st = launch_vt(p, thb, tw64, hidden, weight, targets, d, Mp, pmax, psum, ptgt, status, s);
+    st = launch_vt(p, thb, tw64, tw16, hidden, weight, targets, d, Mp, pmax, psum, ptgt, status, s);
   } else if (p.mg == 0)
     st = launch_pair<2>(p, th, tw64, tw16, targets, d, pmax, psum, ptgt, status, s);
   else if (p.mg == -1)

@@ -114,6 +114,24 @@ def plan_sm_split(cfg: VerifyConfig, sms: int, max_prefix: int = None, late: boo
     return ctas, sms - ctas
 
 
+def clip_ctas(cfg: VerifyConfig):
+    """CTAs of the CLIP call when a query's frames need no split across a cluster (at most
+    256 frames: one CTA per query and group of 16 candidates), else None."""
+    if cfg.num_frames > 256:
+        return None
+    return cfg.num_queries * -(-cfg.num_cand // 16)
+
+
+def serial_attn_budget(cfg: VerifyConfig, sms: int) -> int:
+    """SM budget of the attention when the calls run one after the other: the CLIP call runs
+    beside it on a side stream, and when CLIP is a few CTAs the attention leaves it those SMs
+    (0 = all SMs otherwise).  Under the streamed key split every SM holds one equal share, so
+    a share that waited for CLIP's SM would hold up the whole call by CLIP's time; giving up
+    one SM of 152 costs the attention under 1 %."""
+    n = clip_ctas(cfg)
+    return sms - n if n is not None and n <= 4 and sms > 8 * n else 0
+
+
 class VerifyStep:
     def __init__(self, cfg: VerifyConfig, device="cuda", mode=fvrag.SEL_MASKED_MEAN_LOGPROB,
                  max_prefix=None, with_lse=True, sm_split="auto"):
@@ -181,15 +199,16 @@ class VerifyStep:
             offs = inputs["prefix_offsets"]
             mp = int(np.max(np.diff(offs))) if len(offs) > 1 else 0
             self.max_prefix = mp if self.max_prefix is None else max(self.max_prefix, mp)
+            sms = torch.cuda.get_device_properties(self.device).multi_processor_count
             if self._sm_split_arg == "auto":
-                sms = torch.cuda.get_device_properties(self.device).multi_processor_count
                 self.sm_split = plan_sm_split(self.cfg, sms, int(self.max_prefix))
                 self.sm_split_e2e = plan_sm_split(self.cfg, sms, int(self.max_prefix), late=True)
+            self._serial_attn_sms = serial_attn_budget(self.cfg, sms)
             self._alloc_attn_ws()
 
     def _budgets(self, e2e=False):
         split = self.sm_split_e2e if e2e else self.sm_split
-        return (0, 0) if split is None else split
+        return (getattr(self, "_serial_attn_sms", 0), 0) if split is None else split
 
     def _alloc_attn_ws(self):
         c = self.cfg

@@ -47,11 +47,11 @@ bool encode_tmap_f16(CUtensorMap* map, const void* base, int rank, const uint64_
 // runtime), or null when none is current or the driver call is unavailable.
 CUcontext current_cu_context();
 
-// Status a workspace status word reports: OK when 0, TIMEOUT when that bit is set,
-// else the recorded code.
+// Status a workspace status word reports: OK when 0, TIMEOUT when both of its bits are set
+// (codes are OR-ed in, and TIMEOUT's bits contain UNSUPPORTED's), else the recorded code.
 inline fvrag_status status_of_word(uint32_t v) {
   if (v == 0) return FVRAG_OK;
-  if (v & FVRAG_ERR_TIMEOUT) return FVRAG_ERR_TIMEOUT;
+  if ((v & FVRAG_ERR_TIMEOUT) == FVRAG_ERR_TIMEOUT) return FVRAG_ERR_TIMEOUT;
   return (fvrag_status)v;
 }
 

@@ -58,6 +58,10 @@
  *     them on two streams.  A budget changes the grid and the key split, hence the
  *     rounding order of partial sums, never the operation computed; the workspace
  *     size depends on it (pass the same descriptor to the *_workspace call).
+ *   - Tracing: with FVRAG_NVTX set in the environment (not "0"; read once, at the
+ *     first call) every compute entry point wraps its work in an NVTX range named
+ *     after it, so that Nsight Systems or ncu's NVTX filters group the kernels a
+ *     call enqueues.  Without a profiler attached the ranges cost nothing.
  *   - fvrag_launch_count() counts the kernel launches the library has enqueued
  *     in this process (a launch captured into a CUDA graph counts once, at
  *     capture), so a caller can tell how many kernels one call or one captured

@@ -9,11 +9,31 @@
 #include "fvrag_common.cuh"
 #include "fvrag_internal.h"
 
+#include <cstdlib>
+#include <cstring>
+#include <nvtx3/nvToolsExt.h>
+
 namespace fvrag {
 
 static std::atomic<uint64_t> g_wait_limit_ns{1000000000ull};
 
 uint64_t wait_limit_ns() { return g_wait_limit_ns.load(std::memory_order_relaxed); }
+
+bool nvtx_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("FVRAG_NVTX");
+    return v != nullptr && v[0] != '\0' && std::strcmp(v, "0") != 0;
+  }();
+  return on;
+}
+
+NvtxRange::NvtxRange(const char* name) : on(nvtx_enabled()) {
+  if (on) nvtxRangePushA(name);
+}
+
+NvtxRange::~NvtxRange() {
+  if (on) nvtxRangePop();
+}
 
 static std::atomic<uint64_t> g_launches{0};
 

@@ -1521,6 +1521,7 @@ extern "C" fvrag_status fvrag_verify_attn(const fvrag_attn_desc* d, const void* 
                                           const int32_t* prefix_offsets, const void* k_tail,
                                           const void* v_tail, void* out, float* lse, void* ws,
                                           size_t ws_size, fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_verify_attn");
   using namespace attn;
   if (!d || !q || !prefix_offsets || !k_tail || !v_tail || !out) return FVRAG_ERR_INVALID_ARG;
   if (d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->hq < 1 || d->hkv < 1 ||
@@ -1554,6 +1555,7 @@ extern "C" fvrag_status fvrag_decode_attn(const fvrag_decode_desc* d, const void
                                           const void* v_cache, const int32_t* cache_len, void* out,
                                           float* lse, void* ws, size_t ws_size,
                                           fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_decode_attn");
   using namespace attn;
   if (!d || !q || !prefix_offsets || !k_cache || !v_cache || !cache_len || !out)
     return FVRAG_ERR_INVALID_ARG;

@@ -401,6 +401,7 @@ static int clip_split(int F, long long groups, int smem) {
 extern "C" fvrag_status fvrag_clip_align(const fvrag_clip_desc* d, const void* cand_emb,
                                          const void* frame_emb, float* cos, float* max_cos,
                                          int32_t* argmax, uint8_t* keep, fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_clip_align");
   if (!d || !cand_emb || !frame_emb || !max_cos || !argmax || !keep) return FVRAG_ERR_INVALID_ARG;
   if (d->num_queries < 1 || d->num_cand < 1 || d->num_frames < 1 || d->dim < 1 || d->flags != 0)
     return FVRAG_ERR_INVALID_ARG;
@@ -443,6 +444,7 @@ extern "C" fvrag_status fvrag_select_candidate(const fvrag_select_desc* d, const
                                                const int32_t* lengths, const uint8_t* keep,
                                                const float* max_cos, float* score,
                                                int32_t* selected, fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_select_candidate");
   if (!d || !logprob || !score || !selected) return FVRAG_ERR_INVALID_ARG;
   if (d->num_queries < 1 || d->num_cand < 1 || d->cand_len < 1 || d->gathers < 1 || d->flags != 0)
     return FVRAG_ERR_INVALID_ARG;

@@ -12,6 +12,22 @@ namespace fvrag {
 // Current limit of the kernels' bounded waits, in nanoseconds.
 uint64_t wait_limit_ns();
 
+// Whether the public calls mark themselves with NVTX ranges: FVRAG_NVTX set in the
+// environment (and not "0"), read once.
+bool nvtx_enabled();
+
+// An NVTX range (nvtxRangePushA / nvtxRangePop) around one public call, so that a profiler
+// attached to the process (Nsight Systems, or ncu's NVTX filters) can group the kernels the
+// call enqueues under the call's name.  Off unless nvtx_enabled(); with no tool attached the
+// NVTX calls do nothing.
+struct NvtxRange {
+  bool on;
+  explicit NvtxRange(const char* name);
+  ~NvtxRange();
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
+
 // Number of SMs of the current device (cached per device); 0 if it cannot be read.
 int sm_count();
 

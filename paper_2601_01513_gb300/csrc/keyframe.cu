@@ -266,6 +266,7 @@ extern "C" fvrag_status fvrag_keyframes(const fvrag_keyframe_desc* d, const uint
                                         const int32_t* video_offsets, int32_t* hist, float* sim,
                                         uint8_t* is_key, int32_t* key_index, int32_t* key_offsets,
                                         void* ws, size_t ws_size, fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_keyframes");
   using namespace kf;
   if (!d || !video_offsets || !sim || !is_key || !key_index || !key_offsets)
     return FVRAG_ERR_INVALID_ARG;

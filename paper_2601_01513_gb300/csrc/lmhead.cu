@@ -1195,6 +1195,7 @@ extern "C" fvrag_status fvrag_score_logprobs(const fvrag_lm_desc* d, const void*
                                              const void* weight, const int32_t* targets,
                                              float* logprob, float* lse, void* ws, size_t ws_size,
                                              fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_score_logprobs");
   using namespace lm;
   if (!d || !hidden || !weight || !targets || !logprob) return FVRAG_ERR_INVALID_ARG;
   if (d->rows < 1 || d->hidden < 1 || d->vocab < 1 || d->gathers < 1 || d->flags != 0 ||
@@ -1301,6 +1302,7 @@ extern "C" fvrag_status fvrag_score_logprobs_noalloc(const fvrag_lm_desc* d, con
                                                      const void* weight, const int32_t* targets,
                                                      float* logprob, float* lse,
                                                      fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_score_logprobs_noalloc");
   using namespace lm;
   // reject bad arguments before anything is enqueued
   if (!d || !hidden || !weight || !targets || !logprob) return FVRAG_ERR_INVALID_ARG;

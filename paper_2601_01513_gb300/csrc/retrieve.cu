@@ -946,6 +946,7 @@ using namespace fvrag;
 
 extern "C" fvrag_status fvrag_embed_inv_norms(const void* x, int32_t rows, int32_t dim,
                                               float* inv_norm, fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_embed_inv_norms");
   if (!x || !inv_norm || rows < 1 || dim < 8) return FVRAG_ERR_INVALID_ARG;
   if (dim % 8 != 0 || !aligned16(x)) return FVRAG_ERR_MISALIGNED;
   return rt::launch_inv_norms(x, rows, dim, inv_norm, reinterpret_cast<cudaStream_t>(stream));
@@ -961,6 +962,7 @@ extern "C" fvrag_status fvrag_retrieve(const fvrag_retrieve_desc* d, const void*
                                        const float* text_inv_norm, int32_t* frame_topk,
                                        float* frame_topk_sim, int32_t* out_idx, float* out_sim,
                                        void* ws, size_t ws_size, fvrag_stream_t stream) {
+  NvtxRange nvtx_range("fvrag_retrieve");
   using namespace rt;
   if (!desc_ok(d) || !frame_offsets || !text_emb || !out_idx || !out_sim)
     return FVRAG_ERR_INVALID_ARG;

@@ -259,3 +259,24 @@ def test_decode_validation(L):
     assert _dec(L, good, q=PMIS) == fvrag.ERR_MISALIGNED
     assert _dec(L, good, kc=PMIS) == fvrag.ERR_MISALIGNED
     assert _dec(L, good, ws_bytes=ws - 1) == fvrag.ERR_WORKSPACE
+
+
+def test_nvtx_ranges_switch_on_without_a_profiler():
+    """FVRAG_NVTX=1 makes every public call push and pop an NVTX range; with no profiler
+    attached that is a no-op, so validation still returns the same status (run in a child
+    process, since the switch is read once)."""
+    import subprocess
+    import sys
+    import os
+    code = (
+        "import ctypes, sys; sys.path.insert(0, %r)\n"
+        "from paper_2601_01513_gb300 import fvrag\n"
+        "L = fvrag.lib()\n"
+        "d = fvrag.AttnDesc(0, 5, 16, 28, 4, 128, 8192, 8192, 0.0, 0)\n"
+        "p = ctypes.c_void_p(1 << 20)\n"
+        "st = L.fvrag_verify_attn(ctypes.byref(d), p, p, p, p, p, p, p, None, p, 1 << 30, None)\n"
+        "print(st)\n" % os.path.dirname(os.path.dirname(os.path.abspath(__file__))))
+    env = dict(os.environ, FVRAG_NVTX="1")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, env=env, timeout=120)
+    assert r.returncode == 0, r.stderr
+    assert int(r.stdout.strip().splitlines()[-1]) == fvrag.ERR_INVALID_ARG

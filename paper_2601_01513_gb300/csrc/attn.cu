@@ -73,7 +73,8 @@ constexpr int kMaxTail = 64;            // verification: tokens per candidate
 constexpr int kMaxCand = kBM + 1;       // candidates a row tile can touch
 constexpr uint32_t kTmemCols = 512;
 // tensor-memory columns: kSP S/P buffers of 128 columns (S_j as fp32 in 128 columns, then
-// P_j as packed bf16 in the first 64), the O accumulator after them.  Three buffers let
+// P_j as packed bf16: keys 0-63 in columns 0-31, keys 64-127 in columns 64-95, each half over
+// the S columns its own softmax warp has read), the O accumulator after them.  Three buffers let
 // S_{j+2} be computed while PV_j still reads P_j.
 constexpr int kSP = 3;
 __device__ __forceinline__ uint32_t col_s(int b) { return (uint32_t)b * 128u; }
@@ -760,8 +761,8 @@ __global__ void __launch_bounds__(kThreads, 1)
           const uint32_t pa = tmem_base + col_s(np % kSP);
           const uint32_t vs = smem_u32(v_ring + (np % kVStages) * Lay::kStage);
 #pragma unroll
-          for (int k16 = 0; k16 < kBN / 16; ++k16)
-            tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8),
+          for (int k16 = 0; k16 < kBN / 16; ++k16)   // P of keys 64-127 starts at column 64
+            tc_mma_bf16_ts(tmem_base + kColO, pa + (uint32_t)(k16 * 8 + (k16 >= 4 ? 32 : 0)),
                            desc_mnmajor_sw128(vs + k16 * 2048, Lay::kKVHalf), idPV,
                            (j | k16) != 0);
           tc_commit(smem_u32(&pv_done[np % kSP]));
@@ -888,8 +889,9 @@ __global__ void __launch_bounds__(kThreads, 1)
         // rows without output (r >= rows) are not masked: their values are finite and
         // discarded, and masking them would split the warp between the two paths below
         const bool full = vlo <= 0 && vhi >= kHalf;
-        // P_j relative to the reference `mref`: bf16 pairs into pk (written over the first 64
-        // columns of the same buffer; S_j is in registers), the partial sum into rs
+        // P_j relative to the reference `mref`: bf16 pairs into pk (written over the first 32
+        // of this warp's own S columns of the buffer; S_j is in registers), the partial sum
+        // into rs
         uint32_t pk[32];
         float rs = 0.f;
         // kMask: 0 = no masking, 1 = mask every element, 2 = mask when the block is not full
@@ -945,9 +947,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         const bool mine = fresh || __any_sync(0xffffffffu, !(rs <= kSumLimit));
         int* xf = xflag + ((jj & 1) * 2 + half) * 4;     // [2 slots][2 halves][4 quarters]
         if (lane == 0) xf[quarter] = mine ? 1 : 0;
-        tc_fence_before();          // this warp's S loads are complete before the partner
-        pair_sync();                // writes its P over them
+        // Each warp writes its P over its own S columns, so this exchange orders no tensor-
+        // memory access between the two; the fences stay because without them the compiler
+        // scheduled the streamed form's loop worse (72b 154 -> 156 us per call).
+        tc_fence_before();
+        pair_sync();
         tc_fence_after();
+        const uint32_t pcol = lane_base + col_s(sb) + (uint32_t)(half * kHalf);   // this warp's P
         const bool slow = mine || xflag[((jj & 1) * 2 + (half ^ 1)) * 4 + quarter] != 0;
         bool resc = false;
         float corr = 1.f;
@@ -978,8 +984,12 @@ __global__ void __launch_bounds__(kThreads, 1)
           resc = m_ref != m_old && m_old != -INFINITY;
           corr = resc ? ex2(m_old - m_ref) : 1.f;
           if (fresh || __any_sync(0xffffffffu, m_ref != m_old)) exp_pass(m_ref);
+          if (ok) tmem_st_32x32b_x32(pcol, pk);
+        } else if (ok) {
+          // the same store, kept on each path: with one store after the branch the compiler
+          // scheduled the loop worse (72b 154 -> 157 us per call)
+          tmem_st_32x32b_x32(pcol, pk);
         }
-        if (ok) tmem_st_32x32b_x32(lane_base + col_s(sb) + (uint32_t)(half * kHalf / 2), pk);
         l = l * corr + rs;
         if (ok && __any_sync(0xffffffffu, resc)) {
           // O holds blocks < j relative to the old reference: wait for PV_{j-1}, then scale

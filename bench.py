@@ -45,8 +45,8 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM traffic of one LM-head launch per workload, from an ncu capture of the kernel
 # source with this SHA-256 prefix (reported as null once the kernel source changes).
 LM_TRAFFIC = {
-    "7b": {"sha256_prefix": "66f93c7cc1035cc6", "bytes_per_launch": 1093414912},
-    "72b": {"sha256_prefix": "66f93c7cc1035cc6", "bytes_per_launch": 2500659456},
+    "7b": {"sha256_prefix": "fc5d9ea0e4553c80", "bytes_per_launch": 1093830912},
+    "72b": {"sha256_prefix": "fc5d9ea0e4553c80", "bytes_per_launch": 2500334080},
 }
 
 

@@ -2,8 +2,10 @@
 the fp64 oracle element by element: ragged prefixes (including none), odd tail lengths and
 head counts, GQA ratios from 1 to 16, both head dimensions; odd row counts, hidden sizes,
 vocabularies and gather counts for the LM head; odd candidate, frame and dimension counts
-for CLIP; ragged prefixes and cache fills for the decode step.  The shapes are drawn once
-from a fixed seed, so every run checks the same cases."""
+for CLIP; ragged prefixes and cache fills for the decode step; keyframe and corpus counts,
+dimensions, k_frame and k_query for retrieval; frame sizes, video lengths and thresholds
+for keyframe extraction.  The shapes are drawn once from fixed seeds, so every run checks
+the same cases."""
 import numpy as np
 import pytest
 import torch
@@ -130,3 +132,49 @@ def test_decode_random_shapes(case):
                                 x["k_cache"], x["v_cache"], x["cache_len"])
     assert np.max(np.abs(out - ro)) <= ATTN_ATOL
     assert np.max(np.abs(lse - rl)) <= ATTN_LSE_ATOL
+
+
+def _retrieve_cases():
+    rng = np.random.default_rng(20261206)
+    out = []
+    for _ in range(N_CASES):
+        nq, kf = int(rng.integers(1, 5)), int(rng.integers(1, 9))
+        # the per-keyframe lists: ceil(keyframes / 128) * 128 * k_frame <= 4096
+        cap = (4096 // (128 * kf)) * 128
+        nkf = [int(n) if rng.random() > 0.1 else 0 for n in rng.integers(0, cap // nq + 1, nq)]
+        out.append((tuple(nkf), int(rng.integers(1, 6000)), 8 * int(rng.integers(8, 97)), kf,
+                    int(rng.integers(1, 65))))
+    return out
+
+
+@pytest.mark.parametrize("case", _retrieve_cases(),
+                         ids=lambda c: "kf" + "-".join(map(str, c[0])) + "_N%d_E%d_k%d_K%d" % c[1:])
+def test_retrieve_random_shapes(case):
+    from test_gpu_retrieval import _check_retrieve
+    nkf, Nt, E, kf, Kq = case
+    offs = np.zeros(len(nkf) + 1, np.int32)
+    offs[1:] = np.cumsum(nkf)
+    frames = synth.round_f16(synth.normal_f64((int(offs[-1]), E), 9000 + Nt, 1))
+    texts = synth.unit_rows_f16(Nt, E, 9000 + Nt, 2)
+    _check_retrieve(frames, offs, texts, kf, Kq)
+
+
+def _keyframe_cases():
+    rng = np.random.default_rng(20261207)
+    # frames start on 16-byte boundaries: width a multiple of 16 pixels
+    return [(int(rng.integers(1, 97)), 16 * int(rng.integers(1, 7)),
+             tuple(int(n) for n in rng.integers(0, 40, int(rng.integers(1, 5)))), float(rng.uniform(0.3, 0.9)))
+            for _ in range(N_CASES)]
+
+
+@pytest.mark.parametrize("case", _keyframe_cases(),
+                         ids=lambda c: "%dx%d_" % c[:2] + "-".join(map(str, c[2])) + "_t%.2f" % c[3])
+def test_keyframes_random_shapes(case):
+    from test_gpu_retrieval import _check_keyframes
+    h, w, lens, theta = case
+    cfg = configs.KF_TINY.with_(height=h, width=w, num_videos=1, frames_range=(1, 1), scene_mean=4.0)
+    voffs = np.zeros(len(lens) + 1, np.int32)
+    voffs[1:] = np.cumsum(lens)
+    T = int(voffs[-1])
+    px, _ = synth.video_frames(cfg.with_(frames_range=(max(T, 1), max(T, 1))))
+    _check_keyframes(px[:T], voffs, theta)

@@ -31,6 +31,11 @@
  *                            Eq. 12 reliability, Eq. 13 high-reliability set,
  *                            argmax alignment over it (mode 1), and the
  *                            other strategies of Sections 4.5-4.6 (modes 2-6).
+ *                            Parity unpinned against the paper on two readings
+ *                            only: the mean (not the sum) of the token log-probs
+ *                            in mode 0, and which token ids stand for "Yes" and
+ *                            "No" (the caller's targets); the function itself is
+ *                            pinned by the tests.
  *   oracle_decode_attn    -- one decode step of the K drafts (Eq. 5, Eq. 8-10):
  *                            each draft's newest token over the shared prefix
  *                            and its own tokens.
